@@ -1,0 +1,466 @@
+/*
+ * mikv_oracle.c — plain CPU oracle for the MiKV decode path (arxiv 2402.18096).
+ *
+ * TEST INFRASTRUCTURE ONLY: used by the tests, the smoke check and the benchmark's CPU-baseline
+ * leg to check the CUDA library; the product path never calls it. It is deliberately simple:
+ * one loop per formula, no blocking, no vectorisation, no reordering beyond what the formulas state.
+ *
+ * Build: gcc -O2 -ffp-contract=off -fno-fast-math -shared -fPIC (see oracle/__init__.py).
+ *
+ * Sections of the paper followed:
+ *   Eq. 1  (Sec. 3.1, "Retaining Evicted KVs with Quantization"): asymmetric N-bit round-to-nearest
+ *          quantizer, alpha = (max - min) / (2^N - 1), beta = min, per token.
+ *   Sec. 3.2 ("Low-bit KV Quantization with Dynamic Outlier Awareness"): group size of half the
+ *          head dimension; Eq. 2 channel balancer from prefill maxima; Eq. 3 keys multiplied by the
+ *          balancer before the quantizer; Eq. 4 query divided by it.
+ *   Fig. 4 and Sec. 3: important KV pairs kept in high precision and chosen by an accumulated
+ *          attention-score (heavy-hitter) policy; the others retained in low precision.
+ *   Sec. 3.4 ("Accelerating the Mixed-Precision KV Cache"): attention is permutation invariant, so
+ *          the important and retained sets are stored apart and attended together.
+ *   Tables 2-3 ("Cache size" columns): memory accounting.
+ * Readings where the paper is silent are stated next to the code that takes them.
+ */
+#include "mikv_oracle.h"
+
+#include <math.h>
+#include <stdlib.h>
+#include <string.h>
+
+/* ---------------------------------------------------------------- number formats */
+
+static float bf16_to_f32(uint16_t h) {
+  uint32_t u = (uint32_t)h << 16;
+  float f;
+  memcpy(&f, &u, sizeof f);
+  return f;
+}
+
+double mikv_ref_f16_to_f64(uint16_t h) {
+  int sign = h >> 15, e = (h >> 10) & 31, m = h & 1023;
+  double v;
+  if (e == 0)
+    v = ldexp((double)m, -24); /* subnormal: m * 2^-24 */
+  else if (e == 31)
+    v = m ? NAN : INFINITY;
+  else
+    v = ldexp((double)(1024 + m), e - 25); /* (1 + m/1024) * 2^(e-15) */
+  return sign ? -v : v;
+}
+
+/* Encode a finite double that is exactly representable in fp16 (|v| <= 65504). */
+static uint16_t encode_f16_exact(double v) {
+  uint16_t sign = signbit(v) ? 0x8000 : 0;
+  double a = fabs(v);
+  if (a == 0.0) return sign;
+  int ex;
+  frexp(a, &ex);
+  int E = ex - 1; /* a in [2^E, 2^(E+1)) */
+  if (E < -14) return (uint16_t)(sign | (uint16_t)ldexp(a, 24));
+  int mant = (int)ldexp(a, 10 - E) - 1024;
+  return (uint16_t)(sign | ((E + 15) << 10) | mant);
+}
+
+/* IEEE 754 binary32 -> binary16 conversion with the given rounding direction. */
+uint16_t mikv_ref_f32_to_f16(float f, int mode) {
+  if (isnan(f)) return 0x7E00;
+  uint16_t sign = signbit(f) ? 0x8000 : 0;
+  if (isinf(f)) return sign | 0x7C00;
+  double a = fabs((double)f);
+  if (a == 0.0) return sign;
+  int ex;
+  frexp(a, &ex);
+  int E = ex - 1;
+  if (E > 15) { /* beyond the largest binade */
+    if (mode == 0) return sign | 0x7C00;
+    if (mode < 0) return sign ? 0xFC00 : 0x7BFF;
+    return sign ? 0xFBFF : 0x7C00;
+  }
+  if (E < -14) E = -14; /* subnormal range shares the quantum 2^-24 */
+  double m = ldexp((double)f, 10 - E); /* exact: f has a 24-bit significand */
+  double r = mode < 0 ? floor(m) : (mode > 0 ? ceil(m) : nearbyint(m));
+  double v = ldexp(r, E - 10);
+  if (fabs(v) > 65504.0) return sign | 0x7C00; /* rounded past the largest finite value */
+  return encode_f16_exact(v);
+}
+
+/* ---------------------------------------------------------------- Eq. 1 quantizer */
+
+/*
+ * Eq. 1 on one group. Readings (the paper gives the formula, not the storage):
+ *  - beta and alpha are stored in fp16. beta16 = fp16 rounded toward -inf of min(x) and
+ *    alpha16 = fp16 rounded toward +inf of fp32((max(x) - beta16) / (2^N - 1)), so that the stored
+ *    grid beta16 + alpha16 * [0, 2^N - 1] covers [min, max].
+ *  - the code is round-half-to-even of the fp32 quotient (x - beta16) / alpha16, clamped to
+ *    [0, 2^N - 1].
+ *  - a group whose values all equal an fp16 number has span 0; alpha16 is then 1.0 and every code 0.
+ */
+int mikv_ref_quantize_group(const float* x, int g, int bits, int32_t* codes, uint16_t* alpha16,
+                            uint16_t* beta16) {
+  float mn = x[0], mx = x[0];
+  for (int i = 1; i < g; ++i) {
+    if (x[i] < mn) mn = x[i];
+    if (x[i] > mx) mx = x[i];
+  }
+  const int qmax = (1 << bits) - 1;
+  uint16_t b16 = mikv_ref_f32_to_f16(mn, -1);
+  float beta = (float)mikv_ref_f16_to_f64(b16);
+  float span = mx - beta;
+  uint16_t a16 = span == 0.0f ? (uint16_t)0x3C00 : mikv_ref_f32_to_f16(span / (float)qmax, +1);
+  float alpha = (float)mikv_ref_f16_to_f64(a16);
+  for (int i = 0; i < g; ++i) {
+    float t = (x[i] - beta) / alpha;
+    int c = (int)nearbyintf(t);
+    if (c < 0) c = 0;
+    if (c > qmax) c = qmax;
+    codes[i] = c;
+  }
+  *alpha16 = a16;
+  *beta16 = b16;
+  return 0;
+}
+
+/* ---------------------------------------------------------------- bit packing */
+
+/*
+ * Packed row layout (our own definition, d = 128). Channel c is written c = 16 m + u with
+ * u = c mod 16 and m = c div 16. A plane is a sequence of little-endian 16-bit units.
+ *  - plane of f-bit fields, f in {2, 4, 8}: P = 16 / f codes per unit; the code of channel c sits in
+ *    unit 8 * (2 * (m div P) + (u div 8)) + (u mod 8), at bits [f * (m mod P), f * (m mod P) + f).
+ *  - plane of 1-bit fields: the bit of channel c sits in unit (u mod 8), at bit 8 * (u div 8) + m.
+ * N = 2, 4, 8: one plane of N-bit fields. N = 3: a plane of 2-bit fields holding bits 0..1 of each
+ * code, then a plane of 1-bit fields holding bit 2. A row takes 16 * N bytes.
+ */
+static void field_position(int c, int f, int* unit, int* bit) {
+  int u = c % 16, m = c / 16;
+  if (f == 1) {
+    *unit = u % 8;
+    *bit = 8 * (u / 8) + m;
+    return;
+  }
+  int P = 16 / f;
+  *unit = 8 * (2 * (m / P) + u / 8) + u % 8;
+  *bit = f * (m % P);
+}
+
+static int plane_count(int bits) { return bits == 3 ? 2 : 1; }
+static int plane_width(int bits, int p) { return bits == 3 ? (p == 0 ? 2 : 1) : bits; }
+static int plane_shift(int bits, int p) { return bits == 3 && p == 1 ? 2 : 0; }
+
+static int valid_bits(int bits) { return bits == 2 || bits == 3 || bits == 4 || bits == 8; }
+
+int mikv_ref_pack_row(const int32_t* codes, int d, int bits, uint8_t* packed) {
+  if (!valid_bits(bits) || d != 128) return -1;
+  memset(packed, 0, (size_t)d * bits / 8);
+  size_t offset = 0;
+  for (int p = 0; p < plane_count(bits); ++p) {
+    int f = plane_width(bits, p), sh = plane_shift(bits, p);
+    uint32_t mask = (1u << f) - 1;
+    for (int c = 0; c < d; ++c) {
+      int unit, b;
+      field_position(c, f, &unit, &b);
+      uint32_t v = (((uint32_t)codes[c] >> sh) & mask) << b;
+      uint8_t* at = packed + offset + 2 * (size_t)unit;
+      at[0] |= (uint8_t)(v & 0xFF);
+      at[1] |= (uint8_t)(v >> 8);
+    }
+    offset += (size_t)d * f / 8;
+  }
+  return 0;
+}
+
+int mikv_ref_unpack_row(const uint8_t* packed, int d, int bits, int32_t* codes) {
+  if (!valid_bits(bits) || d != 128) return -1;
+  for (int c = 0; c < d; ++c) codes[c] = 0;
+  size_t offset = 0;
+  for (int p = 0; p < plane_count(bits); ++p) {
+    int f = plane_width(bits, p), sh = plane_shift(bits, p);
+    uint32_t mask = (1u << f) - 1;
+    for (int c = 0; c < d; ++c) {
+      int unit, b;
+      field_position(c, f, &unit, &b);
+      const uint8_t* at = packed + offset + 2 * (size_t)unit;
+      uint32_t word = (uint32_t)at[0] | (uint32_t)at[1] << 8;
+      codes[c] |= (int32_t)(((word >> b) & mask) << sh);
+    }
+    offset += (size_t)d * f / 8;
+  }
+  return 0;
+}
+
+/* ---------------------------------------------------------------- rows */
+
+int mikv_ref_quantize_row(const float* x, int d, int bits, int g, uint8_t* packed, uint16_t* params) {
+  if (!valid_bits(bits) || g <= 0 || d % g || d != 128) return -1;
+  int32_t* codes = (int32_t*)malloc(sizeof(int32_t) * (size_t)d);
+  if (!codes) return -1;
+  for (int j = 0; j < d / g; ++j)
+    mikv_ref_quantize_group(x + (size_t)j * g, g, bits, codes + (size_t)j * g, &params[2 * j],
+                            &params[2 * j + 1]);
+  mikv_ref_pack_row(codes, d, bits, packed);
+  free(codes);
+  return 0;
+}
+
+int mikv_ref_dequantize_row(const uint8_t* packed, const uint16_t* params, int d, int bits, int g,
+                            double* x_hat) {
+  if (!valid_bits(bits) || g <= 0 || d % g || d != 128) return -1;
+  int32_t* codes = (int32_t*)malloc(sizeof(int32_t) * (size_t)d);
+  if (!codes) return -1;
+  mikv_ref_unpack_row(packed, d, bits, codes);
+  for (int i = 0; i < d; ++i) {
+    double alpha = mikv_ref_f16_to_f64(params[2 * (i / g)]);
+    double beta = mikv_ref_f16_to_f64(params[2 * (i / g) + 1]);
+    x_hat[i] = alpha * codes[i] + beta; /* Eq. 1: alpha * round((x - beta) / alpha) + beta */
+  }
+  free(codes);
+  return 0;
+}
+
+/* ---------------------------------------------------------------- Eq. 2 balancer */
+
+/*
+ * Eq. 2. Readings: the maxima run over every batch row and prefill token (the equation has no batch
+ * index); under grouped-query attention the query maximum also runs over the G query heads sharing
+ * the KV head, since the balanced keys are shared by them. A zero maximum on either side gives 1.
+ * fp32: sqrt(max|q| / max|k|), IEEE division and square root.
+ */
+int mikv_ref_balancer(int B, int Hq, int Hkv, int T, int d, const uint16_t* q_pre,
+                      const uint16_t* k_pre, float* balancer) {
+  if (B <= 0 || Hkv <= 0 || Hq % Hkv || T <= 0 || d <= 0) return -1;
+  int G = Hq / Hkv;
+  for (int h = 0; h < Hkv; ++h) {
+    for (int c = 0; c < d; ++c) {
+      float mq = 0.0f, mk = 0.0f;
+      for (int b = 0; b < B; ++b)
+        for (int t = 0; t < T; ++t) {
+          for (int j = 0; j < G; ++j) {
+            float v = fabsf(bf16_to_f32(q_pre[(((size_t)b * Hq + h * G + j) * T + t) * d + c]));
+            if (v > mq) mq = v;
+          }
+          float v = fabsf(bf16_to_f32(k_pre[(((size_t)b * Hkv + h) * T + t) * d + c]));
+          if (v > mk) mk = v;
+        }
+      balancer[(size_t)h * d + c] = (mq == 0.0f || mk == 0.0f) ? 1.0f : sqrtf(mq / mk);
+    }
+  }
+  return 0;
+}
+
+/* ---------------------------------------------------------------- demotion (quantize + pack) */
+
+int mikv_ref_quantize_pack(int B, int Hkv, int d, int bits, int g, int lo_cap, const uint16_t* k_src,
+                           const uint16_t* v_src, const int32_t* src_tok, int n_src,
+                           const int32_t* rows, int n_rows, int lo_start, const float* balancer,
+                           uint8_t* k_codes, uint8_t* v_codes, uint16_t* k_params,
+                           uint16_t* v_params, int32_t* lo_tok) {
+  if (!valid_bits(bits) || g <= 0 || d % g || d != 128 || n_rows < 0 || lo_start < 0 ||
+      lo_start + n_rows > lo_cap)
+    return -1;
+  size_t row_bytes = (size_t)d * bits / 8, ngroups = (size_t)(d / g);
+  float* x = (float*)malloc(sizeof(float) * (size_t)d);
+  if (!x) return -1;
+  for (int b = 0; b < B; ++b)
+    for (int h = 0; h < Hkv; ++h)
+      for (int i = 0; i < n_rows; ++i) {
+        size_t bh = (size_t)b * Hkv + h;
+        int r = rows[bh * n_rows + i];
+        if (r < 0 || r >= n_src) { free(x); return -1; }
+        size_t pos = bh * lo_cap + (size_t)(lo_start + i);
+        const uint16_t* krow = k_src + (bh * n_src + r) * d;
+        const uint16_t* vrow = v_src + (bh * n_src + r) * d;
+        for (int c = 0; c < d; ++c) /* Eq. 3: key times balancer before the quantizer */
+          x[c] = bf16_to_f32(krow[c]) * (balancer ? balancer[(size_t)h * d + c] : 1.0f);
+        mikv_ref_quantize_row(x, d, bits, g, k_codes + pos * row_bytes, k_params + pos * ngroups * 2);
+        for (int c = 0; c < d; ++c) x[c] = bf16_to_f32(vrow[c]);
+        mikv_ref_quantize_row(x, d, bits, g, v_codes + pos * row_bytes, v_params + pos * ngroups * 2);
+        lo_tok[pos] = src_tok ? src_tok[bh * n_src + r] : r;
+      }
+  free(x);
+  return 0;
+}
+
+/* ---------------------------------------------------------------- decode attention */
+
+/*
+ * softmax(s) V over the union of the important set (bf16 keys/values, attended with q) and the
+ * retained set (dequantized balanced keys attended with q / balancer, Eq. 3-4; dequantized values).
+ * The union is unordered (Sec. 3.4 permutation invariance). s = sm_scale * q.k.
+ * Reading: important keys are stored without the balancer and attended with the plain query; in exact
+ * arithmetic (q / b).(k * b) = q.k, so this is the same attention.
+ */
+int mikv_ref_decode_attention(int B, int Hq, int Hkv, int d, int bits, int g, int hi_cap, int lo_cap,
+                              int n_lo, const uint16_t* k_hi, const uint16_t* v_hi,
+                              const uint8_t* k_codes, const uint8_t* v_codes,
+                              const uint16_t* k_params, const uint16_t* v_params,
+                              const float* balancer, const uint16_t* q, double sm_scale,
+                              double* out, double* hi_logits, double* ml) {
+  if (B <= 0 || Hkv <= 0 || Hq % Hkv || !valid_bits(bits) || g <= 0 || d % g || d != 128 ||
+      hi_cap < 0 || n_lo < 0 || n_lo > lo_cap || hi_cap + n_lo == 0)
+    return -1;
+  int G = Hq / Hkv;
+  size_t row_bytes = (size_t)d * bits / 8, ngroups = (size_t)(d / g);
+  int n = hi_cap + n_lo;
+  double* s = (double*)malloc(sizeof(double) * (size_t)n);
+  double* qv = (double*)malloc(sizeof(double) * (size_t)d);
+  double* qhat = (double*)malloc(sizeof(double) * (size_t)d);
+  double* xr = (double*)malloc(sizeof(double) * (size_t)d);
+  if (!s || !qv || !qhat || !xr) { free(s); free(qv); free(qhat); free(xr); return -1; }
+  for (int b = 0; b < B; ++b)
+    for (int hq = 0; hq < Hq; ++hq) {
+      int h = hq / G;
+      size_t bh = (size_t)b * Hkv + h, bq = (size_t)b * Hq + hq;
+      for (int c = 0; c < d; ++c) {
+        qv[c] = bf16_to_f32(q[bq * d + c]);
+        qhat[c] = qv[c] / (balancer ? (double)balancer[(size_t)h * d + c] : 1.0); /* Eq. 4 */
+      }
+      /* logits */
+      for (int i = 0; i < hi_cap; ++i) {
+        double acc = 0.0;
+        for (int c = 0; c < d; ++c) acc += qv[c] * bf16_to_f32(k_hi[(bh * hi_cap + i) * d + c]);
+        s[i] = sm_scale * acc;
+      }
+      for (int t = 0; t < n_lo; ++t) {
+        size_t pos = bh * lo_cap + t;
+        mikv_ref_dequantize_row(k_codes + pos * row_bytes, k_params + pos * ngroups * 2, d, bits, g, xr);
+        double acc = 0.0;
+        for (int c = 0; c < d; ++c) acc += qhat[c] * xr[c];
+        s[hi_cap + t] = sm_scale * acc;
+      }
+      /* softmax */
+      double m = -INFINITY;
+      for (int i = 0; i < n; ++i)
+        if (s[i] > m) m = s[i];
+      double l = 0.0;
+      for (int i = 0; i < n; ++i) l += exp(s[i] - m);
+      /* weighted values */
+      double* o = out + bq * d;
+      for (int c = 0; c < d; ++c) o[c] = 0.0;
+      for (int i = 0; i < hi_cap; ++i) {
+        double p = exp(s[i] - m) / l;
+        for (int c = 0; c < d; ++c) o[c] += p * bf16_to_f32(v_hi[(bh * hi_cap + i) * d + c]);
+      }
+      for (int t = 0; t < n_lo; ++t) {
+        size_t pos = bh * lo_cap + t;
+        double p = exp(s[hi_cap + t] - m) / l;
+        mikv_ref_dequantize_row(v_codes + pos * row_bytes, v_params + pos * ngroups * 2, d, bits, g, xr);
+        for (int c = 0; c < d; ++c) o[c] += p * xr[c];
+      }
+      if (hi_logits)
+        for (int i = 0; i < hi_cap; ++i) hi_logits[bq * hi_cap + i] = s[i];
+      if (ml) {
+        ml[2 * bq] = m;
+        ml[2 * bq + 1] = l;
+      }
+    }
+  free(s); free(qv); free(qhat); free(xr);
+  return 0;
+}
+
+/* ---------------------------------------------------------------- importance policy */
+
+/*
+ * Heavy-hitter importance (the accumulated-attention policy the paper plugs in, Fig. 4 / Sec. 3):
+ * each important slot's score grows by the attention weight it receives at this step, summed over the
+ * query heads that read it. Reading: retained tokens are not tracked (their high-precision values are
+ * gone, so they cannot be promoted back) and no recent-token window is kept.
+ */
+int mikv_ref_update_importance(int B, int Hq, int Hkv, int hi_cap, const float* hi_logits,
+                               const float* ml, float* acc) {
+  if (B <= 0 || Hkv <= 0 || Hq % Hkv || hi_cap < 0) return -1;
+  int G = Hq / Hkv;
+  for (int b = 0; b < B; ++b)
+    for (int h = 0; h < Hkv; ++h)
+      for (int i = 0; i < hi_cap; ++i) {
+        size_t bh = (size_t)b * Hkv + h;
+        double add = 0.0;
+        for (int j = 0; j < G; ++j) {
+          size_t bq = (size_t)b * Hq + (size_t)h * G + j;
+          add += exp((double)hi_logits[bq * hi_cap + i] - (double)ml[2 * bq]) / (double)ml[2 * bq + 1];
+        }
+        acc[bh * hi_cap + i] = (float)((double)acc[bh * hi_cap + i] + add);
+      }
+  return 0;
+}
+
+static int key_less(float sa, int32_t ia, float sb, int32_t ib) {
+  if (sa < sb) return 1;
+  if (sb < sa) return 0;
+  return ia < ib;
+}
+
+/*
+ * Demotion choice: the n_demote slots with the lowest (score, token id) leave the important set.
+ * Reading: ties on the score go to the older (smaller id) token; results are listed by slot.
+ * A slot's rank is the number of slots whose key is smaller (keys are distinct because ids are).
+ */
+int mikv_ref_select_demote(int B, int Hkv, int n, int n_demote, const float* scores,
+                           const int32_t* ids, int32_t* demoted, int32_t* kept) {
+  if (B <= 0 || Hkv <= 0 || n < 0 || n_demote < 0 || n_demote > n) return -1;
+  for (int b = 0; b < B; ++b)
+    for (int h = 0; h < Hkv; ++h) {
+      size_t bh = (size_t)b * Hkv + h;
+      const float* sc = scores + bh * n;
+      int nd = 0, nk = 0;
+      for (int i = 0; i < n; ++i) {
+        int32_t idi = ids ? ids[bh * n + i] : i;
+        int rank = 0;
+        for (int j = 0; j < n; ++j) {
+          int32_t idj = ids ? ids[bh * n + j] : j;
+          if (j != i && key_less(sc[j], idj, sc[i], idi)) ++rank;
+        }
+        if (rank < n_demote)
+          demoted[bh * n_demote + nd++] = i;
+        else if (kept)
+          kept[bh * (n - n_demote) + nk++] = i;
+      }
+    }
+  return 0;
+}
+
+int mikv_ref_insert_token(int B, int Hkv, int d, int hi_cap, const uint16_t* k_new,
+                          const uint16_t* v_new, int tok, const int32_t* slots, uint16_t* k_hi,
+                          uint16_t* v_hi, int32_t* hi_tok, float* acc) {
+  for (int b = 0; b < B; ++b)
+    for (int h = 0; h < Hkv; ++h) {
+      size_t bh = (size_t)b * Hkv + h;
+      int s = slots[bh];
+      if (s < 0 || s >= hi_cap) return -1;
+      memcpy(k_hi + (bh * hi_cap + s) * d, k_new + bh * d, sizeof(uint16_t) * (size_t)d);
+      memcpy(v_hi + (bh * hi_cap + s) * d, v_new + bh * d, sizeof(uint16_t) * (size_t)d);
+      hi_tok[bh * hi_cap + s] = tok;
+      acc[bh * hi_cap + s] = 0.0f;
+    }
+  return 0;
+}
+
+int mikv_ref_gather_hi(int B, int Hkv, int d, int hi_cap, const uint16_t* k_src,
+                       const uint16_t* v_src, const int32_t* src_tok, const float* src_scores,
+                       int n_src, const int32_t* rows, int n_rows, uint16_t* k_hi, uint16_t* v_hi,
+                       int32_t* hi_tok, float* acc) {
+  if (n_rows > hi_cap || n_rows < 0) return -1;
+  for (int b = 0; b < B; ++b)
+    for (int h = 0; h < Hkv; ++h)
+      for (int i = 0; i < n_rows; ++i) {
+        size_t bh = (size_t)b * Hkv + h;
+        int r = rows[bh * n_rows + i];
+        if (r < 0 || r >= n_src) return -1;
+        memcpy(k_hi + (bh * hi_cap + i) * d, k_src + (bh * n_src + r) * d, sizeof(uint16_t) * (size_t)d);
+        memcpy(v_hi + (bh * hi_cap + i) * d, v_src + (bh * n_src + r) * d, sizeof(uint16_t) * (size_t)d);
+        hi_tok[bh * hi_cap + i] = src_tok ? src_tok[bh * n_src + r] : r;
+        acc[bh * hi_cap + i] = src_scores ? src_scores[bh * n_src + r] : 0.0f;
+      }
+  return 0;
+}
+
+/* ---------------------------------------------------------------- memory accounting */
+
+/*
+ * Cache size relative to fp16 for every token (the "Cache size" columns of Tables 2-3): a token in
+ * the important set costs hi_bits per element (plus 32/g bits of fp16 alpha and beta when it is itself
+ * quantized), a retained token bits + 32/g. Returned as a fraction.
+ */
+double mikv_ref_cache_fraction(int bits, int g, double ratio, int hi_bits) {
+  double hi = hi_bits >= 16 ? 1.0 : (hi_bits + 32.0 / g) / 16.0;
+  double lo = (bits + 32.0 / g) / 16.0;
+  return ratio * hi + (1.0 - ratio) * lo;
+}
