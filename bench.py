@@ -1,0 +1,409 @@
+"""Benchmark of the MiKV decode hot path on GB300.
+
+A step = one decode token through every layer of the workload: per layer, insert the new KV pair,
+attend over the mixed-precision cache (bf16 important set + low-bit retained set), update the
+accumulated-attention scores, pick the least important slot and quantize/pack it into the retained set.
+The metric is the compressed-KV bytes the attention reads per step divided by the step time (GB/s),
+with ms per step alongside. Inputs are seeded synthetic tensors resident in HBM before timing; the cache
+(tens of GB) is far larger than L2, so no flush is needed between steps.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload mistral-7b|llama2-7b|llama2-13b|tiny]
+  python bench.py --impl reference ...   # the CPU oracle on a bounded sample of the same workload
+
+Multi-GPU (torchrun, one process per GPU): the (batch, head) units are independent, so every rank runs
+its own batch of the workload with no data-path collective (weak scaling); ranks only meet at the
+timing barrier and a max-reduce of the elapsed time.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import torch  # noqa: E402
+
+import mikv_inputs as mi  # noqa: E402
+
+METRIC = "decode-attn compressed-KV GB/s and % of GB300 HBM peak; us per decode step"
+UNIT = "GB/s"
+DEFAULT_WORKLOAD = "mistral-7b"
+
+
+def _peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = os.path.join("/tmp", f"mikv_clocks_{os.getpid()}.csv")
+
+    def start(self):
+        try:
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=self.fh, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.fh.close()
+        sm, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    mx = max(mx, float(parts[2]))
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[5:9]):
+                    if v.lower() == "active":
+                        reasons.add(n)
+        os.unlink(self.path)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def _dist():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        return dist, rank, world, local
+    return None, 0, 1, local
+
+
+def _max_over_ranks(dist, x: float) -> float:
+    if dist is None:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def build_model(w, steps_cap: int, dev, rank: int):
+    """All layers' caches, built from seeded prefill tensors with the library's own kernels."""
+    import paper_2402_18096_gb300 as pkg
+    from paper_2402_18096_gb300.layer import MixedPrecisionLayer
+    shape = pkg.Shape(w.batch, w.heads_q, w.heads_kv, w.bits, w.group, w.hi_cap, w.lo_cap_for(steps_cap))
+    wr = mi.scaled(w, seed=w.seed + 7919 * rank)  # each rank owns a different batch
+    layers = []
+    for li in range(w.layers):
+        k, v = mi.prefill_kv(wr, li, dev)
+        scores = mi.initial_scores(wr, li, dev)
+        q_pre = mi.prefill_queries(wr, li, dev)
+        layers.append(MixedPrecisionLayer.from_prefill(shape, k, v, scores, q_pre, device=dev))
+        del k, v, scores, q_pre
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+    return shape, layers
+
+
+def run_mikv(args):
+    import paper_2402_18096_gb300 as pkg
+    dist, rank, world, local = _dist()
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    pkg.load()
+    w = mi.WORKLOADS[args.workload]
+    if args.batch:
+        w = mi.scaled(w, batch=args.batch)
+    if args.layers:
+        w = mi.scaled(w, layers=args.layers)
+    K, W = args.steps, args.warmup
+    e2e_steps = max(2, K // 2)
+    attn_reps = 2
+    steps_cap = W + K + W + e2e_steps + 4
+    shape, layers = build_model(w, steps_cap, dev, rank)
+    L = len(layers)
+    # per-step decode inputs, resident on the device
+    n_in = W + K
+    inputs = [[mi.decode_inputs(mi.scaled(w, seed=w.seed + 7919 * rank), li, s, dev) for li in range(L)]
+              for s in range(n_in)]
+    out = torch.empty(w.batch, w.heads_q, w.head_dim, dtype=torch.bfloat16, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step(s):
+        for li, layer in enumerate(layers):
+            q, kn, vn = inputs[s][li]
+            layer.step(q, kn, vn, out)
+
+    def compressed_bytes():
+        return sum(layer.cache.nbytes_attended(layer.n_lo) for layer in layers)
+
+    for s in range(W):
+        step(s)
+    torch.cuda.synchronize()
+    for layer in layers:
+        pkg.mikv_workspace_check(layer.ws)
+
+    bytes_before = compressed_bytes()
+    clocks = ClockSampler(torch.cuda.current_device()) if rank == 0 else None
+    if clocks:
+        clocks.start()
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for s in range(K):
+        step(W + s)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    clk = clocks.stop() if clocks else None
+    bytes_after = compressed_bytes()
+    # bytes attended over the K steps: n_lo grows by one per step per layer
+    bytes_per_step = (bytes_before + bytes_after) / 2 - sum(
+        layer.cache.nbytes_attended(1) - layer.cache.nbytes_attended(0) for layer in layers) / 2
+    ms = e0.elapsed_time(e1) / K
+    ms = _max_over_ranks(dist, ms)
+    for layer in layers:
+        pkg.mikv_workspace_check(layer.ws)
+
+    # ---- dominant kernel alone: decode attention (split-K kernel + merge), same caches, events on stream
+    ws_attn = [torch.zeros(pkg.mikv_workspace_bytes(shape, pkg.WS_ATTENTION, layer.n_lo) + 256, dtype=torch.uint8,
+                           device=dev) for layer in layers[:1]]
+    q0 = inputs[0][0][0]
+    a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    a0.record(stream)
+    for _ in range(attn_reps):
+        for layer in layers:
+            pkg.mikv_decode_attention(layer.cache, layer.n_lo, q0, layer.sm_scale, out, ws_attn[0])
+    a1.record(stream)
+    torch.cuda.synchronize()
+    attn_ms = a0.elapsed_time(a1) / (attn_reps * L)
+    attn_bytes = sum(layer.cache.nbytes_attended(layer.n_lo) for layer in layers) / L
+
+    # ---- end to end through the C ABI with host buffers: H2D inputs, D2H outputs, every step
+    per_in = [inputs[0][li] for li in range(L)]
+    host_in = [[t.cpu().pin_memory() for t in trip] for trip in per_in]
+    host_out = torch.empty(L, w.batch, w.heads_q, w.head_dim, dtype=torch.bfloat16).pin_memory()
+    dev_in = [[torch.empty_like(t) for t in trip] for trip in per_in]
+    dev_out = torch.empty(L, w.batch, w.heads_q, w.head_dim, dtype=torch.bfloat16, device=dev)
+    h2d = sum(t.numel() * t.element_size() for trip in host_in for t in trip)
+    d2h = host_out.numel() * host_out.element_size()
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    t0 = time.perf_counter()
+    for s in range(e2e_steps):
+        for li, layer in enumerate(layers):
+            for d, h in zip(dev_in[li], host_in[li]):
+                d.copy_(h, non_blocking=True)
+            layer.step(dev_in[li][0], dev_in[li][1], dev_in[li][2], dev_out[li])
+        host_out.copy_(dev_out, non_blocking=True)
+        torch.cuda.current_stream().synchronize()
+    e2e_ms = (time.perf_counter() - t0) * 1e3 / e2e_steps
+    e2e_ms = _max_over_ranks(dist, e2e_ms)
+    for layer in layers:
+        pkg.mikv_workspace_check(layer.ws)
+
+    peak, peak_kind = _peaks()
+    value = world * bytes_per_step / (ms * 1e-3) / 1e9
+    achieved = attn_bytes / (attn_ms * 1e-3) / 1e9
+    line = {
+        "metric": METRIC,
+        "value": round(value, 1),
+        "unit": UNIT,
+        "n_gpus": world,
+        "steps": K,
+        "warmup": W,
+        "ms_per_step": round(ms, 4),
+        "us_per_step": round(ms * 1e3, 1),
+        "pct_of_hbm_peak": round(100 * value / world / peak, 1),
+        "hbm_peak_gbs": peak,
+        "hbm_peak_kind": peak_kind,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16+int%d" % w.bits,
+        "data": "synthetic",
+        "config": {"workload": w.name, "batch": w.batch, "layers": L, "heads_q": w.heads_q, "heads_kv": w.heads_kv,
+                   "context": w.context, "bits": w.bits, "group": w.group, "importance_ratio": w.ratio,
+                   "compressed_bytes_per_step": int(bytes_per_step), "l2": "cache larger than L2, no flush",
+                   "parallelism": f"replicas{world}"},
+        "roofline": {"kernel": "decode attention (split-K + merge)", "bound": "hbm", "achieved": round(achieved, 1),
+                     "peak": peak, "unit": "GB/s", "frac": round(achieved / peak, 3),
+                     "traffic": None, "bytes_per_launch": int(attn_bytes), "avg_launch_us": round(attn_ms * 1e3, 2)},
+        "e2e": {"value": round(world * bytes_per_step / (e2e_ms * 1e-3) / 1e9, 1), "unit": UNIT,
+                "ms_per_step": round(e2e_ms, 4), "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": K * L * 6,
+    }
+    if clk:
+        line["clocks"] = clk
+    if rank == 0 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(w, seconds=args.cpu_seconds)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+# ------------------------------------------------------------------ CPU oracle (reference arm)
+
+def _oracle_head(w, b, h, steps_cap):
+    """Oracle cache of one (batch row, KV head) built from seeded prefill tensors of that head (drawn on
+    the GPU when there is one, only to save time, then copied to the host)."""
+    import numpy as np
+    import oracle
+    gen_dev = "cuda" if torch.cuda.is_available() else "cpu"
+    G = w.heads_q // w.heads_kv
+    k, v = mi.prefill_kv(w, 0, gen_dev, heads=[h])
+    scores = mi.initial_scores(w, 0, gen_dev, rows=[b], heads=[h]).cpu()
+    q_pre = mi.prefill_queries(w, 0, gen_dev, heads=list(range(h * G, (h + 1) * G)))
+    bal = oracle.balancer(mi.bf16_bits(q_pre), mi.bf16_bits(k))
+    ks, vs = mi.bf16_bits(k[b:b + 1]), mi.bf16_bits(v[b:b + 1])
+    sc = scores.numpy()
+    del k, v, q_pre
+    dem, kept = oracle.select_demote(sc, w.context - w.budget)
+    c = oracle.empty_cache(1, 1, w.head_dim, w.bits, w.group, w.hi_cap, w.lo_cap_for(steps_cap))
+    oracle.gather_hi(c, ks, vs, kept, src_scores=sc)
+    oracle.quantize_pack(c, ks, vs, dem, 0, balancer_=bal)
+    return c, bal, np.array([[w.budget]], np.int32)
+
+
+def _oracle_step(w, c, bal, slots, n_lo, pos, q, kn, vn):
+    """One decode step of one KV head on the oracle, in the library's order."""
+    import numpy as np
+    import oracle
+    G = w.heads_q // w.heads_kv
+    oracle.insert_token(c, kn, vn, pos, slots)
+    _, hl, ml = oracle.decode_attention(c, q, n_lo, 1 / math.sqrt(w.head_dim), balancer_=bal)
+    c["acc"] = oracle.update_importance(c["acc"], hl.astype(np.float32), ml.astype(np.float32), G)
+    dem, _ = oracle.select_demote(c["acc"], 1, c["hi_tok"], want_kept=False)
+    oracle.quantize_pack(c, c["k_hi"], c["v_hi"], dem, n_lo, src_tok=c["hi_tok"], balancer_=bal)
+    return dem[0]
+
+
+def _head_bytes(w, n_lo):
+    lo = 2 * (w.head_dim * w.bits // 8 + 4 * (w.head_dim // w.group))
+    return w.hi_cap * 4 * w.head_dim + n_lo * lo
+
+
+def cpu_baseline(w, seconds: float = 15.0, steps=None):
+    """The oracle, as it stands, on a bounded sample: whole decode steps of single KV heads."""
+    import oracle
+    oracle.build()
+    G = w.heads_q // w.heads_kv
+    c, bal, slots = _oracle_head(w, 0, 0, 64)
+    n_lo = w.n_lo0
+    done_bytes, elapsed, n = 0, 0.0, 0
+    while (steps is None and elapsed < seconds) or (steps is not None and n < steps):
+        q, kn, vn = mi.decode_inputs(w, 0, n, "cpu", rows=[0], kv_heads=[0])
+        qb = mi.bf16_bits(q[:, :G])
+        kb, vb = mi.bf16_bits(kn[:, :1]), mi.bf16_bits(vn[:, :1])
+        t0 = time.perf_counter()
+        slots = _oracle_step(w, c, bal, slots, n_lo, w.context + n, qb, kb, vb)
+        elapsed += time.perf_counter() - t0
+        done_bytes += _head_bytes(w, n_lo)
+        n_lo += 1
+        n += 1
+        if n_lo >= c["k_codes"].shape[2]:
+            break
+    return {"value": round(done_bytes / elapsed / 1e9, 4), "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"{n} whole decode steps of one KV head (batch row 0, head 0, layer 0) of {w.name}; "
+                      f"single-threaded C, fp64 attention; bytes = that head's compressed KV",
+            "ms_per_head_step": round(1e3 * elapsed / n, 3)}
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    w = mi.WORKLOADS[args.workload]
+    K, W = args.steps, args.warmup
+    import oracle
+    oracle.build()
+    G = w.heads_q // w.heads_kv
+    c, bal, slots = _oracle_head(w, 0, 0, W + K + 4)
+    n_lo = w.n_lo0
+    times, nbytes = [], []
+    for s in range(W + K):
+        q, kn, vn = mi.decode_inputs(w, 0, s, "cpu", rows=[0], kv_heads=[0])
+        qb, kb, vb = mi.bf16_bits(q[:, :G]), mi.bf16_bits(kn[:, :1]), mi.bf16_bits(vn[:, :1])
+        t0 = time.perf_counter()
+        slots = _oracle_step(w, c, bal, slots, n_lo, w.context + s, qb, kb, vb)
+        dt = time.perf_counter() - t0
+        if s >= W:
+            times.append(dt)
+            nbytes.append(_head_bytes(w, n_lo))
+        n_lo += 1
+    value = sum(nbytes) / sum(times) / 1e9
+    ms = 1e3 * sum(times) / K
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": UNIT, "n_gpus": 0,
+        "steps": K, "warmup": W, "ms_per_step": round(ms, 3), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64 attention, f32 quantizer", "data": "synthetic",
+        "config": {"workload": w.name, "sample": "one KV head (batch row 0, head 0) of layer 0 per step"},
+        "cpu_baseline": {"value": round(value, 4), "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": f"{K} whole decode steps of one KV head of {w.name}, single-threaded C"},
+        "e2e": {"value": round(value, 4), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="mikv", choices=["mikv", "reference"])
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(mi.WORKLOADS))
+    ap.add_argument("--batch", type=int, default=0, help="smaller batch (profiling cases only)")
+    ap.add_argument("--layers", type=int, default=0, help="fewer layers (profiling cases only)")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "mikv" and not (args.batch or args.layers):
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_mikv(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -14,7 +14,7 @@ Mistral-7b, Sec. 4.1), which are not available here:
 """
 from __future__ import annotations
 
-from dataclasses import dataclass, field, replace
+from dataclasses import dataclass, replace
 from typing import List, Optional
 
 import torch
@@ -86,6 +86,22 @@ def scaled(w: Workload, **kw) -> Workload:
 
 
 # ------------------------------------------------------------------ random tensors
+#
+# Every tensor is drawn in independent chunks, one per (batch row, head), each from its own seeded
+# generator, so any subset of rows and heads can be produced alone (the CPU oracle draws only the heads
+# it checks) and equals the same slice of the full tensor drawn on the same device.
+
+KIND_K, KIND_V, KIND_QPRE, KIND_SCORES, KIND_Q, KIND_KNEW, KIND_VNEW = range(7)
+_MASK63 = (1 << 63) - 1
+
+
+def _seed(w: Workload, layer: int, kind: int, b: int, h: int, step: int = 0) -> int:
+    x = w.seed
+    for v in (layer, kind, b, h, step):
+        x = (x * 6364136223846793005 + 1442695040888963407 + v) & _MASK63
+        x ^= x >> 29
+    return x
+
 
 def _gen(device, seed: int) -> torch.Generator:
     g = torch.Generator(device=device)
@@ -95,7 +111,7 @@ def _gen(device, seed: int) -> torch.Generator:
 
 def outlier_channels(w: Workload, layer: int) -> torch.Tensor:
     """int64 [Hkv, 4]: the outlier key channels of each KV head of `layer` (CPU)."""
-    g = _gen("cpu", w.seed * 1000003 + 7919 * layer + 17)
+    g = _gen("cpu", _seed(w, layer, 99, 0, 0))
     half = w.head_dim // 2
     out = torch.empty(w.heads_kv, 4, dtype=torch.int64)
     for h in range(w.heads_kv):
@@ -104,59 +120,79 @@ def outlier_channels(w: Workload, layer: int) -> torch.Tensor:
     return out
 
 
-def prefill_kv(w: Workload, layer: int, device="cpu", batch: Optional[int] = None,
-               context: Optional[int] = None):
-    """bf16 K, V [B, Hkv, T, d] of one layer's prefill, keys with 4 outlier channels per head x10."""
-    B = w.batch if batch is None else batch
-    T = w.context if context is None else context
-    g = _gen(device, w.seed * 1000003 + 1000 * layer + 1)
-    k = torch.randn(B, w.heads_kv, T, w.head_dim, generator=g, device=device)
-    v = torch.randn(B, w.heads_kv, T, w.head_dim, generator=g, device=device)
-    oc = outlier_channels(w, layer).to(device)
-    scale = torch.ones(w.heads_kv, w.head_dim, device=device)
-    scale.scatter_(1, oc, OUTLIER_SCALE)
-    k.mul_(scale[None, :, None, :])
-    return k.to(torch.bfloat16), v.to(torch.bfloat16)
+def _channel_scale(w: Workload, layer: int, device) -> torch.Tensor:
+    """fp32 [Hkv, d]: 10 on each KV head's outlier channels, 1 elsewhere."""
+    scale = torch.ones(w.heads_kv, w.head_dim)
+    scale.scatter_(1, outlier_channels(w, layer), OUTLIER_SCALE)
+    return scale.to(device)
 
 
-def prefill_queries(w: Workload, layer: int, device="cpu", batch: Optional[int] = None,
-                    context: Optional[int] = None):
-    """bf16 Q [B, Hq, T, d] of one layer's prefill, with the query side of the outlier channels
-    (the same channels as the keys of the KV head, scaled x10)."""
-    B = w.batch if batch is None else batch
-    T = w.context if context is None else context
-    g = _gen(device, w.seed * 1000003 + 1000 * layer + 2)
-    q = torch.randn(B, w.heads_q, T, w.head_dim, generator=g, device=device)
+def _draw(w, layer, kind, rows, heads, n, device, scale_of_head=None, step=0):
+    out = torch.empty(len(rows), len(heads), *n, dtype=torch.bfloat16, device=device)
+    for i, b in enumerate(rows):
+        for j, h in enumerate(heads):
+            x = torch.randn(*n, generator=_gen(device, _seed(w, layer, kind, b, h, step)), device=device)
+            if scale_of_head is not None:
+                x.mul_(scale_of_head(h))
+            out[i, j] = x.to(torch.bfloat16)
+    return out
+
+
+def prefill_kv(w: Workload, layer: int, device="cpu", rows=None, heads=None):
+    """bf16 K, V [B, Hkv, T, d] of one layer's prefill; keys carry 4 outlier channels per head x10.
+    rows / heads select batch rows and KV heads (default: all)."""
+    rows = range(w.batch) if rows is None else rows
+    heads = range(w.heads_kv) if heads is None else heads
+    sc = _channel_scale(w, layer, device)
+    n = (w.context, w.head_dim)
+    k = _draw(w, layer, KIND_K, rows, heads, n, device, lambda h: sc[h])
+    v = _draw(w, layer, KIND_V, rows, heads, n, device)
+    return k, v
+
+
+def prefill_queries(w: Workload, layer: int, device="cpu", rows=None, heads=None):
+    """bf16 Q [B, Hq, T, d] of one layer's prefill; query heads carry the outlier channels of their KV
+    head, scaled x10. heads selects query heads."""
+    rows = range(w.batch) if rows is None else rows
+    heads = range(w.heads_q) if heads is None else heads
     G = w.heads_q // w.heads_kv
-    oc = outlier_channels(w, layer).to(device)
-    scale = torch.ones(w.heads_kv, w.head_dim, device=device)
-    scale.scatter_(1, oc, OUTLIER_SCALE)
-    q.mul_(scale.repeat_interleave(G, 0)[None, :, None, :])
-    return q.to(torch.bfloat16)
+    sc = _channel_scale(w, layer, device)
+    return _draw(w, layer, KIND_QPRE, rows, heads, (w.context, w.head_dim), device, lambda h: sc[h // G])
 
 
-def initial_scores(w: Workload, layer: int, device="cpu", batch: Optional[int] = None,
-                   context: Optional[int] = None):
+def initial_scores(w: Workload, layer: int, device="cpu", rows=None, heads=None):
     """fp32 [B, Hkv, T] synthetic accumulated-attention scores of the prefill tokens."""
-    B = w.batch if batch is None else batch
-    T = w.context if context is None else context
-    g = _gen(device, w.seed * 1000003 + 1000 * layer + 3)
-    return torch.randn(B, w.heads_kv, T, generator=g, device=device).exp_()
+    rows = range(w.batch) if rows is None else rows
+    heads = range(w.heads_kv) if heads is None else heads
+    out = torch.empty(len(rows), len(heads), w.context, dtype=torch.float32, device=device)
+    for i, b in enumerate(rows):
+        for j, h in enumerate(heads):
+            g = _gen(device, _seed(w, layer, KIND_SCORES, b, h))
+            out[i, j] = torch.randn(w.context, generator=g, device=device).exp_()
+    return out
 
 
-def decode_inputs(w: Workload, layer: int, step: int, device="cpu", batch: Optional[int] = None):
-    """(q bf16 [B, Hq, d], k_new bf16 [B, Hkv, d], v_new bf16 [B, Hkv, d]) of one decode step;
-    the new key carries the layer's outlier channels like the prefill keys."""
-    B = w.batch if batch is None else batch
-    g = _gen(device, w.seed * 1000003 + 1000 * layer + 10 + 7 * step)
-    q = torch.randn(B, w.heads_q, w.head_dim, generator=g, device=device)
-    k = torch.randn(B, w.heads_kv, w.head_dim, generator=g, device=device)
-    v = torch.randn(B, w.heads_kv, w.head_dim, generator=g, device=device)
-    oc = outlier_channels(w, layer).to(device)
-    scale = torch.ones(w.heads_kv, w.head_dim, device=device)
-    scale.scatter_(1, oc, OUTLIER_SCALE)
-    k.mul_(scale[None])
-    return q.to(torch.bfloat16), k.to(torch.bfloat16), v.to(torch.bfloat16)
+def decode_inputs(w: Workload, layer: int, step: int, device="cpu", rows=None, kv_heads=None):
+    """(q bf16 [B, Hq, d], k_new bf16 [B, Hkv, d], v_new bf16 [B, Hkv, d]) of one decode step; the new
+    key carries the layer's outlier channels. Drawn per batch row (all heads at once); kv_heads selects
+    KV heads (and their query heads) from the drawn rows."""
+    rows = range(w.batch) if rows is None else rows
+    G = w.heads_q // w.heads_kv
+    sc = _channel_scale(w, layer, device)
+    q = torch.empty(len(rows), w.heads_q, w.head_dim, dtype=torch.bfloat16, device=device)
+    k = torch.empty(len(rows), w.heads_kv, w.head_dim, dtype=torch.bfloat16, device=device)
+    v = torch.empty_like(k)
+    for i, b in enumerate(rows):
+        q[i] = torch.randn(w.heads_q, w.head_dim, device=device,
+                           generator=_gen(device, _seed(w, layer, KIND_Q, b, 0, step))).to(torch.bfloat16)
+        k[i] = (torch.randn(w.heads_kv, w.head_dim, device=device,
+                            generator=_gen(device, _seed(w, layer, KIND_KNEW, b, 0, step))) * sc).to(torch.bfloat16)
+        v[i] = torch.randn(w.heads_kv, w.head_dim, device=device,
+                           generator=_gen(device, _seed(w, layer, KIND_VNEW, b, 0, step))).to(torch.bfloat16)
+    if kv_heads is not None:
+        qh = [h * G + j for h in kv_heads for j in range(G)]
+        q, k, v = q[:, qh].contiguous(), k[:, list(kv_heads)].contiguous(), v[:, list(kv_heads)].contiguous()
+    return q, k, v
 
 
 def bf16_bits(t: torch.Tensor):

@@ -1,0 +1,367 @@
+// mikv_abi.cu — host side of the libmikv C ABI (include/mikv.h): argument validation, tensor-map
+// encoding for TMA, workspace layout and kernel dispatch. Nothing here allocates device memory or
+// synchronises, except mikv_workspace_check which reads the status word on request.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <mutex>
+
+#include "mikv_device.cuh"
+#include "mikv_internal.h"
+
+using namespace mikv;
+
+namespace {
+
+mikv_status cuda_status(cudaError_t e) { return e == cudaSuccess ? MIKV_OK : MIKV_ERR_CUDA; }
+
+int num_sms() {
+  int dev = 0, n = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 148;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) return 148;
+  return n;
+}
+
+bool shape_ok(const mikv_shape* s) {
+  return s && s->batch > 0 && s->heads_q > 0 && s->heads_kv > 0 && s->heads_q % s->heads_kv == 0 &&
+         s->head_dim > 0 && s->bits > 0 && s->group > 0 && s->hi_cap >= 0 && s->hi_stride >= s->hi_cap &&
+         s->hi_stride % 16 == 0 && s->lo_cap >= 0 && s->lo_cap % 16 == 0;
+}
+
+mikv_status shape_supported(const mikv_shape* s) {
+  if (!shape_ok(s)) return MIKV_ERR_ARG;
+  const int G = s->heads_q / s->heads_kv;
+  if (s->head_dim != kHeadDim) return MIKV_ERR_UNSUPPORTED;
+  if (s->bits < 2 || s->bits > 4) return MIKV_ERR_UNSUPPORTED;
+  if (s->group != 32 && s->group != 64 && s->group != 128) return MIKV_ERR_UNSUPPORTED;
+  if (G != 1 && G != 2 && G != 4 && G != 8) return MIKV_ERR_UNSUPPORTED;
+  return MIKV_OK;
+}
+
+bool cache_ok(const mikv_cache* c) {
+  return c && c->k_hi && c->v_hi && c->hi_tok && c->acc && c->k_codes && c->v_codes && c->k_params &&
+         c->v_params && c->lo_tok;
+}
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+// ------------------------------------------------------------------ tensor maps
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+struct MapKey {
+  const void* ptr;
+  uint64_t inner, rows, stride;
+  uint32_t bx, by;
+  int dtype, swz;
+  bool operator==(const MapKey& o) const { return memcmp(this, &o, sizeof(MapKey)) == 0; }
+};
+
+// Encoded maps are kept per (pointer, geometry): a layer's cache arrays are reused every step.
+bool make_map(CUtensorMap* out, const void* ptr, CUtensorMapDataType dtype, uint64_t inner, uint64_t rows,
+              uint64_t stride_bytes, uint32_t bx, uint32_t by, CUtensorMapSwizzle swz) {
+  static std::mutex mu;
+  static MapKey keys[64];
+  static CUtensorMap maps[64];
+  static int used = 0, next = 0;
+  MapKey k;
+  memset(&k, 0, sizeof k);
+  k.ptr = ptr;
+  k.inner = inner;
+  k.rows = rows;
+  k.stride = stride_bytes;
+  k.bx = bx;
+  k.by = by;
+  k.dtype = (int)dtype;
+  k.swz = (int)swz;
+  std::lock_guard<std::mutex> lock(mu);
+  for (int i = 0; i < used; ++i)
+    if (keys[i] == k) {
+      *out = maps[i];
+      return true;
+    }
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) return false;
+  const cuuint64_t dims[2] = {inner, rows};
+  const cuuint64_t strides[1] = {stride_bytes};
+  const cuuint32_t box[2] = {bx, by};
+  const cuuint32_t estr[2] = {1, 1};
+  CUtensorMap m;
+  if (enc(&m, dtype, 2, const_cast<void*>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
+          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return false;
+  const int slot = used < 64 ? used++ : (next++ & 63);
+  keys[slot] = k;
+  maps[slot] = m;
+  *out = m;
+  return true;
+}
+
+struct StepLayout {
+  size_t attn, logits, ml, total;
+};
+
+StepLayout step_layout(const mikv_shape* s, int n_lo_max) {
+  StepLayout L;
+  L.attn = attention_workspace_bytes(*s, n_lo_max, num_sms());
+  const size_t logits = (size_t)s->batch * s->heads_q * s->hi_stride * sizeof(float);
+  const size_t ml = (size_t)s->batch * s->heads_q * 2 * sizeof(float);
+  L.logits = L.attn;
+  L.ml = L.logits + (logits + 255) / 256 * 256;
+  L.total = L.ml + (ml + 255) / 256 * 256;
+  return L;
+}
+
+mikv_status attention_impl(const mikv_shape* s, const mikv_cache* c, int32_t n_lo, const void* q, float sm_scale,
+                           void* out, int32_t out_dtype, float* hi_logits, float* ml, void* ws, size_t ws_bytes,
+                           cudaStream_t st) {
+  const int sms = num_sms();
+  const AttnPlan plan = plan_attention(*s, n_lo, sms);
+  if (ws_bytes < attention_workspace_bytes(*s, n_lo, sms)) return MIKV_ERR_WORKSPACE;
+  const int G = s->heads_q / s->heads_kv;
+  AttnArgs a;
+  memset(&a, 0, sizeof a);
+  const uint64_t hi_rows = (uint64_t)s->batch * s->heads_kv * s->hi_stride;
+  const uint64_t lo_rows = (uint64_t)s->batch * s->heads_kv * s->lo_cap;
+  const uint64_t row_bytes = 16ull * s->bits;
+  bool ok = make_map(&a.map_k_hi, c->k_hi, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, kHeadDim, hi_rows, 2 * kHeadDim, 64,
+                     16, CU_TENSOR_MAP_SWIZZLE_128B) &&
+            make_map(&a.map_v_hi, c->v_hi, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, kHeadDim, hi_rows, 2 * kHeadDim, 64,
+                     16, CU_TENSOR_MAP_SWIZZLE_128B);
+  if (ok && lo_rows > 0) {
+    if (s->bits == 3) {
+      ok = make_map(&a.map_k_lo, c->k_codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, row_bytes, lo_rows, row_bytes, 32, 16,
+                    CU_TENSOR_MAP_SWIZZLE_32B) &&
+           make_map(&a.map_v_lo, c->v_codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, row_bytes, lo_rows, row_bytes, 32, 16,
+                    CU_TENSOR_MAP_SWIZZLE_32B) &&
+           make_map(&a.map_k_lo1, c->k_codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, row_bytes, lo_rows, row_bytes, 16,
+                    16, CU_TENSOR_MAP_SWIZZLE_NONE) &&
+           make_map(&a.map_v_lo1, c->v_codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, row_bytes, lo_rows, row_bytes, 16,
+                    16, CU_TENSOR_MAP_SWIZZLE_NONE);
+    } else {
+      const CUtensorMapSwizzle swz = s->bits == 2 ? CU_TENSOR_MAP_SWIZZLE_32B : CU_TENSOR_MAP_SWIZZLE_64B;
+      ok = make_map(&a.map_k_lo, c->k_codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, row_bytes, lo_rows, row_bytes,
+                    (uint32_t)row_bytes, 16, swz) &&
+           make_map(&a.map_v_lo, c->v_codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, row_bytes, lo_rows, row_bytes,
+                    (uint32_t)row_bytes, 16, swz);
+    }
+  }
+  if (!ok) return MIKV_ERR_CUDA;
+  a.k_params = c->k_params;
+  a.v_params = c->v_params;
+  a.q = q;
+  a.balancer = c->balancer;
+  a.hi_logits = hi_logits;
+  char* wsb = static_cast<char*>(ws);
+  a.status = reinterpret_cast<int*>(wsb);
+  a.part_o = reinterpret_cast<float*>(wsb + kWsHeader);
+  a.part_ml = a.part_o + (size_t)plan.n_items * G * kHeadDim;
+  a.batch = s->batch;
+  a.heads_q = s->heads_q;
+  a.heads_kv = s->heads_kv;
+  a.hi_cap = s->hi_cap;
+  a.hi_stride = s->hi_stride;
+  a.lo_cap = s->lo_cap;
+  a.n_lo = n_lo;
+  a.hi_blocks = (s->hi_cap + 15) / 16;
+  a.lo_blocks = (n_lo + 15) / 16;
+  a.n_split = plan.n_split;
+  a.n_items = plan.n_items;
+  a.sm_scale = sm_scale;
+  cudaError_t e = launch_attention(a, s->bits, s->group, G, plan.grid, st);
+  if (e != cudaSuccess) return MIKV_ERR_CUDA;
+  MergeArgs m;
+  m.part_o = a.part_o;
+  m.part_ml = a.part_ml;
+  m.out = out;
+  m.ml = ml;
+  m.batch = s->batch;
+  m.heads_q = s->heads_q;
+  m.heads_kv = s->heads_kv;
+  m.n_split = plan.n_split;
+  e = launch_merge(m, G, out_dtype == MIKV_OUT_F32, st);
+  return cuda_status(e);
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* mikv_status_string(mikv_status s) {
+  switch (s) {
+    case MIKV_OK: return "ok";
+    case MIKV_ERR_ARG: return "invalid argument";
+    case MIKV_ERR_UNSUPPORTED: return "unsupported configuration";
+    case MIKV_ERR_CAPACITY: return "capacity exceeded";
+    case MIKV_ERR_CUDA: return "CUDA error";
+    case MIKV_ERR_WORKSPACE: return "workspace missing, too small or misaligned";
+    case MIKV_ERR_DEVICE: return "a kernel reported an internal failure";
+  }
+  return "unknown status";
+}
+
+size_t mikv_workspace_bytes(const mikv_shape* shape, int32_t op, int32_t n_lo_max) {
+  if (shape_supported(shape) != MIKV_OK || n_lo_max < 0) return 0;
+  switch (op) {
+    case MIKV_WS_ATTENTION: return attention_workspace_bytes(*shape, n_lo_max, num_sms());
+    case MIKV_WS_BALANCER: return kWsHeader + 2 * (size_t)shape->heads_kv * kHeadDim * sizeof(uint32_t);
+    case MIKV_WS_STEP: return step_layout(shape, n_lo_max).total;
+  }
+  return 0;
+}
+
+mikv_status mikv_workspace_reset(void* workspace, size_t ws_bytes, void* stream) {
+  if (!workspace || ws_bytes < kWsHeader) return MIKV_ERR_WORKSPACE;
+  return cuda_status(cudaMemsetAsync(workspace, 0, sizeof(int), static_cast<cudaStream_t>(stream)));
+}
+
+mikv_status mikv_workspace_check(const void* workspace, void* stream) {
+  if (!workspace) return MIKV_ERR_WORKSPACE;
+  int v = 0;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (cudaMemcpyAsync(&v, workspace, sizeof v, cudaMemcpyDeviceToHost, st) != cudaSuccess) return MIKV_ERR_CUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return MIKV_ERR_CUDA;
+  return v == 0 ? MIKV_OK : MIKV_ERR_DEVICE;
+}
+
+mikv_status mikv_compute_balancer(const mikv_shape* shape, const void* q_pre, const void* k_pre, int32_t T,
+                                  float* balancer_out, void* workspace, size_t ws_bytes, void* stream) {
+  mikv_status st = shape_supported(shape);
+  if (st != MIKV_OK) return st;
+  if (!q_pre || !k_pre || !balancer_out || T <= 0) return MIKV_ERR_ARG;
+  if (!workspace || !aligned(workspace, 256) ||
+      ws_bytes < mikv_workspace_bytes(shape, MIKV_WS_BALANCER, 0))
+    return MIKV_ERR_WORKSPACE;
+  uint32_t* ws = reinterpret_cast<uint32_t*>(static_cast<char*>(workspace) + kWsHeader);
+  return cuda_status(launch_balancer(*shape, q_pre, k_pre, T, balancer_out, ws, static_cast<cudaStream_t>(stream)));
+}
+
+mikv_status mikv_quantize_pack(const mikv_shape* shape, const mikv_cache* cache, const void* k_src,
+                               const void* v_src, const int32_t* src_tok, int32_t n_src, const int32_t* rows,
+                               int32_t n_rows, int32_t lo_start, void* stream) {
+  mikv_status st = shape_supported(shape);
+  if (st != MIKV_OK) return st;
+  if (!cache_ok(cache) || !k_src || !v_src || n_src <= 0 || n_rows < 0 || lo_start < 0 || (n_rows > 0 && !rows))
+    return MIKV_ERR_ARG;
+  if ((int64_t)lo_start + n_rows > shape->lo_cap) return MIKV_ERR_CAPACITY;
+  if ((int64_t)(n_rows + 3) / 4 > 2147483647 || (int64_t)shape->batch * shape->heads_kv > 65535)
+    return MIKV_ERR_UNSUPPORTED;
+  return cuda_status(launch_quantize_pack(*shape, *cache, k_src, v_src, src_tok, n_src, rows, n_rows, lo_start,
+                                          static_cast<cudaStream_t>(stream)));
+}
+
+mikv_status mikv_decode_attention(const mikv_shape* shape, const mikv_cache* cache, int32_t n_lo, const void* q,
+                                  float sm_scale, void* out, int32_t out_dtype, float* hi_logits, float* ml,
+                                  void* workspace, size_t ws_bytes, void* stream) {
+  mikv_status st = shape_supported(shape);
+  if (st != MIKV_OK) return st;
+  if (!cache_ok(cache) || !q || !out || n_lo < 0 || (out_dtype != MIKV_OUT_BF16 && out_dtype != MIKV_OUT_F32))
+    return MIKV_ERR_ARG;
+  if (n_lo > shape->lo_cap) return MIKV_ERR_CAPACITY;
+  if (shape->hi_cap + n_lo < 1) return MIKV_ERR_ARG;
+  if (!aligned(cache->k_hi, 16) || !aligned(cache->v_hi, 16) || !aligned(cache->k_codes, 16) ||
+      !aligned(cache->v_codes, 16) || !aligned(cache->k_params, 16) || !aligned(cache->v_params, 16) ||
+      !aligned(q, 4) || (cache->balancer && !aligned(cache->balancer, 16)))
+    return MIKV_ERR_ARG;
+  if (!workspace || !aligned(workspace, 256)) return MIKV_ERR_WORKSPACE;
+  return attention_impl(shape, cache, n_lo, q, sm_scale, out, out_dtype, hi_logits, ml, workspace, ws_bytes,
+                        static_cast<cudaStream_t>(stream));
+}
+
+mikv_status mikv_update_importance(const mikv_shape* shape, const mikv_cache* cache, const float* hi_logits,
+                                   const float* ml, void* stream) {
+  mikv_status st = shape_supported(shape);
+  if (st != MIKV_OK) return st;
+  if (!cache_ok(cache) || !hi_logits || !ml) return MIKV_ERR_ARG;
+  if (shape->hi_cap == 0) return MIKV_OK;
+  return cuda_status(launch_update_importance(*shape, *cache, hi_logits, ml, static_cast<cudaStream_t>(stream)));
+}
+
+mikv_status mikv_select_demote(int32_t batch, int32_t heads, const float* scores, const int32_t* ids, int32_t n,
+                               int32_t stride, int32_t n_demote, int32_t* demoted, int32_t* kept, void* stream) {
+  if (batch <= 0 || heads <= 0 || !scores || n < 0 || stride < n || n_demote < 0 || n_demote > n) return MIKV_ERR_ARG;
+  if (n_demote > 0 && !demoted) return MIKV_ERR_ARG;
+  if ((int64_t)batch * heads > 2147483647) return MIKV_ERR_UNSUPPORTED;
+  if (n == 0) return MIKV_OK;
+  return cuda_status(launch_select(batch, heads, scores, ids, n, stride, n_demote, demoted, kept,
+                                   static_cast<cudaStream_t>(stream)));
+}
+
+mikv_status mikv_insert_token(const mikv_shape* shape, const mikv_cache* cache, const void* k_new,
+                              const void* v_new, int32_t tok, const int32_t* slots, void* stream) {
+  mikv_status st = shape_supported(shape);
+  if (st != MIKV_OK) return st;
+  if (!cache_ok(cache) || !k_new || !v_new || !slots) return MIKV_ERR_ARG;
+  if (shape->hi_cap < 1) return MIKV_ERR_CAPACITY;
+  return cuda_status(launch_insert(*shape, *cache, k_new, v_new, tok, slots, static_cast<cudaStream_t>(stream)));
+}
+
+mikv_status mikv_gather_hi(const mikv_shape* shape, const mikv_cache* cache, const void* k_src, const void* v_src,
+                           const int32_t* src_tok, const float* src_scores, int32_t n_src, const int32_t* rows,
+                           int32_t n_rows, void* stream) {
+  mikv_status st = shape_supported(shape);
+  if (st != MIKV_OK) return st;
+  if (!cache_ok(cache) || !k_src || !v_src || n_src <= 0 || n_rows < 0 || (n_rows > 0 && !rows))
+    return MIKV_ERR_ARG;
+  if (n_rows > shape->hi_cap) return MIKV_ERR_CAPACITY;
+  return cuda_status(launch_gather(*shape, *cache, k_src, v_src, src_tok, src_scores, n_src, rows, n_rows,
+                                   static_cast<cudaStream_t>(stream)));
+}
+
+mikv_status mikv_decode_step(const mikv_shape* shape, const mikv_cache* cache, int32_t n_lo, const void* q,
+                             const void* k_new, const void* v_new, int32_t tok, int32_t* slots, float sm_scale,
+                             void* out, int32_t out_dtype, void* workspace, size_t ws_bytes, void* stream) {
+  mikv_status st = shape_supported(shape);
+  if (st != MIKV_OK) return st;
+  if (!cache_ok(cache) || !q || !k_new || !v_new || !slots || !out || n_lo < 0) return MIKV_ERR_ARG;
+  if (shape->hi_cap < 1) return MIKV_ERR_CAPACITY;
+  if ((int64_t)n_lo + 1 > shape->lo_cap) return MIKV_ERR_CAPACITY;
+  if (!workspace || !aligned(workspace, 256)) return MIKV_ERR_WORKSPACE;
+  const StepLayout L = step_layout(shape, n_lo);
+  if (ws_bytes < L.total) return MIKV_ERR_WORKSPACE;
+  char* wsb = static_cast<char*>(workspace);
+  float* logits = reinterpret_cast<float*>(wsb + L.logits);
+  float* ml = reinterpret_cast<float*>(wsb + L.ml);
+  if ((st = mikv_insert_token(shape, cache, k_new, v_new, tok, slots, stream)) != MIKV_OK) return st;
+  if ((st = mikv_decode_attention(shape, cache, n_lo, q, sm_scale, out, out_dtype, logits, ml, workspace, L.attn,
+                                  stream)) != MIKV_OK)
+    return st;
+  if ((st = mikv_update_importance(shape, cache, logits, ml, stream)) != MIKV_OK) return st;
+  if ((st = mikv_select_demote(shape->batch, shape->heads_kv, cache->acc, cache->hi_tok, shape->hi_cap,
+                               shape->hi_stride, 1, slots, nullptr, stream)) != MIKV_OK)
+    return st;
+  return mikv_quantize_pack(shape, cache, cache->k_hi, cache->v_hi, cache->hi_tok, shape->hi_stride, slots, 1, n_lo,
+                            stream);
+}
+
+double mikv_cache_fraction(int32_t bits, int32_t group, double ratio, int32_t hi_bits) {
+  if (group <= 0) return -1.0;
+  const double hi = hi_bits >= 16 ? 1.0 : (hi_bits + 32.0 / group) / 16.0;
+  const double lo = (bits + 32.0 / group) / 16.0;
+  return ratio * hi + (1.0 - ratio) * lo;
+}
+
+size_t mikv_retained_row_bytes(int32_t bits, int32_t group, int32_t head_dim) {
+  if (bits <= 0 || group <= 0 || head_dim <= 0 || head_dim % group) return 0;
+  return (size_t)head_dim * bits / 8 + (size_t)4 * (head_dim / group);
+}
+
+}  // extern "C"

@@ -1,0 +1,193 @@
+// mikv_quant.cu — demotion of KV rows into the retained set (Eq. 1 with the Eq. 3 key balancer) and
+// the channel balancer itself (Eq. 2), arxiv 2402.18096.
+//
+// quantize_pack: one warp per (row, K or V); each lane owns 4 consecutive channels. Group minima and
+// maxima come from butterfly shuffles over the GROUP/4 lanes of a group; scale and zero are rounded
+// to fp16 toward -inf (beta) and +inf (alpha) so the stored grid covers the group's range; codes are
+// round-half-even of the IEEE fp32 quotient (x - beta) / alpha. Every step uses explicitly rounded
+// intrinsics so the result is bit-identical to a plain IEEE evaluation. Codes are OR-ed into the
+// row's packed layout in shared memory and written out as whole words.
+#include "mikv_device.cuh"
+#include "mikv_internal.h"
+
+namespace mikv {
+namespace {
+
+struct QPArgs {
+  const __nv_bfloat16* k_src;
+  const __nv_bfloat16* v_src;
+  const int32_t* src_tok;
+  const int32_t* rows;
+  const float* balancer;
+  uint8_t* k_codes;
+  uint8_t* v_codes;
+  __half2* k_params;
+  __half2* v_params;
+  int32_t* lo_tok;
+  int heads_kv, n_src, n_rows, lo_start, lo_cap;
+};
+
+// Bit position of channel c (= 16 m + u) in a plane of f-bit fields: 16-bit unit and bit offset.
+__device__ __forceinline__ void field_pos(int c, int f, int& unit, int& bit) {
+  const int u = c & 15, m = c >> 4;
+  if (f == 1) {
+    unit = u & 7;
+    bit = 8 * (u >> 3) + m;
+  } else {
+    const int P = 16 / f;
+    unit = 8 * (2 * (m / P) + (u >> 3)) + (u & 7);
+    bit = f * (m % P);
+  }
+}
+
+template <int BITS, int GROUP>
+__global__ void __launch_bounds__(256) quantize_pack_kernel(const QPArgs a) {
+  constexpr int QMAX = (1 << BITS) - 1;
+  constexpr int LANES = GROUP / 4;       // lanes per quantization group
+  constexpr int WORDS = 4 * BITS;        // 32-bit words of one packed row
+  __shared__ uint32_t buf[8][16];
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int i = blockIdx.x * 4 + (w >> 1);
+  const bool is_v = (w & 1) != 0;
+  const int bh = blockIdx.y, h = bh % a.heads_kv;
+  if (lane < 16) buf[w][lane] = 0u;
+  __syncwarp();
+  if (i >= a.n_rows) return;
+  const int r = a.rows[(size_t)bh * a.n_rows + i];
+  if (r < 0 || r >= a.n_src) return;  // out-of-range rows are skipped (documented in the ABI)
+
+  const __nv_bfloat16* src = (is_v ? a.v_src : a.k_src) + ((size_t)bh * a.n_src + r) * kHeadDim + 4 * lane;
+  const uint2 raw = *reinterpret_cast<const uint2*>(src);
+  float x[4] = {__uint_as_float(raw.x << 16), __uint_as_float(raw.x & 0xffff0000u),
+                __uint_as_float(raw.y << 16), __uint_as_float(raw.y & 0xffff0000u)};
+  if (!is_v && a.balancer) {  // Eq. 3: keys times the balancer before the quantizer
+    const float4 b = *reinterpret_cast<const float4*>(a.balancer + h * kHeadDim + 4 * lane);
+    x[0] = __fmul_rn(x[0], b.x);
+    x[1] = __fmul_rn(x[1], b.y);
+    x[2] = __fmul_rn(x[2], b.z);
+    x[3] = __fmul_rn(x[3], b.w);
+  }
+  float mn = fminf(fminf(x[0], x[1]), fminf(x[2], x[3]));
+  float mx = fmaxf(fmaxf(x[0], x[1]), fmaxf(x[2], x[3]));
+#pragma unroll
+  for (int off = 1; off < LANES; off <<= 1) {
+    mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, off));
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+  }
+  // Eq. 1: beta = min, alpha = (max - min) / (2^N - 1), stored in fp16 with outward rounding.
+  const __half beta16 = __float2half_rd(mn);
+  const float beta = __half2float(beta16);
+  const float span = __fsub_rn(mx, beta);
+  const __half alpha16 = span == 0.f ? __float2half_rn(1.f) : __float2half_ru(__fdiv_rn(span, (float)QMAX));
+  const float alpha = __half2float(alpha16);
+
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    int code = __float2int_rn(__fdiv_rn(__fsub_rn(x[e], beta), alpha));
+    code = code < 0 ? 0 : (code > QMAX ? QMAX : code);
+    const int c = 4 * lane + e;
+    int unit, bit;
+    field_pos(c, BITS == 3 ? 2 : BITS, unit, bit);
+    const uint32_t fmask = BITS == 3 ? 3u : (uint32_t)QMAX;
+    atomicOr(&buf[w][unit >> 1], (((uint32_t)code & fmask) << bit) << (16 * (unit & 1)));
+    if (BITS == 3) {
+      field_pos(c, 1, unit, bit);
+      atomicOr(&buf[w][8 + (unit >> 1)], (((uint32_t)code >> 2) << bit) << (16 * (unit & 1)));
+    }
+  }
+  __syncwarp();
+  const size_t pos = (size_t)bh * a.lo_cap + a.lo_start + i;
+  uint32_t* dst = reinterpret_cast<uint32_t*>((is_v ? a.v_codes : a.k_codes) + pos * (16 * BITS));
+  if (lane < WORDS) dst[lane] = buf[w][lane];
+  if ((lane & (LANES - 1)) == 0) {
+    __half2* params = is_v ? a.v_params : a.k_params;
+    params[pos * (kHeadDim / GROUP) + (4 * lane) / GROUP] = __halves2half2(alpha16, beta16);
+  }
+  if (!is_v && lane == 0) a.lo_tok[pos] = a.src_tok ? a.src_tok[(size_t)bh * a.n_src + r] : r;
+}
+
+template <int BITS>
+cudaError_t qp_group(const QPArgs& a, int group, dim3 grid, cudaStream_t st) {
+  switch (group) {
+    case 32: quantize_pack_kernel<BITS, 32><<<grid, 256, 0, st>>>(a); break;
+    case 64: quantize_pack_kernel<BITS, 64><<<grid, 256, 0, st>>>(a); break;
+    case 128: quantize_pack_kernel<BITS, 128><<<grid, 256, 0, st>>>(a); break;
+    default: return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------- Eq. 2 balancer
+
+// Per (token chunk, batch row, head): column maxima of |x| folded into ws with atomicMax on the bit
+// patterns (non-negative floats order like their bits). Rows y < B*Hq are queries, the rest keys.
+__global__ void __launch_bounds__(128) absmax_kernel(const __nv_bfloat16* q_pre, const __nv_bfloat16* k_pre,
+                                                      int B, int Hq, int Hkv, int T, int chunk,
+                                                      uint32_t* ws) {
+  const int y = blockIdx.y, c = threadIdx.x;
+  const bool is_q = y < B * Hq;
+  const int yy = is_q ? y : y - B * Hq;
+  const int heads = is_q ? Hq : Hkv;
+  const int head = yy % heads;
+  const int h = is_q ? head / (Hq / Hkv) : head;
+  const __nv_bfloat16* base = (is_q ? q_pre : k_pre) + (size_t)yy * T * kHeadDim + c;
+  const int t0 = blockIdx.x * chunk, t1 = min(T, t0 + chunk);
+  float m = 0.f;
+  for (int t = t0; t < t1; ++t) m = fmaxf(m, fabsf(__bfloat162float(base[(size_t)t * kHeadDim])));
+  atomicMax(&ws[(is_q ? 0 : Hkv * kHeadDim) + h * kHeadDim + c], __float_as_uint(m));
+}
+
+__global__ void __launch_bounds__(128) balancer_kernel(const uint32_t* ws, int Hkv, float* out) {
+  const int h = blockIdx.x, c = threadIdx.x;
+  const float mq = __uint_as_float(ws[h * kHeadDim + c]);
+  const float mk = __uint_as_float(ws[Hkv * kHeadDim + h * kHeadDim + c]);
+  out[h * kHeadDim + c] = (mq == 0.f || mk == 0.f) ? 1.f : __fsqrt_rn(__fdiv_rn(mq, mk));
+}
+
+}  // namespace
+
+cudaError_t launch_quantize_pack(const mikv_shape& s, const mikv_cache& c, const void* k_src,
+                                 const void* v_src, const int32_t* src_tok, int n_src,
+                                 const int32_t* rows, int n_rows, int lo_start, cudaStream_t st) {
+  if (n_rows == 0) return cudaSuccess;
+  QPArgs a;
+  a.k_src = static_cast<const __nv_bfloat16*>(k_src);
+  a.v_src = static_cast<const __nv_bfloat16*>(v_src);
+  a.src_tok = src_tok;
+  a.rows = rows;
+  a.balancer = c.balancer;
+  a.k_codes = static_cast<uint8_t*>(c.k_codes);
+  a.v_codes = static_cast<uint8_t*>(c.v_codes);
+  a.k_params = static_cast<__half2*>(c.k_params);
+  a.v_params = static_cast<__half2*>(c.v_params);
+  a.lo_tok = c.lo_tok;
+  a.heads_kv = s.heads_kv;
+  a.n_src = n_src;
+  a.n_rows = n_rows;
+  a.lo_start = lo_start;
+  a.lo_cap = s.lo_cap;
+  const dim3 grid((n_rows + 3) / 4, s.batch * s.heads_kv);
+  switch (s.bits) {
+    case 2: return qp_group<2>(a, s.group, grid, st);
+    case 3: return qp_group<3>(a, s.group, grid, st);
+    case 4: return qp_group<4>(a, s.group, grid, st);
+  }
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_balancer(const mikv_shape& s, const void* q_pre, const void* k_pre, int T, float* out,
+                            uint32_t* ws_max, cudaStream_t st) {
+  cudaError_t e = cudaMemsetAsync(ws_max, 0, sizeof(uint32_t) * 2 * s.heads_kv * kHeadDim, st);
+  if (e != cudaSuccess) return e;
+  const int chunk = 256;
+  const dim3 grid((T + chunk - 1) / chunk, s.batch * (s.heads_q + s.heads_kv));
+  absmax_kernel<<<grid, kHeadDim, 0, st>>>(static_cast<const __nv_bfloat16*>(q_pre),
+                                           static_cast<const __nv_bfloat16*>(k_pre), s.batch, s.heads_q,
+                                           s.heads_kv, T, chunk, ws_max);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  balancer_kernel<<<s.heads_kv, kHeadDim, 0, st>>>(ws_max, s.heads_kv, out);
+  return cudaGetLastError();
+}
+
+}  // namespace mikv

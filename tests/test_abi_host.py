@@ -1,0 +1,129 @@
+"""Host-side checks of the C ABI (no GPU needed): the library builds and loads, exports every function
+include/mikv.h declares, validates arguments before launching anything, and its host-only helpers
+agree with the paper's memory accounting."""
+import ctypes
+import json
+import math
+import os
+import re
+
+import pytest
+
+import oracle
+import paper_2402_18096_gb300 as pkg
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "mikv.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    return pkg.load()
+
+
+def _declared():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?[a-z_0-9]+\s*\*?\s*(mikv_[a-z_0-9]+)\s*\(", text, re.M)))
+
+
+def test_exports_every_declared_symbol(lib):
+    names = _declared()
+    assert len(names) >= 14, names
+    for n in ["mikv_quantize_pack", "mikv_decode_attention", "mikv_update_importance", "mikv_select_demote"]:
+        assert n in names
+    for n in names:
+        assert hasattr(lib, n), n
+    # every name the header declares is a plain C symbol (no C++ mangling)
+    nm = os.popen(f"nm -D --defined-only {pkg._build.LIB}").read()
+    for n in names:
+        assert re.search(rf"\bT {n}$", nm, re.M), n
+
+
+def test_status_strings(lib):
+    for code in range(7):
+        assert pkg.mikv_status_string(code) not in ("", "unknown status")
+    assert pkg.mikv_status_string(99) == "unknown status"
+
+
+def test_cache_fraction_matches_oracle_and_tables(lib):
+    for bits in (2, 3, 4, 8):
+        for g in (32, 64, 128):
+            for r in (0.0, 0.05, 0.2, 0.5, 1.0):
+                for hb in (16, 8, 4, 2):
+                    assert pkg.mikv_cache_fraction(bits, g, r, hb) == pytest.approx(
+                        oracle.cache_fraction(bits, g, r, hb), rel=1e-15)
+    with open(os.path.join(ROOT, "tests", "golden", "cache_size_tables.json")) as f:
+        for row in json.load(f)["rows"]:
+            frac = pkg.mikv_cache_fraction(row["retained_bits"], row["group"], row["ratio"], row["importance_bits"])
+            assert math.floor(frac * 100 + 0.5) == row["cache_size_percent"]
+
+
+def test_row_bytes(lib):
+    assert pkg.mikv_retained_row_bytes(2, 32) == 32 + 16
+    assert pkg.mikv_retained_row_bytes(3, 64) == 48 + 8
+    assert pkg.mikv_retained_row_bytes(4, 128) == 64 + 4
+    assert pkg.mikv_retained_row_bytes(2, 48) == 0  # group must divide d
+
+
+def _shape(**kw):
+    s = dict(batch=2, heads_q=8, heads_kv=2, head_dim=128, bits=2, group=32, hi_cap=20, hi_stride=32, lo_cap=64)
+    s.update(kw)
+    return pkg._Shape(*[s[n] for n, _ in pkg._Shape._fields_])
+
+
+def _fake_cache():
+    # never dereferenced: validation rejects or the test stops before any launch
+    return pkg._Cache(*([0x10000] * 9 + [None]))
+
+
+def test_workspace_sizes_monotone(lib):
+    s = _shape()
+    sizes = [lib.mikv_workspace_bytes(ctypes.byref(s), 0, n) for n in (0, 16, 100, 1000, 5000)]
+    assert all(x > 0 for x in sizes)
+    assert sizes == sorted(sizes)
+    assert lib.mikv_workspace_bytes(ctypes.byref(s), 2, 64) >= lib.mikv_workspace_bytes(ctypes.byref(s), 0, 64)
+    assert lib.mikv_workspace_bytes(ctypes.byref(_shape(head_dim=64)), 0, 16) == 0
+    assert lib.mikv_workspace_bytes(ctypes.byref(_shape(bits=5)), 0, 16) == 0
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(head_dim=64), 2), (dict(bits=5), 2), (dict(bits=8), 2), (dict(group=48), 2),
+    (dict(heads_q=6, heads_kv=2), 2), (dict(heads_q=7), 1), (dict(hi_stride=24), 1),
+    (dict(lo_cap=60), 1), (dict(batch=0), 1), (dict(hi_stride=16, hi_cap=20), 1),
+])
+def test_shape_validation(lib, kw, code):
+    s = _shape(**kw)
+    c = _fake_cache()
+    rc = lib.mikv_quantize_pack(ctypes.byref(s), ctypes.byref(c), 0x10000, 0x10000, None, 4, 0x10000, 1, 0, None)
+    assert rc == code
+
+
+def test_argument_validation_before_launch(lib):
+    s = _shape()
+    c = _fake_cache()
+    P = 0x10000
+    # retained capacity: lo_start + n_rows > lo_cap
+    assert lib.mikv_quantize_pack(ctypes.byref(s), ctypes.byref(c), P, P, None, 4, P, 5, 60, None) == 3
+    # null cache member
+    bad = pkg._Cache(*([P] * 8 + [None, None]))
+    assert lib.mikv_quantize_pack(ctypes.byref(s), ctypes.byref(bad), P, P, None, 4, P, 1, 0, None) == 1
+    # attention: n_lo beyond capacity, bad output type, missing or misaligned workspace
+    assert lib.mikv_decode_attention(ctypes.byref(s), ctypes.byref(c), 65, P, 1.0, P, 0, None, None, P, 1 << 20,
+                                     None) == 3
+    assert lib.mikv_decode_attention(ctypes.byref(s), ctypes.byref(c), 3, P, 1.0, P, 7, None, None, P, 1 << 20,
+                                     None) == 1
+    assert lib.mikv_decode_attention(ctypes.byref(s), ctypes.byref(c), 3, P, 1.0, P, 0, None, None, None, 0,
+                                     None) == 5
+    assert lib.mikv_decode_attention(ctypes.byref(s), ctypes.byref(c), 3, P, 1.0, P, 0, None, None, P + 8, 1 << 20,
+                                     None) == 5
+    assert lib.mikv_decode_attention(ctypes.byref(s), ctypes.byref(c), 3, P, 1.0, P, 0, None, None, P, 16,
+                                     None) == 5
+    # selection: more demoted than entries, stride below n
+    assert lib.mikv_select_demote(2, 2, P, None, 10, 10, 11, P, None, None) == 1
+    assert lib.mikv_select_demote(2, 2, P, None, 10, 8, 1, P, None, None) == 1
+    # step: retained set full
+    full = _shape(lo_cap=16)
+    assert lib.mikv_decode_step(ctypes.byref(full), ctypes.byref(c), 16, P, P, P, 0, P, 1.0, P, 0, P, 1 << 30,
+                                None) == 3
+    # gather beyond the important capacity
+    assert lib.mikv_gather_hi(ctypes.byref(s), ctypes.byref(c), P, P, None, None, 40, P, 21, None) == 3
