@@ -112,12 +112,18 @@ def _dist():
     return None, 0, 1, local
 
 
-def _max_over_ranks(dist, x: float) -> float:
+def max_over_ranks(dist, x: float, device="cuda") -> float:
+    """The slowest rank's time: every rank contributes x, all receive the maximum."""
     if dist is None:
         return x
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    t = torch.tensor([x], dtype=torch.float64, device=device)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def rank_workload(w, rank: int):
+    """Weak scaling: every rank runs the same shape on its own batch (its own seeds)."""
+    return mi.scaled(w, seed=w.seed + 7919 * rank)
 
 
 def build_model(w, steps_cap: int, dev, rank: int):
@@ -125,7 +131,7 @@ def build_model(w, steps_cap: int, dev, rank: int):
     import paper_2402_18096_gb300 as pkg
     from paper_2402_18096_gb300.layer import MixedPrecisionLayer
     shape = pkg.Shape(w.batch, w.heads_q, w.heads_kv, w.bits, w.group, w.hi_cap, w.lo_cap_for(steps_cap))
-    wr = mi.scaled(w, seed=w.seed + 7919 * rank)  # each rank owns a different batch
+    wr = rank_workload(w, rank)  # each rank owns a different batch
     layers = []
     for li in range(w.layers):
         k, v = mi.prefill_kv(wr, li, dev)
@@ -157,7 +163,7 @@ def run_mikv(args):
     L = len(layers)
     # per-step decode inputs, resident on the device
     n_in = W + K
-    inputs = [[mi.decode_inputs(mi.scaled(w, seed=w.seed + 7919 * rank), li, s, dev) for li in range(L)]
+    inputs = [[mi.decode_inputs(rank_workload(w, rank), li, s, dev) for li in range(L)]
               for s in range(n_in)]
     out = torch.empty(w.batch, w.heads_q, w.head_dim, dtype=torch.bfloat16, device=dev)
     stream = torch.cuda.current_stream()
@@ -197,7 +203,7 @@ def run_mikv(args):
     bytes_per_step = (bytes_before + bytes_after) / 2 - sum(
         layer.cache.nbytes_attended(1) - layer.cache.nbytes_attended(0) for layer in layers) / 2
     ms = e0.elapsed_time(e1) / K
-    ms = _max_over_ranks(dist, ms)
+    ms = max_over_ranks(dist, ms)
     for layer in layers:
         pkg.mikv_workspace_check(layer.ws)
 
@@ -236,7 +242,7 @@ def run_mikv(args):
         host_out.copy_(dev_out, non_blocking=True)
         torch.cuda.current_stream().synchronize()
     e2e_ms = (time.perf_counter() - t0) * 1e3 / e2e_steps
-    e2e_ms = _max_over_ranks(dist, e2e_ms)
+    e2e_ms = max_over_ranks(dist, e2e_ms)
     for layer in layers:
         pkg.mikv_workspace_check(layer.ws)
 

@@ -136,6 +136,7 @@ mikv_status attention_impl(const mikv_shape* s, const mikv_cache* c, int32_t n_l
   const int sms = num_sms();
   const AttnPlan plan = plan_attention(*s, n_lo, sms);
   if (ws_bytes < attention_workspace_bytes(*s, n_lo, sms)) return MIKV_ERR_WORKSPACE;
+  if ((long long)s->batch * s->heads_kv * plan.n_u > 2000000000LL) return MIKV_ERR_UNSUPPORTED;
   const int G = s->heads_q / s->heads_kv;
   AttnArgs a;
   memset(&a, 0, sizeof a);
@@ -147,33 +148,42 @@ mikv_status attention_impl(const mikv_shape* s, const mikv_cache* c, int32_t n_l
             make_map(&a.map_v_hi, c->v_hi, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, kHeadDim, hi_rows, 2 * kHeadDim, 64,
                      16, CU_TENSOR_MAP_SWIZZLE_128B);
   if (ok && lo_rows > 0) {
+    // retained arrays: one box covers a whole unit of U.blocks blocks of 16 rows
+    const LoUnit U = lo_unit_layout(s->bits, s->group);
+    const uint32_t box_rows = 16u * U.blocks;
     if (s->bits == 3) {
-      ok = make_map(&a.map_k_lo, c->k_codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, row_bytes, lo_rows, row_bytes, 32, 16,
-                    CU_TENSOR_MAP_SWIZZLE_32B) &&
-           make_map(&a.map_v_lo, c->v_codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, row_bytes, lo_rows, row_bytes, 32, 16,
-                    CU_TENSOR_MAP_SWIZZLE_32B) &&
+      ok = make_map(&a.map_k_lo, c->k_codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, row_bytes, lo_rows, row_bytes, 32,
+                    box_rows, CU_TENSOR_MAP_SWIZZLE_32B) &&
+           make_map(&a.map_v_lo, c->v_codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, row_bytes, lo_rows, row_bytes, 32,
+                    box_rows, CU_TENSOR_MAP_SWIZZLE_32B) &&
            make_map(&a.map_k_lo1, c->k_codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, row_bytes, lo_rows, row_bytes, 16,
-                    16, CU_TENSOR_MAP_SWIZZLE_NONE) &&
+                    box_rows, CU_TENSOR_MAP_SWIZZLE_NONE) &&
            make_map(&a.map_v_lo1, c->v_codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, row_bytes, lo_rows, row_bytes, 16,
-                    16, CU_TENSOR_MAP_SWIZZLE_NONE);
+                    box_rows, CU_TENSOR_MAP_SWIZZLE_NONE);
     } else {
       const CUtensorMapSwizzle swz = s->bits == 2 ? CU_TENSOR_MAP_SWIZZLE_32B : CU_TENSOR_MAP_SWIZZLE_64B;
       ok = make_map(&a.map_k_lo, c->k_codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, row_bytes, lo_rows, row_bytes,
-                    (uint32_t)row_bytes, 16, swz) &&
+                    (uint32_t)row_bytes, box_rows, swz) &&
            make_map(&a.map_v_lo, c->v_codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, row_bytes, lo_rows, row_bytes,
-                    (uint32_t)row_bytes, 16, swz);
+                    (uint32_t)row_bytes, box_rows, swz);
     }
+    // (alpha, beta) pairs viewed as rows of 16 bytes: U.param_row / 16 rows per token
+    const uint64_t par_rows = lo_rows * (uint64_t)U.param_row / 16;
+    const uint32_t par_box = box_rows * U.param_row / 16;
+    ok = ok &&
+         make_map(&a.map_k_par, c->k_params, CU_TENSOR_MAP_DATA_TYPE_UINT8, 16, par_rows, 16, 16, par_box,
+                  CU_TENSOR_MAP_SWIZZLE_NONE) &&
+         make_map(&a.map_v_par, c->v_params, CU_TENSOR_MAP_DATA_TYPE_UINT8, 16, par_rows, 16, 16, par_box,
+                  CU_TENSOR_MAP_SWIZZLE_NONE);
   }
   if (!ok) return MIKV_ERR_CUDA;
-  a.k_params = c->k_params;
-  a.v_params = c->v_params;
   a.q = q;
   a.balancer = c->balancer;
   a.hi_logits = hi_logits;
   char* wsb = static_cast<char*>(ws);
   a.status = reinterpret_cast<int*>(wsb);
   a.part_o = reinterpret_cast<float*>(wsb + kWsHeader);
-  a.part_ml = a.part_o + (size_t)plan.n_items * G * kHeadDim;
+  a.part_ml = a.part_o + (size_t)plan.n_slots * G * kHeadDim;
   a.batch = s->batch;
   a.heads_q = s->heads_q;
   a.heads_kv = s->heads_kv;
@@ -181,10 +191,11 @@ mikv_status attention_impl(const mikv_shape* s, const mikv_cache* c, int32_t n_l
   a.hi_stride = s->hi_stride;
   a.lo_cap = s->lo_cap;
   a.n_lo = n_lo;
-  a.hi_blocks = (s->hi_cap + 15) / 16;
-  a.lo_blocks = (n_lo + 15) / 16;
-  a.n_split = plan.n_split;
-  a.n_items = plan.n_items;
+  a.hi_units = plan.hi_units;
+  a.lo_blocks = plan.lo_blocks;
+  a.n_u = plan.n_u;
+  a.n_units = plan.n_units;
+  a.n_warps = plan.n_warps;
   a.sm_scale = sm_scale;
   cudaError_t e = launch_attention(a, s->bits, s->group, G, plan.grid, st);
   if (e != cudaSuccess) return MIKV_ERR_CUDA;
@@ -196,7 +207,9 @@ mikv_status attention_impl(const mikv_shape* s, const mikv_cache* c, int32_t n_l
   m.batch = s->batch;
   m.heads_q = s->heads_q;
   m.heads_kv = s->heads_kv;
-  m.n_split = plan.n_split;
+  m.n_u = plan.n_u;
+  m.n_units = plan.n_units;
+  m.n_warps = plan.n_warps;
   e = launch_merge(m, G, out_dtype == MIKV_OUT_F32, st);
   return cuda_status(e);
 }

@@ -6,18 +6,25 @@
 // unordered set for attention (Sec. 3.4), so they are streamed separately and merged by the online
 // softmax.
 //
-// Design (per CTA: 4 consumer warps + 1 producer warp, 2 CTAs per SM, persistent over work items):
-//  * work item = (b, h, context split); splits are contiguous ranges of 16-token blocks;
-//  * the producer lane streams blocks into a 3-stage shared-memory ring with TMA: 2-D tensor copies
-//    with hardware swizzle for bf16 rows and packed codes, 1-D bulk copies for (alpha, beta) pairs,
-//    completion tracked by mbarriers (every wait is bounded in time);
-//  * a consumer warp takes one 16-token block at a time: ldmatrix yields the mma.sync fragments
-//    directly (the packed-code layout of the ABI is built for this), codes become fp16 in registers
-//    (exact magic-number conversion, then alpha * c + beta), QK^T and PV run on tensor cores with fp32
-//    accumulation (tokens on M for QK^T, channels on M for PV, query heads on N), online softmax in
-//    fp32; movmatrix turns the probabilities into the PV operand without shared memory;
-//  * the 4 warps' partial (max, sum, output) are combined through shared memory and written per item;
-//    a merge kernel combines the splits of each query head.
+// Work decomposition. Every (b, h) owns the same sequence of "units": an important unit is one block
+// of 16 bf16 tokens (8 KB of K and V), a retained unit is up to eight blocks of 16 coded
+// tokens (about the same bytes). The two kinds are interleaved evenly inside each head's sequence, the
+// sequences of all heads are concatenated, and every warp of the persistent grid takes one contiguous,
+// equal share. A warp therefore streams a balanced mix of bandwidth-heavy and ALU-heavy units and
+// touches one or two heads (a few, for small caches); it writes one partial (max, sum, output) per head
+// it touched, and a merge kernel combines the partials of each query head.
+//
+// Per warp: a private 3-stage shared-memory ring fed by TMA (lane 0 issues 2-D tensor copies: bf16
+// rows and packed codes with hardware swizzle, one box per array per unit, (alpha, beta) pairs as
+// 16-byte rows; one mbarrier per stage, every wait bounded in time). No cross-warp synchronisation.
+//
+// Per 16-token block: ldmatrix yields mma.sync fragments directly (the ABI's code layout is built for
+// this); tokens sit on M for QK^T and channels on M for PV, query heads on N. Codes become exact fp16
+// integers with one LOP3 each (the code bits OR-ed under an fp16 exponent that makes the code's lowest
+// bit weigh 1) and one HSUB2. Keys are then dequantized (alpha * c + beta, HFMA2) for QK^T; for PV the
+// value scale is folded into the probabilities (p * alpha per token and group) and the zero into one
+// extra MMA row (sum of p * beta per group), so values need no HFMA2. Online softmax in fp32;
+// movmatrix turns probabilities into the PV operand without shared memory.
 #include <math.h>
 
 #include "mikv_device.cuh"
@@ -26,61 +33,64 @@
 namespace mikv {
 namespace {
 
-constexpr int kConsumerWarps = 4;
-constexpr int kThreads = (kConsumerWarps + 1) * 32;
-constexpr int kStages = 3;
-constexpr int kStageBytes = 32768;
+constexpr int kWarps = 4;            // independent warps per CTA
+constexpr int kThreads = kWarps * 32;
+constexpr int kNS = 3;               // ring stages per warp
+constexpr int kStageBytes = kUnitBytes;
 constexpr int kHiBlockBytes = 8192;  // K and V of 16 tokens: 4 boxes of 16 rows x 64 bf16
-constexpr int kMinBlocksPerSplit = 8;
 constexpr int kCtasPerSm = 2;
-constexpr int kItemsPerCta = 8;
+constexpr int kUnitsPerWarp = 24;    // target share per warp (sizes the grid for small caches)
 constexpr float kLog2e = 1.4426950408889634f;
 
-template <int BITS, int GROUP>
-struct LoLayout {
-  static constexpr int kRowBytes = 16 * BITS;               // packed codes of one row
-  static constexpr int kCodeBox = 16 * kRowBytes;           // 16 rows of codes
-  static constexpr int kParamRow = 4 * (kHeadDim / GROUP);  // (alpha, beta) fp16 pairs of one row
-  static constexpr int kParamBox = 16 * kParamRow;
-  static constexpr int kTxBytes = 2 * kCodeBox + 2 * kParamBox;
-  static constexpr int kBlockBytes = (kTxBytes + 511) / 512 * 512;  // keeps swizzle atoms aligned
-  static constexpr int kPerWarpRaw = kStageBytes / (kConsumerWarps * kBlockBytes);
-  static constexpr int kBlocksPerWarp = kPerWarpRaw < 8 ? kPerWarpRaw : 8;
-  static constexpr int kK = 0, kV = kCodeBox, kKp = 2 * kCodeBox, kVp = 2 * kCodeBox + kParamBox;
+__host__ __device__ constexpr int smem_bytes() { return 1024 + kWarps * kNS * kStageBytes + kWarps * kNS * 8; }
+
+// Position in the concatenated unit sequence. Unit i of a head (of n_u units, hu of them important)
+// is important when floor((i+1) hu / n_u) > floor(i hu / n_u): important units are spread evenly.
+// The cursor keeps r = (i hu) mod n_u and h = floor(i hu / n_u) so each step is O(1).
+struct Cursor {
+  int bh, i, r, h;
 };
 
-__host__ __device__ constexpr int red_bytes(int G) { return kConsumerWarps * G * 130 * 4; }
-__host__ __device__ constexpr int smem_bytes(int G) {
-  return 1024 + kStages * kStageBytes + red_bytes(G) + 2 * kStages * 8;
+struct UnitKind {
+  bool hi;
+  int index;  // important block index, or retained unit index
+};
+
+__device__ __forceinline__ Cursor cursor_at(int u, int hu, int n_u) {
+  Cursor c;
+  c.bh = u / n_u;
+  c.i = u - c.bh * n_u;
+  const long long p = (long long)c.i * hu;
+  c.h = (int)(p / n_u);
+  c.r = (int)(p - (long long)c.h * n_u);
+  return c;
 }
 
-__device__ __forceinline__ int ceil_div(int a, int b) { return (a + b - 1) / b; }
+__device__ __forceinline__ UnitKind cursor_kind(const Cursor& c, int hu, int n_u) {
+  UnitKind k;
+  k.hi = c.r + hu >= n_u;
+  k.index = k.hi ? c.h : c.i - c.h;
+  return k;
+}
 
-// Stage k of an item with n_hs important stages and n_ls retained stages: alternate while both
-// remain so that bandwidth-heavy (important) and ALU-heavy (retained) stages interleave.
-__device__ __forceinline__ void stage_kind(int k, int n_hs, int n_ls, bool& hi, int& j) {
-  const int m = n_hs < n_ls ? n_hs : n_ls;
-  if (k < 2 * m) {
-    hi = (k & 1) == 0;
-    j = k >> 1;
-  } else {
-    hi = n_hs > n_ls;
-    j = m + (k - 2 * m);
+__device__ __forceinline__ void cursor_next(Cursor& c, int hu, int n_u) {
+  const bool hi = c.r + hu >= n_u;
+  c.r += hu - (hi ? n_u : 0);
+  c.h += hi ? 1 : 0;
+  if (++c.i == n_u) {
+    ++c.bh;
+    c.i = c.r = c.h = 0;
   }
-}
-
-__device__ __forceinline__ void split_range(int total, int n_split, int s, int& b0, int& b1) {
-  b0 = (int)((long long)total * s / n_split);
-  b1 = (int)((long long)total * (s + 1) / n_split);
 }
 
 struct Softmax {
   float m[2], l[2];
 };
 
-// Online-softmax update for one 16-token block. sacc holds raw q.k for (token g, head 2t),
-// (g, 2t+1), (g+8, 2t), (g+8, 2t+1); returns unnormalised probabilities in p.
-__device__ __forceinline__ void softmax_block(const float (&s)[4], Softmax& st, float (&o)[8][4],
+// Online-softmax update for one 16-token block. s holds scaled logits of (token g, head 2t),
+// (g, 2t+1), (g+8, 2t), (g+8, 2t+1) (-inf past the end); returns unnormalised probabilities in p.
+// o (output) and ob (zero-row sums) are running sums at the current max: both are rescaled.
+__device__ __forceinline__ void softmax_block(const float (&s)[4], Softmax& st, float (&o)[8][4], float (&ob)[4],
                                               float (&p)[4]) {
   float bm0 = fmaxf(s[0], s[2]), bm1 = fmaxf(s[1], s[3]);
 #pragma unroll
@@ -101,6 +111,8 @@ __device__ __forceinline__ void softmax_block(const float (&s)[4], Softmax& st, 
       o[mt][2] *= c0;
       o[mt][3] *= c1;
     }
+    ob[0] *= c0;
+    ob[1] *= c1;
     st.m[0] = mn0;
     st.m[1] = mn1;
   }
@@ -116,13 +128,15 @@ __device__ __forceinline__ void softmax_block(const float (&s)[4], Softmax& st, 
 // Scale raw dot products, mask tokens >= valid, and store important-set logits.
 template <int G>
 __device__ __forceinline__ void finish_logits(const float (&acc)[4], float scale, int valid, int g, int t,
-                                              float* logit_base, int hi_stride, int slot0,
-                                              float (&s)[4]) {
-  const float ninf = -INFINITY;
-  s[0] = g < valid ? acc[0] * scale : ninf;
-  s[1] = g < valid ? acc[1] * scale : ninf;
-  s[2] = g + 8 < valid ? acc[2] * scale : ninf;
-  s[3] = g + 8 < valid ? acc[3] * scale : ninf;
+                                              float* logit_base, int hi_stride, int slot0, float (&s)[4]) {
+  s[0] = acc[0] * scale;
+  s[1] = acc[1] * scale;
+  s[2] = acc[2] * scale;
+  s[3] = acc[3] * scale;
+  if (valid < 16) {
+    if (g >= valid) s[0] = s[1] = -INFINITY;
+    if (g + 8 >= valid) s[2] = s[3] = -INFINITY;
+  }
   if (logit_base) {
     const int h0 = 2 * t, h1 = 2 * t + 1;
     if (h0 < G) {
@@ -136,24 +150,65 @@ __device__ __forceinline__ void finish_logits(const float (&acc)[4], float scale
   }
 }
 
-// One block of 16 important tokens (bf16, 128B-swizzled boxes: K ch 0-63, K ch 64-127, V, V).
+// ---------------------------------------------------------------------- code extraction
+//
+// A 32-bit fragment register holds two 16-bit units (two channels or two tokens) whose codes sit at
+// the same bit positions. OR-ing the masked code bits under the fp16 exponent of 2^(10 - pos) gives
+// the exact value 2^(10 - pos) + code (the code's lowest bit then weighs 1); HSUB2 of that power of
+// two leaves the exact code. Positions 10 and up lie in the exponent field and are shifted down first.
+
+__device__ __forceinline__ uint32_t exact_codes(uint32_t x_with_magic, uint32_t magic2) {
+  return h2_as_u32(__hsub2(u32_as_h2(x_with_magic), u32_as_h2(magic2)));
+}
+
+__device__ __forceinline__ uint32_t mag2(int j) {  // fp16 pair 2^(10 - 2j), j = 0..4
+  return j == 0 ? 0x64006400u : j == 1 ? 0x5C005C00u : j == 2 ? 0x54005400u : j == 3 ? 0x4C004C00u : 0x44004400u;
+}
+
+// 2-bit code j (0..7) of each unit of r (r10 = r >> 10): exact fp16 pair.
+__device__ __forceinline__ uint32_t code2(uint32_t r, uint32_t r10, int j) {
+  if (j < 5) return exact_codes(and_or(r, 0x00030003u << (2 * j), mag2(j)), mag2(j));
+  const int jj = j - 5;
+  return exact_codes(and_or(r10, 0x00030003u << (2 * jj), mag2(jj)), mag2(jj));
+}
+
+// 4-bit code p (0..3) of each unit of r (r8 = r >> 8): exact fp16 pair (magics 2^10 and 2^6).
+__device__ __forceinline__ uint32_t code4(uint32_t r, uint32_t r8, int p) {
+  const uint32_t src = p < 2 ? r : r8;
+  const int pp = p & 1;
+  const uint32_t mag = pp ? 0x54005400u : 0x64006400u;
+  return exact_codes(and_or(src, 0x000F000Fu << (4 * pp), mag), mag);
+}
+
+// 3-bit code: bits 0..1 at position j of r, bit 2 at bit hb of each unit of h.
+__device__ __forceinline__ uint32_t code3(uint32_t r, uint32_t h, int j, int hb) {
+  const uint32_t lo = and_or(r >> (2 * j), 0x00030003u, 0x64006400u);
+  return exact_codes(lo | (((h >> hb) << 2) & 0x00040004u), 0x64006400u);
+}
+
+// ---------------------------------------------------------------------- one important block
+
 template <int G>
 __device__ __forceinline__ void process_hi(uint32_t blk, int valid, int slot0, const uint32_t (&qb)[8][2],
                                            float scale, float* logit_base, int hi_stride, Softmax& st,
-                                           float (&o)[8][4], int lane) {
+                                           float (&o)[8][4], float (&ob)[4], int lane) {
   const int g = lane >> 2, t = lane & 3, r8 = lane & 7, j = lane >> 3;
-  float acc[4] = {0.f, 0.f, 0.f, 0.f};
+  float acc0[4] = {0.f, 0.f, 0.f, 0.f}, acc1[4] = {0.f, 0.f, 0.f, 0.f};
   const int krow = r8 + 8 * (j & 1);
 #pragma unroll
   for (int ks = 0; ks < 8; ++ks) {
     const int chunk = 2 * (ks & 3) + (j >> 1);
     uint32_t a[4];
     ldsm_x4(blk + (ks >> 2) * 2048 + krow * 128 + ((chunk ^ (krow & 7)) << 4), a);
-    mma_bf16(acc, a, qb[ks][0], qb[ks][1]);
+    if (ks & 1)
+      mma_bf16(acc1, a, qb[ks][0], qb[ks][1]);
+    else
+      mma_bf16(acc0, a, qb[ks][0], qb[ks][1]);
   }
+  const float acc[4] = {acc0[0] + acc1[0], acc0[1] + acc1[1], acc0[2] + acc1[2], acc0[3] + acc1[3]};
   float s[4], p[4];
   finish_logits<G>(acc, scale, valid, g, t, logit_base, hi_stride, slot0, s);
-  softmax_block(s, st, o, p);
+  softmax_block(s, st, o, ob, p);
   const uint32_t pb0 = movmatrix_t(pack_bf16(p[0], p[1]));
   const uint32_t pb1 = movmatrix_t(pack_bf16(p[2], p[3]));
   uint32_t m01 = 0xffffffffu, m89 = 0xffffffffu;
@@ -167,374 +222,369 @@ __device__ __forceinline__ void process_hi(uint32_t blk, int valid, int slot0, c
     const int chunk = 2 * (mt & 3) + (j & 1);
     uint32_t a[4];
     ldsm_x4_t(blk + 4096 + (mt >> 2) * 2048 + vtok * 128 + ((chunk ^ (vtok & 7)) << 4), a);
-    a[0] &= m01;
-    a[1] &= m01;
-    a[2] &= m89;
-    a[3] &= m89;
+    if (valid < 16) {  // rows past the end may hold any bits: zero them (P is 0 there, NaN * 0 is not)
+      a[0] &= m01;
+      a[1] &= m01;
+      a[2] &= m89;
+      a[3] &= m89;
+    }
     mma_bf16(o[mt], a, pb0, pb1);
   }
 }
 
-// One block of 16 retained tokens: packed codes (swizzled boxes), then (alpha, beta) rows.
+// ---------------------------------------------------------------------- one retained block
+
 template <int BITS, int GROUP, int G>
-__device__ __forceinline__ void process_lo(uint32_t blk, int valid, const uint32_t (&qh)[8][2], float scale,
-                                           Softmax& st, float (&o)[8][4], int lane) {
-  using L = LoLayout<BITS, GROUP>;
+__device__ __forceinline__ void process_lo(uint32_t unit, int b, int valid, const uint32_t (&qh)[8][2], float scale,
+                                           Softmax& st, float (&o)[8][4], float (&ob)[4], int lane) {
+  constexpr LoUnit U = lo_unit_layout(BITS, GROUP);
   constexpr int NG = kHeadDim / GROUP;
+  constexpr int PR = U.param_row;
+  // this block's rows inside the unit's sections
+  const uint32_t ka = unit + U.k_a + b * 16 * U.plane_a_bytes, kb = unit + U.k_b + b * 16 * U.plane_b_bytes;
+  const uint32_t va = unit + U.v_a + b * 16 * U.plane_a_bytes, vb = unit + U.v_b + b * 16 * U.plane_b_bytes;
+  const uint32_t kp = unit + U.k_p + b * 16 * PR, vp = unit + U.v_p + b * 16 * PR;
+  constexpr int NR = BITS == 4 ? 8 : 4;
   const int g = lane >> 2, t = lane & 3, r8 = lane & 7, j = lane >> 3;
 
-  // ---- keys: codes of tokens g and g+8
-  uint32_t kr[BITS == 4 ? 8 : 4];
+  // ---- keys of tokens g and g+8
+  uint32_t kr[NR], kh[NR];
   uint32_t kb0 = 0, kb1 = 0;
   {
     const int tok = r8 + 8 * (j & 1);
     if (BITS == 4) {
       const int o0 = tok * 64 + 16 * (j >> 1), sw = ((tok >> 1) & 3) << 4;
       uint32_t r0[4], r1[4];
-      ldsm_x4(blk + L::kK + (o0 ^ sw), r0);
-      ldsm_x4(blk + L::kK + ((o0 + 32) ^ sw), r1);
+      ldsm_x4(ka + (o0 ^ sw), r0);
+      ldsm_x4(ka + ((o0 + 32) ^ sw), r1);
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
         kr[i] = r0[i];
-        kr[(BITS == 4 ? 4 : 0) + i] = r1[i];
+        kr[(NR == 8 ? 4 : 0) + i] = r1[i];
       }
     } else {
       const int o0 = tok * 32 + 16 * (j >> 1), sw = ((tok >> 2) & 1) << 4;
       uint32_t r0[4];
-      ldsm_x4(blk + L::kK + (o0 ^ sw), r0);
+      ldsm_x4(ka + (o0 ^ sw), r0);
 #pragma unroll
       for (int i = 0; i < 4; ++i) kr[i] = r0[i];
-      if (BITS == 3) ldsm_x2(blk + L::kK + 512 + (lane & 15) * 16, kb0, kb1);
+      if (BITS == 3) ldsm_x2(kb + (lane & 15) * 16, kb0, kb1);
     }
+#pragma unroll
+    for (int i = 0; i < NR; ++i) kh[i] = kr[i] >> (BITS == 4 ? 8 : 10);
   }
   uint32_t pk0[NG], pk1[NG];
-#pragma unroll
-  for (int gi = 0; gi < NG; ++gi) {
-    pk0[gi] = lds32(blk + L::kKp + g * L::kParamRow + 4 * gi);
-    pk1[gi] = lds32(blk + L::kKp + (g + 8) * L::kParamRow + 4 * gi);
-  }
-  float acc[4] = {0.f, 0.f, 0.f, 0.f};
+  lds_vec<NG>(kp + g * PR, pk0);
+  lds_vec<NG>(kp + (g + 8) * PR, pk1);
+  float acc0[4] = {0.f, 0.f, 0.f, 0.f}, acc1[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
   for (int ks = 0; ks < 8; ++ks) {
     const int gi = (16 * ks) / GROUP;
     const uint32_t al0 = prmt(pk0[gi], pk0[gi], 0x1010u), be0 = prmt(pk0[gi], pk0[gi], 0x3232u);
     const uint32_t al1 = prmt(pk1[gi], pk1[gi], 0x1010u), be1 = prmt(pk1[gi], pk1[gi], 0x3232u);
-    uint32_t x0, x1, x2, x3;
+    uint32_t c[4];
     if (BITS == 4) {
-      const int ri = (ks >> 2) * 4, sh = 4 * (ks & 3);
-      x0 = and_or(kr[ri + 0] >> sh, 0x000f000fu, 0x64006400u);
-      x1 = and_or(kr[ri + 1] >> sh, 0x000f000fu, 0x64006400u);
-      x2 = and_or(kr[ri + 2] >> sh, 0x000f000fu, 0x64006400u);
-      x3 = and_or(kr[ri + 3] >> sh, 0x000f000fu, 0x64006400u);
+      const int ri = (ks >> 2) * 4, p = ks & 3;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) c[i] = code4(kr[ri + i], kh[ri + i], p);
+    } else if (BITS == 2) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) c[i] = code2(kr[i], kh[i], ks);
     } else {
-      const int sh = 2 * ks;
-      x0 = and_or(kr[0] >> sh, 0x00030003u, 0x64006400u);
-      x1 = and_or(kr[1] >> sh, 0x00030003u, 0x64006400u);
-      x2 = and_or(kr[2] >> sh, 0x00030003u, 0x64006400u);
-      x3 = and_or(kr[3] >> sh, 0x00030003u, 0x64006400u);
-      if (BITS == 3) {
-        x0 |= ((kb0 >> ks) << 2) & 0x00040004u;
-        x1 |= ((kb1 >> ks) << 2) & 0x00040004u;
-        x2 |= ((kb0 >> (8 + ks)) << 2) & 0x00040004u;
-        x3 |= ((kb1 >> (8 + ks)) << 2) & 0x00040004u;
-      }
+      c[0] = code3(kr[0], kb0, ks, ks);
+      c[1] = code3(kr[1], kb1, ks, ks);
+      c[2] = code3(kr[2], kb0, ks, 8 + ks);
+      c[3] = code3(kr[3], kb1, ks, 8 + ks);
     }
-    const uint32_t a[4] = {dequant_pair(x0, al0, be0), dequant_pair(x1, al1, be1), dequant_pair(x2, al0, be0),
-                           dequant_pair(x3, al1, be1)};
-    mma_f16(acc, a, qh[ks][0], qh[ks][1]);
+    const uint32_t a[4] = {h2_as_u32(__hfma2(u32_as_h2(c[0]), u32_as_h2(al0), u32_as_h2(be0))),
+                           h2_as_u32(__hfma2(u32_as_h2(c[1]), u32_as_h2(al1), u32_as_h2(be1))),
+                           h2_as_u32(__hfma2(u32_as_h2(c[2]), u32_as_h2(al0), u32_as_h2(be0))),
+                           h2_as_u32(__hfma2(u32_as_h2(c[3]), u32_as_h2(al1), u32_as_h2(be1)))};
+    if (ks & 1)
+      mma_f16(acc1, a, qh[ks][0], qh[ks][1]);
+    else
+      mma_f16(acc0, a, qh[ks][0], qh[ks][1]);
   }
+  const float acc[4] = {acc0[0] + acc1[0], acc0[1] + acc1[1], acc0[2] + acc1[2], acc0[3] + acc1[3]};
   float s[4], p[4];
   finish_logits<G>(acc, scale, valid, g, t, nullptr, 0, 0, s);
-  softmax_block(s, st, o, p);
-  const uint32_t pb0 = movmatrix_t(pack_f16(p[0], p[1]));
-  const uint32_t pb1 = movmatrix_t(pack_f16(p[2], p[3]));
+  softmax_block(s, st, o, ob, p);
+  const uint32_t pb0 = movmatrix_t(pack_f16(p[0], p[1]));  // (P[2t][head g], P[2t+1][head g])
+  const uint32_t pb1 = movmatrix_t(pack_f16(p[2], p[3]));  // tokens 2t+8, 2t+9
 
-  // ---- values: codes of tokens (2t, 2t+1) and (2t+8, 2t+9) for channels 16 mt + g (+8)
-  uint32_t vr[BITS == 4 ? 8 : 4];
+  // ---- values of tokens (2t, 2t+1) and (2t+8, 2t+9), channels 16 mt + g and 16 mt + 8 + g
+  uint32_t vr[NR], vh[NR];
   uint32_t vb0 = 0, vb1 = 0;
   {
     const int tok = r8 + 8 * (j >> 1);
     if (BITS == 4) {
       const int o0 = tok * 64 + 16 * (j & 1), sw = ((tok >> 1) & 3) << 4;
       uint32_t r0[4], r1[4];
-      ldsm_x4_t(blk + L::kV + (o0 ^ sw), r0);
-      ldsm_x4_t(blk + L::kV + ((o0 + 32) ^ sw), r1);
+      ldsm_x4_t(va + (o0 ^ sw), r0);
+      ldsm_x4_t(va + ((o0 + 32) ^ sw), r1);
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
         vr[i] = r0[i];
-        vr[(BITS == 4 ? 4 : 0) + i] = r1[i];
+        vr[(NR == 8 ? 4 : 0) + i] = r1[i];
       }
     } else {
       const int o0 = tok * 32 + 16 * (j & 1), sw = ((tok >> 2) & 1) << 4;
       uint32_t r0[4];
-      ldsm_x4_t(blk + L::kV + (o0 ^ sw), r0);
+      ldsm_x4_t(va + (o0 ^ sw), r0);
 #pragma unroll
       for (int i = 0; i < 4; ++i) vr[i] = r0[i];
-      if (BITS == 3) ldsm_x2_t(blk + L::kV + 512 + (lane & 15) * 16, vb0, vb1);
+      if (BITS == 3) ldsm_x2_t(vb + (lane & 15) * 16, vb0, vb1);
     }
-  }
-  uint32_t pv[4][NG];
 #pragma unroll
-  for (int k = 0; k < 4; ++k) {
-    const int tok = 2 * t + (k & 1) + 8 * (k >> 1);
+    for (int i = 0; i < NR; ++i) vh[i] = vr[i] >> (BITS == 4 ? 8 : 10);
+  }
+  // (alpha, beta) of the four tokens for every group; zero past the end (exact zeros in the sums)
+  const int t0 = 2 * t, t1 = 2 * t + 1, t8 = 2 * t + 8, t9 = 2 * t + 9;
+  uint32_t pv0[NG], pv1[NG], pv8[NG], pv9[NG];
+  lds_vec<NG>(vp + t0 * PR, pv0);
+  lds_vec<NG>(vp + t1 * PR, pv1);
+  lds_vec<NG>(vp + t8 * PR, pv8);
+  lds_vec<NG>(vp + t9 * PR, pv9);
+  // zero-row operand: row g < NG holds beta of group g for this thread's tokens
+  uint32_t bw0 = 0, bw1 = 0, bw8 = 0, bw9 = 0;
+  if (g < NG) {
+    bw0 = lds32(vp + t0 * PR + 4 * g);
+    bw1 = lds32(vp + t1 * PR + 4 * g);
+    bw8 = lds32(vp + t8 * PR + 4 * g);
+    bw9 = lds32(vp + t9 * PR + 4 * g);
+  }
+  if (valid < 16) {
 #pragma unroll
     for (int gi = 0; gi < NG; ++gi) {
-      const uint32_t w = lds32(blk + L::kVp + tok * L::kParamRow + 4 * gi);
-      pv[k][gi] = tok < valid ? w : 0u;  // alpha = beta = 0 makes rows past the end exact zeros
+      if (t0 >= valid) pv0[gi] = 0u;
+      if (t1 >= valid) pv1[gi] = 0u;
+      if (t8 >= valid) pv8[gi] = 0u;
+      if (t9 >= valid) pv9[gi] = 0u;
     }
+    if (t0 >= valid) bw0 = 0u;
+    if (t1 >= valid) bw1 = 0u;
+    if (t8 >= valid) bw8 = 0u;
+    if (t9 >= valid) bw9 = 0u;
+  }
+  {
+    const uint32_t a[4] = {prmt(bw0, bw1, 0x7632u), 0u, prmt(bw8, bw9, 0x7632u), 0u};
+    mma_f16(ob, a, pb0, pb1);  // ob[row g][heads 2t, 2t+1] += sum over tokens of p * beta_g
+  }
+  uint32_t pa0[NG], pa1[NG];  // p * alpha per group: B operand of the code MMAs
+#pragma unroll
+  for (int gi = 0; gi < NG; ++gi) {
+    pa0[gi] = h2_as_u32(__hmul2(u32_as_h2(pb0), u32_as_h2(prmt(pv0[gi], pv1[gi], 0x5410u))));
+    pa1[gi] = h2_as_u32(__hmul2(u32_as_h2(pb1), u32_as_h2(prmt(pv8[gi], pv9[gi], 0x5410u))));
   }
 #pragma unroll
   for (int mt = 0; mt < 8; ++mt) {
     const int gi = (16 * mt) / GROUP;
-    const uint32_t a01 = prmt(pv[0][gi], pv[1][gi], 0x5410u), b01 = prmt(pv[0][gi], pv[1][gi], 0x7632u);
-    const uint32_t a89 = prmt(pv[2][gi], pv[3][gi], 0x5410u), b89 = prmt(pv[2][gi], pv[3][gi], 0x7632u);
-    uint32_t y0, y1, y2, y3;
+    uint32_t a[4];
     if (BITS == 4) {
-      const int ri = (mt >> 2) * 4, sh = 4 * (mt & 3);
-      y0 = and_or(vr[ri + 0] >> sh, 0x000f000fu, 0x64006400u);
-      y1 = and_or(vr[ri + 1] >> sh, 0x000f000fu, 0x64006400u);
-      y2 = and_or(vr[ri + 2] >> sh, 0x000f000fu, 0x64006400u);
-      y3 = and_or(vr[ri + 3] >> sh, 0x000f000fu, 0x64006400u);
+      const int ri = (mt >> 2) * 4, pp = mt & 3;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) a[i] = code4(vr[ri + i], vh[ri + i], pp);
+    } else if (BITS == 2) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) a[i] = code2(vr[i], vh[i], mt);
     } else {
-      const int sh = 2 * mt;
-      y0 = and_or(vr[0] >> sh, 0x00030003u, 0x64006400u);
-      y1 = and_or(vr[1] >> sh, 0x00030003u, 0x64006400u);
-      y2 = and_or(vr[2] >> sh, 0x00030003u, 0x64006400u);
-      y3 = and_or(vr[3] >> sh, 0x00030003u, 0x64006400u);
-      if (BITS == 3) {
-        y0 |= ((vb0 >> mt) << 2) & 0x00040004u;
-        y1 |= ((vb0 >> (8 + mt)) << 2) & 0x00040004u;
-        y2 |= ((vb1 >> mt) << 2) & 0x00040004u;
-        y3 |= ((vb1 >> (8 + mt)) << 2) & 0x00040004u;
-      }
+      a[0] = code3(vr[0], vb0, mt, mt);
+      a[1] = code3(vr[1], vb0, mt, 8 + mt);
+      a[2] = code3(vr[2], vb1, mt, mt);
+      a[3] = code3(vr[3], vb1, mt, 8 + mt);
     }
-    const uint32_t a[4] = {dequant_pair(y0, a01, b01), dequant_pair(y1, a01, b01), dequant_pair(y2, a89, b89),
-                           dequant_pair(y3, a89, b89)};
-    mma_f16(o[mt], a, pb0, pb1);
+    mma_f16(o[mt], a, pa0[gi], pa1[gi]);
   }
 }
 
+// Write this warp's partial for one head: unnormalised output (plus the zero-row terms), max, sum.
+template <int GROUP, int G>
+__device__ __forceinline__ void write_partial(const AttnArgs& a, int slot, Softmax& st, const float (&o)[8][4],
+                                              const float (&ob)[4], int lane) {
+  const int g = lane >> 2, t = lane & 3;
+#pragma unroll
+  for (int off = 4; off < 32; off <<= 1) {
+    st.l[0] += __shfl_xor_sync(0xffffffffu, st.l[0], off);
+    st.l[1] += __shfl_xor_sync(0xffffffffu, st.l[1], off);
+  }
+  constexpr int NG = kHeadDim / GROUP;
+  float bz0[NG], bz1[NG];  // sum p * beta of group gi for heads 2t, 2t+1, held by lane 4 gi + t
+#pragma unroll
+  for (int gi = 0; gi < NG; ++gi) {
+    bz0[gi] = __shfl_sync(0xffffffffu, ob[0], gi * 4 + t);
+    bz1[gi] = __shfl_sync(0xffffffffu, ob[1], gi * 4 + t);
+  }
+#pragma unroll
+  for (int hd = 0; hd < 2; ++hd) {
+    const int head = 2 * t + hd;
+    if (head < G) {
+      float* po = a.part_o + ((size_t)slot * G + head) * kHeadDim;
+#pragma unroll
+      for (int mt = 0; mt < 8; ++mt) {
+        const int gi = (16 * mt) / GROUP;
+        const float z = hd ? bz1[gi] : bz0[gi];
+        po[16 * mt + g] = o[mt][hd] + z;
+        po[16 * mt + 8 + g] = o[mt][2 + hd] + z;
+      }
+      if (g == 0) {
+        a.part_ml[((size_t)slot * G + head) * 2] = st.m[hd];
+        a.part_ml[((size_t)slot * G + head) * 2 + 1] = st.l[hd];
+      }
+    }
+  }
+}
+
+template <int BITS, int GROUP>
+__device__ __forceinline__ void issue_unit(const AttnArgs& a, const Cursor& c, uint32_t dst, uint32_t bar) {
+  constexpr LoUnit U = lo_unit_layout(BITS, GROUP);
+  const UnitKind k = cursor_kind(c, a.hi_units, a.n_u);
+  if (k.hi) {
+    const int row = c.bh * a.hi_stride + 16 * k.index;
+    mbar_arrive_expect_tx(bar, kHiBlockBytes);
+    tma_load_2d(dst, &a.map_k_hi, 0, row, bar);
+    tma_load_2d(dst + 2048, &a.map_k_hi, 64, row, bar);
+    tma_load_2d(dst + 4096, &a.map_v_hi, 0, row, bar);
+    tma_load_2d(dst + 6144, &a.map_v_hi, 64, row, bar);
+  } else {
+    // one box per array covers the whole unit (U.blocks blocks of 16 rows); rows past this head's
+    // retained length are masked by the consumer, rows past the array are zero-filled by TMA
+    const int row = c.bh * a.lo_cap + 16 * U.blocks * k.index;
+    mbar_arrive_expect_tx(bar, U.tx);
+    tma_load_2d(dst + U.k_a, &a.map_k_lo, 0, row, bar);
+    tma_load_2d(dst + U.v_a, &a.map_v_lo, 0, row, bar);
+    if (BITS == 3) {
+      tma_load_2d(dst + U.k_b, &a.map_k_lo1, 32, row, bar);
+      tma_load_2d(dst + U.v_b, &a.map_v_lo1, 32, row, bar);
+    }
+    const int prow = row * U.param_row / 16;
+    tma_load_2d(dst + U.k_p, &a.map_k_par, 0, prow, bar);
+    tma_load_2d(dst + U.v_p, &a.map_v_par, 0, prow, bar);
+  }
+}
+
+__device__ __forceinline__ void fence_proxy_async() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
 template <int BITS, int GROUP, int G>
-__global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_split_kernel(const __grid_constant__ AttnArgs a) {
-  using L = LoLayout<BITS, GROUP>;
-  static_assert(L::kBlocksPerWarp >= 1, "retained block too large for a stage");
+__global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const __grid_constant__ AttnArgs a) {
+  constexpr LoUnit U = lo_unit_layout(BITS, GROUP);
+  static_assert(U.total <= kStageBytes, "retained unit too large for a stage");
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
-  uint8_t* base_ptr = smem_raw + (base - raw);
-  float* red = reinterpret_cast<float*>(base_ptr + kStages * kStageBytes);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(base_ptr + kStages * kStageBytes + red_bytes(G));
-  __shared__ int abort_flag;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
-      mbar_init(smem_u32(&bars[s]), 1);
-      mbar_init(smem_u32(&bars[kStages + s]), kConsumerWarps);
-    }
-    abort_flag = 0;
+  const int wg = blockIdx.x * kWarps + warp;
+  if (wg >= a.n_warps) return;  // no block-wide synchronisation follows
+  const uint32_t ring = base + warp * kNS * kStageBytes;
+  const uint32_t bars = base + kWarps * kNS * kStageBytes + warp * kNS * 8;
+  const int u0 = (int)((long long)wg * a.n_units / a.n_warps);
+  const int u1 = (int)((long long)(wg + 1) * a.n_units / a.n_warps);
+  const int hu = a.hi_units, n_u = a.n_u;
+  Cursor ci = cursor_at(u0, hu, n_u);  // next unit to issue (lane 0)
+  if (lane == 0) {
+    for (int s = 0; s < kNS; ++s) mbar_init(bars + 8 * s, 1);
     fence_mbar_init();
-  }
-  __syncthreads();
-  volatile int* abort_v = &abort_flag;
-
-  if (warp == kConsumerWarps) {
-    // ------------------------------------------------------------------ producer
-    if (lane != 0) return;
     prefetch_tensormap(&a.map_k_hi);
     prefetch_tensormap(&a.map_v_hi);
     if (a.lo_blocks > 0) {  // the retained-set maps are only encoded when the retained arrays exist
       prefetch_tensormap(&a.map_k_lo);
       prefetch_tensormap(&a.map_v_lo);
+      prefetch_tensormap(&a.map_k_par);
+      prefetch_tensormap(&a.map_v_par);
     }
-    uint32_t it = 0;
-    uint32_t issued_mask = 0, last_use[kStages] = {0, 0, 0};
-    bool failed = false;
-    for (int item = blockIdx.x; item < a.n_items && !failed; item += gridDim.x) {
-      const int bh = item / a.n_split, sp = item - bh * a.n_split;
-      int hb0, hb1, lb0, lb1;
-      split_range(a.hi_blocks, a.n_split, sp, hb0, hb1);
-      split_range(a.lo_blocks, a.n_split, sp, lb0, lb1);
-      const int n_hs = ceil_div(hb1 - hb0, kConsumerWarps);
-      const int n_ls = ceil_div(lb1 - lb0, kConsumerWarps * L::kBlocksPerWarp);
-      for (int k = 0; k < n_hs + n_ls; ++k, ++it) {
-        const int s = it % kStages;
-        const uint32_t use = it / kStages;
-        const uint32_t full = smem_u32(&bars[s]), empty = smem_u32(&bars[kStages + s]);
-        if (*abort_v) { failed = true; break; }
-        if (use > 0 && !mbar_wait(empty, (use - 1) & 1)) {
-          record_error(a.status, kErrEmptyTimeout);
-          *abort_v = 1;
-          failed = true;
-          break;
-        }
-        bool hi;
-        int jj;
-        stage_kind(k, n_hs, n_ls, hi, jj);
-        const uint32_t dst = base + s * kStageBytes;
-        if (hi) {
-          const int first = hb0 + jj * kConsumerWarps;
-          const int nb = min(kConsumerWarps, hb1 - first);
-          mbar_arrive_expect_tx(full, nb * kHiBlockBytes);
-          for (int w = 0; w < nb; ++w) {
-            const int row = bh * a.hi_stride + 16 * (first + w);
-            const uint32_t blk = dst + w * kHiBlockBytes;
-            tma_load_2d(blk, &a.map_k_hi, 0, row, full);
-            tma_load_2d(blk + 2048, &a.map_k_hi, 64, row, full);
-            tma_load_2d(blk + 4096, &a.map_v_hi, 0, row, full);
-            tma_load_2d(blk + 6144, &a.map_v_hi, 64, row, full);
+    for (int k = 0; k < kNS && u0 + k < u1; ++k) {
+      issue_unit<BITS, GROUP>(a, ci, ring + k * kStageBytes, bars + 8 * k);
+      cursor_next(ci, hu, n_u);
+    }
+  }
+  __syncwarp();
+
+  const int g = lane >> 2, t = lane & 3;
+  uint32_t qb[8][2], qh[8][2];
+  Softmax st;
+  float o[8][4], ob[4];
+  float* logit_base = nullptr;
+  Cursor cc = cursor_at(u0, hu, n_u);  // unit being consumed
+  int cur = -1;
+  bool failed = false;
+  int u = u0;
+  for (; u < u1; ++u) {
+    if (cc.bh != cur) {
+      if (cur >= 0) write_partial<GROUP, G>(a, wg + cur, st, o, ob, lane);
+      cur = cc.bh;
+      const int b = cur / a.heads_kv, h = cur - b * a.heads_kv;
+      // query fragments (B operand: head g; channels 16 ks + 2t (+1) and 16 ks + 2t + 8 (+9))
+      if (g < G) {
+        const __nv_bfloat16* qp =
+            static_cast<const __nv_bfloat16*>(a.q) + (size_t)(b * a.heads_q + h * G + g) * kHeadDim;
+#pragma unroll
+        for (int ks = 0; ks < 8; ++ks)
+#pragma unroll
+          for (int r = 0; r < 2; ++r) {
+            const int c = 16 * ks + 2 * t + 8 * r;
+            const uint32_t w = *reinterpret_cast<const uint32_t*>(qp + c);
+            qb[ks][r] = w;
+            const float q0 = __uint_as_float(w << 16), q1 = __uint_as_float(w & 0xffff0000u);
+            const float b0 = a.balancer ? a.balancer[h * kHeadDim + c] : 1.f;
+            const float b1 = a.balancer ? a.balancer[h * kHeadDim + c + 1] : 1.f;
+            qh[ks][r] = pack_f16(__fdiv_rn(q0, b0), __fdiv_rn(q1, b1));  // Eq. 4
           }
-        } else {
-          const int first = lb0 + jj * kConsumerWarps * L::kBlocksPerWarp;
-          const int nb = min(kConsumerWarps * L::kBlocksPerWarp, lb1 - first);
-          mbar_arrive_expect_tx(full, nb * L::kTxBytes);
-          for (int i = 0; i < nb; ++i) {
-            const int row = bh * a.lo_cap + 16 * (first + i);
-            const uint32_t blk = dst + i * L::kBlockBytes;
-            tma_load_2d(blk + L::kK, &a.map_k_lo, 0, row, full);
-            tma_load_2d(blk + L::kV, &a.map_v_lo, 0, row, full);
-            if (BITS == 3) {
-              tma_load_2d(blk + L::kK + 512, &a.map_k_lo1, 32, row, full);
-              tma_load_2d(blk + L::kV + 512, &a.map_v_lo1, 32, row, full);
-            }
-            bulk_load(blk + L::kKp, static_cast<const uint8_t*>(a.k_params) + (size_t)row * L::kParamRow,
-                      L::kParamBox, full);
-            bulk_load(blk + L::kVp, static_cast<const uint8_t*>(a.v_params) + (size_t)row * L::kParamRow,
-                      L::kParamBox, full);
-          }
-        }
-        issued_mask |= 1u << s;
-        last_use[s] = use;
+      } else {
+#pragma unroll
+        for (int ks = 0; ks < 8; ++ks) qb[ks][0] = qb[ks][1] = qh[ks][0] = qh[ks][1] = 0u;
       }
+      logit_base = a.hi_logits ? a.hi_logits + (size_t)(b * a.heads_q + h * G) * a.hi_stride : nullptr;
+      st.m[0] = st.m[1] = -INFINITY;
+      st.l[0] = st.l[1] = 0.f;
+#pragma unroll
+      for (int mt = 0; mt < 8; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
+      ob[0] = ob[1] = ob[2] = ob[3] = 0.f;
     }
-    if (failed) {
-      // Leave no copy in flight into this CTA's shared memory: wait (bounded) for every stage issued.
-      for (int s = 0; s < kStages; ++s)
-        if ((issued_mask >> s) & 1u)
-          if (!mbar_wait(smem_u32(&bars[s]), last_use[s] & 1)) record_error(a.status, kErrDrainTimeout);
+    const int s = (u - u0) % kNS;
+    const uint32_t use = (u - u0) / kNS;
+    if (!mbar_wait(bars + 8 * s, use & 1)) {
+      record_error(a.status, kErrFullTimeout);
+      failed = true;
+      break;
     }
+    const uint32_t stage = ring + s * kStageBytes;
+    const UnitKind k = cursor_kind(cc, hu, n_u);
+    if (k.hi) {
+      process_hi<G>(stage, min(16, a.hi_cap - 16 * k.index), 16 * k.index, qb, a.sm_scale, logit_base,
+                    a.hi_stride, st, o, ob, lane);
+    } else {
+      const int first = k.index * U.blocks;
+      const int nb = min(U.blocks, a.lo_blocks - first);
+      for (int b = 0; b < nb; ++b)
+        process_lo<BITS, GROUP, G>(stage, b, min(16, a.n_lo - 16 * (first + b)), qh, a.sm_scale, st, o, ob, lane);
+    }
+    cursor_next(cc, hu, n_u);
+    __syncwarp();
+    if (lane == 0 && u + kNS < u1) {
+      fence_proxy_async();  // our generic reads of this stage precede the next asynchronous write
+      issue_unit<BITS, GROUP>(a, ci, stage, bars + 8 * s);
+      cursor_next(ci, hu, n_u);
+    }
+  }
+  if (failed) {
+    // leave no copy in flight into this warp's ring: wait (bounded) for every unit still issued
+    if (lane == 0)
+      for (int v = u; v < u1 && v < u + kNS; ++v) {
+        const int s = (v - u0) % kNS;
+        if (!mbar_wait(bars + 8 * s, ((v - u0) / kNS) & 1)) record_error(a.status, kErrDrainTimeout);
+      }
     return;
   }
+  if (cur >= 0) write_partial<GROUP, G>(a, wg + cur, st, o, ob, lane);
+}
 
-  // -------------------------------------------------------------------- consumers
-  const int g = lane >> 2, t = lane & 3;
-  uint32_t it = 0;
-  for (int item = blockIdx.x; item < a.n_items; item += gridDim.x) {
-    const int bh = item / a.n_split, sp = item - bh * a.n_split;
-    const int b = bh / a.heads_kv, h = bh - b * a.heads_kv;
-    int hb0, hb1, lb0, lb1;
-    split_range(a.hi_blocks, a.n_split, sp, hb0, hb1);
-    split_range(a.lo_blocks, a.n_split, sp, lb0, lb1);
-    const int n_hs = ceil_div(hb1 - hb0, kConsumerWarps);
-    const int n_ls = ceil_div(lb1 - lb0, kConsumerWarps * L::kBlocksPerWarp);
-
-    // query fragments (B operand, head g, channels 16 ks + 2t (+1) and 16 ks + 2t + 8 (+9))
-    uint32_t qb[8][2], qh[8][2];
-    if (g < G) {
-      const __nv_bfloat16* qp =
-          static_cast<const __nv_bfloat16*>(a.q) + (size_t)(b * a.heads_q + h * G + g) * kHeadDim;
-#pragma unroll
-      for (int ks = 0; ks < 8; ++ks)
-#pragma unroll
-        for (int r = 0; r < 2; ++r) {
-          const int c = 16 * ks + 2 * t + 8 * r;
-          const uint32_t w = *reinterpret_cast<const uint32_t*>(qp + c);
-          qb[ks][r] = w;
-          const float q0 = __uint_as_float(w << 16), q1 = __uint_as_float(w & 0xffff0000u);
-          const float b0 = a.balancer ? a.balancer[h * kHeadDim + c] : 1.f;
-          const float b1 = a.balancer ? a.balancer[h * kHeadDim + c + 1] : 1.f;
-          qh[ks][r] = pack_f16(__fdiv_rn(q0, b0), __fdiv_rn(q1, b1));  // Eq. 4
-        }
-    } else {
-#pragma unroll
-      for (int ks = 0; ks < 8; ++ks) qb[ks][0] = qb[ks][1] = qh[ks][0] = qh[ks][1] = 0u;
-    }
-    float* logit_base =
-        a.hi_logits ? a.hi_logits + (size_t)(b * a.heads_q + h * G) * a.hi_stride : nullptr;
-
-    Softmax st;
-    st.m[0] = st.m[1] = -INFINITY;
-    st.l[0] = st.l[1] = 0.f;
-    float o[8][4];
-#pragma unroll
-    for (int mt = 0; mt < 8; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
-
-    for (int k = 0; k < n_hs + n_ls; ++k, ++it) {
-      if (*abort_v) continue;
-      const int s = it % kStages;
-      const uint32_t use = it / kStages;
-      if (!mbar_wait(smem_u32(&bars[s]), use & 1)) {
-        record_error(a.status, kErrFullTimeout);
-        *abort_v = 1;
-        continue;
-      }
-      bool hi;
-      int jj;
-      stage_kind(k, n_hs, n_ls, hi, jj);
-      const uint32_t dst = base + s * kStageBytes;
-      if (hi) {
-        const int hb = hb0 + jj * kConsumerWarps + warp;
-        if (hb < hb1)
-          process_hi<G>(dst + warp * kHiBlockBytes, min(16, a.hi_cap - 16 * hb), 16 * hb, qb, a.sm_scale,
-                        logit_base, a.hi_stride, st, o, lane);
-      } else {
-        const int first = lb0 + jj * kConsumerWarps * L::kBlocksPerWarp + warp * L::kBlocksPerWarp;
-        for (int i = 0; i < L::kBlocksPerWarp; ++i) {
-          const int lb = first + i;
-          if (lb >= lb1) break;
-          process_lo<BITS, GROUP, G>(dst + (warp * L::kBlocksPerWarp + i) * L::kBlockBytes,
-                                     min(16, a.n_lo - 16 * lb), qh, a.sm_scale, st, o, lane);
-        }
-      }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(smem_u32(&bars[kStages + s]));
-    }
-
-    // ---- combine the 4 warps' partials and write this item's (max, sum, output)
-#pragma unroll
-    for (int off = 4; off < 32; off <<= 1) {
-      st.l[0] += __shfl_xor_sync(0xffffffffu, st.l[0], off);
-      st.l[1] += __shfl_xor_sync(0xffffffffu, st.l[1], off);
-    }
-    float* rw = red + warp * G * 130;
-#pragma unroll
-    for (int hd = 0; hd < 2; ++hd) {
-      const int head = 2 * t + hd;
-      if (head < G) {
-#pragma unroll
-        for (int mt = 0; mt < 8; ++mt) {
-          rw[head * 130 + 16 * mt + g] = o[mt][hd];
-          rw[head * 130 + 16 * mt + 8 + g] = o[mt][2 + hd];
-        }
-        if (g == 0) {
-          rw[head * 130 + 128] = st.m[hd];
-          rw[head * 130 + 129] = st.l[hd];
-        }
-      }
-    }
-    named_bar_sync(1, kConsumerWarps * 32);
-    for (int idx = warp * 32 + lane; idx < G * kHeadDim; idx += kConsumerWarps * 32) {
-      const int head = idx / kHeadDim, ch = idx - head * kHeadDim;
-      float M = -INFINITY;
-#pragma unroll
-      for (int w = 0; w < kConsumerWarps; ++w) M = fmaxf(M, red[(w * G + head) * 130 + 128]);
-      float O = 0.f, Ls = 0.f;
-      if (M != -INFINITY) {
-#pragma unroll
-        for (int w = 0; w < kConsumerWarps; ++w) {
-          const float mw = red[(w * G + head) * 130 + 128];
-          const float wt = mw == -INFINITY ? 0.f : fast_exp2((mw - M) * kLog2e);
-          O += wt * red[(w * G + head) * 130 + ch];
-          Ls += wt * red[(w * G + head) * 130 + 129];
-        }
-      }
-      a.part_o[((size_t)item * G + head) * kHeadDim + ch] = O;
-      if (ch == 0) {
-        a.part_ml[((size_t)item * G + head) * 2] = M;
-        a.part_ml[((size_t)item * G + head) * 2 + 1] = Ls;
-      }
-    }
-    named_bar_sync(1, kConsumerWarps * 32);
-  }
+// Warp that owns unit U under the equal split of n_units units over n_warps warps.
+__device__ __forceinline__ int owner_warp(long long U, long long n_units, int n_warps) {
+  int w = (int)(((U + 1) * n_warps - 1) / n_units);
+  while (w > 0 && (long long)w * n_units / n_warps > U) --w;
+  while (w + 1 < n_warps && (long long)(w + 1) * n_units / n_warps <= U) ++w;
+  return w;
 }
 
 template <int OUT_F32>
@@ -542,17 +592,20 @@ __global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a, int G) {
   const int bq = blockIdx.x;
   const int b = bq / a.heads_q, hq = bq - b * a.heads_q;
   const int h = hq / G, jh = hq - h * G;
+  const int bh = b * a.heads_kv + h;
   const int c = threadIdx.x;
-  const size_t item0 = (size_t)(b * a.heads_kv + h) * a.n_split;
+  const int w0 = owner_warp((long long)bh * a.n_u, a.n_units, a.n_warps);
+  const int w1 = owner_warp((long long)(bh + 1) * a.n_u - 1, a.n_units, a.n_warps);
   float M = -INFINITY;
-  for (int s = 0; s < a.n_split; ++s) M = fmaxf(M, a.part_ml[((item0 + s) * G + jh) * 2]);
+  for (int w = w0; w <= w1; ++w) M = fmaxf(M, a.part_ml[((size_t)(w + bh) * G + jh) * 2]);
   float O = 0.f, Ls = 0.f;
-  for (int s = 0; s < a.n_split; ++s) {
-    const float ms = a.part_ml[((item0 + s) * G + jh) * 2];
+  for (int w = w0; w <= w1; ++w) {
+    const size_t slot = (size_t)(w + bh);
+    const float ms = a.part_ml[(slot * G + jh) * 2];
     if (ms == -INFINITY) continue;
     const float wt = fast_exp2((ms - M) * kLog2e);
-    Ls += wt * a.part_ml[((item0 + s) * G + jh) * 2 + 1];
-    O += wt * a.part_o[((item0 + s) * G + jh) * kHeadDim + c];
+    Ls += wt * a.part_ml[(slot * G + jh) * 2 + 1];
+    O += wt * a.part_o[(slot * G + jh) * kHeadDim + c];
   }
   const float r = O / Ls;
   if (OUT_F32)
@@ -566,10 +619,10 @@ __global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a, int G) {
 }
 
 template <int BITS, int GROUP, int G>
-cudaError_t launch_split(const AttnArgs& a, int grid, cudaStream_t st) {
-  auto kern = attention_split_kernel<BITS, GROUP, G>;
+cudaError_t launch_kernel(const AttnArgs& a, int grid, cudaStream_t st) {
+  auto kern = attention_kernel<BITS, GROUP, G>;
   static bool configured = false;
-  const int smem = smem_bytes(G);
+  const int smem = smem_bytes();
   if (!configured) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
@@ -582,10 +635,10 @@ cudaError_t launch_split(const AttnArgs& a, int grid, cudaStream_t st) {
 template <int BITS, int GROUP>
 cudaError_t dispatch_g(const AttnArgs& a, int G, int grid, cudaStream_t st) {
   switch (G) {
-    case 1: return launch_split<BITS, GROUP, 1>(a, grid, st);
-    case 2: return launch_split<BITS, GROUP, 2>(a, grid, st);
-    case 4: return launch_split<BITS, GROUP, 4>(a, grid, st);
-    case 8: return launch_split<BITS, GROUP, 8>(a, grid, st);
+    case 1: return launch_kernel<BITS, GROUP, 1>(a, grid, st);
+    case 2: return launch_kernel<BITS, GROUP, 2>(a, grid, st);
+    case 4: return launch_kernel<BITS, GROUP, 4>(a, grid, st);
+    case 8: return launch_kernel<BITS, GROUP, 8>(a, grid, st);
   }
   return cudaErrorInvalidValue;
 }
@@ -604,22 +657,31 @@ cudaError_t dispatch_group(const AttnArgs& a, int group, int G, int grid, cudaSt
 
 AttnPlan plan_attention(const mikv_shape& s, int n_lo, int num_sms) {
   AttnPlan p;
-  const int hb = (s.hi_cap + 15) / 16, lb = (n_lo + 15) / 16;
-  const int bh = s.batch * s.heads_kv;
-  const int grid_cap = num_sms * kCtasPerSm;
-  const int want = (kItemsPerCta * grid_cap + bh - 1) / bh;
-  const int cap = (hb + lb + kMinBlocksPerSplit - 1) / kMinBlocksPerSplit;
-  p.n_split = want < cap ? want : cap;
-  if (p.n_split < 1) p.n_split = 1;
-  p.n_items = bh * p.n_split;
-  p.grid = p.n_items < grid_cap ? p.n_items : grid_cap;
+  p.hi_units = (s.hi_cap + 15) / 16;
+  p.lo_blocks = (n_lo + 15) / 16;
+  const int k = lo_unit_layout(s.bits, s.group).blocks;
+  p.lo_units = (p.lo_blocks + k - 1) / k;
+  p.n_u = p.hi_units + p.lo_units;
+  const long long bh = (long long)s.batch * s.heads_kv;
+  p.n_units = bh * p.n_u;
+  const long long cap = (long long)num_sms * kCtasPerSm * kWarps;
+  long long w = (p.n_units + kUnitsPerWarp - 1) / kUnitsPerWarp;
+  if (w < cap) w = p.n_units < cap ? p.n_units : cap;  // spread small caches over the whole GPU
+  if (w > cap) w = cap;
+  if (w < 1) w = 1;
+  p.n_warps = (int)w;
+  p.grid = (p.n_warps + kWarps - 1) / kWarps;
+  p.n_slots = p.n_warps + (int)bh;
   return p;
 }
 
 size_t attention_workspace_bytes(const mikv_shape& s, int n_lo_max, int num_sms) {
+  // the slot count grows with n_lo only through n_warps, which is capped: size for the cap
   const AttnPlan p = plan_attention(s, n_lo_max, num_sms);
+  const long long cap = (long long)num_sms * kCtasPerSm * kWarps;
+  const long long slots = cap + (long long)s.batch * s.heads_kv;
   const int G = s.heads_q / s.heads_kv;
-  const size_t part = (size_t)p.n_items * G * (kHeadDim + 2) * sizeof(float);
+  const size_t part = (size_t)(slots > p.n_slots ? slots : p.n_slots) * G * (kHeadDim + 2) * sizeof(float);
   return kWsHeader + (part + 255) / 256 * 256;
 }
 

@@ -126,6 +126,19 @@ __device__ __forceinline__ uint32_t lds32(uint32_t addr) {
   return r;
 }
 
+// N consecutive 32-bit words from shared memory (N = 1, 2 or 4; address aligned to 4 N bytes).
+template <int N>
+__device__ __forceinline__ void lds_vec(uint32_t addr, uint32_t (&r)[N]) {
+  if constexpr (N == 4) {
+    asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];" : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr) : "memory");
+  } else if constexpr (N == 2) {
+    asm volatile("ld.shared.v2.b32 {%0, %1}, [%2];" : "=r"(r[0]), "=r"(r[1]) : "r"(addr) : "memory");
+  } else {
+    r[0] = lds32(addr);
+  }
+}
+
 __device__ __forceinline__ uint32_t movmatrix_t(uint32_t x) {
   uint32_t r;
   asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(r) : "r"(x));

@@ -11,28 +11,74 @@
 
 namespace mikv {
 
-// Attention split plan: per (b, kv-head) the important blocks [0, hi_blocks) and retained blocks
-// [0, lo_blocks) of 16 tokens are divided into n_split contiguous ranges.
+// Shared-memory layout of one retained unit: up to `blocks` consecutive 16-token blocks loaded with
+// one TMA box per array (codes of K, codes of V, parameters of K, parameters of V; N = 3 adds the
+// 1-bit planes). Offsets are in bytes from the unit's stage; each section starts on the alignment its
+// swizzle needs (256 B for 32-byte swizzle, 512 B for 64-byte swizzle, 128 B otherwise).
+struct LoUnit {
+  int blocks;
+  int row_bytes, plane_a_bytes, plane_b_bytes;  // per token: codes, and the two planes (N = 3)
+  int param_row;                                 // bytes of (alpha, beta) pairs per token
+  int k_a, k_b, v_a, v_b, k_p, v_p;              // section offsets (k_b, v_b only for N = 3)
+  int total;                                     // bytes used
+  int tx;                                        // bytes the TMA boxes deliver
+};
+
+constexpr int kUnitBytes = 8192;
+
+__host__ __device__ constexpr int align_up(int x, int a) { return (x + a - 1) / a * a; }
+
+__host__ __device__ constexpr LoUnit lo_unit_layout_n(int bits, int group, int n) {
+  LoUnit u{};
+  u.blocks = n;
+  u.row_bytes = 16 * bits;
+  u.plane_a_bytes = bits == 3 ? 32 : 16 * bits;
+  u.plane_b_bytes = bits == 3 ? 16 : 0;
+  u.param_row = 4 * (128 / group);
+  const int rows = 16 * n;
+  const int code_align = bits == 4 ? 512 : 256;
+  u.k_a = 0;
+  u.k_b = align_up(u.k_a + rows * u.plane_a_bytes, 128);
+  u.v_a = align_up(u.k_b + rows * u.plane_b_bytes, code_align);
+  u.v_b = align_up(u.v_a + rows * u.plane_a_bytes, 128);
+  u.k_p = align_up(u.v_b + rows * u.plane_b_bytes, 128);
+  u.v_p = align_up(u.k_p + rows * u.param_row, 128);
+  u.total = u.v_p + rows * u.param_row;
+  u.tx = 2 * rows * (u.plane_a_bytes + u.plane_b_bytes) + 2 * rows * u.param_row;
+  return u;
+}
+
+// The largest unit (at most 8 blocks) that fits one stage.
+__host__ __device__ constexpr LoUnit lo_unit_layout(int bits, int group) {
+  int n = 8;
+  while (n > 1 && lo_unit_layout_n(bits, group, n).total > kUnitBytes) --n;
+  return lo_unit_layout_n(bits, group, n);
+}
+
+// Attention work plan: per (b, kv-head) a sequence of n_u units (hi_units important blocks of 16
+// tokens, lo_units groups of retained blocks), all heads concatenated into n_units units and split
+// into n_warps equal contiguous shares; warp w writes the partial of head bh into slot w + bh.
 struct AttnPlan {
-  int n_split;
-  int n_items;  // B * Hkv * n_split
-  int grid;     // persistent CTAs
+  int hi_units, lo_blocks, lo_units, n_u;
+  int n_units;
+  int n_warps;
+  int grid;
+  int n_slots;
 };
 
 struct AttnArgs {
   CUtensorMap map_k_hi, map_v_hi;    // bf16 rows of 128 channels, box 64 x 16, 128B swizzle
-  CUtensorMap map_k_lo, map_v_lo;    // packed codes (bits 0..1 plane for N = 3), box row x 16
-  CUtensorMap map_k_lo1, map_v_lo1;  // N = 3 only: 1-bit plane, box 16 B x 16
-  const void* k_params;
-  const void* v_params;
+  CUtensorMap map_k_lo, map_v_lo;    // packed codes (bits 0..1 plane for N = 3), box plane x 16 blocks
+  CUtensorMap map_k_lo1, map_v_lo1;  // N = 3 only: 1-bit plane
+  CUtensorMap map_k_par, map_v_par;  // (alpha, beta) pairs viewed as 16-byte rows
   const void* q;
   const float* balancer;
   float* hi_logits;
-  float* part_o;   // [n_items][G][128]
-  float* part_ml;  // [n_items][G][2]
+  float* part_o;   // [n_slots][G][128]
+  float* part_ml;  // [n_slots][G][2]
   int* status;
   int batch, heads_q, heads_kv, hi_cap, hi_stride, lo_cap, n_lo;
-  int hi_blocks, lo_blocks, n_split, n_items;
+  int hi_units, lo_blocks, n_u, n_units, n_warps;
   float sm_scale;
 };
 
@@ -41,7 +87,8 @@ struct MergeArgs {
   const float* part_ml;
   void* out;
   float* ml;
-  int batch, heads_q, heads_kv, n_split;
+  int batch, heads_q, heads_kv;
+  int n_u, n_units, n_warps;
 };
 
 AttnPlan plan_attention(const mikv_shape& s, int n_lo, int num_sms);

@@ -120,6 +120,7 @@ def test_decode_steps_trajectory():
     dev = torch.device("cuda")
     slots_ref = {(r["b"], r["h"]): np.array([[w.budget]], np.int32) for r in refs}
     near_ties = 0
+    acc_tol = {}
     for step in range(steps):
         q, k_new, v_new = mi.decode_inputs(w, 0, step)
         out = torch.empty(w.batch, w.heads_q, w.head_dim, dtype=torch.float32, device=dev)
@@ -139,9 +140,11 @@ def test_decode_steps_trajectory():
             assert np.all(err <= 2e-3 * vmax[b, h]), (step, b, h, err.max())
             acc_before = c["acc"][0, 0].astype(np.float64)
             c["acc"] = oracle.update_importance(c["acc"], hl.astype(np.float32), ml.astype(np.float32), G)
-            # one step's increment is a softmax weight; its relative error follows the logit error
-            # (fp16 query / key operands, about 1e-3 at most here)
-            acc_tol = 3e-3 * np.abs(c["acc"][0, 0] - acc_before) + 2e-6 * np.abs(acc_before) + 1e-7
+            # each step's increment is a softmax weight whose relative error follows the logit error
+            # (fp16 query / key operands, about 1e-3 at most here); errors add up over the steps
+            tol = acc_tol.setdefault((b, h), np.zeros(w.hi_cap))
+            tol[slot[0, 0]] = 0.0
+            tol += 3e-3 * np.abs(c["acc"][0, 0] - acc_before) + 2e-7 * np.abs(acc_before) + 1e-9
             acc_gpu = layer.cache.acc[b, h, :w.hi_cap].cpu().numpy()
             dem, _ = oracle.select_demote(c["acc"], 1, c["hi_tok"], want_kept=False)
             victim = int(dem[0, 0, 0])
@@ -152,7 +155,7 @@ def test_decode_steps_trajectory():
                 assert abs(a_sorted[1] - a_sorted[0]) < 1e-5 * max(1.0, abs(a_sorted[0])), (step, b, h)
                 near_ties += 1
                 victim = int(gslots[b, h])
-            assert np.all(np.abs(acc_gpu - c["acc"][0, 0]) <= acc_tol), (step, b, h)
+            assert np.all(np.abs(acc_gpu - c["acc"][0, 0]) <= tol), (step, b, h)
             oracle.quantize_pack(c, c["k_hi"], c["v_hi"], np.array([[[victim]]], np.int32), n_lo,
                                  src_tok=c["hi_tok"], balancer_=r["balancer"])
             np.testing.assert_array_equal(layer.cache.k_codes[b, h, n_lo].cpu().numpy(), c["k_codes"][0, 0, n_lo])
