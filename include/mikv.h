@@ -49,7 +49,9 @@ typedef enum {
   MIKV_ERR_CAPACITY = 3,    /* a write would pass lo_cap / hi_cap */
   MIKV_ERR_CUDA = 4,        /* a CUDA call failed; cudaGetLastError() was consumed */
   MIKV_ERR_WORKSPACE = 5,   /* workspace missing, too small or misaligned */
-  MIKV_ERR_DEVICE = 6       /* a kernel reported a failure through the workspace status word */
+  MIKV_ERR_DEVICE = 6,      /* a kernel reported a failure through the workspace status word */
+  MIKV_ERR_SCRATCH = 7      /* the problem needs more scratch than mikv_decode_attention_noalloc's
+                               built-in buffer holds (MIKV_NOALLOC_SCRATCH_BYTES) */
 } mikv_status;
 
 /* Shape of one layer's mixed-precision cache. */
@@ -212,6 +214,32 @@ mikv_status mikv_decode_step(const mikv_shape* shape, const mikv_cache* cache, i
                              const void* q, const void* k_new, const void* v_new, int32_t tok,
                              int32_t* slots, float sm_scale, void* out, int32_t out_dtype,
                              void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * Decode attention without a caller-provided workspace and without any allocation (there is no
+ * counterpart in the paper; this is a deployment convenience).
+ *
+ * Some callers cannot allocate device memory on the decode path: an inference engine that owns every
+ * byte of device memory through its own pool and forbids plugins from calling the CUDA allocator, or a
+ * latency-critical serving loop that must not call cudaMalloc (it can synchronise the device). This
+ * entry point computes exactly what mikv_decode_attention computes, with the same arguments minus the
+ * workspace, and keeps its split partials in a scratch buffer that the library itself declares as a
+ * fixed-size device array of MIKV_NOALLOC_SCRATCH_BYTES bytes. Every GPU that loads the library holds
+ * that buffer until the process exits.
+ *   - The first call on a device looks up the buffer's device address (cudaGetSymbolAddress) with that
+ *     device current; make that first call before any stream capture.
+ *   - The call itself allocates nothing and frees nothing; it zeroes the buffer's status word on
+ *     `stream` before launching.
+ *   - All calls share the one buffer: calls that can overlap on the GPU (different streams without
+ *     ordering between them) race on it and must not be issued.
+ *   - A problem whose scratch (mikv_workspace_bytes(shape, MIKV_WS_ATTENTION, n_lo)) exceeds the
+ *     buffer returns MIKV_ERR_SCRATCH and launches nothing.
+ *   - A kernel-side failure is recorded in the buffer's status word only; it is not reported here.
+ */
+#define MIKV_NOALLOC_SCRATCH_BYTES (8u << 20)
+mikv_status mikv_decode_attention_noalloc(const mikv_shape* shape, const mikv_cache* cache, int32_t n_lo,
+                                          const void* q, float sm_scale, void* out, int32_t out_dtype,
+                                          float* hi_logits, float* ml, void* stream);
 
 /*
  * KV-cache size as a fraction of an all-fp16 cache (the "Cache size" columns of Tables 2-3): a ratio

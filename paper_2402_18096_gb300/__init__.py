@@ -21,6 +21,7 @@ __all__ = [
     "mikv_workspace_reset", "mikv_workspace_check", "mikv_compute_balancer", "mikv_quantize_pack",
     "mikv_decode_attention", "mikv_update_importance", "mikv_select_demote", "mikv_insert_token",
     "mikv_gather_hi", "mikv_decode_step", "mikv_cache_fraction", "mikv_retained_row_bytes",
+    "mikv_decode_attention_noalloc", "NOALLOC_SCRATCH_BYTES",
     "WS_ATTENTION", "WS_BALANCER", "WS_STEP", "OUT_BF16", "OUT_F32", "HEAD_DIM",
 ]
 
@@ -28,7 +29,8 @@ HEAD_DIM = 128
 OUT_BF16, OUT_F32 = 0, 1
 WS_ATTENTION, WS_BALANCER, WS_STEP = 0, 1, 2
 STATUS = {0: "MIKV_OK", 1: "MIKV_ERR_ARG", 2: "MIKV_ERR_UNSUPPORTED", 3: "MIKV_ERR_CAPACITY",
-          4: "MIKV_ERR_CUDA", 5: "MIKV_ERR_WORKSPACE", 6: "MIKV_ERR_DEVICE"}
+          4: "MIKV_ERR_CUDA", 5: "MIKV_ERR_WORKSPACE", 6: "MIKV_ERR_DEVICE", 7: "MIKV_ERR_SCRATCH"}
+NOALLOC_SCRATCH_BYTES = 8 << 20
 
 
 class MikvError(RuntimeError):
@@ -79,6 +81,7 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
                 "mikv_insert_token": (I, [SP, CP, P, P, I, P, P]),
                 "mikv_gather_hi": (I, [SP, CP, P, P, P, P, I, P, I, P]),
                 "mikv_decode_step": (I, [SP, CP, I, P, P, P, I, P, F, P, I, P, Z, P]),
+                "mikv_decode_attention_noalloc": (I, [SP, CP, I, P, F, P, I, P, P, P]),
                 "mikv_cache_fraction": (ctypes.c_double, [I, I, ctypes.c_double, I]),
                 "mikv_retained_row_bytes": (Z, [I, I, I]),
             }
@@ -200,6 +203,16 @@ def mikv_decode_attention(cache: LayerCache, n_lo: int, q, sm_scale: float, out,
     _check("mikv_decode_attention", load().mikv_decode_attention(
         ctypes.byref(cache.shape.c()), ctypes.byref(cache.c()), n_lo, _ptr(q), float(sm_scale), _ptr(out),
         out_dtype, _ptr(hi_logits), _ptr(ml), _ptr(workspace), workspace.numel(), _stream(stream)))
+
+
+def mikv_decode_attention_noalloc(cache: LayerCache, n_lo: int, q, sm_scale: float, out, hi_logits=None,
+                                  ml=None, stream=None):
+    """mikv_decode_attention with the library's built-in scratch buffer instead of a workspace; for
+    callers that may not allocate device memory. Calls must not overlap on the GPU (one shared buffer)."""
+    out_dtype = OUT_F32 if out.dtype == torch.float32 else OUT_BF16
+    _check("mikv_decode_attention_noalloc", load().mikv_decode_attention_noalloc(
+        ctypes.byref(cache.shape.c()), ctypes.byref(cache.c()), n_lo, _ptr(q), float(sm_scale), _ptr(out),
+        out_dtype, _ptr(hi_logits), _ptr(ml), _stream(stream)))
 
 
 def mikv_update_importance(cache: LayerCache, hi_logits, ml, stream=None):

@@ -227,6 +227,7 @@ const char* mikv_status_string(mikv_status s) {
     case MIKV_ERR_CUDA: return "CUDA error";
     case MIKV_ERR_WORKSPACE: return "workspace missing, too small or misaligned";
     case MIKV_ERR_DEVICE: return "a kernel reported an internal failure";
+    case MIKV_ERR_SCRATCH: return "problem needs more scratch than the built-in no-allocation buffer holds";
   }
   return "unknown status";
 }
@@ -378,3 +379,60 @@ size_t mikv_retained_row_bytes(int32_t bits, int32_t group, int32_t head_dim) {
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------- no-allocation entry
+//
+// For callers that may not allocate device memory on the decode path (an engine that owns all device
+// memory and forbids plugins to call the CUDA allocator, or a serving loop that cannot afford a
+// synchronising cudaMalloc): decode attention whose split partials live in a fixed file-scope device
+// buffer of the library instead of a caller workspace. The buffer is part of the loaded module, so
+// every device that loads the library holds it until the process exits.
+
+namespace {
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[MIKV_NOALLOC_SCRATCH_BYTES];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_noalloc_mu;
+void* g_noalloc_ptr[kMaxDevices] = {};
+
+// Device address of the buffer on the current device, looked up once per device. The name of a
+// __device__ array in host code is only a host-side stand-in, so the address must come from the runtime.
+mikv_status noalloc_scratch(void** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return MIKV_ERR_CUDA;
+  if (dev < 0 || dev >= kMaxDevices) return MIKV_ERR_UNSUPPORTED;
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  if (!g_noalloc_ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return MIKV_ERR_CUDA;
+    g_noalloc_ptr[dev] = p;
+  }
+  *out = g_noalloc_ptr[dev];
+  return MIKV_OK;
+}
+
+}  // namespace
+
+extern "C" mikv_status mikv_decode_attention_noalloc(const mikv_shape* shape, const mikv_cache* cache, int32_t n_lo,
+                                                     const void* q, float sm_scale, void* out, int32_t out_dtype,
+                                                     float* hi_logits, float* ml, void* stream) {
+  mikv_status st = shape_supported(shape);
+  if (st != MIKV_OK) return st;
+  if (!cache_ok(cache) || !q || !out || n_lo < 0 || (out_dtype != MIKV_OUT_BF16 && out_dtype != MIKV_OUT_F32))
+    return MIKV_ERR_ARG;
+  if (n_lo > shape->lo_cap) return MIKV_ERR_CAPACITY;
+  if (shape->hi_cap + n_lo < 1) return MIKV_ERR_ARG;
+  if (!aligned(cache->k_hi, 16) || !aligned(cache->v_hi, 16) || !aligned(cache->k_codes, 16) ||
+      !aligned(cache->v_codes, 16) || !aligned(cache->k_params, 16) || !aligned(cache->v_params, 16) ||
+      !aligned(q, 4) || (cache->balancer && !aligned(cache->balancer, 16)))
+    return MIKV_ERR_ARG;
+  const size_t need = attention_workspace_bytes(*shape, n_lo, num_sms());
+  if (need > MIKV_NOALLOC_SCRATCH_BYTES) return MIKV_ERR_SCRATCH;
+  void* ws = nullptr;
+  if ((st = noalloc_scratch(&ws)) != MIKV_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaMemsetAsync(ws, 0, sizeof(int), s) != cudaSuccess) return MIKV_ERR_CUDA;  // status word starts at 0
+  return attention_impl(shape, cache, n_lo, q, sm_scale, out, out_dtype, hi_logits, ml, ws,
+                        MIKV_NOALLOC_SCRATCH_BYTES, s);
+}
