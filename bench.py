@@ -38,6 +38,38 @@ UNIT = "GB/s"
 DEFAULT_WORKLOAD = "mistral-7b"
 
 
+ATTN_SOURCES = ["mikv_attention.cu", "mikv_device.cuh", "mikv_internal.h", "mikv_rows.cuh"]
+TRAFFIC_SUMMARY = os.path.join(ROOT, "profiles", "attention_kernel_mistral7b_b4.md")
+
+
+def attention_source_sha256() -> str:
+    import hashlib
+    h = hashlib.sha256()
+    for f in ATTN_SOURCES:
+        with open(os.path.join(ROOT, "paper_2402_18096_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
+def profiled_traffic_ratio():
+    """DRAM bytes per algorithmic byte of the attention kernel, from the committed ncu summary, if it was
+    taken on the current kernel sources (else None: counters of another kernel do not apply)."""
+    if not os.path.exists(TRAFFIC_SUMMARY):
+        return None
+    vals = {}
+    with open(TRAFFIC_SUMMARY) as f:
+        for line in f:
+            if ":" in line and line.strip().startswith("- `"):
+                k, v = line.strip()[3:].split("`", 1)
+                vals[k] = v.split(":", 1)[1].strip()
+    try:
+        if vals.get("kernel_source_sha256") != attention_source_sha256():
+            return None
+        return float(vals["dram_bytes_per_algorithmic_byte"])
+    except (KeyError, ValueError):
+        return None
+
+
 def _peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -247,6 +279,8 @@ def run_mikv(args):
         pkg.mikv_workspace_check(layer.ws)
 
     peak, peak_kind = _peaks()
+    ratio = profiled_traffic_ratio()
+    traffic = None if ratio is None else int(ratio * attn_bytes)
     value = world * bytes_per_step / (ms * 1e-3) / 1e9
     achieved = attn_bytes / (attn_ms * 1e-3) / 1e9
     line = {
@@ -272,10 +306,10 @@ def run_mikv(args):
                    "parallelism": f"replicas{world}"},
         "roofline": {"kernel": "decode attention (split-K + merge)", "bound": "hbm", "achieved": round(achieved, 1),
                      "peak": peak, "unit": "GB/s", "frac": round(achieved / peak, 3),
-                     "traffic": None, "bytes_per_launch": int(attn_bytes), "avg_launch_us": round(attn_ms * 1e3, 2)},
+                     "traffic": traffic, "bytes_per_launch": int(attn_bytes), "avg_launch_us": round(attn_ms * 1e3, 2)},
         "e2e": {"value": round(world * bytes_per_step / (e2e_ms * 1e-3) / 1e9, 1), "unit": UNIT,
                 "ms_per_step": round(e2e_ms, 4), "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-        "gpu_launches": K * L * 6,
+        "gpu_launches": K * L * 3,  # per layer step: insert, attention, fused tail
     }
     if clk:
         line["clocks"] = clk

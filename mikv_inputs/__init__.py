@@ -96,9 +96,9 @@ _MASK63 = (1 << 63) - 1
 
 
 def _seed(w: Workload, layer: int, kind: int, b: int, h: int, step: int = 0) -> int:
-    x = w.seed
+    x = int(w.seed)
     for v in (layer, kind, b, h, step):
-        x = (x * 6364136223846793005 + 1442695040888963407 + v) & _MASK63
+        x = (x * 6364136223846793005 + 1442695040888963407 + int(v)) & _MASK63
         x ^= x >> 29
     return x
 

@@ -115,24 +115,40 @@ bool make_map(CUtensorMap* out, const void* ptr, CUtensorMapDataType dtype, uint
   return true;
 }
 
+// Checks shared by every attention entry point (nothing is launched when they fail).
+mikv_status attention_args_ok(const mikv_shape* shape, const mikv_cache* cache, int32_t n_lo, const void* q,
+                              const void* out, int32_t out_dtype) {
+  mikv_status st = shape_supported(shape);
+  if (st != MIKV_OK) return st;
+  if (!cache_ok(cache) || !q || !out || n_lo < 0 || (out_dtype != MIKV_OUT_BF16 && out_dtype != MIKV_OUT_F32))
+    return MIKV_ERR_ARG;
+  if (n_lo > shape->lo_cap) return MIKV_ERR_CAPACITY;
+  if (shape->hi_cap + n_lo < 1) return MIKV_ERR_ARG;
+  if (!aligned(cache->k_hi, 16) || !aligned(cache->v_hi, 16) || !aligned(cache->k_codes, 16) ||
+      !aligned(cache->v_codes, 16) || !aligned(cache->k_params, 16) || !aligned(cache->v_params, 16) ||
+      !aligned(q, 4) || (cache->balancer && !aligned(cache->balancer, 16)))
+    return MIKV_ERR_ARG;
+  return MIKV_OK;
+}
+
 struct StepLayout {
-  size_t attn, logits, ml, total;
+  size_t attn, logits, total;
 };
 
 StepLayout step_layout(const mikv_shape* s, int n_lo_max) {
   StepLayout L;
   L.attn = attention_workspace_bytes(*s, n_lo_max, num_sms());
   const size_t logits = (size_t)s->batch * s->heads_q * s->hi_stride * sizeof(float);
-  const size_t ml = (size_t)s->batch * s->heads_q * 2 * sizeof(float);
   L.logits = L.attn;
-  L.ml = L.logits + (logits + 255) / 256 * 256;
-  L.total = L.ml + (ml + 255) / 256 * 256;
+  L.total = L.logits + (logits + 255) / 256 * 256;
   return L;
 }
 
+// Launches the attention kernel and, when `merge` is set, the merge of its partials into out / ml.
+// With `merge` unset the partials stay in the workspace and *args_out describes them.
 mikv_status attention_impl(const mikv_shape* s, const mikv_cache* c, int32_t n_lo, const void* q, float sm_scale,
                            void* out, int32_t out_dtype, float* hi_logits, float* ml, void* ws, size_t ws_bytes,
-                           cudaStream_t st) {
+                           cudaStream_t st, bool merge = true, AttnArgs* args_out = nullptr) {
   const int sms = num_sms();
   const AttnPlan plan = plan_attention(*s, n_lo, sms);
   if (ws_bytes < attention_workspace_bytes(*s, n_lo, sms)) return MIKV_ERR_WORKSPACE;
@@ -199,6 +215,8 @@ mikv_status attention_impl(const mikv_shape* s, const mikv_cache* c, int32_t n_l
   a.sm_scale = sm_scale;
   cudaError_t e = launch_attention(a, s->bits, s->group, G, plan.grid, st);
   if (e != cudaSuccess) return MIKV_ERR_CUDA;
+  if (args_out) *args_out = a;
+  if (!merge) return MIKV_OK;
   MergeArgs m;
   m.part_o = a.part_o;
   m.part_ml = a.part_ml;
@@ -285,16 +303,8 @@ mikv_status mikv_quantize_pack(const mikv_shape* shape, const mikv_cache* cache,
 mikv_status mikv_decode_attention(const mikv_shape* shape, const mikv_cache* cache, int32_t n_lo, const void* q,
                                   float sm_scale, void* out, int32_t out_dtype, float* hi_logits, float* ml,
                                   void* workspace, size_t ws_bytes, void* stream) {
-  mikv_status st = shape_supported(shape);
+  mikv_status st = attention_args_ok(shape, cache, n_lo, q, out, out_dtype);
   if (st != MIKV_OK) return st;
-  if (!cache_ok(cache) || !q || !out || n_lo < 0 || (out_dtype != MIKV_OUT_BF16 && out_dtype != MIKV_OUT_F32))
-    return MIKV_ERR_ARG;
-  if (n_lo > shape->lo_cap) return MIKV_ERR_CAPACITY;
-  if (shape->hi_cap + n_lo < 1) return MIKV_ERR_ARG;
-  if (!aligned(cache->k_hi, 16) || !aligned(cache->v_hi, 16) || !aligned(cache->k_codes, 16) ||
-      !aligned(cache->v_codes, 16) || !aligned(cache->k_params, 16) || !aligned(cache->v_params, 16) ||
-      !aligned(q, 4) || (cache->balancer && !aligned(cache->balancer, 16)))
-    return MIKV_ERR_ARG;
   if (!workspace || !aligned(workspace, 256)) return MIKV_ERR_WORKSPACE;
   return attention_impl(shape, cache, n_lo, q, sm_scale, out, out_dtype, hi_logits, ml, workspace, ws_bytes,
                         static_cast<cudaStream_t>(stream));
@@ -353,17 +363,42 @@ mikv_status mikv_decode_step(const mikv_shape* shape, const mikv_cache* cache, i
   if (ws_bytes < L.total) return MIKV_ERR_WORKSPACE;
   char* wsb = static_cast<char*>(workspace);
   float* logits = reinterpret_cast<float*>(wsb + L.logits);
-  float* ml = reinterpret_cast<float*>(wsb + L.ml);
+  if ((st = attention_args_ok(shape, cache, n_lo, q, out, out_dtype)) != MIKV_OK) return st;
+  if (!aligned(k_new, 8) || !aligned(v_new, 8)) return MIKV_ERR_ARG;
   if ((st = mikv_insert_token(shape, cache, k_new, v_new, tok, slots, stream)) != MIKV_OK) return st;
-  if ((st = mikv_decode_attention(shape, cache, n_lo, q, sm_scale, out, out_dtype, logits, ml, workspace, L.attn,
-                                  stream)) != MIKV_OK)
+  // attention without its separate merge: the fused tail below merges, updates, selects and demotes
+  AttnArgs a;
+  if ((st = attention_impl(shape, cache, n_lo, q, sm_scale, out, out_dtype, logits, nullptr, workspace, L.attn,
+                           static_cast<cudaStream_t>(stream), false, &a)) != MIKV_OK)
     return st;
-  if ((st = mikv_update_importance(shape, cache, logits, ml, stream)) != MIKV_OK) return st;
-  if ((st = mikv_select_demote(shape->batch, shape->heads_kv, cache->acc, cache->hi_tok, shape->hi_cap,
-                               shape->hi_stride, 1, slots, nullptr, stream)) != MIKV_OK)
-    return st;
-  return mikv_quantize_pack(shape, cache, cache->k_hi, cache->v_hi, cache->hi_tok, shape->hi_stride, slots, 1, n_lo,
-                            stream);
+  StepPostArgs p;
+  p.part_o = a.part_o;
+  p.part_ml = a.part_ml;
+  p.out = out;
+  p.hi_logits = logits;
+  p.acc = cache->acc;
+  p.hi_tok = cache->hi_tok;
+  p.k_hi = cache->k_hi;
+  p.v_hi = cache->v_hi;
+  p.balancer = cache->balancer;
+  p.k_codes = cache->k_codes;
+  p.v_codes = cache->v_codes;
+  p.k_params = cache->k_params;
+  p.v_params = cache->v_params;
+  p.lo_tok = cache->lo_tok;
+  p.slots = slots;
+  p.batch = shape->batch;
+  p.heads_q = shape->heads_q;
+  p.heads_kv = shape->heads_kv;
+  p.hi_cap = shape->hi_cap;
+  p.hi_stride = shape->hi_stride;
+  p.lo_cap = shape->lo_cap;
+  p.n_lo = n_lo;
+  p.n_u = a.n_u;
+  p.n_units = a.n_units;
+  p.n_warps = a.n_warps;
+  return cuda_status(launch_step_post(p, shape->bits, shape->group, shape->heads_q / shape->heads_kv,
+                                      out_dtype == MIKV_OUT_F32, static_cast<cudaStream_t>(stream)));
 }
 
 double mikv_cache_fraction(int32_t bits, int32_t group, double ratio, int32_t hi_bits) {
@@ -417,16 +452,8 @@ mikv_status noalloc_scratch(void** out) {
 extern "C" mikv_status mikv_decode_attention_noalloc(const mikv_shape* shape, const mikv_cache* cache, int32_t n_lo,
                                                      const void* q, float sm_scale, void* out, int32_t out_dtype,
                                                      float* hi_logits, float* ml, void* stream) {
-  mikv_status st = shape_supported(shape);
+  mikv_status st = attention_args_ok(shape, cache, n_lo, q, out, out_dtype);
   if (st != MIKV_OK) return st;
-  if (!cache_ok(cache) || !q || !out || n_lo < 0 || (out_dtype != MIKV_OUT_BF16 && out_dtype != MIKV_OUT_F32))
-    return MIKV_ERR_ARG;
-  if (n_lo > shape->lo_cap) return MIKV_ERR_CAPACITY;
-  if (shape->hi_cap + n_lo < 1) return MIKV_ERR_ARG;
-  if (!aligned(cache->k_hi, 16) || !aligned(cache->v_hi, 16) || !aligned(cache->k_codes, 16) ||
-      !aligned(cache->v_codes, 16) || !aligned(cache->k_params, 16) || !aligned(cache->v_params, 16) ||
-      !aligned(q, 4) || (cache->balancer && !aligned(cache->balancer, 16)))
-    return MIKV_ERR_ARG;
   const size_t need = attention_workspace_bytes(*shape, n_lo, num_sms());
   if (need > MIKV_NOALLOC_SCRATCH_BYTES) return MIKV_ERR_SCRATCH;
   void* ws = nullptr;

@@ -14,7 +14,7 @@
 // touches one or two heads (a few, for small caches); it writes one partial (max, sum, output) per head
 // it touched, and a merge kernel combines the partials of each query head.
 //
-// Per warp: a private 3-stage shared-memory ring fed by TMA (lane 0 issues 2-D tensor copies: bf16
+// Per warp: a private shared-memory ring (2 stages by default) fed by TMA (lane 0 issues 2-D tensor copies: bf16
 // rows and packed codes with hardware swizzle, one box per array per unit, (alpha, beta) pairs as
 // 16-byte rows; one mbarrier per stage, every wait bounded in time). No cross-warp synchronisation.
 //
@@ -29,16 +29,31 @@
 
 #include "mikv_device.cuh"
 #include "mikv_internal.h"
+#include "mikv_rows.cuh"
 
 namespace mikv {
 namespace {
 
-constexpr int kWarps = 4;            // independent warps per CTA
+// Launch shape (compile-time tuning knobs; the defaults are the measured best on GB300).
+#ifndef MIKV_ATTN_WARPS
+#define MIKV_ATTN_WARPS 6
+#endif
+#ifndef MIKV_ATTN_STAGES
+#define MIKV_ATTN_STAGES 2
+#endif
+#ifndef MIKV_ATTN_CTAS
+#define MIKV_ATTN_CTAS 2
+#endif
+#ifndef MIKV_QK_ACC
+#define MIKV_QK_ACC 2
+#endif
+constexpr int kWarps = MIKV_ATTN_WARPS;     // independent warps per CTA
 constexpr int kThreads = kWarps * 32;
-constexpr int kNS = 3;               // ring stages per warp
+constexpr int kNS = MIKV_ATTN_STAGES;       // ring stages per warp
 constexpr int kStageBytes = kUnitBytes;
-constexpr int kHiBlockBytes = 8192;  // K and V of 16 tokens: 4 boxes of 16 rows x 64 bf16
-constexpr int kCtasPerSm = 2;
+constexpr int kHiBlockBytes = 8192;         // K and V of 16 tokens: 4 boxes of 16 rows x 64 bf16
+constexpr int kCtasPerSm = MIKV_ATTN_CTAS;
+constexpr int kQkAcc = MIKV_QK_ACC;         // independent accumulators of the QK^T MMA chain
 constexpr int kUnitsPerWarp = 24;    // target share per warp (sizes the grid for small caches)
 constexpr float kLog2e = 1.4426950408889634f;
 
@@ -86,6 +101,16 @@ __device__ __forceinline__ void cursor_next(Cursor& c, int hu, int n_u) {
 struct Softmax {
   float m[2], l[2];
 };
+
+__device__ __forceinline__ void sum_acc(const float (&accs)[kQkAcc][4], float (&acc)[4]) {
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    float v = accs[0][e];
+#pragma unroll
+    for (int q = 1; q < kQkAcc; ++q) v += accs[q][e];
+    acc[e] = v;
+  }
+}
 
 // Online-softmax update for one 16-token block. s holds scaled logits of (token g, head 2t),
 // (g, 2t+1), (g+8, 2t), (g+8, 2t+1) (-inf past the end); returns unnormalised probabilities in p.
@@ -193,19 +218,19 @@ __device__ __forceinline__ void process_hi(uint32_t blk, int valid, int slot0, c
                                            float scale, float* logit_base, int hi_stride, Softmax& st,
                                            float (&o)[8][4], float (&ob)[4], int lane) {
   const int g = lane >> 2, t = lane & 3, r8 = lane & 7, j = lane >> 3;
-  float acc0[4] = {0.f, 0.f, 0.f, 0.f}, acc1[4] = {0.f, 0.f, 0.f, 0.f};
+  float accs[kQkAcc][4];
+#pragma unroll
+  for (int q = 0; q < kQkAcc; ++q) accs[q][0] = accs[q][1] = accs[q][2] = accs[q][3] = 0.f;
   const int krow = r8 + 8 * (j & 1);
 #pragma unroll
   for (int ks = 0; ks < 8; ++ks) {
     const int chunk = 2 * (ks & 3) + (j >> 1);
     uint32_t a[4];
     ldsm_x4(blk + (ks >> 2) * 2048 + krow * 128 + ((chunk ^ (krow & 7)) << 4), a);
-    if (ks & 1)
-      mma_bf16(acc1, a, qb[ks][0], qb[ks][1]);
-    else
-      mma_bf16(acc0, a, qb[ks][0], qb[ks][1]);
+    mma_bf16(accs[ks % kQkAcc], a, qb[ks][0], qb[ks][1]);
   }
-  const float acc[4] = {acc0[0] + acc1[0], acc0[1] + acc1[1], acc0[2] + acc1[2], acc0[3] + acc1[3]};
+  float acc[4];
+  sum_acc(accs, acc);
   float s[4], p[4];
   finish_logits<G>(acc, scale, valid, g, t, logit_base, hi_stride, slot0, s);
   softmax_block(s, st, o, ob, p);
@@ -276,7 +301,9 @@ __device__ __forceinline__ void process_lo(uint32_t unit, int b, int valid, cons
   uint32_t pk0[NG], pk1[NG];
   lds_vec<NG>(kp + g * PR, pk0);
   lds_vec<NG>(kp + (g + 8) * PR, pk1);
-  float acc0[4] = {0.f, 0.f, 0.f, 0.f}, acc1[4] = {0.f, 0.f, 0.f, 0.f};
+  float accs[kQkAcc][4];
+#pragma unroll
+  for (int q = 0; q < kQkAcc; ++q) accs[q][0] = accs[q][1] = accs[q][2] = accs[q][3] = 0.f;
 #pragma unroll
   for (int ks = 0; ks < 8; ++ks) {
     const int gi = (16 * ks) / GROUP;
@@ -300,12 +327,10 @@ __device__ __forceinline__ void process_lo(uint32_t unit, int b, int valid, cons
                            h2_as_u32(__hfma2(u32_as_h2(c[1]), u32_as_h2(al1), u32_as_h2(be1))),
                            h2_as_u32(__hfma2(u32_as_h2(c[2]), u32_as_h2(al0), u32_as_h2(be0))),
                            h2_as_u32(__hfma2(u32_as_h2(c[3]), u32_as_h2(al1), u32_as_h2(be1)))};
-    if (ks & 1)
-      mma_f16(acc1, a, qh[ks][0], qh[ks][1]);
-    else
-      mma_f16(acc0, a, qh[ks][0], qh[ks][1]);
+    mma_f16(accs[ks % kQkAcc], a, qh[ks][0], qh[ks][1]);
   }
-  const float acc[4] = {acc0[0] + acc1[0], acc0[1] + acc1[1], acc0[2] + acc1[2], acc0[3] + acc1[3]};
+  float acc[4];
+  sum_acc(accs, acc);
   float s[4], p[4];
   finish_logits<G>(acc, scale, valid, g, t, nullptr, 0, 0, s);
   softmax_block(s, st, o, ob, p);
@@ -579,14 +604,6 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
   if (cur >= 0) write_partial<GROUP, G>(a, wg + cur, st, o, ob, lane);
 }
 
-// Warp that owns unit U under the equal split of n_units units over n_warps warps.
-__device__ __forceinline__ int owner_warp(long long U, long long n_units, int n_warps) {
-  int w = (int)(((U + 1) * n_warps - 1) / n_units);
-  while (w > 0 && (long long)w * n_units / n_warps > U) --w;
-  while (w + 1 < n_warps && (long long)(w + 1) * n_units / n_warps <= U) ++w;
-  return w;
-}
-
 template <int OUT_F32>
 __global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a, int G) {
   const int bq = blockIdx.x;
@@ -596,25 +613,15 @@ __global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a, int G) {
   const int c = threadIdx.x;
   const int w0 = owner_warp((long long)bh * a.n_u, a.n_units, a.n_warps);
   const int w1 = owner_warp((long long)(bh + 1) * a.n_u - 1, a.n_units, a.n_warps);
-  float M = -INFINITY;
-  for (int w = w0; w <= w1; ++w) M = fmaxf(M, a.part_ml[((size_t)(w + bh) * G + jh) * 2]);
-  float O = 0.f, Ls = 0.f;
-  for (int w = w0; w <= w1; ++w) {
-    const size_t slot = (size_t)(w + bh);
-    const float ms = a.part_ml[(slot * G + jh) * 2];
-    if (ms == -INFINITY) continue;
-    const float wt = fast_exp2((ms - M) * kLog2e);
-    Ls += wt * a.part_ml[(slot * G + jh) * 2 + 1];
-    O += wt * a.part_o[(slot * G + jh) * kHeadDim + c];
-  }
-  const float r = O / Ls;
+  float r[1], M, L;
+  merge_head<1>(a.part_o, a.part_ml, G, bh, jh, w0, w1, c, r, M, L);
   if (OUT_F32)
-    static_cast<float*>(a.out)[(size_t)bq * kHeadDim + c] = r;
+    static_cast<float*>(a.out)[(size_t)bq * kHeadDim + c] = r[0];
   else
-    static_cast<__nv_bfloat16*>(a.out)[(size_t)bq * kHeadDim + c] = __float2bfloat16_rn(r);
+    static_cast<__nv_bfloat16*>(a.out)[(size_t)bq * kHeadDim + c] = __float2bfloat16_rn(r[0]);
   if (c == 0 && a.ml) {
     a.ml[2 * bq] = M;
-    a.ml[2 * bq + 1] = Ls;
+    a.ml[2 * bq + 1] = L;
   }
 }
 

@@ -91,6 +91,29 @@ struct MergeArgs {
   int n_u, n_units, n_warps;
 };
 
+// Fused tail of a decode step (mikv_step.cu): merge + importance update + argmin + demotion.
+struct StepPostArgs {
+  const float* part_o;
+  const float* part_ml;
+  void* out;
+  const float* hi_logits;
+  float* acc;
+  const int32_t* hi_tok;
+  const void* k_hi;
+  const void* v_hi;
+  const float* balancer;
+  void* k_codes;
+  void* v_codes;
+  void* k_params;
+  void* v_params;
+  int32_t* lo_tok;
+  int32_t* slots;
+  int batch, heads_q, heads_kv, hi_cap, hi_stride, lo_cap, n_lo;
+  int n_u, n_units, n_warps;
+};
+
+cudaError_t launch_step_post(const StepPostArgs& a, int bits, int group, int G, int out_f32, cudaStream_t st);
+
 AttnPlan plan_attention(const mikv_shape& s, int n_lo, int num_sms);
 size_t attention_workspace_bytes(const mikv_shape& s, int n_lo_max, int num_sms);
 cudaError_t launch_attention(const AttnArgs& a, int bits, int group, int G, int grid, cudaStream_t st);

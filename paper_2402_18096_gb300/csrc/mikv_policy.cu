@@ -3,6 +3,7 @@
 // important set, insertion of the new token and the important-set build from prefill rows.
 #include "mikv_device.cuh"
 #include "mikv_internal.h"
+#include "mikv_rows.cuh"
 
 namespace mikv {
 namespace {
@@ -21,13 +22,6 @@ __global__ void __launch_bounds__(128) update_importance_kernel(float* acc, cons
     add += expf(hi_logits[(size_t)bq * hi_stride + i] - ml[2 * bq]) / ml[2 * bq + 1];
   }
   acc[(size_t)bh * hi_stride + i] += add;
-}
-
-// Total order of (score, id): ascending score, then ascending id. -0 is folded into +0.
-__device__ __forceinline__ unsigned long long order_key(float s, int32_t id) {
-  uint32_t u = __float_as_uint(s == 0.f ? 0.f : s);
-  u = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
-  return ((unsigned long long)u << 32) | (uint32_t)(id ^ (int32_t)0x80000000);
 }
 
 constexpr int kSelThreads = 1024;

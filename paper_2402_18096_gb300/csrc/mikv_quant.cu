@@ -1,14 +1,14 @@
 // mikv_quant.cu — demotion of KV rows into the retained set (Eq. 1 with the Eq. 3 key balancer) and
 // the channel balancer itself (Eq. 2), arxiv 2402.18096.
 //
-// quantize_pack: one warp per (row, K or V); each lane owns 4 consecutive channels. Group minima and
-// maxima come from butterfly shuffles over the GROUP/4 lanes of a group; scale and zero are rounded
-// to fp16 toward -inf (beta) and +inf (alpha) so the stored grid covers the group's range; codes are
-// round-half-even of the IEEE fp32 quotient (x - beta) / alpha. Every step uses explicitly rounded
-// intrinsics so the result is bit-identical to a plain IEEE evaluation. Codes are OR-ed into the
-// row's packed layout in shared memory and written out as whole words.
+// quantize_pack: one warp per (row, K or V) running quantize_row_warp (mikv_rows.cuh): each lane owns
+// 4 consecutive channels, group minima and maxima come from butterfly shuffles, scale and zero are
+// rounded to fp16 outward so the stored grid covers the group's range, codes are round-half-even of
+// the IEEE fp32 quotient (x - beta) / alpha, OR-ed into the packed layout in shared memory and written
+// out as whole words.
 #include "mikv_device.cuh"
 #include "mikv_internal.h"
+#include "mikv_rows.cuh"
 
 namespace mikv {
 namespace {
@@ -27,82 +27,21 @@ struct QPArgs {
   int heads_kv, n_src, n_rows, lo_start, lo_cap;
 };
 
-// Bit position of channel c (= 16 m + u) in a plane of f-bit fields: 16-bit unit and bit offset.
-__device__ __forceinline__ void field_pos(int c, int f, int& unit, int& bit) {
-  const int u = c & 15, m = c >> 4;
-  if (f == 1) {
-    unit = u & 7;
-    bit = 8 * (u >> 3) + m;
-  } else {
-    const int P = 16 / f;
-    unit = 8 * (2 * (m / P) + (u >> 3)) + (u & 7);
-    bit = f * (m % P);
-  }
-}
-
 template <int BITS, int GROUP>
 __global__ void __launch_bounds__(256) quantize_pack_kernel(const QPArgs a) {
-  constexpr int QMAX = (1 << BITS) - 1;
-  constexpr int LANES = GROUP / 4;       // lanes per quantization group
-  constexpr int WORDS = 4 * BITS;        // 32-bit words of one packed row
   __shared__ uint32_t buf[8][16];
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int i = blockIdx.x * 4 + (w >> 1);
   const bool is_v = (w & 1) != 0;
   const int bh = blockIdx.y, h = bh % a.heads_kv;
-  if (lane < 16) buf[w][lane] = 0u;
-  __syncwarp();
   if (i >= a.n_rows) return;
   const int r = a.rows[(size_t)bh * a.n_rows + i];
   if (r < 0 || r >= a.n_src) return;  // out-of-range rows are skipped (documented in the ABI)
-
-  const __nv_bfloat16* src = (is_v ? a.v_src : a.k_src) + ((size_t)bh * a.n_src + r) * kHeadDim + 4 * lane;
-  const uint2 raw = *reinterpret_cast<const uint2*>(src);
-  float x[4] = {__uint_as_float(raw.x << 16), __uint_as_float(raw.x & 0xffff0000u),
-                __uint_as_float(raw.y << 16), __uint_as_float(raw.y & 0xffff0000u)};
-  if (!is_v && a.balancer) {  // Eq. 3: keys times the balancer before the quantizer
-    const float4 b = *reinterpret_cast<const float4*>(a.balancer + h * kHeadDim + 4 * lane);
-    x[0] = __fmul_rn(x[0], b.x);
-    x[1] = __fmul_rn(x[1], b.y);
-    x[2] = __fmul_rn(x[2], b.z);
-    x[3] = __fmul_rn(x[3], b.w);
-  }
-  float mn = fminf(fminf(x[0], x[1]), fminf(x[2], x[3]));
-  float mx = fmaxf(fmaxf(x[0], x[1]), fmaxf(x[2], x[3]));
-#pragma unroll
-  for (int off = 1; off < LANES; off <<= 1) {
-    mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, off));
-    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-  }
-  // Eq. 1: beta = min, alpha = (max - min) / (2^N - 1), stored in fp16 with outward rounding.
-  const __half beta16 = __float2half_rd(mn);
-  const float beta = __half2float(beta16);
-  const float span = __fsub_rn(mx, beta);
-  const __half alpha16 = span == 0.f ? __float2half_rn(1.f) : __float2half_ru(__fdiv_rn(span, (float)QMAX));
-  const float alpha = __half2float(alpha16);
-
-#pragma unroll
-  for (int e = 0; e < 4; ++e) {
-    int code = __float2int_rn(__fdiv_rn(__fsub_rn(x[e], beta), alpha));
-    code = code < 0 ? 0 : (code > QMAX ? QMAX : code);
-    const int c = 4 * lane + e;
-    int unit, bit;
-    field_pos(c, BITS == 3 ? 2 : BITS, unit, bit);
-    const uint32_t fmask = BITS == 3 ? 3u : (uint32_t)QMAX;
-    atomicOr(&buf[w][unit >> 1], (((uint32_t)code & fmask) << bit) << (16 * (unit & 1)));
-    if (BITS == 3) {
-      field_pos(c, 1, unit, bit);
-      atomicOr(&buf[w][8 + (unit >> 1)], (((uint32_t)code >> 2) << bit) << (16 * (unit & 1)));
-    }
-  }
-  __syncwarp();
   const size_t pos = (size_t)bh * a.lo_cap + a.lo_start + i;
-  uint32_t* dst = reinterpret_cast<uint32_t*>((is_v ? a.v_codes : a.k_codes) + pos * (16 * BITS));
-  if (lane < WORDS) dst[lane] = buf[w][lane];
-  if ((lane & (LANES - 1)) == 0) {
-    __half2* params = is_v ? a.v_params : a.k_params;
-    params[pos * (kHeadDim / GROUP) + (4 * lane) / GROUP] = __halves2half2(alpha16, beta16);
-  }
+  const __nv_bfloat16* src = (is_v ? a.v_src : a.k_src) + ((size_t)bh * a.n_src + r) * kHeadDim;
+  quantize_row_warp<BITS, GROUP>(src, is_v ? nullptr : (a.balancer ? a.balancer + h * kHeadDim : nullptr),
+                                 (is_v ? a.v_codes : a.k_codes) + pos * (16 * BITS),
+                                 (is_v ? a.v_params : a.k_params) + pos * (kHeadDim / GROUP), buf[w], lane);
   if (!is_v && lane == 0) a.lo_tok[pos] = a.src_tok ? a.src_tok[(size_t)bh * a.n_src + r] : r;
 }
 

@@ -1,0 +1,176 @@
+// mikv_step.cu — the tail of one decode step, fused into one kernel per (batch b, KV head h):
+// combine the attention partials of the G query heads (output and softmax statistics), add this
+// step's attention weights to the accumulated importance of every important slot (heavy-hitter
+// policy, Fig. 4 / Sec. 3 of arxiv 2402.18096), pick the least important slot by (score, token id),
+// and quantize/pack its key and value rows into the next retained row (Eq. 1, Eq. 3).
+//
+// Each part performs the same arithmetic, in the same order, as the standalone kernels behind
+// mikv_decode_attention's merge, mikv_update_importance, mikv_select_demote and mikv_quantize_pack,
+// so a step through mikv_decode_step gives the same bits as the four separate calls.
+#include <math.h>
+
+#include "mikv_device.cuh"
+#include "mikv_internal.h"
+#include "mikv_rows.cuh"
+
+namespace mikv {
+namespace {
+
+constexpr int kPostThreads = 1024;
+constexpr int kPostUnroll = 4;  // independent slots in flight per thread
+
+template <int BITS, int GROUP, int G, int OUT_F32>
+__global__ void __launch_bounds__(kPostThreads) step_post_kernel(const StepPostArgs a) {
+  __shared__ float s_m[8], s_l[8];
+  __shared__ unsigned long long s_best[kPostThreads / 32];
+  __shared__ int s_slot[kPostThreads / 32];
+  __shared__ int s_victim;
+  __shared__ uint32_t buf[2][16];
+  const int bh = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int b = bh / a.heads_kv, h = bh - b * a.heads_kv;
+
+  // 1. combine the split partials of query heads h*G .. h*G+G-1 (one warp per query head)
+  if (warp < G) {
+    const int w0 = owner_warp((long long)bh * a.n_u, a.n_units, a.n_warps);
+    const int w1 = owner_warp((long long)(bh + 1) * a.n_u - 1, a.n_units, a.n_warps);
+    float r[4], M, L;
+    merge_head<4>(a.part_o, a.part_ml, G, bh, warp, w0, w1, 4 * lane, r, M, L);
+    const size_t bq = (size_t)b * a.heads_q + h * G + warp;
+    if (OUT_F32) {
+      reinterpret_cast<float4*>(static_cast<float*>(a.out) + bq * kHeadDim)[lane] = make_float4(r[0], r[1], r[2], r[3]);
+    } else {
+      __nv_bfloat162 v0 = __floats2bfloat162_rn(r[0], r[1]), v1 = __floats2bfloat162_rn(r[2], r[3]);
+      uint2 u;
+      u.x = *reinterpret_cast<uint32_t*>(&v0);
+      u.y = *reinterpret_cast<uint32_t*>(&v1);
+      reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(a.out) + bq * kHeadDim)[lane] = u;
+    }
+    if (lane == 0) {
+      s_m[warp] = M;
+      s_l[warp] = L;
+    }
+  }
+  __syncthreads();
+
+  // 2. importance update and the least important slot (keys are unique: ids are distinct)
+  float* acc = a.acc + (size_t)bh * a.hi_stride;
+  const int32_t* tok = a.hi_tok + (size_t)bh * a.hi_stride;
+  const float* logit = a.hi_logits + (size_t)(b * a.heads_q + h * G) * a.hi_stride;
+  unsigned long long best = ~0ull;
+  int best_slot = -1;
+  for (int i0 = tid; i0 < a.hi_cap; i0 += kPostThreads * kPostUnroll) {
+    float lg[kPostUnroll][G], ac[kPostUnroll];
+    int32_t tk[kPostUnroll];
+#pragma unroll
+    for (int r = 0; r < kPostUnroll; ++r) {  // issue every load of this round before using any
+      const int i = i0 + r * kPostThreads;
+      const bool ok = i < a.hi_cap;
+#pragma unroll
+      for (int j = 0; j < G; ++j) lg[r][j] = ok ? logit[(size_t)j * a.hi_stride + i] : 0.f;
+      ac[r] = ok ? acc[i] : 0.f;
+      tk[r] = ok ? tok[i] : 0;
+    }
+#pragma unroll
+    for (int r = 0; r < kPostUnroll; ++r) {
+      const int i = i0 + r * kPostThreads;
+      if (i >= a.hi_cap) continue;
+      float add = 0.f;
+#pragma unroll
+      for (int j = 0; j < G; ++j) add += expf(lg[r][j] - s_m[j]) / s_l[j];
+      const float v = ac[r] + add;
+      acc[i] = v;
+      const unsigned long long k = order_key(v, tk[r]);
+      if (k < best) {
+        best = k;
+        best_slot = i;
+      }
+    }
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    const unsigned long long o = __shfl_xor_sync(0xffffffffu, best, off);
+    const int os = __shfl_xor_sync(0xffffffffu, best_slot, off);
+    if (o < best) {
+      best = o;
+      best_slot = os;
+    }
+  }
+  if (lane == 0) {
+    s_best[warp] = best;
+    s_slot[warp] = best_slot;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    unsigned long long bb = s_best[0];
+    int bs = s_slot[0];
+    for (int w = 1; w < kPostThreads / 32; ++w)
+      if (s_best[w] < bb) {
+        bb = s_best[w];
+        bs = s_slot[w];
+      }
+    s_victim = bs;
+  }
+  __syncthreads();
+  const int victim = s_victim;
+  if (victim < 0) return;  // unreachable for valid scores (hi_cap >= 1, no NaN)
+
+  // 3. demote the victim: quantize its key (balanced, Eq. 3) and value rows into retained row n_lo
+  if (warp < 2) {
+    const bool is_v = warp == 1;
+    const size_t pos = (size_t)bh * a.lo_cap + a.n_lo;
+    const __nv_bfloat16* src = static_cast<const __nv_bfloat16*>(is_v ? a.v_hi : a.k_hi) +
+                               ((size_t)bh * a.hi_stride + victim) * kHeadDim;
+    quantize_row_warp<BITS, GROUP>(src, is_v ? nullptr : (a.balancer ? a.balancer + h * kHeadDim : nullptr),
+                                   static_cast<uint8_t*>(is_v ? a.v_codes : a.k_codes) + pos * (16 * BITS),
+                                   static_cast<__half2*>(is_v ? a.v_params : a.k_params) + pos * (kHeadDim / GROUP),
+                                   buf[warp], lane);
+    if (!is_v && lane == 0) {
+      a.lo_tok[pos] = tok[victim];
+      a.slots[bh] = victim;
+    }
+  }
+}
+
+template <int BITS, int GROUP, int G>
+cudaError_t post_out(const StepPostArgs& a, int out_f32, cudaStream_t st) {
+  const int grid = a.batch * a.heads_kv;
+  if (out_f32)
+    step_post_kernel<BITS, GROUP, G, 1><<<grid, kPostThreads, 0, st>>>(a);
+  else
+    step_post_kernel<BITS, GROUP, G, 0><<<grid, kPostThreads, 0, st>>>(a);
+  return cudaGetLastError();
+}
+
+template <int BITS, int GROUP>
+cudaError_t post_g(const StepPostArgs& a, int G, int out_f32, cudaStream_t st) {
+  switch (G) {
+    case 1: return post_out<BITS, GROUP, 1>(a, out_f32, st);
+    case 2: return post_out<BITS, GROUP, 2>(a, out_f32, st);
+    case 4: return post_out<BITS, GROUP, 4>(a, out_f32, st);
+    case 8: return post_out<BITS, GROUP, 8>(a, out_f32, st);
+  }
+  return cudaErrorInvalidValue;
+}
+
+template <int BITS>
+cudaError_t post_group(const StepPostArgs& a, int group, int G, int out_f32, cudaStream_t st) {
+  switch (group) {
+    case 32: return post_g<BITS, 32>(a, G, out_f32, st);
+    case 64: return post_g<BITS, 64>(a, G, out_f32, st);
+    case 128: return post_g<BITS, 128>(a, G, out_f32, st);
+  }
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace
+
+cudaError_t launch_step_post(const StepPostArgs& a, int bits, int group, int G, int out_f32, cudaStream_t st) {
+  switch (bits) {
+    case 2: return post_group<2>(a, group, G, out_f32, st);
+    case 3: return post_group<3>(a, group, G, out_f32, st);
+    case 4: return post_group<4>(a, group, G, out_f32, st);
+  }
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace mikv

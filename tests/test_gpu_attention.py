@@ -165,11 +165,14 @@ def test_decode_steps_trajectory():
     assert near_ties <= 2
 
 
-@pytest.mark.parametrize("wname,heads", [("llama2-7b", [(0, 0), (7, 31)]), ("mistral-7b", [(31, 7)]),
-                                        ("llama2-13b", [(15, 39)])])
+@pytest.mark.parametrize("wname,heads", [("llama2-7b", [(0, 0), (3, 17), (7, 31)]),
+                                        ("mistral-7b", [(0, 0), (13, 5), (31, 7)]),
+                                        ("llama2-13b", [(9, 21), (15, 39)])])
 def test_full_size_layer_sampled_heads(wname, heads):
-    """One layer at the benchmark's full size, built and attended in the benchmark's launch
-    configuration; the oracle checks sampled (batch, KV head) pairs one by one."""
+    """One layer at the benchmark's full size, built and stepped in the benchmark's launch
+    configuration (decode step: insert, attention, fused merge / update / select / demote); the oracle
+    checks sampled (batch, KV head) pairs one by one: retained codes, output, softmax max and sum, the
+    demoted slot and its packed row."""
     w = mi.WORKLOADS[wname]
     dev = torch.device("cuda")
     k, v = mi.prefill_kv(w, 0, dev)
@@ -181,9 +184,16 @@ def test_full_size_layer_sampled_heads(wname, heads):
     layer = MixedPrecisionLayer.from_prefill(shape, k, v, scores, q_pre, device=dev)
     G = w.heads_q // w.heads_kv
     q, k_new, v_new = mi.decode_inputs(w, 0, 0, dev)
+    # attention with statistics on a copy of the inserted state, then the real fused step
+    pkg.mikv_insert_token(layer.cache, k_new, v_new, w.context, layer.slots)
+    ml = torch.empty(w.batch, w.heads_q, 2, device=dev)
+    out_a = torch.empty(w.batch, w.heads_q, w.head_dim, dtype=torch.float32, device=dev)
+    ws = new_workspace(shape, pkg.WS_ATTENTION, w.n_lo0)
+    pkg.mikv_decode_attention(layer.cache, w.n_lo0, q, sm_scale(), out_a, ws, ml=ml)
     out = torch.empty(w.batch, w.heads_q, w.head_dim, dtype=torch.bfloat16, device=dev)
-    layer.step(q, k_new, v_new, out)
+    layer.step(q, k_new, v_new, out)  # re-inserts the same token into the same slot: idempotent
     pkg.mikv_workspace_check(layer.ws)
+    victims = layer.slots.cpu().numpy()
     for b, h in heads:
         raw = (k[:, h:h + 1].cpu(), v[:, h:h + 1].cpu(), scores[:, h:h + 1].cpu(),
                q_pre[:, h * G:(h + 1) * G].cpu())
@@ -196,9 +206,26 @@ def test_full_size_layer_sampled_heads(wname, heads):
                                       .view(np.uint16), c["v_params"][0, 0, :n_lo])
         oracle.insert_token(c, bits16(k_new[b:b + 1, h:h + 1]), bits16(v_new[b:b + 1, h:h + 1]), w.context,
                             np.array([[w.budget]], np.int32))
-        ref_o, _, _ = oracle.decode_attention(c, bits16(q[b:b + 1, h * G:(h + 1) * G]), n_lo, sm_scale(),
-                                              balancer_=ref["balancer"])
+        qb = bits16(q[b:b + 1, h * G:(h + 1) * G])
+        ref_o, hl, rml = oracle.decode_attention(c, qb, n_lo, sm_scale(), balancer_=ref["balancer"])
         vmax = max(float(v[b, h].float().abs().max()), float(v_new[b, h].float().abs().max()))
         got = out[b, h * G:(h + 1) * G].float().cpu().numpy()
         tol = attention_tolerance(vmax, ref_o[0], True)
         assert np.all(np.abs(got - ref_o[0]) <= tol), np.abs(got - ref_o[0]).max()
+        got_a = out_a[b, h * G:(h + 1) * G].cpu().numpy()
+        assert np.all(np.abs(got_a - ref_o[0]) <= attention_tolerance(vmax, ref_o[0], False))
+        # softmax statistics: every token is counted once (a lost or doubled block moves l by >= 0.1 %)
+        bound = _logit_bound(c, qb, ref["balancer"], w, n_lo)
+        gm = ml[b, h * G:(h + 1) * G].cpu().numpy()
+        assert np.all(np.abs(gm[:, 0] - rml[0, :, 0]) <= bound)
+        np.testing.assert_allclose(gm[:, 1], rml[0, :, 1], rtol=4 * float(bound.max()) + 1e-5)
+        # the demoted slot and its packed rows
+        acc = oracle.update_importance(c["acc"], hl.astype(np.float32), rml.astype(np.float32), G)
+        dem, _ = oracle.select_demote(acc, 1, c["hi_tok"], want_kept=False)
+        if int(dem[0, 0, 0]) == int(victims[b, h]):
+            oracle.quantize_pack(c, c["k_hi"], c["v_hi"], dem, n_lo, src_tok=c["hi_tok"], balancer_=ref["balancer"])
+            np.testing.assert_array_equal(layer.cache.v_codes[b, h, n_lo].cpu().numpy(), c["v_codes"][0, 0, n_lo])
+            assert int(layer.cache.lo_tok[b, h, n_lo]) == int(c["lo_tok"][0, 0, n_lo])
+        else:  # only a near tie of fp32 scores may pick another slot
+            a_sorted = np.sort(acc[0, 0])
+            assert abs(a_sorted[1] - a_sorted[0]) < 1e-5 * max(1.0, abs(a_sorted[0]))
