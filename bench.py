@@ -389,6 +389,61 @@ def cpu_baseline(w, seconds: float = 15.0, steps=None):
             "ms_per_head_step": round(1e3 * elapsed / n, 3)}
 
 
+def run_sweep(args):
+    """Every point of the batch-64 sweep (bits x importance ratio x group): whole decode steps on one
+    layer (insert, attention, importance update, one demotion per head), plus attention alone."""
+    import paper_2402_18096_gb300 as pkg
+    from paper_2402_18096_gb300.layer import MixedPrecisionLayer
+    dev = torch.device("cuda")
+    pkg.load()
+    peak, peak_kind = _peaks()
+    points = []
+    for w in mi.sweep_workloads():
+        K, W = args.steps, args.warmup
+        shape = pkg.Shape(w.batch, w.heads_q, w.heads_kv, w.bits, w.group, w.hi_cap, w.lo_cap_for(K + W + 4))
+        k, v = mi.prefill_kv(w, 0, dev)
+        sc = mi.initial_scores(w, 0, dev)
+        qp = mi.prefill_queries(w, 0, dev)
+        layer = MixedPrecisionLayer.from_prefill(shape, k, v, sc, qp, device=dev)
+        del k, v, qp
+        ins = [mi.decode_inputs(w, 0, s, dev) for s in range(K + W)]
+        out = torch.empty(w.batch, w.heads_q, w.head_dim, dtype=torch.bfloat16, device=dev)
+        for s in range(W):
+            layer.step(*ins[s], out)
+        torch.cuda.synchronize()
+        b0 = layer.cache.nbytes_attended(layer.n_lo)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for s in range(K):
+            layer.step(*ins[W + s], out)
+        e1.record()
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / K
+        nbytes = (b0 + layer.cache.nbytes_attended(layer.n_lo)) / 2 - (layer.cache.nbytes_attended(1)
+                                                                     - layer.cache.nbytes_attended(0)) / 2
+        ws = torch.zeros(pkg.mikv_workspace_bytes(shape, pkg.WS_ATTENTION, layer.n_lo) + 256, dtype=torch.uint8,
+                         device=dev)
+        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a0.record()
+        for _ in range(K):
+            pkg.mikv_decode_attention(layer.cache, layer.n_lo, ins[0][0], layer.sm_scale, out, ws)
+        a1.record()
+        torch.cuda.synchronize()
+        attn_ms = a0.elapsed_time(a1) / K
+        ab = layer.cache.nbytes_attended(layer.n_lo)
+        pkg.mikv_workspace_check(layer.ws)
+        pkg.mikv_workspace_check(ws)
+        points.append({"bits": w.bits, "group": w.group, "ratio": w.ratio, "compressed_bytes": int(nbytes),
+                       "us_per_step": round(ms * 1e3, 1), "step_gbs": round(nbytes / ms / 1e6, 1),
+                       "attn_us": round(attn_ms * 1e3, 1), "attn_gbs": round(ab / attn_ms / 1e6, 1),
+                       "attn_frac": round(ab / attn_ms / 1e6 / peak, 3)})
+        del layer, ins
+        torch.cuda.empty_cache()
+    print(json.dumps({"sweep": "batch 64, 32 heads, T 4096, one layer; bits x ratio x group",
+                      "metric": METRIC, "unit": UNIT, "peak": peak, "peak_kind": peak_kind, "steps": args.steps,
+                      "warmup": args.warmup, "points": points}), flush=True)
+
+
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -436,11 +491,14 @@ def main():
     ap.add_argument("--layers", type=int, default=0, help="fewer layers (profiling cases only)")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sweep", action="store_true", help="the batch-64 bits x ratio x group sweep (one layer)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "mikv" and not (args.batch or args.layers):
         ap.error("--warmup must be >= 3")
     if args.impl == "reference":
         run_reference(args)
+    elif args.sweep:
+        run_sweep(args)
     else:
         run_mikv(args)
 

@@ -47,9 +47,17 @@ namespace {
 #ifndef MIKV_QK_ACC
 #define MIKV_QK_ACC 2
 #endif
+#ifndef MIKV_LO_PAIR
+#define MIKV_LO_PAIR 1
+#endif
+#ifndef MIKV_PAIR_ACC
+#define MIKV_PAIR_ACC 1
+#endif
 constexpr int kWarps = MIKV_ATTN_WARPS;     // independent warps per CTA
 constexpr int kThreads = kWarps * 32;
 constexpr int kNS = MIKV_ATTN_STAGES;       // ring stages per warp
+constexpr bool kLoPair = MIKV_LO_PAIR != 0;  // retained blocks processed two at a time
+constexpr int kPairAcc = MIKV_PAIR_ACC;      // QK^T accumulators per block when paired
 constexpr int kStageBytes = kUnitBytes;
 constexpr int kHiBlockBytes = 8192;         // K and V of 16 tokens: 4 boxes of 16 rows x 64 bf16
 constexpr int kCtasPerSm = MIKV_ATTN_CTAS;
@@ -98,33 +106,49 @@ __device__ __forceinline__ void cursor_next(Cursor& c, int hu, int n_u) {
   }
 }
 
+// Running softmax state of heads 2t, 2t+1: reference max m (warp-uniform per head), sum l of
+// exp(logit - m) over this thread's tokens, and mx, the largest logit this thread has seen.
 struct Softmax {
-  float m[2], l[2];
+  float m[2], l[2], mx[2];
 };
 
-__device__ __forceinline__ void sum_acc(const float (&accs)[kQkAcc][4], float (&acc)[4]) {
+template <int Q>
+__device__ __forceinline__ void sum_acc(const float (&accs)[Q][4], float (&acc)[4]) {
 #pragma unroll
   for (int e = 0; e < 4; ++e) {
     float v = accs[0][e];
 #pragma unroll
-    for (int q = 1; q < kQkAcc; ++q) v += accs[q][e];
+    for (int q = 1; q < Q; ++q) v += accs[q][e];
     acc[e] = v;
   }
 }
 
-// Online-softmax update for one 16-token block. s holds scaled logits of (token g, head 2t),
-// (g, 2t+1), (g+8, 2t), (g+8, 2t+1) (-inf past the end); returns unnormalised probabilities in p.
-// o (output) and ob (zero-row sums) are running sums at the current max: both are rescaled.
-__device__ __forceinline__ void softmax_block(const float (&s)[4], Softmax& st, float (&o)[8][4], float (&ob)[4],
-                                              float (&p)[4]) {
-  float bm0 = fmaxf(s[0], s[2]), bm1 = fmaxf(s[1], s[3]);
+// Online-softmax update for NK 16-token blocks. s[k] holds scaled logits of (token g, head 2t),
+// (g, 2t+1), (g+8, 2t), (g+8, 2t+1) of block k (-inf past the end); returns unnormalised
+// probabilities in p.
+// o (output) and ob (zero-row and alpha sums) are running sums at the current reference max m: all are
+// rescaled when m moves. The reference is only moved (one cross-lane reduction) when some logit exceeds it by
+// more than kLazy; otherwise the block reuses the old reference, so probabilities stay below e^kLazy.
+constexpr float kLazy = 4.f;
+
+template <int NB, int NK>
+__device__ __forceinline__ void softmax_blocks(const float (&s)[NK][4], Softmax& st, float (&o)[8][4],
+                                               float (&ob)[NB][4], float (&p)[NK][4]) {
+  float bm0 = fmaxf(s[0][0], s[0][2]), bm1 = fmaxf(s[0][1], s[0][3]);
 #pragma unroll
-  for (int off = 4; off < 32; off <<= 1) {
-    bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, off));
-    bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, off));
+  for (int k = 1; k < NK; ++k) {
+    bm0 = fmaxf(bm0, fmaxf(s[k][0], s[k][2]));
+    bm1 = fmaxf(bm1, fmaxf(s[k][1], s[k][3]));
   }
-  const float mn0 = fmaxf(st.m[0], bm0), mn1 = fmaxf(st.m[1], bm1);
-  if (__any_sync(0xffffffffu, mn0 > st.m[0] || mn1 > st.m[1])) {
+  st.mx[0] = fmaxf(st.mx[0], bm0);
+  st.mx[1] = fmaxf(st.mx[1], bm1);
+  if (__any_sync(0xffffffffu, bm0 > st.m[0] + kLazy || bm1 > st.m[1] + kLazy)) {
+#pragma unroll
+    for (int off = 4; off < 32; off <<= 1) {
+      bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, off));
+      bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, off));
+    }
+    const float mn0 = fmaxf(st.m[0], bm0), mn1 = fmaxf(st.m[1], bm1);
     const float c0 = mn0 == st.m[0] ? 1.f : fast_exp2((st.m[0] - mn0) * kLog2e);
     const float c1 = mn1 == st.m[1] ? 1.f : fast_exp2((st.m[1] - mn1) * kLog2e);
     st.l[0] *= c0;
@@ -136,18 +160,26 @@ __device__ __forceinline__ void softmax_block(const float (&s)[4], Softmax& st, 
       o[mt][2] *= c0;
       o[mt][3] *= c1;
     }
-    ob[0] *= c0;
-    ob[1] *= c1;
+#pragma unroll
+    for (int i = 0; i < NB; ++i) {
+      ob[i][0] *= c0;
+      ob[i][1] *= c1;
+      ob[i][2] *= c0;
+      ob[i][3] *= c1;
+    }
     st.m[0] = mn0;
     st.m[1] = mn1;
   }
   const float ml0 = st.m[0] * kLog2e, ml1 = st.m[1] * kLog2e;
-  p[0] = fast_exp2(fmaf(s[0], kLog2e, -ml0));
-  p[1] = fast_exp2(fmaf(s[1], kLog2e, -ml1));
-  p[2] = fast_exp2(fmaf(s[2], kLog2e, -ml0));
-  p[3] = fast_exp2(fmaf(s[3], kLog2e, -ml1));
-  st.l[0] += p[0] + p[2];
-  st.l[1] += p[1] + p[3];
+#pragma unroll
+  for (int k = 0; k < NK; ++k) {
+    p[k][0] = fast_exp2(fmaf(s[k][0], kLog2e, -ml0));
+    p[k][1] = fast_exp2(fmaf(s[k][1], kLog2e, -ml1));
+    p[k][2] = fast_exp2(fmaf(s[k][2], kLog2e, -ml0));
+    p[k][3] = fast_exp2(fmaf(s[k][3], kLog2e, -ml1));
+    st.l[0] += p[k][0] + p[k][2];
+    st.l[1] += p[k][1] + p[k][3];
+  }
 }
 
 // Scale raw dot products, mask tokens >= valid, and store important-set logits.
@@ -211,12 +243,35 @@ __device__ __forceinline__ uint32_t code3(uint32_t r, uint32_t h, int j, int hb)
   return exact_codes(lo | (((h >> hb) << 2) & 0x00040004u), 0x64006400u);
 }
 
+// Value codes (N = 2, 4) skip the subtraction: the code is placed at a mantissa position where it
+// weighs 1 under a magic M in {4, 16, 64}, so the fp16 pair holds M + code exactly. The PV sums then
+// carry M * sum(p * alpha) per channel on top of the wanted sum; that term is measured by a ones-row
+// MMA on the same fp16 operands and removed in write_partial. M stays small (<= 64) so the removal
+// costs only a few bits of the fp32 accumulator.
+// N = 2: code j of r sits at bits 2j of each unit. Four shifted copies (r << 6, r << 2, r >> 2, r >> 6)
+// bring codes 2i and 2i + 1 to bits 6..7 (M = 16) and 8..9 (M = 4).
+__device__ __forceinline__ uint32_t vcode2(const uint32_t (&sh)[4], int j) {
+  return (j & 1) ? and_or(sh[j >> 1], 0x03000300u, 0x44004400u) : and_or(sh[j >> 1], 0x00C000C0u, 0x4C004C00u);
+}
+__host__ __device__ constexpr float voff2(int j) { return (j & 1) ? 4.f : 16.f; }
+// N = 4: nibble p of r at bits 4p. Nibbles 0 and 1 are read at bits 4..7 of r << 4 and r (M = 64),
+// nibbles 2 and 3 at bits 6..9 of r >> 2 and r >> 6 (M = 16).
+__device__ __forceinline__ uint32_t vcode4(const uint32_t (&sh)[4], int p) {
+  return p < 2 ? and_or(sh[p], 0x00F000F0u, 0x54005400u) : and_or(sh[p], 0x03C003C0u, 0x4C004C00u);
+}
+__host__ __device__ constexpr float voff4(int p) { return p < 2 ? 64.f : 16.f; }
+
+template <int BITS>
+__host__ __device__ constexpr float voff(int mt) {
+  return BITS == 2 ? voff2(mt) : BITS == 4 ? voff4(mt & 3) : 0.f;
+}
+
 // ---------------------------------------------------------------------- one important block
 
-template <int G>
+template <int G, int NB>
 __device__ __forceinline__ void process_hi(uint32_t blk, int valid, int slot0, const uint32_t (&qb)[8][2],
                                            float scale, float* logit_base, int hi_stride, Softmax& st,
-                                           float (&o)[8][4], float (&ob)[4], int lane) {
+                                           float (&o)[8][4], float (&ob)[NB][4], int lane) {
   const int g = lane >> 2, t = lane & 3, r8 = lane & 7, j = lane >> 3;
   float accs[kQkAcc][4];
 #pragma unroll
@@ -231,11 +286,11 @@ __device__ __forceinline__ void process_hi(uint32_t blk, int valid, int slot0, c
   }
   float acc[4];
   sum_acc(accs, acc);
-  float s[4], p[4];
-  finish_logits<G>(acc, scale, valid, g, t, logit_base, hi_stride, slot0, s);
-  softmax_block(s, st, o, ob, p);
-  const uint32_t pb0 = movmatrix_t(pack_bf16(p[0], p[1]));
-  const uint32_t pb1 = movmatrix_t(pack_bf16(p[2], p[3]));
+  float s[1][4], p[1][4];
+  finish_logits<G>(acc, scale, valid, g, t, logit_base, hi_stride, slot0, s[0]);
+  softmax_blocks(s, st, o, ob, p);
+  const uint32_t pb0 = movmatrix_t(pack_bf16(p[0][0], p[0][1]));
+  const uint32_t pb1 = movmatrix_t(pack_bf16(p[0][2], p[0][3]));
   uint32_t m01 = 0xffffffffu, m89 = 0xffffffffu;
   if (valid < 16) {
     m01 = (2 * t < valid ? 0x0000ffffu : 0u) | (2 * t + 1 < valid ? 0xffff0000u : 0u);
@@ -259,16 +314,16 @@ __device__ __forceinline__ void process_hi(uint32_t blk, int valid, int slot0, c
 
 // ---------------------------------------------------------------------- one retained block
 
-template <int BITS, int GROUP, int G>
-__device__ __forceinline__ void process_lo(uint32_t unit, int b, int valid, const uint32_t (&qh)[8][2], float scale,
-                                           Softmax& st, float (&o)[8][4], float (&ob)[4], int lane) {
+// Key side of retained block b of a unit: scaled logits s, -inf past valid.
+template <int BITS, int GROUP, int G, int QACC>
+__device__ __forceinline__ void lo_logits(uint32_t unit, int b, int valid, const uint32_t (&qh)[8][2], float scale,
+                                          float (&s)[4], int lane) {
   constexpr LoUnit U = lo_unit_layout(BITS, GROUP);
   constexpr int NG = kHeadDim / GROUP;
   constexpr int PR = U.param_row;
   // this block's rows inside the unit's sections
   const uint32_t ka = unit + U.k_a + b * 16 * U.plane_a_bytes, kb = unit + U.k_b + b * 16 * U.plane_b_bytes;
-  const uint32_t va = unit + U.v_a + b * 16 * U.plane_a_bytes, vb = unit + U.v_b + b * 16 * U.plane_b_bytes;
-  const uint32_t kp = unit + U.k_p + b * 16 * PR, vp = unit + U.v_p + b * 16 * PR;
+  const uint32_t kp = unit + U.k_p + b * 16 * PR;
   constexpr int NR = BITS == 4 ? 8 : 4;
   const int g = lane >> 2, t = lane & 3, r8 = lane & 7, j = lane >> 3;
 
@@ -301,9 +356,9 @@ __device__ __forceinline__ void process_lo(uint32_t unit, int b, int valid, cons
   uint32_t pk0[NG], pk1[NG];
   lds_vec<NG>(kp + g * PR, pk0);
   lds_vec<NG>(kp + (g + 8) * PR, pk1);
-  float accs[kQkAcc][4];
+  float accs[QACC][4];
 #pragma unroll
-  for (int q = 0; q < kQkAcc; ++q) accs[q][0] = accs[q][1] = accs[q][2] = accs[q][3] = 0.f;
+  for (int q = 0; q < QACC; ++q) accs[q][0] = accs[q][1] = accs[q][2] = accs[q][3] = 0.f;
 #pragma unroll
   for (int ks = 0; ks < 8; ++ks) {
     const int gi = (16 * ks) / GROUP;
@@ -327,18 +382,29 @@ __device__ __forceinline__ void process_lo(uint32_t unit, int b, int valid, cons
                            h2_as_u32(__hfma2(u32_as_h2(c[1]), u32_as_h2(al1), u32_as_h2(be1))),
                            h2_as_u32(__hfma2(u32_as_h2(c[2]), u32_as_h2(al0), u32_as_h2(be0))),
                            h2_as_u32(__hfma2(u32_as_h2(c[3]), u32_as_h2(al1), u32_as_h2(be1)))};
-    mma_f16(accs[ks % kQkAcc], a, qh[ks][0], qh[ks][1]);
+    mma_f16(accs[ks % QACC], a, qh[ks][0], qh[ks][1]);
   }
   float acc[4];
   sum_acc(accs, acc);
-  float s[4], p[4];
   finish_logits<G>(acc, scale, valid, g, t, nullptr, 0, 0, s);
-  softmax_block(s, st, o, ob, p);
+}
+
+// Value side of retained block b: o, ob += P (this block's probabilities p) times the block's values.
+template <int BITS, int GROUP, int NB>
+__device__ __forceinline__ void lo_values(uint32_t unit, int b, int valid, const float (&p)[4], float (&o)[8][4],
+                                          float (&ob)[NB][4], int lane) {
+  constexpr LoUnit U = lo_unit_layout(BITS, GROUP);
+  constexpr int NG = kHeadDim / GROUP;
+  constexpr int PR = U.param_row;
+  const uint32_t va = unit + U.v_a + b * 16 * U.plane_a_bytes, vb = unit + U.v_b + b * 16 * U.plane_b_bytes;
+  const uint32_t vp = unit + U.v_p + b * 16 * PR;
+  constexpr int NR = BITS == 4 ? 8 : 4;
+  const int g = lane >> 2, t = lane & 3, r8 = lane & 7, j = lane >> 3;
   const uint32_t pb0 = movmatrix_t(pack_f16(p[0], p[1]));  // (P[2t][head g], P[2t+1][head g])
   const uint32_t pb1 = movmatrix_t(pack_f16(p[2], p[3]));  // tokens 2t+8, 2t+9
 
   // ---- values of tokens (2t, 2t+1) and (2t+8, 2t+9), channels 16 mt + g and 16 mt + 8 + g
-  uint32_t vr[NR], vh[NR];
+  uint32_t vr[NR];
   uint32_t vb0 = 0, vb1 = 0;
   {
     const int tok = r8 + 8 * (j >> 1);
@@ -360,8 +426,6 @@ __device__ __forceinline__ void process_lo(uint32_t unit, int b, int valid, cons
       for (int i = 0; i < 4; ++i) vr[i] = r0[i];
       if (BITS == 3) ldsm_x2_t(vb + (lane & 15) * 16, vb0, vb1);
     }
-#pragma unroll
-    for (int i = 0; i < NR; ++i) vh[i] = vr[i] >> (BITS == 4 ? 8 : 10);
   }
   // (alpha, beta) of the four tokens for every group; zero past the end (exact zeros in the sums)
   const int t0 = 2 * t, t1 = 2 * t + 1, t8 = 2 * t + 8, t9 = 2 * t + 9;
@@ -370,7 +434,7 @@ __device__ __forceinline__ void process_lo(uint32_t unit, int b, int valid, cons
   lds_vec<NG>(vp + t1 * PR, pv1);
   lds_vec<NG>(vp + t8 * PR, pv8);
   lds_vec<NG>(vp + t9 * PR, pv9);
-  // zero-row operand: row g < NG holds beta of group g for this thread's tokens
+  // zero rows: row g < NG of the beta operand holds beta of group g for this thread's tokens
   uint32_t bw0 = 0, bw1 = 0, bw8 = 0, bw9 = 0;
   if (g < NG) {
     bw0 = lds32(vp + t0 * PR + 4 * g);
@@ -393,13 +457,24 @@ __device__ __forceinline__ void process_lo(uint32_t unit, int b, int valid, cons
   }
   {
     const uint32_t a[4] = {prmt(bw0, bw1, 0x7632u), 0u, prmt(bw8, bw9, 0x7632u), 0u};
-    mma_f16(ob, a, pb0, pb1);  // ob[row g][heads 2t, 2t+1] += sum over tokens of p * beta_g
+    mma_f16(ob[0], a, pb0, pb1);  // ob[0][row gi][heads 2t, 2t+1] += sum over tokens of p * beta
   }
   uint32_t pa0[NG], pa1[NG];  // p * alpha per group: B operand of the code MMAs
 #pragma unroll
   for (int gi = 0; gi < NG; ++gi) {
     pa0[gi] = h2_as_u32(__hmul2(u32_as_h2(pb0), u32_as_h2(prmt(pv0[gi], pv1[gi], 0x5410u))));
     pa1[gi] = h2_as_u32(__hmul2(u32_as_h2(pb1), u32_as_h2(prmt(pv8[gi], pv9[gi], 0x5410u))));
+  }
+  if (BITS != 3) {
+    // sum of p * alpha per group, from the same fp16 operands as the code MMAs: ones in rows 0..7
+    // (even groups) or 8..15 (odd groups), so ob[1 + gi / 2] holds two groups per fragment
+    constexpr uint32_t kOne = 0x3C003C00u;
+#pragma unroll
+    for (int gi = 0; gi < NG; ++gi) {
+      const uint32_t e = (gi & 1) ? 0u : kOne, d = (gi & 1) ? kOne : 0u;
+      const uint32_t a[4] = {e, d, e, d};
+      mma_f16(ob[1 + gi / 2], a, pa0[gi], pa1[gi]);
+    }
   }
 #pragma unroll
   for (int mt = 0; mt < 8; ++mt) {
@@ -408,36 +483,67 @@ __device__ __forceinline__ void process_lo(uint32_t unit, int b, int valid, cons
     if (BITS == 4) {
       const int ri = (mt >> 2) * 4, pp = mt & 3;
 #pragma unroll
-      for (int i = 0; i < 4; ++i) a[i] = code4(vr[ri + i], vh[ri + i], pp);
+      for (int i = 0; i < 4; ++i) {
+        const uint32_t w = vr[ri + i];
+        const uint32_t c4[4] = {w << 4, w, w >> 2, w >> 6};  // shared by the four mt of this word
+        a[i] = vcode4(c4, pp);
+      }
     } else if (BITS == 2) {
 #pragma unroll
-      for (int i = 0; i < 4; ++i) a[i] = code2(vr[i], vh[i], mt);
+      for (int i = 0; i < 4; ++i) {
+        const uint32_t c2[4] = {vr[i] << 6, vr[i] << 2, vr[i] >> 2, vr[i] >> 6};  // shared by all mt
+        a[i] = vcode2(c2, mt);
+      }
     } else {
       a[0] = code3(vr[0], vb0, mt, mt);
       a[1] = code3(vr[1], vb0, mt, 8 + mt);
       a[2] = code3(vr[2], vb1, mt, mt);
       a[3] = code3(vr[3], vb1, mt, 8 + mt);
     }
-    mma_f16(o[mt], a, pa0[gi], pa1[gi]);
+    mma_f16(o[mt], a, pa0[gi], pa1[gi]);  // sums p * alpha * (code + offset)
   }
 }
 
-// Write this warp's partial for one head: unnormalised output (plus the zero-row terms), max, sum.
-template <int GROUP, int G>
+// NK consecutive retained blocks b .. b + NK - 1 of a unit (n_left = valid tokens from block b on, at
+// least 16 (NK - 1) + 1): the key sides first, one softmax update over all NK blocks, then the value
+// sides, so the dependency chains of the blocks overlap.
+template <int BITS, int GROUP, int G, int NB, int NK>
+__device__ __forceinline__ void process_lo(uint32_t unit, int b, int n_left, const uint32_t (&qh)[8][2], float scale,
+                                           Softmax& st, float (&o)[8][4], float (&ob)[NB][4], int lane) {
+  float s[NK][4], p[NK][4];
+#pragma unroll
+  for (int k = 0; k < NK; ++k)
+    lo_logits<BITS, GROUP, G, NK == 1 ? kQkAcc : kPairAcc>(unit, b + k, min(16, n_left - 16 * k), qh, scale, s[k],
+                                                           lane);
+  softmax_blocks(s, st, o, ob, p);
+#pragma unroll
+  for (int k = 0; k < NK; ++k) lo_values<BITS, GROUP, NB>(unit, b + k, min(16, n_left - 16 * k), p[k], o, ob, lane);
+}
+
+// Write this warp's partial for one head: output (plus the zero-row terms, minus the value-code offsets),
+// true max and sum. The running sums are at the reference max m; they are rescaled here to the largest
+// logit seen, so the partial's (max, sum) are the exact statistics of its tokens.
+template <int BITS, int GROUP, int G, int NB>
 __device__ __forceinline__ void write_partial(const AttnArgs& a, int slot, Softmax& st, const float (&o)[8][4],
-                                              const float (&ob)[4], int lane) {
+                                              const float (&ob)[NB][4], int lane) {
   const int g = lane >> 2, t = lane & 3;
 #pragma unroll
   for (int off = 4; off < 32; off <<= 1) {
     st.l[0] += __shfl_xor_sync(0xffffffffu, st.l[0], off);
     st.l[1] += __shfl_xor_sync(0xffffffffu, st.l[1], off);
+    st.mx[0] = fmaxf(st.mx[0], __shfl_xor_sync(0xffffffffu, st.mx[0], off));
+    st.mx[1] = fmaxf(st.mx[1], __shfl_xor_sync(0xffffffffu, st.mx[1], off));
   }
+  float c[2];
+#pragma unroll
+  for (int hd = 0; hd < 2; ++hd)  // m <= mx <= m + kLazy; equal (also both -inf) gives 1
+    c[hd] = st.mx[hd] == st.m[hd] ? 1.f : fast_exp2((st.m[hd] - st.mx[hd]) * kLog2e);
   constexpr int NG = kHeadDim / GROUP;
   float bz0[NG], bz1[NG];  // sum p * beta of group gi for heads 2t, 2t+1, held by lane 4 gi + t
 #pragma unroll
   for (int gi = 0; gi < NG; ++gi) {
-    bz0[gi] = __shfl_sync(0xffffffffu, ob[0], gi * 4 + t);
-    bz1[gi] = __shfl_sync(0xffffffffu, ob[1], gi * 4 + t);
+    bz0[gi] = __shfl_sync(0xffffffffu, ob[0][0], gi * 4 + t);
+    bz1[gi] = __shfl_sync(0xffffffffu, ob[0][1], gi * 4 + t);
   }
 #pragma unroll
   for (int hd = 0; hd < 2; ++hd) {
@@ -447,13 +553,14 @@ __device__ __forceinline__ void write_partial(const AttnArgs& a, int slot, Softm
 #pragma unroll
       for (int mt = 0; mt < 8; ++mt) {
         const int gi = (16 * mt) / GROUP;
-        const float z = hd ? bz1[gi] : bz0[gi];
-        po[16 * mt + g] = o[mt][hd] + z;
-        po[16 * mt + 8 + g] = o[mt][2 + hd] + z;
+        float z = hd ? bz1[gi] : bz0[gi];
+        if (BITS != 3) z = fmaf(-voff<BITS>(mt), ob[1 + gi / 2][2 * (gi & 1) + hd], z);
+        po[16 * mt + g] = (o[mt][hd] + z) * c[hd];
+        po[16 * mt + 8 + g] = (o[mt][2 + hd] + z) * c[hd];
       }
       if (g == 0) {
-        a.part_ml[((size_t)slot * G + head) * 2] = st.m[hd];
-        a.part_ml[((size_t)slot * G + head) * 2 + 1] = st.l[hd];
+        a.part_ml[((size_t)slot * G + head) * 2] = st.mx[hd];
+        a.part_ml[((size_t)slot * G + head) * 2 + 1] = st.l[hd] * c[hd];
       }
     }
   }
@@ -527,8 +634,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
 
   const int g = lane >> 2, t = lane & 3;
   uint32_t qb[8][2], qh[8][2];
+  constexpr int NB = 1 + (BITS == 3 ? 0 : (kHeadDim / GROUP + 1) / 2);  // beta rows + alpha-sum pairs
   Softmax st;
-  float o[8][4], ob[4];
+  float o[8][4], ob[NB][4];
   float* logit_base = nullptr;
   Cursor cc = cursor_at(u0, hu, n_u);  // unit being consumed
   int cur = -1;
@@ -536,7 +644,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
   int u = u0;
   for (; u < u1; ++u) {
     if (cc.bh != cur) {
-      if (cur >= 0) write_partial<GROUP, G>(a, wg + cur, st, o, ob, lane);
+      if (cur >= 0) write_partial<BITS, GROUP, G, NB>(a, wg + cur, st, o, ob, lane);
       cur = cc.bh;
       const int b = cur / a.heads_kv, h = cur - b * a.heads_kv;
       // query fragments (B operand: head g; channels 16 ks + 2t (+1) and 16 ks + 2t + 8 (+9))
@@ -562,9 +670,11 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
       logit_base = a.hi_logits ? a.hi_logits + (size_t)(b * a.heads_q + h * G) * a.hi_stride : nullptr;
       st.m[0] = st.m[1] = -INFINITY;
       st.l[0] = st.l[1] = 0.f;
+      st.mx[0] = st.mx[1] = -INFINITY;
 #pragma unroll
       for (int mt = 0; mt < 8; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
-      ob[0] = ob[1] = ob[2] = ob[3] = 0.f;
+#pragma unroll
+      for (int i = 0; i < NB; ++i) ob[i][0] = ob[i][1] = ob[i][2] = ob[i][3] = 0.f;
     }
     const int s = (u - u0) % kNS;
     const uint32_t use = (u - u0) / kNS;
@@ -576,13 +686,17 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
     const uint32_t stage = ring + s * kStageBytes;
     const UnitKind k = cursor_kind(cc, hu, n_u);
     if (k.hi) {
-      process_hi<G>(stage, min(16, a.hi_cap - 16 * k.index), 16 * k.index, qb, a.sm_scale, logit_base,
+      process_hi<G, NB>(stage, min(16, a.hi_cap - 16 * k.index), 16 * k.index, qb, a.sm_scale, logit_base,
                     a.hi_stride, st, o, ob, lane);
     } else {
       const int first = k.index * U.blocks;
       const int nb = min(U.blocks, a.lo_blocks - first);
-      for (int b = 0; b < nb; ++b)
-        process_lo<BITS, GROUP, G>(stage, b, min(16, a.n_lo - 16 * (first + b)), qh, a.sm_scale, st, o, ob, lane);
+      int b = 0;
+      if (kLoPair)
+        for (; b + 1 < nb; b += 2)
+          process_lo<BITS, GROUP, G, NB, 2>(stage, b, a.n_lo - 16 * (first + b), qh, a.sm_scale, st, o, ob, lane);
+      for (; b < nb; ++b)
+        process_lo<BITS, GROUP, G, NB, 1>(stage, b, a.n_lo - 16 * (first + b), qh, a.sm_scale, st, o, ob, lane);
     }
     cursor_next(cc, hu, n_u);
     __syncwarp();
@@ -601,25 +715,32 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
       }
     return;
   }
-  if (cur >= 0) write_partial<GROUP, G>(a, wg + cur, st, o, ob, lane);
+  if (cur >= 0) write_partial<BITS, GROUP, G, NB>(a, wg + cur, st, o, ob, lane);
 }
 
+// Combination of the split partials: one warp per query head (4 heads per block), 4 channels per lane.
 template <int OUT_F32>
 __global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a, int G) {
-  const int bq = blockIdx.x;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int bq = blockIdx.x * 4 + warp;
+  if (bq >= a.batch * a.heads_q) return;
   const int b = bq / a.heads_q, hq = bq - b * a.heads_q;
   const int h = hq / G, jh = hq - h * G;
   const int bh = b * a.heads_kv + h;
-  const int c = threadIdx.x;
   const int w0 = owner_warp((long long)bh * a.n_u, a.n_units, a.n_warps);
   const int w1 = owner_warp((long long)(bh + 1) * a.n_u - 1, a.n_units, a.n_warps);
-  float r[1], M, L;
-  merge_head<1>(a.part_o, a.part_ml, G, bh, jh, w0, w1, c, r, M, L);
-  if (OUT_F32)
-    static_cast<float*>(a.out)[(size_t)bq * kHeadDim + c] = r[0];
-  else
-    static_cast<__nv_bfloat16*>(a.out)[(size_t)bq * kHeadDim + c] = __float2bfloat16_rn(r[0]);
-  if (c == 0 && a.ml) {
+  float r[4], M, L;
+  merge_head_warp(a.part_o, a.part_ml, G, bh, jh, w0, w1, lane, r, M, L);
+  if (OUT_F32) {
+    reinterpret_cast<float4*>(static_cast<float*>(a.out) + (size_t)bq * kHeadDim)[lane] = make_float4(r[0], r[1], r[2], r[3]);
+  } else {
+    __nv_bfloat162 v0 = __floats2bfloat162_rn(r[0], r[1]), v1 = __floats2bfloat162_rn(r[2], r[3]);
+    uint2 u;
+    u.x = *reinterpret_cast<uint32_t*>(&v0);
+    u.y = *reinterpret_cast<uint32_t*>(&v1);
+    reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(a.out) + (size_t)bq * kHeadDim)[lane] = u;
+  }
+  if (lane == 0 && a.ml) {
     a.ml[2 * bq] = M;
     a.ml[2 * bq + 1] = L;
   }
@@ -702,11 +823,11 @@ cudaError_t launch_attention(const AttnArgs& a, int bits, int group, int G, int 
 }
 
 cudaError_t launch_merge(const MergeArgs& a, int G, int out_f32, cudaStream_t st) {
-  const int grid = a.batch * a.heads_q;
+  const int grid = (a.batch * a.heads_q + 3) / 4;
   if (out_f32)
-    merge_kernel<1><<<grid, kHeadDim, 0, st>>>(a, G);
+    merge_kernel<1><<<grid, 128, 0, st>>>(a, G);
   else
-    merge_kernel<0><<<grid, kHeadDim, 0, st>>>(a, G);
+    merge_kernel<0><<<grid, 128, 0, st>>>(a, G);
   return cudaGetLastError();
 }
 

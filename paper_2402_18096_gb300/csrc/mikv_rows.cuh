@@ -90,29 +90,50 @@ __device__ __forceinline__ int owner_warp(long long U, long long n_units, int n_
   return w;
 }
 
-// Combine the split partials of query head jh of KV head bh (warps w0..w1 wrote slots w + bh):
-// returns (M, L) and the normalised output of channels c0..c0+NC-1.
-template <int NC>
-__device__ __forceinline__ void merge_head(const float* part_o, const float* part_ml, int G, int bh, int jh, int w0,
-                                           int w1, int c0, float (&out)[NC], float& M, float& L) {
+// One warp combines the split partials of query head jh of KV head bh (warps w0..w1 of the attention
+// kernel wrote slots w + bh): lane l returns the normalised output of channels 4l..4l+3, and every lane
+// returns (M, L) = (max logit, sum of exp(logit - M)). The per-slot statistics are read by all lanes at
+// once and broadcast with shuffles, so the merge costs a few dependent loads whatever the slot count.
+__device__ __forceinline__ void merge_head_warp(const float* part_o, const float* part_ml, int G, int bh, int jh,
+                                                int w0, int w1, int lane, float (&out)[4], float& M, float& L) {
   constexpr float kLog2e = 1.4426950408889634f;
+  const int n = w1 - w0 + 1;
   M = -INFINITY;
-  for (int w = w0; w <= w1; ++w) M = fmaxf(M, part_ml[((size_t)(w + bh) * G + jh) * 2]);
-  float O[NC];
-#pragma unroll
-  for (int i = 0; i < NC; ++i) O[i] = 0.f;
-  L = 0.f;
-  for (int w = w0; w <= w1; ++w) {
-    const size_t slot = (size_t)(w + bh);
-    const float ms = part_ml[(slot * G + jh) * 2];
-    if (ms == -INFINITY) continue;
-    const float wt = fast_exp2((ms - M) * kLog2e);
-    L += wt * part_ml[(slot * G + jh) * 2 + 1];
-#pragma unroll
-    for (int i = 0; i < NC; ++i) O[i] += wt * part_o[(slot * G + jh) * kHeadDim + c0 + i];
+  for (int c0 = 0; c0 < n; c0 += 32) {
+    const int i = c0 + lane;
+    if (i < n) M = fmaxf(M, part_ml[((size_t)(w0 + i + bh) * G + jh) * 2]);
   }
 #pragma unroll
-  for (int i = 0; i < NC; ++i) out[i] = O[i] / L;
+  for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+  float O[4] = {0.f, 0.f, 0.f, 0.f};
+  float Lp = 0.f;
+  for (int c0 = 0; c0 < n; c0 += 32) {
+    const int i = c0 + lane;
+    float wt = 0.f;
+    if (i < n) {
+      const size_t slot = (size_t)(w0 + i + bh);
+      const float ms = part_ml[(slot * G + jh) * 2];
+      if (ms != -INFINITY) {
+        wt = fast_exp2((ms - M) * kLog2e);
+        Lp += wt * part_ml[(slot * G + jh) * 2 + 1];
+      }
+    }
+    const int cnt = min(32, n - c0);
+    for (int k = 0; k < cnt; ++k) {
+      const float ws = __shfl_sync(0xffffffffu, wt, k);
+      const size_t slot = (size_t)(w0 + c0 + k + bh);
+      const float4 po = reinterpret_cast<const float4*>(part_o + (slot * G + jh) * kHeadDim)[lane];
+      O[0] += ws * po.x;
+      O[1] += ws * po.y;
+      O[2] += ws * po.z;
+      O[3] += ws * po.w;
+    }
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) Lp += __shfl_xor_sync(0xffffffffu, Lp, off);
+  L = Lp;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) out[i] = O[i] / L;
 }
 
 }  // namespace mikv

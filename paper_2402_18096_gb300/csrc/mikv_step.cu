@@ -34,7 +34,7 @@ __global__ void __launch_bounds__(kPostThreads) step_post_kernel(const StepPostA
     const int w0 = owner_warp((long long)bh * a.n_u, a.n_units, a.n_warps);
     const int w1 = owner_warp((long long)(bh + 1) * a.n_u - 1, a.n_units, a.n_warps);
     float r[4], M, L;
-    merge_head<4>(a.part_o, a.part_ml, G, bh, warp, w0, w1, 4 * lane, r, M, L);
+    merge_head_warp(a.part_o, a.part_ml, G, bh, warp, w0, w1, lane, r, M, L);
     const size_t bq = (size_t)b * a.heads_q + h * G + warp;
     if (OUT_F32) {
       reinterpret_cast<float4*>(static_cast<float*>(a.out) + bq * kHeadDim)[lane] = make_float4(r[0], r[1], r[2], r[3]);

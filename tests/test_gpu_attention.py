@@ -229,3 +229,38 @@ def test_full_size_layer_sampled_heads(wname, heads):
         else:  # only a near tie of fp32 scores may pick another slot
             a_sorted = np.sort(acc[0, 0])
             assert abs(a_sorted[1] - a_sorted[0]) < 1e-5 * max(1.0, abs(a_sorted[0]))
+
+
+@pytest.mark.parametrize("w", mi.sweep_workloads(), ids=lambda w: f"int{w.bits}-g{w.group}-r{int(w.ratio * 100)}")
+def test_sweep_points_one_step(w):
+    """Every point of the batch-64 sweep (bits x importance ratio x group) at batch 2: one whole decode
+    step (insert, attention, importance update, demotion) against the oracle on one sampled KV head."""
+    w = mi.scaled(w, batch=2, seed=w.bits * 100 + w.group + int(w.ratio * 1000))
+    raw = raw_inputs(w)
+    layer = gpu_layer(w, raw, steps=2)
+    b, h = 1, (w.bits * 7 + w.group) % w.heads_kv
+    ref = oracle_layer(w, raw, layer.shape.lo_cap, heads=[(b, h)])[0]
+    c = ref["cache"]
+    q, k_new, v_new = mi.decode_inputs(w, 0, 0)
+    dev = torch.device("cuda")
+    out = torch.empty(w.batch, w.heads_q, w.head_dim, dtype=torch.float32, device=dev)
+    n_lo = layer.n_lo
+    layer.step(q.to(dev), k_new.to(dev), v_new.to(dev), out)
+    pkg.mikv_workspace_check(layer.ws)
+    oracle.insert_token(c, bits16(k_new[b:b + 1, h:h + 1]), bits16(v_new[b:b + 1, h:h + 1]), w.context,
+                        np.array([[w.budget]], np.int32))
+    ref_o, hl, ml = oracle.decode_attention(c, bits16(q[b:b + 1, h:h + 1]), n_lo, sm_scale(), balancer_=ref["balancer"])
+    vmax = max(float(raw[1][b, h].float().abs().max()), float(v_new[b, h].float().abs().max()))
+    err = np.abs(out[b, h:h + 1].cpu().numpy() - ref_o[0])
+    assert np.all(err <= 2e-3 * vmax), err.max()
+    acc = oracle.update_importance(c["acc"], hl.astype(np.float32), ml.astype(np.float32), 1)
+    dem, _ = oracle.select_demote(acc, 1, c["hi_tok"], want_kept=False)
+    victim = int(layer.slots[b, h])
+    if victim == int(dem[0, 0, 0]):
+        oracle.quantize_pack(c, c["k_hi"], c["v_hi"], dem, n_lo, src_tok=c["hi_tok"], balancer_=ref["balancer"])
+        np.testing.assert_array_equal(layer.cache.k_codes[b, h, n_lo].cpu().numpy(), c["k_codes"][0, 0, n_lo])
+        np.testing.assert_array_equal(layer.cache.k_params[b, h, n_lo].cpu().view(torch.int16).numpy().view(np.uint16),
+                                      c["k_params"][0, 0, n_lo])
+    else:
+        a_sorted = np.sort(acc[0, 0])
+        assert abs(a_sorted[1] - a_sorted[0]) < 1e-5 * max(1.0, abs(a_sorted[0]))
