@@ -158,39 +158,27 @@ mikv_status attention_impl(const mikv_shape* s, const mikv_cache* c, int32_t n_l
   memset(&a, 0, sizeof a);
   const uint64_t hi_rows = (uint64_t)s->batch * s->heads_kv * s->hi_stride;
   const uint64_t lo_rows = (uint64_t)s->batch * s->heads_kv * s->lo_cap;
-  const uint64_t row_bytes = 16ull * s->bits;
   bool ok = make_map(&a.map_k_hi, c->k_hi, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, kHeadDim, hi_rows, 2 * kHeadDim, 64,
                      16, CU_TENSOR_MAP_SWIZZLE_128B) &&
             make_map(&a.map_v_hi, c->v_hi, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, kHeadDim, hi_rows, 2 * kHeadDim, 64,
                      16, CU_TENSOR_MAP_SWIZZLE_128B);
   if (ok && lo_rows > 0) {
-    // retained arrays: one box covers a whole unit of U.blocks blocks of 16 rows
+    // retained arrays: each is viewed as rows of U.map_w (codes) or U.param_w (alpha, beta) bytes, and
+    // one box covers a whole unit of 16 * U.blocks tokens (lo_cap % 16 == 0 keeps units row-aligned)
     const LoUnit U = lo_unit_layout(s->bits, s->group);
-    const uint32_t box_rows = 16u * U.blocks;
-    if (s->bits == 3) {
-      ok = make_map(&a.map_k_lo, c->k_codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, row_bytes, lo_rows, row_bytes, 32,
-                    box_rows, CU_TENSOR_MAP_SWIZZLE_32B) &&
-           make_map(&a.map_v_lo, c->v_codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, row_bytes, lo_rows, row_bytes, 32,
-                    box_rows, CU_TENSOR_MAP_SWIZZLE_32B) &&
-           make_map(&a.map_k_lo1, c->k_codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, row_bytes, lo_rows, row_bytes, 16,
-                    box_rows, CU_TENSOR_MAP_SWIZZLE_NONE) &&
-           make_map(&a.map_v_lo1, c->v_codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, row_bytes, lo_rows, row_bytes, 16,
-                    box_rows, CU_TENSOR_MAP_SWIZZLE_NONE);
-    } else {
-      const CUtensorMapSwizzle swz = s->bits == 2 ? CU_TENSOR_MAP_SWIZZLE_32B : CU_TENSOR_MAP_SWIZZLE_64B;
-      ok = make_map(&a.map_k_lo, c->k_codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, row_bytes, lo_rows, row_bytes,
-                    (uint32_t)row_bytes, box_rows, swz) &&
-           make_map(&a.map_v_lo, c->v_codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, row_bytes, lo_rows, row_bytes,
-                    (uint32_t)row_bytes, box_rows, swz);
-    }
-    // (alpha, beta) pairs viewed as rows of 16 bytes: U.param_row / 16 rows per token
-    const uint64_t par_rows = lo_rows * (uint64_t)U.param_row / 16;
-    const uint32_t par_box = box_rows * U.param_row / 16;
-    ok = ok &&
-         make_map(&a.map_k_par, c->k_params, CU_TENSOR_MAP_DATA_TYPE_UINT8, 16, par_rows, 16, 16, par_box,
-                  CU_TENSOR_MAP_SWIZZLE_NONE) &&
-         make_map(&a.map_v_par, c->v_params, CU_TENSOR_MAP_DATA_TYPE_UINT8, 16, par_rows, 16, 16, par_box,
-                  CU_TENSOR_MAP_SWIZZLE_NONE);
+    const uint64_t code_rows = lo_rows * U.pitch / U.map_w;
+    const uint32_t code_box = 16u * U.blocks * U.pitch / U.map_w;
+    const CUtensorMapSwizzle swz = s->bits == 3 ? CU_TENSOR_MAP_SWIZZLE_NONE : CU_TENSOR_MAP_SWIZZLE_64B;
+    const uint64_t par_rows = lo_rows * U.param_row / U.param_w;
+    const uint32_t par_box = 16u * U.blocks * U.param_row / U.param_w;
+    ok = make_map(&a.map_k_lo, c->k_codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, U.map_w, code_rows, U.map_w, U.map_w,
+                  code_box, swz) &&
+         make_map(&a.map_v_lo, c->v_codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, U.map_w, code_rows, U.map_w, U.map_w,
+                  code_box, swz) &&
+         make_map(&a.map_k_par, c->k_params, CU_TENSOR_MAP_DATA_TYPE_UINT8, U.param_w, par_rows, U.param_w,
+                  U.param_w, par_box, CU_TENSOR_MAP_SWIZZLE_NONE) &&
+         make_map(&a.map_v_par, c->v_params, CU_TENSOR_MAP_DATA_TYPE_UINT8, U.param_w, par_rows, U.param_w,
+                  U.param_w, par_box, CU_TENSOR_MAP_SWIZZLE_NONE);
   }
   if (!ok) return MIKV_ERR_CUDA;
   a.q = q;

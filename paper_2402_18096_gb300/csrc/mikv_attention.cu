@@ -248,12 +248,16 @@ __device__ __forceinline__ uint32_t code3(uint32_t r, uint32_t h, int j, int hb)
 // carry M * sum(p * alpha) per channel on top of the wanted sum; that term is measured by a ones-row
 // MMA on the same fp16 operands and removed in write_partial. M stays small (<= 64) so the removal
 // costs only a few bits of the fp32 accumulator.
-// N = 2: code j of r sits at bits 2j of each unit. Four shifted copies (r << 6, r << 2, r >> 2, r >> 6)
-// bring codes 2i and 2i + 1 to bits 6..7 (M = 16) and 8..9 (M = 4).
-__device__ __forceinline__ uint32_t vcode2(const uint32_t (&sh)[4], int j) {
-  return (j & 1) ? and_or(sh[j >> 1], 0x03000300u, 0x44004400u) : and_or(sh[j >> 1], 0x00C000C0u, 0x4C004C00u);
+// N = 2: code j of r sits at bits 2j of each unit. Codes 0..2 are read from r << 4 (bits 4, 6, 8), codes
+// 3, 4 from r itself (bits 6, 8), codes 5..7 from r >> 6 (bits 4, 6, 8): offsets 64, 16, 4, 16, 4, 64, 16, 4.
+__device__ __forceinline__ uint32_t vcode2(uint32_t rl4, uint32_t r, uint32_t rr6, int j) {
+  const uint32_t src = j < 3 ? rl4 : (j < 5 ? r : rr6);
+  const int pos = j < 3 ? j + 2 : (j < 5 ? j : j - 3);  // 2-bit field index of the code in src
+  return and_or(src, 0x00030003u << (2 * pos), mag2(pos));
 }
-__host__ __device__ constexpr float voff2(int j) { return (j & 1) ? 4.f : 16.f; }
+__host__ __device__ constexpr float voff2(int j) {
+  return (j == 0 || j == 5) ? 64.f : (j == 2 || j == 4 || j == 7) ? 4.f : 16.f;
+}
 // N = 4: nibble p of r at bits 4p. Nibbles 0 and 1 are read at bits 4..7 of r << 4 and r (M = 64),
 // nibbles 2 and 3 at bits 6..9 of r >> 2 and r >> 6 (M = 16).
 __device__ __forceinline__ uint32_t vcode4(const uint32_t (&sh)[4], int p) {
@@ -322,7 +326,7 @@ __device__ __forceinline__ void lo_logits(uint32_t unit, int b, int valid, const
   constexpr int NG = kHeadDim / GROUP;
   constexpr int PR = U.param_row;
   // this block's rows inside the unit's sections
-  const uint32_t ka = unit + U.k_a + b * 16 * U.plane_a_bytes, kb = unit + U.k_b + b * 16 * U.plane_b_bytes;
+  const uint32_t ka = unit + U.k_a + b * 16 * U.pitch;
   const uint32_t kp = unit + U.k_p + b * 16 * PR;
   constexpr int NR = BITS == 4 ? 8 : 4;
   const int g = lane >> 2, t = lane & 3, r8 = lane & 7, j = lane >> 3;
@@ -343,12 +347,13 @@ __device__ __forceinline__ void lo_logits(uint32_t unit, int b, int valid, const
         kr[(NR == 8 ? 4 : 0) + i] = r1[i];
       }
     } else {
-      const int o0 = tok * 32 + 16 * (j >> 1), sw = ((tok >> 2) & 1) << 4;
+      // N = 2: 32-byte tokens under the 64B swizzle (bits 4..5 ^= bits 7..8); N = 3: 48-byte tokens, unswizzled
+      const int o0 = tok * U.pitch + 16 * (j >> 1), sw = BITS == 2 ? ((tok >> 2) & 3) << 4 : 0;
       uint32_t r0[4];
       ldsm_x4(ka + (o0 ^ sw), r0);
 #pragma unroll
       for (int i = 0; i < 4; ++i) kr[i] = r0[i];
-      if (BITS == 3) ldsm_x2(kb + (lane & 15) * 16, kb0, kb1);
+      if (BITS == 3) ldsm_x2(ka + (lane & 15) * U.pitch + U.plane_b, kb0, kb1);
     }
 #pragma unroll
     for (int i = 0; i < NR; ++i) kh[i] = kr[i] >> (BITS == 4 ? 8 : 10);
@@ -362,8 +367,10 @@ __device__ __forceinline__ void lo_logits(uint32_t unit, int b, int valid, const
 #pragma unroll
   for (int ks = 0; ks < 8; ++ks) {
     const int gi = (16 * ks) / GROUP;
-    const uint32_t al0 = prmt(pk0[gi], pk0[gi], 0x1010u), be0 = prmt(pk0[gi], pk0[gi], 0x3232u);
-    const uint32_t al1 = prmt(pk1[gi], pk1[gi], 0x1010u), be1 = prmt(pk1[gi], pk1[gi], 0x3232u);
+    // (alpha, alpha) and (beta, beta) of tokens g and g + 8: half-broadcasts the HFMA2 operand selectors absorb
+    const __half2 p0 = u32_as_h2(pk0[gi]), p1 = u32_as_h2(pk1[gi]);
+    const uint32_t al0 = h2_as_u32(__low2half2(p0)), be0 = h2_as_u32(__high2half2(p0));
+    const uint32_t al1 = h2_as_u32(__low2half2(p1)), be1 = h2_as_u32(__high2half2(p1));
     uint32_t c[4];
     if (BITS == 4) {
       const int ri = (ks >> 2) * 4, p = ks & 3;
@@ -396,7 +403,7 @@ __device__ __forceinline__ void lo_values(uint32_t unit, int b, int valid, const
   constexpr LoUnit U = lo_unit_layout(BITS, GROUP);
   constexpr int NG = kHeadDim / GROUP;
   constexpr int PR = U.param_row;
-  const uint32_t va = unit + U.v_a + b * 16 * U.plane_a_bytes, vb = unit + U.v_b + b * 16 * U.plane_b_bytes;
+  const uint32_t va = unit + U.v_a + b * 16 * U.pitch;
   const uint32_t vp = unit + U.v_p + b * 16 * PR;
   constexpr int NR = BITS == 4 ? 8 : 4;
   const int g = lane >> 2, t = lane & 3, r8 = lane & 7, j = lane >> 3;
@@ -419,12 +426,12 @@ __device__ __forceinline__ void lo_values(uint32_t unit, int b, int valid, const
         vr[(NR == 8 ? 4 : 0) + i] = r1[i];
       }
     } else {
-      const int o0 = tok * 32 + 16 * (j & 1), sw = ((tok >> 2) & 1) << 4;
+      const int o0 = tok * U.pitch + 16 * (j & 1), sw = BITS == 2 ? ((tok >> 2) & 3) << 4 : 0;
       uint32_t r0[4];
       ldsm_x4_t(va + (o0 ^ sw), r0);
 #pragma unroll
       for (int i = 0; i < 4; ++i) vr[i] = r0[i];
-      if (BITS == 3) ldsm_x2_t(vb + (lane & 15) * 16, vb0, vb1);
+      if (BITS == 3) ldsm_x2_t(va + (lane & 15) * U.pitch + U.plane_b, vb0, vb1);
     }
   }
   // (alpha, beta) of the four tokens for every group; zero past the end (exact zeros in the sums)
@@ -491,8 +498,7 @@ __device__ __forceinline__ void lo_values(uint32_t unit, int b, int valid, const
     } else if (BITS == 2) {
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
-        const uint32_t c2[4] = {vr[i] << 6, vr[i] << 2, vr[i] >> 2, vr[i] >> 6};  // shared by all mt
-        a[i] = vcode2(c2, mt);
+        a[i] = vcode2(vr[i] << 4, vr[i], vr[i] >> 6, mt);  // the shifted copies are shared by all mt
       }
     } else {
       a[0] = code3(vr[0], vb0, mt, mt);
@@ -580,15 +586,11 @@ __device__ __forceinline__ void issue_unit(const AttnArgs& a, const Cursor& c, u
   } else {
     // one box per array covers the whole unit (U.blocks blocks of 16 rows); rows past this head's
     // retained length are masked by the consumer, rows past the array are zero-filled by TMA
-    const int row = c.bh * a.lo_cap + 16 * U.blocks * k.index;
+    const long long row = (long long)c.bh * a.lo_cap + 16 * U.blocks * k.index;  // first token row
     mbar_arrive_expect_tx(bar, U.tx);
-    tma_load_2d(dst + U.k_a, &a.map_k_lo, 0, row, bar);
-    tma_load_2d(dst + U.v_a, &a.map_v_lo, 0, row, bar);
-    if (BITS == 3) {
-      tma_load_2d(dst + U.k_b, &a.map_k_lo1, 32, row, bar);
-      tma_load_2d(dst + U.v_b, &a.map_v_lo1, 32, row, bar);
-    }
-    const int prow = row * U.param_row / 16;
+    const int crow = (int)(row * U.pitch / U.map_w), prow = (int)(row * U.param_row / U.param_w);
+    tma_load_2d(dst + U.k_a, &a.map_k_lo, 0, crow, bar);
+    tma_load_2d(dst + U.v_a, &a.map_v_lo, 0, crow, bar);
     tma_load_2d(dst + U.k_p, &a.map_k_par, 0, prow, bar);
     tma_load_2d(dst + U.v_p, &a.map_v_par, 0, prow, bar);
   }

@@ -17,34 +17,40 @@ namespace mikv {
 // swizzle needs (256 B for 32-byte swizzle, 512 B for 64-byte swizzle, 128 B otherwise).
 struct LoUnit {
   int blocks;
-  int row_bytes, plane_a_bytes, plane_b_bytes;  // per token: codes, and the two planes (N = 3)
-  int param_row;                                 // bytes of (alpha, beta) pairs per token
-  int k_a, k_b, v_a, v_b, k_p, v_p;              // section offsets (k_b, v_b only for N = 3)
-  int total;                                     // bytes used
-  int tx;                                        // bytes the TMA boxes deliver
+  int pitch;      // bytes of codes per token (both planes for N = 3), in HBM and in the stage
+  int plane_b;    // N = 3: offset of the 1-bit plane inside a token's codes
+  int map_w;      // the code arrays are copied as rows of map_w bytes (several tokens per row)
+  int param_row;  // bytes of (alpha, beta) pairs per token
+  int param_w;    // the parameter arrays are copied as rows of param_w bytes
+  int k_a, v_a, k_p, v_p;  // section offsets in the stage
+  int total;               // bytes used
+  int tx;                  // bytes the TMA boxes deliver
 };
 
 constexpr int kUnitBytes = 8192;
 
 __host__ __device__ constexpr int align_up(int x, int a) { return (x + a - 1) / a * a; }
 
+// A unit's rows of one array are contiguous in HBM (16 n tokens of one head), so TMA copies them as
+// wide rows: 64-byte rows with the 64B swizzle for N = 2 (two tokens per row) and N = 4 (one token),
+// unswizzled 128-byte rows for N = 3 (48-byte tokens, whose pitch alone spreads ldmatrix rows over all
+// banks). Few wide rows per unit keep the TMA request rate far below what HBM needs.
 __host__ __device__ constexpr LoUnit lo_unit_layout_n(int bits, int group, int n) {
   LoUnit u{};
   u.blocks = n;
-  u.row_bytes = 16 * bits;
-  u.plane_a_bytes = bits == 3 ? 32 : 16 * bits;
-  u.plane_b_bytes = bits == 3 ? 16 : 0;
+  u.pitch = bits == 3 ? 48 : 16 * bits;
+  u.plane_b = bits == 3 ? 32 : 0;
+  u.map_w = bits == 3 ? 128 : 64;
   u.param_row = 4 * (128 / group);
+  u.param_w = u.param_row == 4 ? 64 : 128;
   const int rows = 16 * n;
-  const int code_align = bits == 4 ? 512 : 256;
+  const int code_align = bits == 3 ? 128 : 512;  // the 64B swizzle pattern repeats every 512 bytes
   u.k_a = 0;
-  u.k_b = align_up(u.k_a + rows * u.plane_a_bytes, 128);
-  u.v_a = align_up(u.k_b + rows * u.plane_b_bytes, code_align);
-  u.v_b = align_up(u.v_a + rows * u.plane_a_bytes, 128);
-  u.k_p = align_up(u.v_b + rows * u.plane_b_bytes, 128);
+  u.v_a = align_up(u.k_a + rows * u.pitch, code_align);
+  u.k_p = align_up(u.v_a + rows * u.pitch, 128);
   u.v_p = align_up(u.k_p + rows * u.param_row, 128);
   u.total = u.v_p + rows * u.param_row;
-  u.tx = 2 * rows * (u.plane_a_bytes + u.plane_b_bytes) + 2 * rows * u.param_row;
+  u.tx = 2 * rows * u.pitch + 2 * rows * u.param_row;
   return u;
 }
 
@@ -68,9 +74,8 @@ struct AttnPlan {
 
 struct AttnArgs {
   CUtensorMap map_k_hi, map_v_hi;    // bf16 rows of 128 channels, box 64 x 16, 128B swizzle
-  CUtensorMap map_k_lo, map_v_lo;    // packed codes (bits 0..1 plane for N = 3), box plane x 16 blocks
-  CUtensorMap map_k_lo1, map_v_lo1;  // N = 3 only: 1-bit plane
-  CUtensorMap map_k_par, map_v_par;  // (alpha, beta) pairs viewed as 16-byte rows
+  CUtensorMap map_k_lo, map_v_lo;    // packed codes viewed as rows of LoUnit::map_w bytes, box = one unit
+  CUtensorMap map_k_par, map_v_par;  // (alpha, beta) pairs viewed as rows of LoUnit::param_w bytes
   const void* q;
   const float* balancer;
   float* hi_logits;

@@ -31,6 +31,10 @@ CASES = {
     "one-token": mi.Workload("t1", 1, 4, 4, 1, 1, 3, 32, 0.2, seed=6),
     "exact-16": mi.Workload("x16", 1, 4, 1, 160, 1, 4, 32, 0.09375, seed=7),  # hi_cap = 16
 }
+# every retained layout (bits x group): ragged lengths, several units per head
+for _b in (2, 3, 4):
+    for _g in (32, 64, 128):
+        CASES[f"layout-int{_b}-g{_g}"] = mi.Workload(f"l{_b}{_g}", 1, 4, 2, 611, 1, _b, _g, 0.15, seed=10 * _b + _g)
 
 
 def _check_cache(layer, refs, w):
