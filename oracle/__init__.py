@@ -15,6 +15,8 @@ Functions follow the paper:
   * ``update_importance`` / ``select_demote``: accumulated-attention (heavy-hitter) importance policy
     that decides which tokens stay in high precision (Fig. 4, Sec. 3).
   * ``cache_fraction``: the "Cache size" columns of Tables 2-3.
+  * caches with ``hi_bits < 16``: the reduced-precision important set of Sec. 3.3 / Table 3
+    (important rows quantized like retained rows; demotion re-quantizes their dequantized values).
 
 Readings where the paper is silent are documented in ``mikv_oracle.c`` next to the code.
 """
@@ -71,6 +73,12 @@ def _load():
                 "mikv_ref_insert_token": (I, [I, I, I, I, P, P, I, P, P, P, P, P]),
                 "mikv_ref_gather_hi": (I, [I, I, I, I, P, P, P, P, I, P, I, P, P, P, P]),
                 "mikv_ref_cache_fraction": (D, [I, I, D, I]),
+                "mikv_ref_dequantize_row_f32": (I, [P, P, I, I, I, P]),
+                "mikv_ref_gather_hi_q": (I, [I, I, I, I, I, I, P, P, P, P, I, P, I, P, P, P, P, P, P, P]),
+                "mikv_ref_insert_token_q": (I, [I, I, I, I, I, I, P, P, I, P, P, P, P, P, P, P, P]),
+                "mikv_ref_decode_attention_q": (I, [I, I, I, I, I, I, I, I, I, I, I, P, P, P, P, P, P, P, P,
+                                                    P, P, D, P, P, P]),
+                "mikv_ref_demote_hi_q": (I, [I, I, I, I, I, I, I, I, I, P, I, P, P, P, P, P, P, P, P, P, P]),
             }
             for name, (res, args) in sig.items():
                 fn = getattr(lib, name)
@@ -197,6 +205,8 @@ def decode_attention(cache: dict, q, n_lo: int, sm_scale: float, balancer_=None)
     cache: numpy dict with k_hi, v_hi (uint16 [B, Hkv, hi_cap, d]), k_codes, v_codes
     (uint8 [B, Hkv, lo_cap, 16*bits]), k_params, v_params (uint16 [B, Hkv, lo_cap, d/g, 2]).
     q: uint16 bf16 bits [B, Hq, d]."""
+    if cache.get("hi_bits", 16) < 16:
+        return _decode_attention_q(cache, q, n_lo, sm_scale, balancer_)
     q = _arr(q, np.uint16)
     B, Hq, d = q.shape
     k_hi = _arr(cache["k_hi"], np.uint16)
@@ -215,6 +225,29 @@ def decode_attention(cache: dict, q, n_lo: int, sm_scale: float, balancer_=None)
     _check(_load().mikv_ref_decode_attention(
         B, Hq, Hkv, d, bits, g, hi_cap, lo_cap, n_lo, _p(k_hi), _p(v_hi), _p(kc), _p(vc), _p(kp),
         _p(vp), _p(bal), _p(q), float(sm_scale), _p(out), _p(hl), _p(ml)), "decode_attention")
+    return out, hl, ml
+
+
+def _decode_attention_q(cache: dict, q, n_lo: int, sm_scale: float, balancer_=None):
+    q = _arr(q, np.uint16)
+    B, Hq, d = q.shape
+    hb, hg = cache["hi_bits"], cache["hi_group"]
+    khc, vhc = _arr(cache["k_hi"], np.uint8), _arr(cache["v_hi"], np.uint8)
+    khp, vhp = _arr(cache["k_hp"], np.uint16), _arr(cache["v_hp"], np.uint16)
+    Hkv, hi_cap = khc.shape[1], khc.shape[2]
+    kc = _arr(cache["k_codes"], np.uint8)
+    vc = _arr(cache["v_codes"], np.uint8)
+    kp = _arr(cache["k_params"], np.uint16)
+    vp = _arr(cache["v_params"], np.uint16)
+    lo_cap, bits = kc.shape[2], kc.shape[3] // 16
+    g = d // kp.shape[3]
+    bal = _arr(balancer_, np.float32)
+    out = np.zeros((B, Hq, d), np.float64)
+    hl = np.zeros((B, Hq, hi_cap), np.float64)
+    ml = np.zeros((B, Hq, 2), np.float64)
+    _check(_load().mikv_ref_decode_attention_q(
+        B, Hq, Hkv, d, hb, hg, bits, g, hi_cap, lo_cap, n_lo, _p(khc), _p(vhc), _p(khp), _p(vhp), _p(kc),
+        _p(vc), _p(kp), _p(vp), _p(bal), _p(q), float(sm_scale), _p(out), _p(hl), _p(ml)), "decode_attention_q")
     return out, hl, ml
 
 
@@ -242,37 +275,98 @@ def select_demote(scores, n_demote: int, ids=None, want_kept: bool = True):
     return dem, kept
 
 
-def insert_token(cache: dict, k_new, v_new, tok: int, slots):
-    """Write the new token (uint16 [B, Hkv, d]) into slot ``slots[b, h]`` of the important set."""
+def insert_token(cache: dict, k_new, v_new, tok: int, slots, balancer_=None):
+    """Write the new token (uint16 [B, Hkv, d]) into slot ``slots[b, h]`` of the important set (quantized,
+    keys balanced, when the cache's important set is reduced-precision)."""
     k_new = _arr(k_new, np.uint16)
     v_new = _arr(v_new, np.uint16)
     slots = _arr(slots, np.int32)
+    if cache.get("hi_bits", 16) < 16:
+        B, Hkv, hi_cap = cache["hi_tok"].shape
+        d = k_new.shape[2]
+        _check(_load().mikv_ref_insert_token_q(
+            B, Hkv, d, hi_cap, cache["hi_bits"], cache["hi_group"], _p(k_new), _p(v_new), tok, _p(slots),
+            _p(_arr(balancer_, np.float32)), _p(cache["k_hi"]), _p(cache["v_hi"]), _p(cache["k_hp"]),
+            _p(cache["v_hp"]), _p(cache["hi_tok"]), _p(cache["acc"])), "insert_token_q")
+        return
     B, Hkv, hi_cap, d = cache["k_hi"].shape
     _check(_load().mikv_ref_insert_token(B, Hkv, d, hi_cap, _p(k_new), _p(v_new), tok, _p(slots),
                                          _p(cache["k_hi"]), _p(cache["v_hi"]), _p(cache["hi_tok"]),
                                          _p(cache["acc"])), "insert_token")
 
 
-def gather_hi(cache: dict, k_src, v_src, rows, src_tok=None, src_scores=None):
+def gather_hi(cache: dict, k_src, v_src, rows, src_tok=None, src_scores=None, balancer_=None):
+    """Important-set build: slot i of (b, h) receives source row rows[b, h, i] (quantized, keys balanced,
+    for a reduced-precision important set)."""
     k_src = _arr(k_src, np.uint16)
     v_src = _arr(v_src, np.uint16)
     rows = _arr(rows, np.int32)
     src_tok = _arr(src_tok, np.int32)
     src_scores = _arr(src_scores, np.float32)
     B, Hkv, n_src, d = k_src.shape
-    hi_cap = cache["k_hi"].shape[2]
+    hi_cap = cache["hi_tok"].shape[2]
+    if cache.get("hi_bits", 16) < 16:
+        _check(_load().mikv_ref_gather_hi_q(
+            B, Hkv, d, hi_cap, cache["hi_bits"], cache["hi_group"], _p(k_src), _p(v_src), _p(src_tok),
+            _p(src_scores), n_src, _p(rows), rows.shape[2], _p(_arr(balancer_, np.float32)), _p(cache["k_hi"]),
+            _p(cache["v_hi"]), _p(cache["k_hp"]), _p(cache["v_hp"]), _p(cache["hi_tok"]), _p(cache["acc"])),
+            "gather_hi_q")
+        return
     _check(_load().mikv_ref_gather_hi(B, Hkv, d, hi_cap, _p(k_src), _p(v_src), _p(src_tok),
                                       _p(src_scores), n_src, _p(rows), rows.shape[2],
                                       _p(cache["k_hi"]), _p(cache["v_hi"]), _p(cache["hi_tok"]),
                                       _p(cache["acc"])), "gather_hi")
 
 
+def demote_hi(cache: dict, slots, lo_pos: int, balancer_=None):
+    """Move important slot ``slots[b, h]`` into retained position ``lo_pos`` (Eq. 1 at the retained
+    precision; a bf16 important row gets the balancer on its key first, a reduced-precision one is
+    re-quantized from its fp32 dequantized values)."""
+    slots = _arr(slots, np.int32)
+    B, Hkv, hi_cap = cache["hi_tok"].shape
+    if cache.get("hi_bits", 16) >= 16:
+        quantize_pack(cache, cache["k_hi"], cache["v_hi"], slots.reshape(B, Hkv, 1), lo_pos, src_tok=cache["hi_tok"],
+                      balancer_=balancer_)
+        return
+    kc = cache["k_codes"]
+    d = cache["k_hp"].shape[3] * cache["hi_group"]
+    lo_cap, bits = kc.shape[2], kc.shape[3] // 16
+    g = d // cache["k_params"].shape[3]
+    _check(_load().mikv_ref_demote_hi_q(
+        B, Hkv, d, hi_cap, cache["hi_bits"], cache["hi_group"], bits, g, lo_cap, _p(slots), lo_pos,
+        _p(cache["k_hi"]), _p(cache["v_hi"]), _p(cache["k_hp"]), _p(cache["v_hp"]), _p(cache["hi_tok"]),
+        _p(cache["k_codes"]), _p(cache["v_codes"]), _p(cache["k_params"]), _p(cache["v_params"]),
+        _p(cache["lo_tok"])), "demote_hi_q")
+
+
+def dequantize_row_f32(packed, params, bits: int, g: int, d: int = 128):
+    """fp32 dequantization alpha16 * code + beta16 (exact product, one rounding) -> float32 [d]."""
+    packed = _arr(packed, np.uint8)
+    params = _arr(params, np.uint16)
+    out = np.zeros(d, np.float32)
+    _check(_load().mikv_ref_dequantize_row_f32(_p(packed), _p(params), d, bits, g, _p(out)), "dequantize_row_f32")
+    return out
+
+
 def cache_fraction(bits: int, g: int, ratio: float, hi_bits: int = 16) -> float:
     return float(_load().mikv_ref_cache_fraction(bits, g, ratio, hi_bits))
 
 
-def empty_cache(B: int, Hkv: int, d: int, bits: int, g: int, hi_cap: int, lo_cap: int) -> dict:
-    """Zero-initialised numpy arrays in the oracle's (dense) layout."""
+def empty_cache(B: int, Hkv: int, d: int, bits: int, g: int, hi_cap: int, lo_cap: int, hi_bits: int = 16,
+                hi_group: int = 64) -> dict:
+    """Zero-initialised numpy arrays in the oracle's (dense) layout. With hi_bits < 16 the important set
+    holds codes (k_hi, v_hi uint8 [B, Hkv, hi_cap, d*hi_bits/8]) and parameters (k_hp, v_hp)."""
+    if hi_bits < 16:
+        c = empty_cache(B, Hkv, d, bits, g, hi_cap, lo_cap)
+        c.update({
+            "hi_bits": hi_bits,
+            "hi_group": hi_group,
+            "k_hi": np.zeros((B, Hkv, hi_cap, d * hi_bits // 8), np.uint8),
+            "v_hi": np.zeros((B, Hkv, hi_cap, d * hi_bits // 8), np.uint8),
+            "k_hp": np.zeros((B, Hkv, hi_cap, d // hi_group, 2), np.uint16),
+            "v_hp": np.zeros((B, Hkv, hi_cap, d // hi_group, 2), np.uint16),
+        })
+        return c
     return {
         "k_hi": np.zeros((B, Hkv, hi_cap, d), np.uint16),
         "v_hi": np.zeros((B, Hkv, hi_cap, d), np.uint16),

@@ -452,6 +452,191 @@ int mikv_ref_gather_hi(int B, int Hkv, int d, int hi_cap, const uint16_t* k_src,
   return 0;
 }
 
+/* ---------------------------------------------------------------- reduced-precision important set */
+
+/*
+ * Sec. 3.3 / Table 3 ("Reducing the Precision of the Importance Cache"): the important rows may
+ * themselves be stored as hi_bits-bit codes with fp16 (alpha, beta) per group of hg channels.
+ * Readings (the paper only reports the resulting sizes and accuracies):
+ *  - the important set is quantized with the same quantizer as the retained set (Eq. 1), keys
+ *    multiplied by the balancer first (Eq. 3) and attended with q / balancer (Eq. 4);
+ *  - a new token enters the important set already quantized (its full-precision row is not kept);
+ *  - a demoted important row is re-quantized from its dequantized values: per channel the fp32 value
+ *    alpha16 * c + beta16 (the product is exact in fp32, the sum rounded once), then Eq. 1 at the
+ *    retained precision. Keys are already balanced and are not multiplied by the balancer again.
+ * Arrays: k_hc, v_hc uint8 [B][Hkv][hi_cap][d * hi_bits / 8]; k_hp, v_hp fp16 [B][Hkv][hi_cap][d/hg][2].
+ */
+static void quantize_kv_row(const uint16_t* krow, const uint16_t* vrow, int d, int h, int bits, int g,
+                            const float* balancer, float* x, uint8_t* kc, uint16_t* kp, uint8_t* vc,
+                            uint16_t* vp) {
+  for (int c = 0; c < d; ++c) /* Eq. 3 */
+    x[c] = bf16_to_f32(krow[c]) * (balancer ? balancer[(size_t)h * d + c] : 1.0f);
+  mikv_ref_quantize_row(x, d, bits, g, kc, kp);
+  for (int c = 0; c < d; ++c) x[c] = bf16_to_f32(vrow[c]);
+  mikv_ref_quantize_row(x, d, bits, g, vc, vp);
+}
+
+static int hi_args_ok(int d, int hi_bits, int hg) {
+  return valid_bits(hi_bits) && hg > 0 && d == 128 && d % hg == 0;
+}
+
+int mikv_ref_dequantize_row_f32(const uint8_t* packed, const uint16_t* params, int d, int bits, int g,
+                                float* x) {
+  if (!valid_bits(bits) || g <= 0 || d % g || d != 128) return -1;
+  int32_t* codes = (int32_t*)malloc(sizeof(int32_t) * (size_t)d);
+  if (!codes) return -1;
+  mikv_ref_unpack_row(packed, d, bits, codes);
+  for (int i = 0; i < d; ++i) {
+    float alpha = (float)mikv_ref_f16_to_f64(params[2 * (i / g)]);
+    float beta = (float)mikv_ref_f16_to_f64(params[2 * (i / g) + 1]);
+    float prod = alpha * (float)codes[i]; /* exact: 11-bit alpha times an 8-bit code */
+    x[i] = prod + beta;                   /* one rounding */
+  }
+  free(codes);
+  return 0;
+}
+
+int mikv_ref_gather_hi_q(int B, int Hkv, int d, int hi_cap, int hi_bits, int hg, const uint16_t* k_src,
+                         const uint16_t* v_src, const int32_t* src_tok, const float* src_scores, int n_src,
+                         const int32_t* rows, int n_rows, const float* balancer, uint8_t* k_hc, uint8_t* v_hc,
+                         uint16_t* k_hp, uint16_t* v_hp, int32_t* hi_tok, float* acc) {
+  if (!hi_args_ok(d, hi_bits, hg) || n_rows > hi_cap || n_rows < 0) return -1;
+  size_t rb = (size_t)d * hi_bits / 8, np = (size_t)(d / hg) * 2;
+  float* x = (float*)malloc(sizeof(float) * (size_t)d);
+  if (!x) return -1;
+  for (int b = 0; b < B; ++b)
+    for (int h = 0; h < Hkv; ++h)
+      for (int i = 0; i < n_rows; ++i) {
+        size_t bh = (size_t)b * Hkv + h, slot = bh * hi_cap + i;
+        int r = rows[bh * n_rows + i];
+        if (r < 0 || r >= n_src) { free(x); return -1; }
+        quantize_kv_row(k_src + (bh * n_src + r) * d, v_src + (bh * n_src + r) * d, d, h, hi_bits, hg, balancer,
+                        x, k_hc + slot * rb, k_hp + slot * np, v_hc + slot * rb, v_hp + slot * np);
+        hi_tok[slot] = src_tok ? src_tok[bh * n_src + r] : r;
+        acc[slot] = src_scores ? src_scores[bh * n_src + r] : 0.0f;
+      }
+  free(x);
+  return 0;
+}
+
+int mikv_ref_insert_token_q(int B, int Hkv, int d, int hi_cap, int hi_bits, int hg, const uint16_t* k_new,
+                            const uint16_t* v_new, int tok, const int32_t* slots, const float* balancer,
+                            uint8_t* k_hc, uint8_t* v_hc, uint16_t* k_hp, uint16_t* v_hp, int32_t* hi_tok,
+                            float* acc) {
+  if (!hi_args_ok(d, hi_bits, hg)) return -1;
+  size_t rb = (size_t)d * hi_bits / 8, np = (size_t)(d / hg) * 2;
+  float* x = (float*)malloc(sizeof(float) * (size_t)d);
+  if (!x) return -1;
+  for (int b = 0; b < B; ++b)
+    for (int h = 0; h < Hkv; ++h) {
+      size_t bh = (size_t)b * Hkv + h;
+      int s = slots[bh];
+      if (s < 0 || s >= hi_cap) { free(x); return -1; }
+      size_t slot = bh * hi_cap + s;
+      quantize_kv_row(k_new + bh * d, v_new + bh * d, d, h, hi_bits, hg, balancer, x, k_hc + slot * rb,
+                      k_hp + slot * np, v_hc + slot * rb, v_hp + slot * np);
+      hi_tok[slot] = tok;
+      acc[slot] = 0.0f;
+    }
+  free(x);
+  return 0;
+}
+
+/*
+ * Decode attention with a reduced-precision important set: like mikv_ref_decode_attention, except
+ * that the important keys are dequantized balanced keys attended with q / balancer (Eq. 3-4) and the
+ * important values are dequantized values.
+ */
+int mikv_ref_decode_attention_q(int B, int Hq, int Hkv, int d, int hi_bits, int hg, int bits, int g, int hi_cap,
+                                int lo_cap, int n_lo, const uint8_t* k_hc, const uint8_t* v_hc,
+                                const uint16_t* k_hp, const uint16_t* v_hp, const uint8_t* k_codes,
+                                const uint8_t* v_codes, const uint16_t* k_params, const uint16_t* v_params,
+                                const float* balancer, const uint16_t* q, double sm_scale, double* out,
+                                double* hi_logits, double* ml) {
+  if (B <= 0 || Hkv <= 0 || Hq % Hkv || !valid_bits(bits) || g <= 0 || d % g || d != 128 ||
+      !hi_args_ok(d, hi_bits, hg) || hi_cap < 0 || n_lo < 0 || n_lo > lo_cap || hi_cap + n_lo == 0)
+    return -1;
+  int G = Hq / Hkv;
+  size_t rb = (size_t)d * bits / 8, np = (size_t)(d / g) * 2;
+  size_t hrb = (size_t)d * hi_bits / 8, hnp = (size_t)(d / hg) * 2;
+  int n = hi_cap + n_lo;
+  double* s = (double*)malloc(sizeof(double) * (size_t)n);
+  double* qhat = (double*)malloc(sizeof(double) * (size_t)d);
+  double* xr = (double*)malloc(sizeof(double) * (size_t)d);
+  if (!s || !qhat || !xr) { free(s); free(qhat); free(xr); return -1; }
+  for (int b = 0; b < B; ++b)
+    for (int hq = 0; hq < Hq; ++hq) {
+      int h = hq / G;
+      size_t bh = (size_t)b * Hkv + h, bq = (size_t)b * Hq + hq;
+      for (int c = 0; c < d; ++c) /* Eq. 4 */
+        qhat[c] = bf16_to_f32(q[bq * d + c]) / (balancer ? (double)balancer[(size_t)h * d + c] : 1.0);
+      for (int i = 0; i < n; ++i) {
+        if (i < hi_cap) {
+          size_t slot = bh * hi_cap + i;
+          mikv_ref_dequantize_row(k_hc + slot * hrb, k_hp + slot * hnp, d, hi_bits, hg, xr);
+        } else {
+          size_t pos = bh * lo_cap + (i - hi_cap);
+          mikv_ref_dequantize_row(k_codes + pos * rb, k_params + pos * np, d, bits, g, xr);
+        }
+        double acc = 0.0;
+        for (int c = 0; c < d; ++c) acc += qhat[c] * xr[c];
+        s[i] = sm_scale * acc;
+      }
+      double m = -INFINITY;
+      for (int i = 0; i < n; ++i)
+        if (s[i] > m) m = s[i];
+      double l = 0.0;
+      for (int i = 0; i < n; ++i) l += exp(s[i] - m);
+      double* o = out + bq * d;
+      for (int c = 0; c < d; ++c) o[c] = 0.0;
+      for (int i = 0; i < n; ++i) {
+        if (i < hi_cap) {
+          size_t slot = bh * hi_cap + i;
+          mikv_ref_dequantize_row(v_hc + slot * hrb, v_hp + slot * hnp, d, hi_bits, hg, xr);
+        } else {
+          size_t pos = bh * lo_cap + (i - hi_cap);
+          mikv_ref_dequantize_row(v_codes + pos * rb, v_params + pos * np, d, bits, g, xr);
+        }
+        double p = exp(s[i] - m) / l;
+        for (int c = 0; c < d; ++c) o[c] += p * xr[c];
+      }
+      if (hi_logits)
+        for (int i = 0; i < hi_cap; ++i) hi_logits[bq * hi_cap + i] = s[i];
+      if (ml) {
+        ml[2 * bq] = m;
+        ml[2 * bq + 1] = l;
+      }
+    }
+  free(s); free(qhat); free(xr);
+  return 0;
+}
+
+int mikv_ref_demote_hi_q(int B, int Hkv, int d, int hi_cap, int hi_bits, int hg, int bits, int g, int lo_cap,
+                         const int32_t* slots, int lo_pos, const uint8_t* k_hc, const uint8_t* v_hc,
+                         const uint16_t* k_hp, const uint16_t* v_hp, const int32_t* hi_tok, uint8_t* k_codes,
+                         uint8_t* v_codes, uint16_t* k_params, uint16_t* v_params, int32_t* lo_tok) {
+  if (!hi_args_ok(d, hi_bits, hg) || !valid_bits(bits) || g <= 0 || d % g || lo_pos < 0 || lo_pos >= lo_cap)
+    return -1;
+  size_t hrb = (size_t)d * hi_bits / 8, hnp = (size_t)(d / hg) * 2;
+  size_t rb = (size_t)d * bits / 8, np = (size_t)(d / g) * 2;
+  float* x = (float*)malloc(sizeof(float) * (size_t)d);
+  if (!x) return -1;
+  for (int b = 0; b < B; ++b)
+    for (int h = 0; h < Hkv; ++h) {
+      size_t bh = (size_t)b * Hkv + h;
+      int s = slots[bh];
+      if (s < 0 || s >= hi_cap) { free(x); return -1; }
+      size_t slot = bh * hi_cap + s, pos = bh * lo_cap + lo_pos;
+      mikv_ref_dequantize_row_f32(k_hc + slot * hrb, k_hp + slot * hnp, d, hi_bits, hg, x);
+      mikv_ref_quantize_row(x, d, bits, g, k_codes + pos * rb, k_params + pos * np);
+      mikv_ref_dequantize_row_f32(v_hc + slot * hrb, v_hp + slot * hnp, d, hi_bits, hg, x);
+      mikv_ref_quantize_row(x, d, bits, g, v_codes + pos * rb, v_params + pos * np);
+      lo_tok[pos] = hi_tok[slot];
+    }
+  free(x);
+  return 0;
+}
+
 /* ---------------------------------------------------------------- memory accounting */
 
 /*

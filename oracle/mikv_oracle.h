@@ -107,6 +107,35 @@ int mikv_ref_gather_hi(int B, int Hkv, int d, int hi_cap, const uint16_t* k_src,
                        int n_src, const int32_t* rows, int n_rows, uint16_t* k_hi, uint16_t* v_hi,
                        int32_t* hi_tok, float* acc);
 
+/* Reduced-precision important set (Sec. 3.3, Table 3): important rows stored as hi_bits-bit codes
+ * with fp16 (alpha, beta) per group of hg channels, keys balanced (Eq. 3) and attended with q / balancer.
+ * k_hc, v_hc uint8 [B][Hkv][hi_cap][d*hi_bits/8]; k_hp, v_hp fp16 [B][Hkv][hi_cap][d/hg][2].
+ * mikv_ref_dequantize_row_f32: x[c] = fp32(alpha16 * code + beta16), the sum rounded once.
+ * gather_hi_q / insert_token_q: as gather_hi / insert_token, quantizing the rows.
+ * decode_attention_q: as decode_attention with the coded important set.
+ * demote_hi_q: slot slots[b][h] is dequantized (fp32) and re-quantized at bits/g into retained
+ * position lo_pos (no second balancer multiply); lo_tok receives its token id. */
+int mikv_ref_dequantize_row_f32(const uint8_t* packed, const uint16_t* params, int d, int bits, int g,
+                                float* x);
+int mikv_ref_gather_hi_q(int B, int Hkv, int d, int hi_cap, int hi_bits, int hg, const uint16_t* k_src,
+                         const uint16_t* v_src, const int32_t* src_tok, const float* src_scores, int n_src,
+                         const int32_t* rows, int n_rows, const float* balancer, uint8_t* k_hc, uint8_t* v_hc,
+                         uint16_t* k_hp, uint16_t* v_hp, int32_t* hi_tok, float* acc);
+int mikv_ref_insert_token_q(int B, int Hkv, int d, int hi_cap, int hi_bits, int hg, const uint16_t* k_new,
+                            const uint16_t* v_new, int tok, const int32_t* slots, const float* balancer,
+                            uint8_t* k_hc, uint8_t* v_hc, uint16_t* k_hp, uint16_t* v_hp, int32_t* hi_tok,
+                            float* acc);
+int mikv_ref_decode_attention_q(int B, int Hq, int Hkv, int d, int hi_bits, int hg, int bits, int g, int hi_cap,
+                                int lo_cap, int n_lo, const uint8_t* k_hc, const uint8_t* v_hc,
+                                const uint16_t* k_hp, const uint16_t* v_hp, const uint8_t* k_codes,
+                                const uint8_t* v_codes, const uint16_t* k_params, const uint16_t* v_params,
+                                const float* balancer, const uint16_t* q, double sm_scale, double* out,
+                                double* hi_logits, double* ml);
+int mikv_ref_demote_hi_q(int B, int Hkv, int d, int hi_cap, int hi_bits, int hg, int bits, int g, int lo_cap,
+                         const int32_t* slots, int lo_pos, const uint8_t* k_hc, const uint8_t* v_hc,
+                         const uint16_t* k_hp, const uint16_t* v_hp, const int32_t* hi_tok, uint8_t* k_codes,
+                         uint8_t* v_codes, uint16_t* k_params, uint16_t* v_params, int32_t* lo_tok);
+
 /* Closed-form KV-cache size as a fraction of an all-fp16 cache: ratio r of tokens at hi_bits
  * (16 = fp16, else hi_bits-bit codes with fp16 alpha/beta per group g) plus (1 - r) at bits-bit codes
  * with fp16 alpha/beta per group g. */
