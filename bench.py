@@ -162,7 +162,8 @@ def build_model(w, steps_cap: int, dev, rank: int):
     """All layers' caches, built from seeded prefill tensors with the library's own kernels."""
     import paper_2402_18096_gb300 as pkg
     from paper_2402_18096_gb300.layer import MixedPrecisionLayer
-    shape = pkg.Shape(w.batch, w.heads_q, w.heads_kv, w.bits, w.group, w.hi_cap, w.lo_cap_for(steps_cap))
+    shape = pkg.Shape(w.batch, w.heads_q, w.heads_kv, w.bits, w.group, w.hi_cap, w.lo_cap_for(steps_cap),
+                      hi_bits=w.hi_bits)
     wr = rank_workload(w, rank)  # each rank owns a different batch
     layers = []
     for li in range(w.layers):
@@ -339,8 +340,8 @@ def _oracle_head(w, b, h, steps_cap):
     sc = scores.numpy()
     del k, v, q_pre
     dem, kept = oracle.select_demote(sc, w.context - w.budget)
-    c = oracle.empty_cache(1, 1, w.head_dim, w.bits, w.group, w.hi_cap, w.lo_cap_for(steps_cap))
-    oracle.gather_hi(c, ks, vs, kept, src_scores=sc)
+    c = oracle.empty_cache(1, 1, w.head_dim, w.bits, w.group, w.hi_cap, w.lo_cap_for(steps_cap), hi_bits=w.hi_bits)
+    oracle.gather_hi(c, ks, vs, kept, src_scores=sc, balancer_=bal)
     oracle.quantize_pack(c, ks, vs, dem, 0, balancer_=bal)
     return c, bal, np.array([[w.budget]], np.int32)
 
@@ -350,17 +351,18 @@ def _oracle_step(w, c, bal, slots, n_lo, pos, q, kn, vn):
     import numpy as np
     import oracle
     G = w.heads_q // w.heads_kv
-    oracle.insert_token(c, kn, vn, pos, slots)
+    oracle.insert_token(c, kn, vn, pos, slots, balancer_=bal)
     _, hl, ml = oracle.decode_attention(c, q, n_lo, 1 / math.sqrt(w.head_dim), balancer_=bal)
     c["acc"] = oracle.update_importance(c["acc"], hl.astype(np.float32), ml.astype(np.float32), G)
     dem, _ = oracle.select_demote(c["acc"], 1, c["hi_tok"], want_kept=False)
-    oracle.quantize_pack(c, c["k_hi"], c["v_hi"], dem, n_lo, src_tok=c["hi_tok"], balancer_=bal)
+    oracle.demote_hi(c, dem[:, :, 0], n_lo, balancer_=bal)
     return dem[0]
 
 
 def _head_bytes(w, n_lo):
     lo = 2 * (w.head_dim * w.bits // 8 + 4 * (w.head_dim // w.group))
-    return w.hi_cap * 4 * w.head_dim + n_lo * lo
+    hi = 4 * w.head_dim if w.hi_bits >= 16 else 2 * (w.head_dim * w.hi_bits // 8 + 4 * (w.head_dim // 64))
+    return w.hi_cap * hi + n_lo * lo
 
 
 def cpu_baseline(w, seconds: float = 15.0, steps=None):
@@ -400,7 +402,8 @@ def run_sweep(args):
     points = []
     for w in mi.sweep_workloads():
         K, W = args.steps, args.warmup
-        shape = pkg.Shape(w.batch, w.heads_q, w.heads_kv, w.bits, w.group, w.hi_cap, w.lo_cap_for(K + W + 4))
+        shape = pkg.Shape(w.batch, w.heads_q, w.heads_kv, w.bits, w.group, w.hi_cap, w.lo_cap_for(K + W + 4),
+                          hi_bits=w.hi_bits)
         k, v = mi.prefill_kv(w, 0, dev)
         sc = mi.initial_scores(w, 0, dev)
         qp = mi.prefill_queries(w, 0, dev)

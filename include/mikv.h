@@ -10,7 +10,9 @@
  *     round-to-nearest codes with fp16 scale/zero (Eq. 1, Sec. 3.1) in the "retained set";
  *   - keys are multiplied by a per-channel balancer before quantization and the query is divided by
  *     it (Eq. 2-4, Sec. 3.2);
- *   - attention treats the two sets as one unordered set (permutation invariance, Sec. 3.4).
+ *   - attention treats the two sets as one unordered set (permutation invariance, Sec. 3.4);
+ *   - optionally (Sec. 3.3, Table 3) the important set itself is kept at reduced precision: INT8,
+ *     INT4 or INT2 codes with fp16 scale/zero per 64 channels, quantized like the retained set.
  *
  * Conventions shared by every entry point:
  *   - All array pointers are DEVICE pointers owned by the caller; the library never allocates,
@@ -25,9 +27,9 @@
  *
  * Packed-code layout of one retained row (d = 128, N bits, 16 * N bytes): channel c is written
  * c = 16 m + u (u = c mod 16, m = c div 16) and a plane is a sequence of little-endian 16-bit units.
- * In a plane of f-bit fields (f in {2, 4}) with P = 16 / f codes per unit, channel c sits in unit
+ * In a plane of f-bit fields (f in {2, 4, 8}) with P = 16 / f codes per unit, channel c sits in unit
  * 8 * (2 * (m div P) + (u div 8)) + (u mod 8) at bits [f * (m mod P), f * (m mod P) + f). In a plane of
- * 1-bit fields, channel c sits in unit (u mod 8) at bit 8 * (u div 8) + m. N = 2 and N = 4 use one
+ * 1-bit fields, channel c sits in unit (u mod 8) at bit 8 * (u div 8) + m. N = 2, 4 and 8 use one
  * plane of N-bit fields; N = 3 uses a plane of 2-bit fields (code bits 0..1) followed by a plane of
  * 1-bit fields (code bit 2). The quantization parameters of a row are d / group pairs of fp16
  * (alpha, beta), alpha first; the dequantized value is alpha * code + beta.
@@ -65,13 +67,16 @@ typedef struct {
   int32_t hi_cap;    /* important slots attended per head: the budget k plus one staging slot */
   int32_t hi_stride; /* rows per head in the important-set arrays: multiple of 16, >= hi_cap */
   int32_t lo_cap;    /* rows per head in the retained-set arrays: multiple of 16 */
+  int32_t hi_bits;   /* important-set precision: 0 or 16 = bf16; 8, 4 or 2 = codes (Sec. 3.3, Table 3) */
+  int32_t hi_group;  /* channels per group of a coded important set: 64 (ignored for bf16) */
 } mikv_shape;
 
 /* Device arrays of one layer's cache. Rows >= hi_cap of the important arrays are padding and are
  * never read as data; retained rows >= the current length likewise. */
 typedef struct {
-  void* k_hi;           /* bf16 [B][Hkv][hi_stride][d], keys WITHOUT the balancer */
-  void* v_hi;           /* bf16 [B][Hkv][hi_stride][d] */
+  void* k_hi;           /* bf16 [B][Hkv][hi_stride][d], keys WITHOUT the balancer; or, for a coded
+                           important set, uint8 [B][Hkv][hi_stride][16 * hi_bits] codes of BALANCED keys */
+  void* v_hi;           /* bf16 [B][Hkv][hi_stride][d]; or uint8 [B][Hkv][hi_stride][16 * hi_bits] */
   int32_t* hi_tok;      /* int32 [B][Hkv][hi_stride], token position held by each slot */
   float* acc;           /* fp32 [B][Hkv][hi_stride], accumulated attention score per slot */
   void* k_codes;        /* uint8 [B][Hkv][lo_cap][16 * bits], codes of balanced keys (Eq. 3) */
@@ -80,6 +85,8 @@ typedef struct {
   void* v_params;       /* fp16 [B][Hkv][lo_cap][d / group][2] */
   int32_t* lo_tok;      /* int32 [B][Hkv][lo_cap], token position of each retained row */
   const float* balancer; /* fp32 [Hkv][d] channel balancer of this layer (Eq. 2), or NULL = 1 */
+  void* k_hi_params;    /* coded important set only (else unused): fp16 [B][Hkv][hi_stride][d / hi_group][2] */
+  void* v_hi_params;    /* coded important set only: fp16 [B][Hkv][hi_stride][d / hi_group][2] */
 } mikv_cache;
 
 /* Output element type of mikv_decode_attention. */
@@ -142,6 +149,8 @@ mikv_status mikv_quantize_pack(const mikv_shape* shape, const mikv_cache* cache,
  *   s_i = sm_scale * q . k_hi[i]                  for the hi_cap important slots (bf16 keys)
  *   s_t = sm_scale * (q / balancer) . k_hat[t]    for retained rows t < n_lo, k_hat = alpha*code+beta
  *   out = sum_j softmax(s)_j * v_j  over both sets (v_hat = alpha * code + beta for retained rows)
+ * A coded important set (hi_bits < 16) is attended like the retained set: s_i = sm_scale *
+ * (q / balancer) . k_hat[i] with its own codes and parameters, values dequantized likewise.
  * Split-K flash decoding: partial (max, sum, unnormalised output) per context split in fp32, merged
  * into `out`. Arithmetic: fp32 accumulation; dot products on tensor cores with bf16 (important) or
  * fp16 (retained: dequantized codes, q / balancer) operands.
@@ -183,7 +192,9 @@ mikv_status mikv_select_demote(int32_t batch, int32_t heads, const float* scores
 /*
  * New-token insertion (Fig. 4: the new KV pair enters the important set in high precision):
  * slot s = slots[b][h] (0 <= s < hi_cap) of every (b, h) receives k_new[b][h], v_new[b][h]
- * (bf16 [B][Hkv][d], keys without balancer), hi_tok = tok and acc = 0.
+ * (bf16 [B][Hkv][d], keys without balancer), hi_tok = tok and acc = 0. With a coded important set
+ * (hi_bits < 16) the rows are quantized on the way in (Eq. 1 at hi_bits, groups of hi_group; the key
+ * multiplied by the balancer first, Eq. 3), exactly as mikv_quantize_pack quantizes retained rows.
  */
 mikv_status mikv_insert_token(const mikv_shape* shape, const mikv_cache* cache, const void* k_new,
                               const void* v_new, int32_t tok, const int32_t* slots, void* stream);
@@ -191,7 +202,8 @@ mikv_status mikv_insert_token(const mikv_shape* shape, const mikv_cache* cache, 
 /*
  * Important-set build from prefill rows: important slot i < n_rows of (b, h) receives source row
  * r = rows[b][h][i] of k_src/v_src (bf16 [B][Hkv][n_src][d]), hi_tok = src_tok ? src_tok[b][h][r] : r
- * and acc = src_scores ? src_scores[b][h][r] : 0. Requires n_rows <= hi_cap.
+ * and acc = src_scores ? src_scores[b][h][r] : 0. Requires n_rows <= hi_cap. A coded important set
+ * receives the quantized rows (as in mikv_insert_token).
  */
 mikv_status mikv_gather_hi(const mikv_shape* shape, const mikv_cache* cache, const void* k_src,
                            const void* v_src, const int32_t* src_tok, const float* src_scores,
@@ -203,7 +215,9 @@ mikv_status mikv_gather_hi(const mikv_shape* shape, const mikv_cache* cache, con
  * update the importance scores (mikv_update_importance), choose the least important slot
  * (mikv_select_demote, n_demote = 1) and demote it to retained row n_lo (mikv_quantize_pack).
  * On return slots[b][h] holds the slot freed by the demotion (the next step's insertion slot);
- * the retained length becomes n_lo + 1.
+ * the retained length becomes n_lo + 1. A coded important slot is demoted from its dequantized values:
+ * per channel the fp32 value alpha * code + beta (rounded once), quantized at bits / group; keys are
+ * already balanced and are not multiplied by the balancer again (Sec. 3.3).
  *   q, k_new, v_new   bf16 [B][Hq][d], [B][Hkv][d], [B][Hkv][d]
  *   slots             int32 [B][Hkv], in/out
  *   out               as in mikv_decode_attention

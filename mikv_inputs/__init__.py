@@ -37,6 +37,7 @@ class Workload:
     ratio: float          # fraction of tokens kept in bf16 (importance ratio)
     seed: int = 0
     head_dim: int = HEAD_DIM
+    hi_bits: int = 16     # important-set precision: 16 = bf16, or 8 / 4 / 2-bit codes in groups of 64
 
     @property
     def budget(self) -> int:
@@ -67,6 +68,12 @@ WORKLOADS = {
     "mistral-7b": Workload("mistral-7b-b32-l32-hq32-hkv8-t32768-int2-g32-r20", 32, 32, 8, 32768, 32, 2,
                            32, 0.20),
 }
+# Table 3 settings (INT2 retained, 20 % important, groups of 64) on the Mistral-7B shape, with the
+# important set itself at reduced precision (Sec. 3.3)
+for _hb in (16, 8, 4, 2):
+    WORKLOADS[f"mistral-7b-t3-hi{_hb}"] = Workload(
+        f"mistral-7b-b32-l32-hq32-hkv8-t32768-int2-g64-r20-hi{_hb}", 32, 32, 8, 32768, 32, 2, 64, 0.20,
+        hi_bits=_hb)
 
 
 def sweep_workloads() -> List[Workload]:

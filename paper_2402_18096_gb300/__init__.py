@@ -42,13 +42,14 @@ class MikvError(RuntimeError):
 
 class _Shape(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in
-                ("batch", "heads_q", "heads_kv", "head_dim", "bits", "group", "hi_cap", "hi_stride", "lo_cap")]
+                ("batch", "heads_q", "heads_kv", "head_dim", "bits", "group", "hi_cap", "hi_stride", "lo_cap",
+                 "hi_bits", "hi_group")]
 
 
 class _Cache(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in
                 ("k_hi", "v_hi", "hi_tok", "acc", "k_codes", "v_codes", "k_params", "v_params", "lo_tok",
-                 "balancer")]
+                 "balancer", "k_hi_params", "v_hi_params")]
 
 
 _lib = None
@@ -123,14 +124,20 @@ class Shape:
     hi_cap: int
     lo_cap: int
     head_dim: int = HEAD_DIM
+    hi_bits: int = 16   # important-set precision: 16 = bf16; 8, 4, 2 = codes (Sec. 3.3, Table 3)
+    hi_group: int = 64  # channels per group of a coded important set
 
     @property
     def hi_stride(self) -> int:
         return (self.hi_cap + 15) // 16 * 16
 
+    @property
+    def hi_coded(self) -> bool:
+        return self.hi_bits not in (0, 16)
+
     def c(self) -> _Shape:
         return _Shape(self.batch, self.heads_q, self.heads_kv, self.head_dim, self.bits, self.group,
-                      self.hi_cap, self.hi_stride, self.lo_cap)
+                      self.hi_cap, self.hi_stride, self.lo_cap, self.hi_bits, self.hi_group)
 
 
 class LayerCache:
@@ -141,8 +148,15 @@ class LayerCache:
         B, H, d = s.batch, s.heads_kv, s.head_dim
         self.shape = s
         z = dict(device=device)
-        self.k_hi = torch.zeros(B, H, s.hi_stride, d, dtype=torch.bfloat16, **z)
-        self.v_hi = torch.zeros(B, H, s.hi_stride, d, dtype=torch.bfloat16, **z)
+        if s.hi_coded:  # codes of balanced keys / values plus (alpha, beta) per group
+            self.k_hi = torch.zeros(B, H, s.hi_stride, 16 * s.hi_bits, dtype=torch.uint8, **z)
+            self.v_hi = torch.zeros(B, H, s.hi_stride, 16 * s.hi_bits, dtype=torch.uint8, **z)
+            self.k_hi_params = torch.zeros(B, H, s.hi_stride, d // s.hi_group, 2, dtype=torch.float16, **z)
+            self.v_hi_params = torch.zeros(B, H, s.hi_stride, d // s.hi_group, 2, dtype=torch.float16, **z)
+        else:
+            self.k_hi = torch.zeros(B, H, s.hi_stride, d, dtype=torch.bfloat16, **z)
+            self.v_hi = torch.zeros(B, H, s.hi_stride, d, dtype=torch.bfloat16, **z)
+            self.k_hi_params = self.v_hi_params = None
         self.hi_tok = torch.zeros(B, H, s.hi_stride, dtype=torch.int32, **z)
         self.acc = torch.zeros(B, H, s.hi_stride, dtype=torch.float32, **z)
         self.k_codes = torch.zeros(B, H, s.lo_cap, 16 * s.bits, dtype=torch.uint8, **z)
@@ -156,13 +170,14 @@ class LayerCache:
     def c(self) -> _Cache:
         return _Cache(*[_ptr(getattr(self, n)) for n in
                         ("k_hi", "v_hi", "hi_tok", "acc", "k_codes", "v_codes", "k_params", "v_params",
-                         "lo_tok", "balancer")])
+                         "lo_tok", "balancer", "k_hi_params", "v_hi_params")])
 
     def nbytes_attended(self, n_lo: int) -> int:
-        """Bytes of cache one decode attention reads: hi_cap bf16 K/V rows + n_lo retained rows."""
+        """Bytes of cache one decode attention reads: hi_cap important K/V rows + n_lo retained rows."""
         s = self.shape
         row_lo = 2 * mikv_retained_row_bytes(s.bits, s.group, s.head_dim)
-        return s.batch * s.heads_kv * (s.hi_cap * 4 * s.head_dim + n_lo * row_lo)
+        row_hi = 2 * mikv_retained_row_bytes(s.hi_bits, s.hi_group, s.head_dim) if s.hi_coded else 4 * s.head_dim
+        return s.batch * s.heads_kv * (s.hi_cap * row_hi + n_lo * row_lo)
 
 
 # ------------------------------------------------------------------ C-ABI functions

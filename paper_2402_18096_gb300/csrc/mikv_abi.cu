@@ -37,15 +37,23 @@ mikv_status shape_supported(const mikv_shape* s) {
   if (s->bits < 2 || s->bits > 4) return MIKV_ERR_UNSUPPORTED;
   if (s->group != 32 && s->group != 64 && s->group != 128) return MIKV_ERR_UNSUPPORTED;
   if (G != 1 && G != 2 && G != 4 && G != 8) return MIKV_ERR_UNSUPPORTED;
+  const int hb = s->hi_bits;
+  if (hb != 0 && hb != 16 && hb != 8 && hb != 4 && hb != 2) return MIKV_ERR_UNSUPPORTED;
+  if (hb != 0 && hb != 16 && s->hi_group != kHiGroup) return MIKV_ERR_UNSUPPORTED;
   return MIKV_OK;
 }
 
-bool cache_ok(const mikv_cache* c) {
-  return c && c->k_hi && c->v_hi && c->hi_tok && c->acc && c->k_codes && c->v_codes && c->k_params &&
-         c->v_params && c->lo_tok;
-}
-
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+// The cache's arrays exist (and, for a coded important set, so do its parameter arrays, 16-byte aligned).
+bool cache_ok(const mikv_cache* c, const mikv_shape* s) {
+  if (!(c && c->k_hi && c->v_hi && c->hi_tok && c->acc && c->k_codes && c->v_codes && c->k_params &&
+        c->v_params && c->lo_tok))
+    return false;
+  if (hi_bits_of(*s) != 16)
+    return c->k_hi_params && c->v_hi_params && aligned(c->k_hi_params, 16) && aligned(c->v_hi_params, 16);
+  return true;
+}
 
 // ------------------------------------------------------------------ tensor maps
 
@@ -120,7 +128,7 @@ mikv_status attention_args_ok(const mikv_shape* shape, const mikv_cache* cache, 
                               const void* out, int32_t out_dtype) {
   mikv_status st = shape_supported(shape);
   if (st != MIKV_OK) return st;
-  if (!cache_ok(cache) || !q || !out || n_lo < 0 || (out_dtype != MIKV_OUT_BF16 && out_dtype != MIKV_OUT_F32))
+  if (!cache_ok(cache, shape) || !q || !out || n_lo < 0 || (out_dtype != MIKV_OUT_BF16 && out_dtype != MIKV_OUT_F32))
     return MIKV_ERR_ARG;
   if (n_lo > shape->lo_cap) return MIKV_ERR_CAPACITY;
   if (shape->hi_cap + n_lo < 1) return MIKV_ERR_ARG;
@@ -158,10 +166,31 @@ mikv_status attention_impl(const mikv_shape* s, const mikv_cache* c, int32_t n_l
   memset(&a, 0, sizeof a);
   const uint64_t hi_rows = (uint64_t)s->batch * s->heads_kv * s->hi_stride;
   const uint64_t lo_rows = (uint64_t)s->batch * s->heads_kv * s->lo_cap;
-  bool ok = make_map(&a.map_k_hi, c->k_hi, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, kHeadDim, hi_rows, 2 * kHeadDim, 64,
-                     16, CU_TENSOR_MAP_SWIZZLE_128B) &&
-            make_map(&a.map_v_hi, c->v_hi, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, kHeadDim, hi_rows, 2 * kHeadDim, 64,
-                     16, CU_TENSOR_MAP_SWIZZLE_128B);
+  const int hb = hi_bits_of(*s);
+  bool ok;
+  if (hb == 16) {
+    ok = make_map(&a.map_k_hi, c->k_hi, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, kHeadDim, hi_rows, 2 * kHeadDim, 64, 16,
+                  CU_TENSOR_MAP_SWIZZLE_128B) &&
+         make_map(&a.map_v_hi, c->v_hi, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, kHeadDim, hi_rows, 2 * kHeadDim, 64, 16,
+                  CU_TENSOR_MAP_SWIZZLE_128B);
+  } else {
+    // coded important rows: viewed like retained codes of layout (hb, 64); hi_stride % 16 == 0 keeps
+    // every unit row-aligned
+    const LoUnit H = lo_unit_layout(hb, kHiGroup);
+    const uint64_t code_rows = hi_rows * H.pitch / H.map_w;
+    const uint32_t code_box = 16u * H.blocks * H.pitch / H.map_w;
+    const CUtensorMapSwizzle swz = hb == 8 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
+    const uint64_t par_rows = hi_rows * H.param_row / H.param_w;
+    const uint32_t par_box = 16u * H.blocks * H.param_row / H.param_w;
+    ok = make_map(&a.map_k_hi, c->k_hi, CU_TENSOR_MAP_DATA_TYPE_UINT8, H.map_w, code_rows, H.map_w, H.map_w,
+                  code_box, swz) &&
+         make_map(&a.map_v_hi, c->v_hi, CU_TENSOR_MAP_DATA_TYPE_UINT8, H.map_w, code_rows, H.map_w, H.map_w,
+                  code_box, swz) &&
+         make_map(&a.map_k_hp, c->k_hi_params, CU_TENSOR_MAP_DATA_TYPE_UINT8, H.param_w, par_rows, H.param_w,
+                  H.param_w, par_box, CU_TENSOR_MAP_SWIZZLE_NONE) &&
+         make_map(&a.map_v_hp, c->v_hi_params, CU_TENSOR_MAP_DATA_TYPE_UINT8, H.param_w, par_rows, H.param_w,
+                  H.param_w, par_box, CU_TENSOR_MAP_SWIZZLE_NONE);
+  }
   if (ok && lo_rows > 0) {
     // retained arrays: each is viewed as rows of U.map_w (codes) or U.param_w (alpha, beta) bytes, and
     // one box covers a whole unit of 16 * U.blocks tokens (lo_cap % 16 == 0 keeps units row-aligned)
@@ -195,13 +224,14 @@ mikv_status attention_impl(const mikv_shape* s, const mikv_cache* c, int32_t n_l
   a.hi_stride = s->hi_stride;
   a.lo_cap = s->lo_cap;
   a.n_lo = n_lo;
+  a.hi_blocks = plan.hi_blocks;
   a.hi_units = plan.hi_units;
   a.lo_blocks = plan.lo_blocks;
   a.n_u = plan.n_u;
   a.n_units = plan.n_units;
   a.n_warps = plan.n_warps;
   a.sm_scale = sm_scale;
-  cudaError_t e = launch_attention(a, s->bits, s->group, G, plan.grid, st);
+  cudaError_t e = launch_attention(a, s->bits, s->group, hb, G, plan.grid, st);
   if (e != cudaSuccess) return MIKV_ERR_CUDA;
   if (args_out) *args_out = a;
   if (!merge) return MIKV_OK;
@@ -279,7 +309,7 @@ mikv_status mikv_quantize_pack(const mikv_shape* shape, const mikv_cache* cache,
                                int32_t n_rows, int32_t lo_start, void* stream) {
   mikv_status st = shape_supported(shape);
   if (st != MIKV_OK) return st;
-  if (!cache_ok(cache) || !k_src || !v_src || n_src <= 0 || n_rows < 0 || lo_start < 0 || (n_rows > 0 && !rows))
+  if (!cache_ok(cache, shape) || !k_src || !v_src || n_src <= 0 || n_rows < 0 || lo_start < 0 || (n_rows > 0 && !rows))
     return MIKV_ERR_ARG;
   if ((int64_t)lo_start + n_rows > shape->lo_cap) return MIKV_ERR_CAPACITY;
   if ((int64_t)(n_rows + 3) / 4 > 2147483647 || (int64_t)shape->batch * shape->heads_kv > 65535)
@@ -302,7 +332,7 @@ mikv_status mikv_update_importance(const mikv_shape* shape, const mikv_cache* ca
                                    const float* ml, void* stream) {
   mikv_status st = shape_supported(shape);
   if (st != MIKV_OK) return st;
-  if (!cache_ok(cache) || !hi_logits || !ml) return MIKV_ERR_ARG;
+  if (!cache_ok(cache, shape) || !hi_logits || !ml) return MIKV_ERR_ARG;
   if (shape->hi_cap == 0) return MIKV_OK;
   return cuda_status(launch_update_importance(*shape, *cache, hi_logits, ml, static_cast<cudaStream_t>(stream)));
 }
@@ -321,7 +351,7 @@ mikv_status mikv_insert_token(const mikv_shape* shape, const mikv_cache* cache, 
                               const void* v_new, int32_t tok, const int32_t* slots, void* stream) {
   mikv_status st = shape_supported(shape);
   if (st != MIKV_OK) return st;
-  if (!cache_ok(cache) || !k_new || !v_new || !slots) return MIKV_ERR_ARG;
+  if (!cache_ok(cache, shape) || !k_new || !v_new || !slots) return MIKV_ERR_ARG;
   if (shape->hi_cap < 1) return MIKV_ERR_CAPACITY;
   return cuda_status(launch_insert(*shape, *cache, k_new, v_new, tok, slots, static_cast<cudaStream_t>(stream)));
 }
@@ -331,7 +361,7 @@ mikv_status mikv_gather_hi(const mikv_shape* shape, const mikv_cache* cache, con
                            int32_t n_rows, void* stream) {
   mikv_status st = shape_supported(shape);
   if (st != MIKV_OK) return st;
-  if (!cache_ok(cache) || !k_src || !v_src || n_src <= 0 || n_rows < 0 || (n_rows > 0 && !rows))
+  if (!cache_ok(cache, shape) || !k_src || !v_src || n_src <= 0 || n_rows < 0 || (n_rows > 0 && !rows))
     return MIKV_ERR_ARG;
   if (n_rows > shape->hi_cap) return MIKV_ERR_CAPACITY;
   return cuda_status(launch_gather(*shape, *cache, k_src, v_src, src_tok, src_scores, n_src, rows, n_rows,
@@ -343,7 +373,7 @@ mikv_status mikv_decode_step(const mikv_shape* shape, const mikv_cache* cache, i
                              void* out, int32_t out_dtype, void* workspace, size_t ws_bytes, void* stream) {
   mikv_status st = shape_supported(shape);
   if (st != MIKV_OK) return st;
-  if (!cache_ok(cache) || !q || !k_new || !v_new || !slots || !out || n_lo < 0) return MIKV_ERR_ARG;
+  if (!cache_ok(cache, shape) || !q || !k_new || !v_new || !slots || !out || n_lo < 0) return MIKV_ERR_ARG;
   if (shape->hi_cap < 1) return MIKV_ERR_CAPACITY;
   if ((int64_t)n_lo + 1 > shape->lo_cap) return MIKV_ERR_CAPACITY;
   if (!workspace || !aligned(workspace, 256)) return MIKV_ERR_WORKSPACE;
@@ -375,6 +405,9 @@ mikv_status mikv_decode_step(const mikv_shape* shape, const mikv_cache* cache, i
   p.v_params = cache->v_params;
   p.lo_tok = cache->lo_tok;
   p.slots = slots;
+  p.k_hi_params = cache->k_hi_params;
+  p.v_hi_params = cache->v_hi_params;
+  p.hi_bits = hi_bits_of(*shape);
   p.batch = shape->batch;
   p.heads_q = shape->heads_q;
   p.heads_kv = shape->heads_kv;

@@ -1,0 +1,875 @@
+// mikv_attention.cuh — split-K flash-decoding over the mixed-precision KV cache (sm_103a): the kernel
+// templates. Each mikv_attn_h*.cu instantiates them for one important-set precision; mikv_attention.cu
+// holds the work plan, the merge kernel and the dispatch.
+//
+// Computes, per (batch b, KV head h) and the G query heads that share it, softmax attention of the
+// new query over the important set (bf16 K/V, attended with q) and the retained set (N-bit codes,
+// keys balanced and attended with q / balancer), Eq. 3-4 of arxiv 2402.18096; the two sets are one
+// unordered set for attention (Sec. 3.4), so they are streamed separately and merged by the online
+// softmax.
+//
+// Work decomposition. Every (b, h) owns the same sequence of "units": an important unit is one block
+// of 16 bf16 tokens (8 KB of K and V), a retained unit is up to eight blocks of 16 coded
+// tokens (about the same bytes). The two kinds are interleaved evenly inside each head's sequence, the
+// sequences of all heads are concatenated, and every warp of the persistent grid takes one contiguous,
+// equal share. A warp therefore streams a balanced mix of bandwidth-heavy and ALU-heavy units and
+// touches one or two heads (a few, for small caches); it writes one partial (max, sum, output) per head
+// it touched, and a merge kernel combines the partials of each query head.
+//
+// Per warp: a private shared-memory ring (2 stages by default) fed by TMA (lane 0 issues 2-D tensor copies: bf16
+// rows and packed codes with hardware swizzle, one box per array per unit, (alpha, beta) pairs as
+// 16-byte rows; one mbarrier per stage, every wait bounded in time). No cross-warp synchronisation.
+//
+// A coded important set (Sec. 3.3, Table 3: INT8 / INT4 / INT2 codes, groups of 64) is streamed in
+// units laid out like retained units and attended with the same block code, with exact value codes
+// and its logits stored for the importance update.
+//
+// Per 16-token block: ldmatrix yields mma.sync fragments directly (the ABI's code layout is built for
+// this); tokens sit on M for QK^T and channels on M for PV, query heads on N. Codes become exact fp16
+// integers with one LOP3 each (the code bits OR-ed under an fp16 exponent that makes the code's lowest
+// bit weigh 1) and one HSUB2. Keys are then dequantized (alpha * c + beta, HFMA2) for QK^T; for PV the
+// value scale is folded into the probabilities (p * alpha per token and group) and the zero into one
+// extra MMA row (sum of p * beta per group), so values need no HFMA2. Online softmax in fp32;
+// movmatrix turns probabilities into the PV operand without shared memory.
+#pragma once
+
+#include <math.h>
+
+#include "mikv_device.cuh"
+#include "mikv_internal.h"
+#include "mikv_rows.cuh"
+
+namespace mikv {
+namespace {
+
+// Launch shape (compile-time tuning knobs; the defaults are the measured best on GB300).
+#ifndef MIKV_ATTN_WARPS
+#define MIKV_ATTN_WARPS 6
+#endif
+#ifndef MIKV_ATTN_STAGES
+#define MIKV_ATTN_STAGES 2
+#endif
+#ifndef MIKV_ATTN_CTAS
+#define MIKV_ATTN_CTAS 2
+#endif
+#ifndef MIKV_QK_ACC
+#define MIKV_QK_ACC 2
+#endif
+#ifndef MIKV_LO_PAIR
+#define MIKV_LO_PAIR 1
+#endif
+#ifndef MIKV_PAIR_ACC
+#define MIKV_PAIR_ACC 1
+#endif
+constexpr int kWarps = MIKV_ATTN_WARPS;     // independent warps per CTA
+constexpr int kThreads = kWarps * 32;
+constexpr int kNS = MIKV_ATTN_STAGES;       // ring stages per warp
+constexpr bool kLoPair = MIKV_LO_PAIR != 0;  // retained blocks processed two at a time
+constexpr int kPairAcc = MIKV_PAIR_ACC;      // QK^T accumulators per block when paired
+constexpr int kStageBytes = kUnitBytes;
+constexpr int kHiBlockBytes = 8192;         // K and V of 16 tokens: 4 boxes of 16 rows x 64 bf16
+constexpr int kCtasPerSm = MIKV_ATTN_CTAS;
+constexpr int kQkAcc = MIKV_QK_ACC;         // independent accumulators of the QK^T MMA chain
+constexpr int kUnitsPerWarp = 24;    // target share per warp (sizes the grid for small caches)
+constexpr float kLog2e = 1.4426950408889634f;
+
+__host__ __device__ constexpr int smem_bytes() { return 1024 + kWarps * kNS * kStageBytes + kWarps * kNS * 8; }
+
+// Position in the concatenated unit sequence. Unit i of a head (of n_u units, hu of them important)
+// is important when floor((i+1) hu / n_u) > floor(i hu / n_u): important units are spread evenly.
+// The cursor keeps r = (i hu) mod n_u and h = floor(i hu / n_u) so each step is O(1).
+struct Cursor {
+  int bh, i, r, h;
+};
+
+struct UnitKind {
+  bool hi;
+  int index;  // important block index, or retained unit index
+};
+
+__device__ __forceinline__ Cursor cursor_at(int u, int hu, int n_u) {
+  Cursor c;
+  c.bh = u / n_u;
+  c.i = u - c.bh * n_u;
+  const long long p = (long long)c.i * hu;
+  c.h = (int)(p / n_u);
+  c.r = (int)(p - (long long)c.h * n_u);
+  return c;
+}
+
+__device__ __forceinline__ UnitKind cursor_kind(const Cursor& c, int hu, int n_u) {
+  UnitKind k;
+  k.hi = c.r + hu >= n_u;
+  k.index = k.hi ? c.h : c.i - c.h;
+  return k;
+}
+
+__device__ __forceinline__ void cursor_next(Cursor& c, int hu, int n_u) {
+  const bool hi = c.r + hu >= n_u;
+  c.r += hu - (hi ? n_u : 0);
+  c.h += hi ? 1 : 0;
+  if (++c.i == n_u) {
+    ++c.bh;
+    c.i = c.r = c.h = 0;
+  }
+}
+
+// Running softmax state of heads 2t, 2t+1: reference max m (warp-uniform per head), sum l of
+// exp(logit - m) over this thread's tokens, and mx, the largest logit this thread has seen.
+struct Softmax {
+  float m[2], l[2], mx[2];
+};
+
+template <int Q>
+__device__ __forceinline__ void sum_acc(const float (&accs)[Q][4], float (&acc)[4]) {
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    float v = accs[0][e];
+#pragma unroll
+    for (int q = 1; q < Q; ++q) v += accs[q][e];
+    acc[e] = v;
+  }
+}
+
+// Online-softmax update for NK 16-token blocks. s[k] holds scaled logits of (token g, head 2t),
+// (g, 2t+1), (g+8, 2t), (g+8, 2t+1) of block k (-inf past the end); returns unnormalised
+// probabilities in p.
+// o (output) and ob (zero-row and alpha sums) are running sums at the current reference max m: all are
+// rescaled when m moves. The reference is only moved (one cross-lane reduction) when some logit exceeds it by
+// more than kLazy; otherwise the block reuses the old reference, so probabilities stay below e^kLazy.
+constexpr float kLazy = 4.f;
+
+template <int NB, int NK>
+__device__ __forceinline__ void softmax_blocks(const float (&s)[NK][4], Softmax& st, float (&o)[8][4],
+                                               float (&ob)[NB][4], float (&p)[NK][4]) {
+  float bm0 = fmaxf(s[0][0], s[0][2]), bm1 = fmaxf(s[0][1], s[0][3]);
+#pragma unroll
+  for (int k = 1; k < NK; ++k) {
+    bm0 = fmaxf(bm0, fmaxf(s[k][0], s[k][2]));
+    bm1 = fmaxf(bm1, fmaxf(s[k][1], s[k][3]));
+  }
+  st.mx[0] = fmaxf(st.mx[0], bm0);
+  st.mx[1] = fmaxf(st.mx[1], bm1);
+  if (__any_sync(0xffffffffu, bm0 > st.m[0] + kLazy || bm1 > st.m[1] + kLazy)) {
+#pragma unroll
+    for (int off = 4; off < 32; off <<= 1) {
+      bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, off));
+      bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, off));
+    }
+    const float mn0 = fmaxf(st.m[0], bm0), mn1 = fmaxf(st.m[1], bm1);
+    const float c0 = mn0 == st.m[0] ? 1.f : fast_exp2((st.m[0] - mn0) * kLog2e);
+    const float c1 = mn1 == st.m[1] ? 1.f : fast_exp2((st.m[1] - mn1) * kLog2e);
+    st.l[0] *= c0;
+    st.l[1] *= c1;
+#pragma unroll
+    for (int mt = 0; mt < 8; ++mt) {
+      o[mt][0] *= c0;
+      o[mt][1] *= c1;
+      o[mt][2] *= c0;
+      o[mt][3] *= c1;
+    }
+#pragma unroll
+    for (int i = 0; i < NB; ++i) {
+      ob[i][0] *= c0;
+      ob[i][1] *= c1;
+      ob[i][2] *= c0;
+      ob[i][3] *= c1;
+    }
+    st.m[0] = mn0;
+    st.m[1] = mn1;
+  }
+  const float ml0 = st.m[0] * kLog2e, ml1 = st.m[1] * kLog2e;
+#pragma unroll
+  for (int k = 0; k < NK; ++k) {
+    p[k][0] = fast_exp2(fmaf(s[k][0], kLog2e, -ml0));
+    p[k][1] = fast_exp2(fmaf(s[k][1], kLog2e, -ml1));
+    p[k][2] = fast_exp2(fmaf(s[k][2], kLog2e, -ml0));
+    p[k][3] = fast_exp2(fmaf(s[k][3], kLog2e, -ml1));
+    st.l[0] += p[k][0] + p[k][2];
+    st.l[1] += p[k][1] + p[k][3];
+  }
+}
+
+// Scale raw dot products, mask tokens >= valid, and store important-set logits.
+template <int G>
+__device__ __forceinline__ void finish_logits(const float (&acc)[4], float scale, int valid, int g, int t,
+                                              float* logit_base, int hi_stride, int slot0, float (&s)[4]) {
+  s[0] = acc[0] * scale;
+  s[1] = acc[1] * scale;
+  s[2] = acc[2] * scale;
+  s[3] = acc[3] * scale;
+  if (valid < 16) {
+    if (g >= valid) s[0] = s[1] = -INFINITY;
+    if (g + 8 >= valid) s[2] = s[3] = -INFINITY;
+  }
+  if (logit_base) {
+    const int h0 = 2 * t, h1 = 2 * t + 1;
+    if (h0 < G) {
+      if (g < valid) logit_base[(size_t)h0 * hi_stride + slot0 + g] = s[0];
+      if (g + 8 < valid) logit_base[(size_t)h0 * hi_stride + slot0 + g + 8] = s[2];
+    }
+    if (h1 < G) {
+      if (g < valid) logit_base[(size_t)h1 * hi_stride + slot0 + g] = s[1];
+      if (g + 8 < valid) logit_base[(size_t)h1 * hi_stride + slot0 + g + 8] = s[3];
+    }
+  }
+}
+
+// ---------------------------------------------------------------------- code extraction
+//
+// A 32-bit fragment register holds two 16-bit units (two channels or two tokens) whose codes sit at
+// the same bit positions. OR-ing the masked code bits under the fp16 exponent of 2^(10 - pos) gives
+// the exact value 2^(10 - pos) + code (the code's lowest bit then weighs 1); HSUB2 of that power of
+// two leaves the exact code. Positions 10 and up lie in the exponent field and are shifted down first.
+
+__device__ __forceinline__ uint32_t exact_codes(uint32_t x_with_magic, uint32_t magic2) {
+  return h2_as_u32(__hsub2(u32_as_h2(x_with_magic), u32_as_h2(magic2)));
+}
+
+__device__ __forceinline__ uint32_t mag2(int j) {  // fp16 pair 2^(10 - 2j), j = 0..4
+  return j == 0 ? 0x64006400u : j == 1 ? 0x5C005C00u : j == 2 ? 0x54005400u : j == 3 ? 0x4C004C00u : 0x44004400u;
+}
+
+// 2-bit code j (0..7) of each unit of r (r10 = r >> 10): exact fp16 pair.
+__device__ __forceinline__ uint32_t code2(uint32_t r, uint32_t r10, int j) {
+  if (j < 5) return exact_codes(and_or(r, 0x00030003u << (2 * j), mag2(j)), mag2(j));
+  const int jj = j - 5;
+  return exact_codes(and_or(r10, 0x00030003u << (2 * jj), mag2(jj)), mag2(jj));
+}
+
+// 4-bit code p (0..3) of each unit of r (r8 = r >> 8): exact fp16 pair (magics 2^10 and 2^6).
+__device__ __forceinline__ uint32_t code4(uint32_t r, uint32_t r8, int p) {
+  const uint32_t src = p < 2 ? r : r8;
+  const int pp = p & 1;
+  const uint32_t mag = pp ? 0x54005400u : 0x64006400u;
+  return exact_codes(and_or(src, 0x000F000Fu << (4 * pp), mag), mag);
+}
+
+// 8-bit code: the low (hi = 0) or high (hi = 1) byte of each unit of r, under the exponent of 1024.
+__device__ __forceinline__ uint32_t code8(uint32_t r, int hi) {
+  return exact_codes(prmt(r, 0x64646464u, hi ? 0x4341u : 0x4240u), 0x64006400u);
+}
+
+// 3-bit code: bits 0..1 at position j of r, bit 2 at bit hb of each unit of h.
+__device__ __forceinline__ uint32_t code3(uint32_t r, uint32_t h, int j, int hb) {
+  const uint32_t lo = and_or(r >> (2 * j), 0x00030003u, 0x64006400u);
+  return exact_codes(lo | (((h >> hb) << 2) & 0x00040004u), 0x64006400u);
+}
+
+// Value codes (N = 2, 4) skip the subtraction: the code is placed at a mantissa position where it
+// weighs 1 under a magic M in {4, 16, 64}, so the fp16 pair holds M + code exactly. The PV sums then
+// carry M * sum(p * alpha) per channel on top of the wanted sum; that term is measured by a ones-row
+// MMA on the same fp16 operands and removed in write_partial. M stays small (<= 64) so the removal
+// costs only a few bits of the fp32 accumulator.
+// N = 2: code j of r sits at bits 2j of each unit. Codes 0..2 are read from r << 4 (bits 4, 6, 8), codes
+// 3, 4 from r itself (bits 6, 8), codes 5..7 from r >> 6 (bits 4, 6, 8): offsets 64, 16, 4, 16, 4, 64, 16, 4.
+__device__ __forceinline__ uint32_t vcode2(uint32_t rl4, uint32_t r, uint32_t rr6, int j) {
+  const uint32_t src = j < 3 ? rl4 : (j < 5 ? r : rr6);
+  const int pos = j < 3 ? j + 2 : (j < 5 ? j : j - 3);  // 2-bit field index of the code in src
+  return and_or(src, 0x00030003u << (2 * pos), mag2(pos));
+}
+__host__ __device__ constexpr float voff2(int j) {
+  return (j == 0 || j == 5) ? 64.f : (j == 2 || j == 4 || j == 7) ? 4.f : 16.f;
+}
+// N = 4: nibble p of r at bits 4p. Nibbles 0 and 1 are read at bits 4..7 of r << 4 and r (M = 64),
+// nibbles 2 and 3 at bits 6..9 of r >> 2 and r >> 6 (M = 16).
+__device__ __forceinline__ uint32_t vcode4(const uint32_t (&sh)[4], int p) {
+  return p < 2 ? and_or(sh[p], 0x00F000F0u, 0x54005400u) : and_or(sh[p], 0x03C003C0u, 0x4C004C00u);
+}
+__host__ __device__ constexpr float voff4(int p) { return p < 2 ? 64.f : 16.f; }
+
+template <int BITS>
+__host__ __device__ constexpr float voff(int mt) {
+  return BITS == 2 ? voff2(mt) : BITS == 4 ? voff4(mt & 3) : 0.f;
+}
+
+// ---------------------------------------------------------------------- one important block
+
+template <int G, int NB>
+__device__ __forceinline__ void process_hi(uint32_t blk, int valid, int slot0, const uint32_t (&qb)[8][2],
+                                           float scale, float* logit_base, int hi_stride, Softmax& st,
+                                           float (&o)[8][4], float (&ob)[NB][4], int lane) {
+  const int g = lane >> 2, t = lane & 3, r8 = lane & 7, j = lane >> 3;
+  float accs[kQkAcc][4];
+#pragma unroll
+  for (int q = 0; q < kQkAcc; ++q) accs[q][0] = accs[q][1] = accs[q][2] = accs[q][3] = 0.f;
+  const int krow = r8 + 8 * (j & 1);
+#pragma unroll
+  for (int ks = 0; ks < 8; ++ks) {
+    const int chunk = 2 * (ks & 3) + (j >> 1);
+    uint32_t a[4];
+    ldsm_x4(blk + (ks >> 2) * 2048 + krow * 128 + ((chunk ^ (krow & 7)) << 4), a);
+    mma_bf16(accs[ks % kQkAcc], a, qb[ks][0], qb[ks][1]);
+  }
+  float acc[4];
+  sum_acc(accs, acc);
+  float s[1][4], p[1][4];
+  finish_logits<G>(acc, scale, valid, g, t, logit_base, hi_stride, slot0, s[0]);
+  softmax_blocks(s, st, o, ob, p);
+  const uint32_t pb0 = movmatrix_t(pack_bf16(p[0][0], p[0][1]));
+  const uint32_t pb1 = movmatrix_t(pack_bf16(p[0][2], p[0][3]));
+  uint32_t m01 = 0xffffffffu, m89 = 0xffffffffu;
+  if (valid < 16) {
+    m01 = (2 * t < valid ? 0x0000ffffu : 0u) | (2 * t + 1 < valid ? 0xffff0000u : 0u);
+    m89 = (2 * t + 8 < valid ? 0x0000ffffu : 0u) | (2 * t + 9 < valid ? 0xffff0000u : 0u);
+  }
+  const int vtok = r8 + 8 * (j >> 1);
+#pragma unroll
+  for (int mt = 0; mt < 8; ++mt) {
+    const int chunk = 2 * (mt & 3) + (j & 1);
+    uint32_t a[4];
+    ldsm_x4_t(blk + 4096 + (mt >> 2) * 2048 + vtok * 128 + ((chunk ^ (vtok & 7)) << 4), a);
+    if (valid < 16) {  // rows past the end may hold any bits: zero them (P is 0 there, NaN * 0 is not)
+      a[0] &= m01;
+      a[1] &= m01;
+      a[2] &= m89;
+      a[3] &= m89;
+    }
+    mma_bf16(o[mt], a, pb0, pb1);
+  }
+}
+
+// ---------------------------------------------------------------------- one retained block
+
+// Key side of coded block b of a unit (retained, or coded important with logit_base set): scaled
+// logits s, -inf past valid; important-set logits are also stored at logit_base[head][slot0 + token].
+template <int BITS, int GROUP, int G, int QACC>
+__device__ __forceinline__ void lo_logits(uint32_t unit, int b, int valid, const uint32_t (&qh)[8][2], float scale,
+                                          float (&s)[4], int lane, float* logit_base = nullptr, int hi_stride = 0,
+                                          int slot0 = 0) {
+  constexpr LoUnit U = lo_unit_layout(BITS, GROUP);
+  constexpr int NG = kHeadDim / GROUP;
+  constexpr int PR = U.param_row;
+  // this block's rows inside the unit's sections
+  const uint32_t ka = unit + U.k_a + b * 16 * U.pitch;
+  const uint32_t kp = unit + U.k_p + b * 16 * PR;
+  constexpr int NR = BITS == 4 ? 8 : 4;
+  const int g = lane >> 2, t = lane & 3, r8 = lane & 7, j = lane >> 3;
+
+  uint32_t pk0[NG], pk1[NG];
+  lds_vec<NG>(kp + g * PR, pk0);
+  lds_vec<NG>(kp + (g + 8) * PR, pk1);
+  float accs[QACC][4];
+#pragma unroll
+  for (int q = 0; q < QACC; ++q) accs[q][0] = accs[q][1] = accs[q][2] = accs[q][3] = 0.f;
+  if constexpr (BITS == 8) {
+    // 128-byte token rows under the 128B swizzle; channels 32 i .. 32 i + 31 (ks = 2 i, 2 i + 1) share
+    // one ldmatrix: each 16-bit unit holds the code of ks = 2 i (low byte) and ks = 2 i + 1 (high byte)
+    const int tok = r8 + 8 * (j & 1);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      uint32_t r[4];
+      ldsm_x4(ka + tok * 128 + (((2 * i + (j >> 1)) ^ (tok & 7)) << 4), r);
+#pragma unroll
+      for (int hb = 0; hb < 2; ++hb) {
+        const int ks = 2 * i + hb, gi = (16 * ks) / GROUP;
+        const __half2 p0 = u32_as_h2(pk0[gi]), p1 = u32_as_h2(pk1[gi]);
+        const __half2 al0 = __low2half2(p0), be0 = __high2half2(p0);
+        const __half2 al1 = __low2half2(p1), be1 = __high2half2(p1);
+        const uint32_t a[4] = {h2_as_u32(__hfma2(u32_as_h2(code8(r[0], hb)), al0, be0)),
+                               h2_as_u32(__hfma2(u32_as_h2(code8(r[1], hb)), al1, be1)),
+                               h2_as_u32(__hfma2(u32_as_h2(code8(r[2], hb)), al0, be0)),
+                               h2_as_u32(__hfma2(u32_as_h2(code8(r[3], hb)), al1, be1))};
+        mma_f16(accs[ks % QACC], a, qh[ks][0], qh[ks][1]);
+      }
+    }
+    float acc[4];
+    sum_acc(accs, acc);
+    finish_logits<G>(acc, scale, valid, g, t, logit_base, hi_stride, slot0, s);
+    return;
+  }
+
+  // ---- keys of tokens g and g+8
+  uint32_t kr[NR], kh[NR];
+  uint32_t kb0 = 0, kb1 = 0;
+  {
+    const int tok = r8 + 8 * (j & 1);
+    if (BITS == 4) {
+      const int o0 = tok * 64 + 16 * (j >> 1), sw = ((tok >> 1) & 3) << 4;
+      uint32_t r0[4], r1[4];
+      ldsm_x4(ka + (o0 ^ sw), r0);
+      ldsm_x4(ka + ((o0 + 32) ^ sw), r1);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        kr[i] = r0[i];
+        kr[(NR == 8 ? 4 : 0) + i] = r1[i];
+      }
+    } else {
+      // N = 2: 32-byte tokens under the 64B swizzle (bits 4..5 ^= bits 7..8); N = 3: 48-byte tokens, unswizzled
+      const int o0 = tok * U.pitch + 16 * (j >> 1), sw = BITS == 2 ? ((tok >> 2) & 3) << 4 : 0;
+      uint32_t r0[4];
+      ldsm_x4(ka + (o0 ^ sw), r0);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) kr[i] = r0[i];
+      if (BITS == 3) ldsm_x2(ka + (lane & 15) * U.pitch + U.plane_b, kb0, kb1);
+    }
+#pragma unroll
+    for (int i = 0; i < NR; ++i) kh[i] = kr[i] >> (BITS == 4 ? 8 : 10);
+  }
+#pragma unroll
+  for (int ks = 0; ks < 8; ++ks) {
+    const int gi = (16 * ks) / GROUP;
+    // (alpha, alpha) and (beta, beta) of tokens g and g + 8: half-broadcasts the HFMA2 operand selectors absorb
+    const __half2 p0 = u32_as_h2(pk0[gi]), p1 = u32_as_h2(pk1[gi]);
+    const uint32_t al0 = h2_as_u32(__low2half2(p0)), be0 = h2_as_u32(__high2half2(p0));
+    const uint32_t al1 = h2_as_u32(__low2half2(p1)), be1 = h2_as_u32(__high2half2(p1));
+    uint32_t c[4];
+    if (BITS == 4) {
+      const int ri = (ks >> 2) * 4, p = ks & 3;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) c[i] = code4(kr[ri + i], kh[ri + i], p);
+    } else if (BITS == 2) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) c[i] = code2(kr[i], kh[i], ks);
+    } else {
+      c[0] = code3(kr[0], kb0, ks, ks);
+      c[1] = code3(kr[1], kb1, ks, ks);
+      c[2] = code3(kr[2], kb0, ks, 8 + ks);
+      c[3] = code3(kr[3], kb1, ks, 8 + ks);
+    }
+    const uint32_t a[4] = {h2_as_u32(__hfma2(u32_as_h2(c[0]), u32_as_h2(al0), u32_as_h2(be0))),
+                           h2_as_u32(__hfma2(u32_as_h2(c[1]), u32_as_h2(al1), u32_as_h2(be1))),
+                           h2_as_u32(__hfma2(u32_as_h2(c[2]), u32_as_h2(al0), u32_as_h2(be0))),
+                           h2_as_u32(__hfma2(u32_as_h2(c[3]), u32_as_h2(al1), u32_as_h2(be1)))};
+    mma_f16(accs[ks % QACC], a, qh[ks][0], qh[ks][1]);
+  }
+  float acc[4];
+  sum_acc(accs, acc);
+  finish_logits<G>(acc, scale, valid, g, t, logit_base, hi_stride, slot0, s);
+}
+
+// Value side of coded block b: o, ob += P (this block's probabilities p) times the block's values.
+// EXACT (coded important blocks): codes enter the MMA as exact integers, so the block adds nothing to
+// the alpha sums that remove the retained set's code offsets.
+template <int BITS, int GROUP, int NB, bool EXACT>
+__device__ __forceinline__ void lo_values(uint32_t unit, int b, int valid, const float (&p)[4], float (&o)[8][4],
+                                          float (&ob)[NB][4], int lane) {
+  constexpr LoUnit U = lo_unit_layout(BITS, GROUP);
+  constexpr int NG = kHeadDim / GROUP;
+  constexpr int PR = U.param_row;
+  const uint32_t va = unit + U.v_a + b * 16 * U.pitch;
+  const uint32_t vp = unit + U.v_p + b * 16 * PR;
+  constexpr int NR = BITS == 4 ? 8 : 4;
+  const int g = lane >> 2, t = lane & 3, r8 = lane & 7, j = lane >> 3;
+  const uint32_t pb0 = movmatrix_t(pack_f16(p[0], p[1]));  // (P[2t][head g], P[2t+1][head g])
+  const uint32_t pb1 = movmatrix_t(pack_f16(p[2], p[3]));  // tokens 2t+8, 2t+9
+
+  // ---- values of tokens (2t, 2t+1) and (2t+8, 2t+9), channels 16 mt + g and 16 mt + 8 + g
+  uint32_t vr[NR];
+  uint32_t vb0 = 0, vb1 = 0;
+  const int vtok = r8 + 8 * (j >> 1);
+  if constexpr (BITS != 8) {
+    const int tok = vtok;
+    if (BITS == 4) {
+      const int o0 = tok * 64 + 16 * (j & 1), sw = ((tok >> 1) & 3) << 4;
+      uint32_t r0[4], r1[4];
+      ldsm_x4_t(va + (o0 ^ sw), r0);
+      ldsm_x4_t(va + ((o0 + 32) ^ sw), r1);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        vr[i] = r0[i];
+        vr[(NR == 8 ? 4 : 0) + i] = r1[i];
+      }
+    } else {
+      const int o0 = tok * U.pitch + 16 * (j & 1), sw = BITS == 2 ? ((tok >> 2) & 3) << 4 : 0;
+      uint32_t r0[4];
+      ldsm_x4_t(va + (o0 ^ sw), r0);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) vr[i] = r0[i];
+      if (BITS == 3) ldsm_x2_t(va + (lane & 15) * U.pitch + U.plane_b, vb0, vb1);
+    }
+  }
+  // (alpha, beta) of the four tokens for every group; zero past the end (exact zeros in the sums)
+  const int t0 = 2 * t, t1 = 2 * t + 1, t8 = 2 * t + 8, t9 = 2 * t + 9;
+  uint32_t pv0[NG], pv1[NG], pv8[NG], pv9[NG];
+  lds_vec<NG>(vp + t0 * PR, pv0);
+  lds_vec<NG>(vp + t1 * PR, pv1);
+  lds_vec<NG>(vp + t8 * PR, pv8);
+  lds_vec<NG>(vp + t9 * PR, pv9);
+  // zero rows: row r < 4 of the beta operand holds, for this thread's tokens, beta of the group that
+  // contains channels 32 r .. 32 r + 31 (a granularity the important and retained sets share)
+  uint32_t bw0 = 0, bw1 = 0, bw8 = 0, bw9 = 0;
+  if (g < 4) {
+    const int pidx = (32 * g) / GROUP;
+    bw0 = lds32(vp + t0 * PR + 4 * pidx);
+    bw1 = lds32(vp + t1 * PR + 4 * pidx);
+    bw8 = lds32(vp + t8 * PR + 4 * pidx);
+    bw9 = lds32(vp + t9 * PR + 4 * pidx);
+  }
+  if (valid < 16) {
+#pragma unroll
+    for (int gi = 0; gi < NG; ++gi) {
+      if (t0 >= valid) pv0[gi] = 0u;
+      if (t1 >= valid) pv1[gi] = 0u;
+      if (t8 >= valid) pv8[gi] = 0u;
+      if (t9 >= valid) pv9[gi] = 0u;
+    }
+    if (t0 >= valid) bw0 = 0u;
+    if (t1 >= valid) bw1 = 0u;
+    if (t8 >= valid) bw8 = 0u;
+    if (t9 >= valid) bw9 = 0u;
+  }
+  {
+    const uint32_t a[4] = {prmt(bw0, bw1, 0x7632u), 0u, prmt(bw8, bw9, 0x7632u), 0u};
+    mma_f16(ob[0], a, pb0, pb1);  // ob[0][row r][heads 2t, 2t+1] += sum over tokens of p * beta
+  }
+  uint32_t pa0[NG], pa1[NG];  // p * alpha per group: B operand of the code MMAs
+#pragma unroll
+  for (int gi = 0; gi < NG; ++gi) {
+    pa0[gi] = h2_as_u32(__hmul2(u32_as_h2(pb0), u32_as_h2(prmt(pv0[gi], pv1[gi], 0x5410u))));
+    pa1[gi] = h2_as_u32(__hmul2(u32_as_h2(pb1), u32_as_h2(prmt(pv8[gi], pv9[gi], 0x5410u))));
+  }
+  if (!EXACT && BITS != 3) {
+    // sum of p * alpha per group, from the same fp16 operands as the code MMAs: ones in rows 0..7
+    // (even groups) or 8..15 (odd groups), so ob[1 + gi / 2] holds two groups per fragment
+    constexpr uint32_t kOne = 0x3C003C00u;
+#pragma unroll
+    for (int gi = 0; gi < NG; ++gi) {
+      const uint32_t e = (gi & 1) ? 0u : kOne, d = (gi & 1) ? kOne : 0u;
+      const uint32_t a[4] = {e, d, e, d};
+      mma_f16(ob[1 + gi / 2], a, pa0[gi], pa1[gi]);
+    }
+  }
+  if constexpr (BITS == 8) {
+    // channels 32 i .. 32 i + 31 (mt = 2 i, 2 i + 1) share one transposed ldmatrix, as for the keys
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      uint32_t r[4];
+      ldsm_x4_t(va + vtok * 128 + (((2 * i + (j & 1)) ^ (vtok & 7)) << 4), r);
+#pragma unroll
+      for (int hb = 0; hb < 2; ++hb) {
+        const int mt = 2 * i + hb, gi = (16 * mt) / GROUP;
+        const uint32_t a[4] = {code8(r[0], hb), code8(r[1], hb), code8(r[2], hb), code8(r[3], hb)};
+        mma_f16(o[mt], a, pa0[gi], pa1[gi]);
+      }
+    }
+    return;
+  }
+#pragma unroll
+  for (int mt = 0; mt < 8; ++mt) {
+    const int gi = (16 * mt) / GROUP;
+    uint32_t a[4];
+    if (BITS == 4) {
+      const int ri = (mt >> 2) * 4, pp = mt & 3;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const uint32_t w = vr[ri + i];
+        if (EXACT) {
+          a[i] = code4(w, w >> 8, pp);
+        } else {
+          const uint32_t c4[4] = {w << 4, w, w >> 2, w >> 6};  // shared by the four mt of this word
+          a[i] = vcode4(c4, pp);
+        }
+      }
+    } else if (BITS == 2) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        if (EXACT)
+          a[i] = code2(vr[i], vr[i] >> 10, mt);
+        else
+          a[i] = vcode2(vr[i] << 4, vr[i], vr[i] >> 6, mt);  // the shifted copies are shared by all mt
+      }
+    } else {
+      a[0] = code3(vr[0], vb0, mt, mt);
+      a[1] = code3(vr[1], vb0, mt, 8 + mt);
+      a[2] = code3(vr[2], vb1, mt, mt);
+      a[3] = code3(vr[3], vb1, mt, 8 + mt);
+    }
+    mma_f16(o[mt], a, pa0[gi], pa1[gi]);  // sums p * alpha * (code + offset)
+  }
+}
+
+// NK consecutive coded blocks b .. b + NK - 1 of a unit (n_left = valid tokens from block b on, at
+// least 16 (NK - 1) + 1): the key sides first, one softmax update over all NK blocks, then the value
+// sides, so the dependency chains of the blocks overlap. HI: blocks of a coded important set (logits
+// stored for the importance update, exact value codes); slot0 = important slot of block b's first row.
+template <int BITS, int GROUP, int G, int NB, int NK, bool HI>
+__device__ __forceinline__ void process_coded(uint32_t unit, int b, int n_left, const uint32_t (&qh)[8][2],
+                                              float scale, Softmax& st, float (&o)[8][4], float (&ob)[NB][4],
+                                              int lane, float* logit_base = nullptr, int hi_stride = 0,
+                                              int slot0 = 0) {
+  float s[NK][4], p[NK][4];
+#pragma unroll
+  for (int k = 0; k < NK; ++k)
+    lo_logits<BITS, GROUP, G, NK == 1 ? kQkAcc : kPairAcc>(unit, b + k, min(16, n_left - 16 * k), qh, scale, s[k],
+                                                           lane, HI ? logit_base : nullptr, hi_stride, slot0 + 16 * k);
+  softmax_blocks(s, st, o, ob, p);
+#pragma unroll
+  for (int k = 0; k < NK; ++k)
+    lo_values<BITS, GROUP, NB, HI>(unit, b + k, min(16, n_left - 16 * k), p[k], o, ob, lane);
+}
+
+// Write this warp's partial for one head: output (plus the zero-row terms, minus the value-code offsets),
+// true max and sum. The running sums are at the reference max m; they are rescaled here to the largest
+// logit seen, so the partial's (max, sum) are the exact statistics of its tokens.
+template <int BITS, int GROUP, int G, int NB>
+__device__ __forceinline__ void write_partial(const AttnArgs& a, int slot, Softmax& st, const float (&o)[8][4],
+                                              const float (&ob)[NB][4], int lane) {
+  const int g = lane >> 2, t = lane & 3;
+#pragma unroll
+  for (int off = 4; off < 32; off <<= 1) {
+    st.l[0] += __shfl_xor_sync(0xffffffffu, st.l[0], off);
+    st.l[1] += __shfl_xor_sync(0xffffffffu, st.l[1], off);
+    st.mx[0] = fmaxf(st.mx[0], __shfl_xor_sync(0xffffffffu, st.mx[0], off));
+    st.mx[1] = fmaxf(st.mx[1], __shfl_xor_sync(0xffffffffu, st.mx[1], off));
+  }
+  float c[2];
+#pragma unroll
+  for (int hd = 0; hd < 2; ++hd)  // m <= mx <= m + kLazy; equal (also both -inf) gives 1
+    c[hd] = st.mx[hd] == st.m[hd] ? 1.f : fast_exp2((st.m[hd] - st.mx[hd]) * kLog2e);
+  float bz0[4], bz1[4];  // sum p * beta over channels 32 r .. 32 r + 31, heads 2t, 2t+1: lane 4 r + t
+#pragma unroll
+  for (int r = 0; r < 4; ++r) {
+    bz0[r] = __shfl_sync(0xffffffffu, ob[0][0], r * 4 + t);
+    bz1[r] = __shfl_sync(0xffffffffu, ob[0][1], r * 4 + t);
+  }
+#pragma unroll
+  for (int hd = 0; hd < 2; ++hd) {
+    const int head = 2 * t + hd;
+    if (head < G) {
+      float* po = a.part_o + ((size_t)slot * G + head) * kHeadDim;
+#pragma unroll
+      for (int mt = 0; mt < 8; ++mt) {
+        const int gi = (16 * mt) / GROUP;
+        float z = hd ? bz1[mt >> 1] : bz0[mt >> 1];
+        if (BITS != 3) z = fmaf(-voff<BITS>(mt), ob[1 + gi / 2][2 * (gi & 1) + hd], z);
+        po[16 * mt + g] = (o[mt][hd] + z) * c[hd];
+        po[16 * mt + 8 + g] = (o[mt][2 + hd] + z) * c[hd];
+      }
+      if (g == 0) {
+        a.part_ml[((size_t)slot * G + head) * 2] = st.mx[hd];
+        a.part_ml[((size_t)slot * G + head) * 2 + 1] = st.l[hd] * c[hd];
+      }
+    }
+  }
+}
+
+template <int BITS, int GROUP, int HB>
+__device__ __forceinline__ void issue_unit(const AttnArgs& a, const Cursor& c, uint32_t dst, uint32_t bar) {
+  constexpr LoUnit U = lo_unit_layout(BITS, GROUP);
+  const UnitKind k = cursor_kind(c, a.hi_units, a.n_u);
+  if constexpr (HB != 16) {
+    if (k.hi) {
+      constexpr LoUnit H = lo_unit_layout(HB, kHiGroup);
+      const long long row = (long long)c.bh * a.hi_stride + 16 * H.blocks * k.index;  // first slot
+      mbar_arrive_expect_tx(bar, H.tx);
+      const int crow = (int)(row * H.pitch / H.map_w), prow = (int)(row * H.param_row / H.param_w);
+      tma_load_2d(dst + H.k_a, &a.map_k_hi, 0, crow, bar);
+      tma_load_2d(dst + H.v_a, &a.map_v_hi, 0, crow, bar);
+      tma_load_2d(dst + H.k_p, &a.map_k_hp, 0, prow, bar);
+      tma_load_2d(dst + H.v_p, &a.map_v_hp, 0, prow, bar);
+      return;
+    }
+  }
+  if (k.hi) {
+    const int row = c.bh * a.hi_stride + 16 * k.index;
+    mbar_arrive_expect_tx(bar, kHiBlockBytes);
+    tma_load_2d(dst, &a.map_k_hi, 0, row, bar);
+    tma_load_2d(dst + 2048, &a.map_k_hi, 64, row, bar);
+    tma_load_2d(dst + 4096, &a.map_v_hi, 0, row, bar);
+    tma_load_2d(dst + 6144, &a.map_v_hi, 64, row, bar);
+  } else {
+    // one box per array covers the whole unit (U.blocks blocks of 16 rows); rows past this head's
+    // retained length are masked by the consumer, rows past the array are zero-filled by TMA
+    const long long row = (long long)c.bh * a.lo_cap + 16 * U.blocks * k.index;  // first token row
+    mbar_arrive_expect_tx(bar, U.tx);
+    const int crow = (int)(row * U.pitch / U.map_w), prow = (int)(row * U.param_row / U.param_w);
+    tma_load_2d(dst + U.k_a, &a.map_k_lo, 0, crow, bar);
+    tma_load_2d(dst + U.v_a, &a.map_v_lo, 0, crow, bar);
+    tma_load_2d(dst + U.k_p, &a.map_k_par, 0, prow, bar);
+    tma_load_2d(dst + U.v_p, &a.map_v_par, 0, prow, bar);
+  }
+}
+
+__device__ __forceinline__ void fence_proxy_async() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+template <int BITS, int GROUP, int HB, int G>
+__global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const __grid_constant__ AttnArgs a) {
+  constexpr LoUnit U = lo_unit_layout(BITS, GROUP);
+  constexpr LoUnit H = lo_unit_layout(HB == 16 ? 2 : HB, kHiGroup);
+  static_assert(U.total <= kStageBytes && H.total <= kStageBytes, "unit too large for a stage");
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int wg = blockIdx.x * kWarps + warp;
+  if (wg >= a.n_warps) return;  // no block-wide synchronisation follows
+  const uint32_t ring = base + warp * kNS * kStageBytes;
+  const uint32_t bars = base + kWarps * kNS * kStageBytes + warp * kNS * 8;
+  const int u0 = (int)((long long)wg * a.n_units / a.n_warps);
+  const int u1 = (int)((long long)(wg + 1) * a.n_units / a.n_warps);
+  const int hu = a.hi_units, n_u = a.n_u;
+  Cursor ci = cursor_at(u0, hu, n_u);  // next unit to issue (lane 0)
+  if (lane == 0) {
+    for (int s = 0; s < kNS; ++s) mbar_init(bars + 8 * s, 1);
+    fence_mbar_init();
+    prefetch_tensormap(&a.map_k_hi);
+    prefetch_tensormap(&a.map_v_hi);
+    if (HB != 16) {
+      prefetch_tensormap(&a.map_k_hp);
+      prefetch_tensormap(&a.map_v_hp);
+    }
+    if (a.lo_blocks > 0) {  // the retained-set maps are only encoded when the retained arrays exist
+      prefetch_tensormap(&a.map_k_lo);
+      prefetch_tensormap(&a.map_v_lo);
+      prefetch_tensormap(&a.map_k_par);
+      prefetch_tensormap(&a.map_v_par);
+    }
+    for (int k = 0; k < kNS && u0 + k < u1; ++k) {
+      issue_unit<BITS, GROUP, HB>(a, ci, ring + k * kStageBytes, bars + 8 * k);
+      cursor_next(ci, hu, n_u);
+    }
+  }
+  __syncwarp();
+
+  const int g = lane >> 2, t = lane & 3;
+  uint32_t qb[8][2], qh[8][2];
+  constexpr int NB = 1 + (BITS == 3 ? 0 : (kHeadDim / GROUP + 1) / 2);  // beta rows + alpha-sum pairs
+  Softmax st;
+  float o[8][4], ob[NB][4];
+  float* logit_base = nullptr;
+  Cursor cc = cursor_at(u0, hu, n_u);  // unit being consumed
+  int cur = -1;
+  bool failed = false;
+  int u = u0;
+  for (; u < u1; ++u) {
+    if (cc.bh != cur) {
+      if (cur >= 0) write_partial<BITS, GROUP, G, NB>(a, wg + cur, st, o, ob, lane);
+      cur = cc.bh;
+      const int b = cur / a.heads_kv, h = cur - b * a.heads_kv;
+      // query fragments (B operand: head g; channels 16 ks + 2t (+1) and 16 ks + 2t + 8 (+9))
+      if (g < G) {
+        const __nv_bfloat16* qp =
+            static_cast<const __nv_bfloat16*>(a.q) + (size_t)(b * a.heads_q + h * G + g) * kHeadDim;
+#pragma unroll
+        for (int ks = 0; ks < 8; ++ks)
+#pragma unroll
+          for (int r = 0; r < 2; ++r) {
+            const int c = 16 * ks + 2 * t + 8 * r;
+            const uint32_t w = *reinterpret_cast<const uint32_t*>(qp + c);
+            qb[ks][r] = w;
+            const float q0 = __uint_as_float(w << 16), q1 = __uint_as_float(w & 0xffff0000u);
+            const float b0 = a.balancer ? a.balancer[h * kHeadDim + c] : 1.f;
+            const float b1 = a.balancer ? a.balancer[h * kHeadDim + c + 1] : 1.f;
+            qh[ks][r] = pack_f16(__fdiv_rn(q0, b0), __fdiv_rn(q1, b1));  // Eq. 4
+          }
+      } else {
+#pragma unroll
+        for (int ks = 0; ks < 8; ++ks) qb[ks][0] = qb[ks][1] = qh[ks][0] = qh[ks][1] = 0u;
+      }
+      logit_base = a.hi_logits ? a.hi_logits + (size_t)(b * a.heads_q + h * G) * a.hi_stride : nullptr;
+      st.m[0] = st.m[1] = -INFINITY;
+      st.l[0] = st.l[1] = 0.f;
+      st.mx[0] = st.mx[1] = -INFINITY;
+#pragma unroll
+      for (int mt = 0; mt < 8; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
+#pragma unroll
+      for (int i = 0; i < NB; ++i) ob[i][0] = ob[i][1] = ob[i][2] = ob[i][3] = 0.f;
+    }
+    const int s = (u - u0) % kNS;
+    const uint32_t use = (u - u0) / kNS;
+    if (!mbar_wait(bars + 8 * s, use & 1)) {
+      record_error(a.status, kErrFullTimeout);
+      failed = true;
+      break;
+    }
+    const uint32_t stage = ring + s * kStageBytes;
+    const UnitKind k = cursor_kind(cc, hu, n_u);
+    if (k.hi) {
+      if constexpr (HB == 16) {
+        process_hi<G, NB>(stage, min(16, a.hi_cap - 16 * k.index), 16 * k.index, qb, a.sm_scale, logit_base,
+                          a.hi_stride, st, o, ob, lane);
+      } else {
+        const int first = k.index * H.blocks;
+        const int nb = min(H.blocks, a.hi_blocks - first);
+        int b = 0;
+        if (kLoPair)
+          for (; b + 1 < nb; b += 2)
+            process_coded<HB, kHiGroup, G, NB, 2, true>(stage, b, a.hi_cap - 16 * (first + b), qh, a.sm_scale, st,
+                                                        o, ob, lane, logit_base, a.hi_stride, 16 * (first + b));
+        for (; b < nb; ++b)
+          process_coded<HB, kHiGroup, G, NB, 1, true>(stage, b, a.hi_cap - 16 * (first + b), qh, a.sm_scale, st, o,
+                                                      ob, lane, logit_base, a.hi_stride, 16 * (first + b));
+      }
+    } else {
+      const int first = k.index * U.blocks;
+      const int nb = min(U.blocks, a.lo_blocks - first);
+      int b = 0;
+      if (kLoPair)
+        for (; b + 1 < nb; b += 2)
+          process_coded<BITS, GROUP, G, NB, 2, false>(stage, b, a.n_lo - 16 * (first + b), qh, a.sm_scale, st, o,
+                                                      ob, lane);
+      for (; b < nb; ++b)
+        process_coded<BITS, GROUP, G, NB, 1, false>(stage, b, a.n_lo - 16 * (first + b), qh, a.sm_scale, st, o, ob,
+                                                    lane);
+    }
+    cursor_next(cc, hu, n_u);
+    __syncwarp();
+    if (lane == 0 && u + kNS < u1) {
+      fence_proxy_async();  // our generic reads of this stage precede the next asynchronous write
+      issue_unit<BITS, GROUP, HB>(a, ci, stage, bars + 8 * s);
+      cursor_next(ci, hu, n_u);
+    }
+  }
+  if (failed) {
+    // leave no copy in flight into this warp's ring: wait (bounded) for every unit still issued
+    if (lane == 0)
+      for (int v = u; v < u1 && v < u + kNS; ++v) {
+        const int s = (v - u0) % kNS;
+        if (!mbar_wait(bars + 8 * s, ((v - u0) / kNS) & 1)) record_error(a.status, kErrDrainTimeout);
+      }
+    return;
+  }
+  if (cur >= 0) write_partial<BITS, GROUP, G, NB>(a, wg + cur, st, o, ob, lane);
+}
+
+template <int BITS, int GROUP, int HB, int G>
+cudaError_t launch_kernel(const AttnArgs& a, int grid, cudaStream_t st) {
+  auto kern = attention_kernel<BITS, GROUP, HB, G>;
+  static bool configured = false;
+  const int smem = smem_bytes();
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
+  kern<<<grid, kThreads, smem, st>>>(a);
+  return cudaGetLastError();
+}
+
+template <int BITS, int GROUP, int HB>
+cudaError_t dispatch_g(const AttnArgs& a, int G, int grid, cudaStream_t st) {
+  switch (G) {
+    case 1: return launch_kernel<BITS, GROUP, HB, 1>(a, grid, st);
+    case 2: return launch_kernel<BITS, GROUP, HB, 2>(a, grid, st);
+    case 4: return launch_kernel<BITS, GROUP, HB, 4>(a, grid, st);
+    case 8: return launch_kernel<BITS, GROUP, HB, 8>(a, grid, st);
+  }
+  return cudaErrorInvalidValue;
+}
+
+template <int BITS, int HB>
+cudaError_t dispatch_group(const AttnArgs& a, int group, int G, int grid, cudaStream_t st) {
+  switch (group) {
+    case 32: return dispatch_g<BITS, 32, HB>(a, G, grid, st);
+    case 64: return dispatch_g<BITS, 64, HB>(a, G, grid, st);
+    case 128: return dispatch_g<BITS, 128, HB>(a, G, grid, st);
+  }
+  return cudaErrorInvalidValue;
+}
+
+// Every (retained bits, group, G) kernel for one important-set precision HB (16 = bf16).
+template <int HB>
+cudaError_t launch_attention_hb(const AttnArgs& a, int bits, int group, int G, int grid, cudaStream_t st) {
+  switch (bits) {
+    case 2: return dispatch_group<2, HB>(a, group, G, grid, st);
+    case 3: return dispatch_group<3, HB>(a, group, G, grid, st);
+    case 4: return dispatch_group<4, HB>(a, group, G, grid, st);
+  }
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace
+}  // namespace mikv

@@ -34,17 +34,19 @@ __host__ __device__ constexpr int align_up(int x, int a) { return (x + a - 1) / 
 // A unit's rows of one array are contiguous in HBM (16 n tokens of one head), so TMA copies them as
 // wide rows: 64-byte rows with the 64B swizzle for N = 2 (two tokens per row) and N = 4 (one token),
 // unswizzled 128-byte rows for N = 3 (48-byte tokens, whose pitch alone spreads ldmatrix rows over all
-// banks). Few wide rows per unit keep the TMA request rate far below what HBM needs.
+// banks), 128-byte rows with the 128B swizzle for N = 8 (coded important sets only). Few wide rows per
+// unit keep the TMA request rate far below what HBM needs.
 __host__ __device__ constexpr LoUnit lo_unit_layout_n(int bits, int group, int n) {
   LoUnit u{};
   u.blocks = n;
   u.pitch = bits == 3 ? 48 : 16 * bits;
   u.plane_b = bits == 3 ? 32 : 0;
-  u.map_w = bits == 3 ? 128 : 64;
+  u.map_w = bits == 3 || bits == 8 ? 128 : 64;
   u.param_row = 4 * (128 / group);
   u.param_w = u.param_row == 4 ? 64 : 128;
   const int rows = 16 * n;
-  const int code_align = bits == 3 ? 128 : 512;  // the 64B swizzle pattern repeats every 512 bytes
+  // the 64B / 128B swizzle patterns repeat every 512 / 1024 bytes
+  const int code_align = bits == 3 ? 128 : (bits == 8 ? 1024 : 512);
   u.k_a = 0;
   u.v_a = align_up(u.k_a + rows * u.pitch, code_align);
   u.k_p = align_up(u.v_a + rows * u.pitch, 128);
@@ -61,11 +63,15 @@ __host__ __device__ constexpr LoUnit lo_unit_layout(int bits, int group) {
   return lo_unit_layout_n(bits, group, n);
 }
 
-// Attention work plan: per (b, kv-head) a sequence of n_u units (hi_units important blocks of 16
-// tokens, lo_units groups of retained blocks), all heads concatenated into n_units units and split
-// into n_warps equal contiguous shares; warp w writes the partial of head bh into slot w + bh.
+// Group size of a coded important set (Sec. 3.3, Table 3).
+constexpr int kHiGroup = 64;
+
+// Attention work plan: per (b, kv-head) a sequence of n_u units (hi_units important units: one bf16
+// block of 16 tokens, or lo_unit_layout(hi_bits, 64).blocks coded blocks; lo_units groups of retained
+// blocks), all heads concatenated into n_units units and split into n_warps equal contiguous shares;
+// warp w writes the partial of head bh into slot w + bh.
 struct AttnPlan {
-  int hi_units, lo_blocks, lo_units, n_u;
+  int hi_blocks, hi_units, lo_blocks, lo_units, n_u;
   int n_units;
   int n_warps;
   int grid;
@@ -73,7 +79,9 @@ struct AttnPlan {
 };
 
 struct AttnArgs {
-  CUtensorMap map_k_hi, map_v_hi;    // bf16 rows of 128 channels, box 64 x 16, 128B swizzle
+  CUtensorMap map_k_hi, map_v_hi;    // bf16 rows of 128 channels, box 64 x 16, 128B swizzle; or coded
+                                     // important rows viewed like retained codes (layout hi_bits, 64)
+  CUtensorMap map_k_hp, map_v_hp;    // coded important set: (alpha, beta) rows like map_k_par
   CUtensorMap map_k_lo, map_v_lo;    // packed codes viewed as rows of LoUnit::map_w bytes, box = one unit
   CUtensorMap map_k_par, map_v_par;  // (alpha, beta) pairs viewed as rows of LoUnit::param_w bytes
   const void* q;
@@ -83,7 +91,7 @@ struct AttnArgs {
   float* part_ml;  // [n_slots][G][2]
   int* status;
   int batch, heads_q, heads_kv, hi_cap, hi_stride, lo_cap, n_lo;
-  int hi_units, lo_blocks, n_u, n_units, n_warps;
+  int hi_blocks, hi_units, lo_blocks, n_u, n_units, n_warps;
   float sm_scale;
 };
 
@@ -113,6 +121,9 @@ struct StepPostArgs {
   void* v_params;
   int32_t* lo_tok;
   int32_t* slots;
+  const void* k_hi_params;  // coded important set: (alpha, beta) of the important rows
+  const void* v_hi_params;
+  int hi_bits;              // 16 = bf16 important rows; 8, 4, 2 = coded (groups of kHiGroup)
   int batch, heads_q, heads_kv, hi_cap, hi_stride, lo_cap, n_lo;
   int n_u, n_units, n_warps;
 };
@@ -121,12 +132,24 @@ cudaError_t launch_step_post(const StepPostArgs& a, int bits, int group, int G, 
 
 AttnPlan plan_attention(const mikv_shape& s, int n_lo, int num_sms);
 size_t attention_workspace_bytes(const mikv_shape& s, int n_lo_max, int num_sms);
-cudaError_t launch_attention(const AttnArgs& a, int bits, int group, int G, int grid, cudaStream_t st);
+cudaError_t launch_attention(const AttnArgs& a, int bits, int group, int hi_bits, int G, int grid, cudaStream_t st);
+// one translation unit per important-set precision (mikv_attn_h*.cu)
+cudaError_t launch_attention_h16(const AttnArgs& a, int bits, int group, int G, int grid, cudaStream_t st);
+cudaError_t launch_attention_h8(const AttnArgs& a, int bits, int group, int G, int grid, cudaStream_t st);
+cudaError_t launch_attention_h4(const AttnArgs& a, int bits, int group, int G, int grid, cudaStream_t st);
+cudaError_t launch_attention_h2(const AttnArgs& a, int bits, int group, int G, int grid, cudaStream_t st);
+// effective important-set precision of a shape: 16 for bf16 (hi_bits 0 or 16)
+inline int hi_bits_of(const mikv_shape& s) { return s.hi_bits == 0 ? 16 : s.hi_bits; }
 cudaError_t launch_merge(const MergeArgs& a, int G, int out_f32, cudaStream_t st);
 
 cudaError_t launch_quantize_pack(const mikv_shape& s, const mikv_cache& c, const void* k_src,
                                  const void* v_src, const int32_t* src_tok, int n_src,
                                  const int32_t* rows, int n_rows, int lo_start, cudaStream_t st);
+
+// insert (rows == nullptr, slots/tok used) or gather (rows/n_rows) into a coded important set
+cudaError_t launch_hi_quant(const mikv_shape& s, const mikv_cache& c, const void* k_src, const void* v_src,
+                            const int32_t* src_tok, const float* src_scores, int n_src, const int32_t* rows,
+                            int n_rows, const int32_t* slots, int tok, cudaStream_t st);
 
 cudaError_t launch_balancer(const mikv_shape& s, const void* q_pre, const void* k_pre, int T,
                             float* out, uint32_t* ws_max, cudaStream_t st);

@@ -206,6 +206,8 @@ cudaError_t launch_select(int batch, int heads, const float* scores, const int32
 
 cudaError_t launch_insert(const mikv_shape& s, const mikv_cache& c, const void* k_new, const void* v_new,
                           int tok, const int32_t* slots, cudaStream_t st) {
+  if (hi_bits_of(s) != 16)
+    return launch_hi_quant(s, c, k_new, v_new, nullptr, nullptr, 0, nullptr, 0, slots, tok, st);
   insert_kernel<<<s.batch * s.heads_kv, 64, 0, st>>>(
       static_cast<__nv_bfloat16*>(c.k_hi), static_cast<__nv_bfloat16*>(c.v_hi), c.hi_tok, c.acc,
       static_cast<const __nv_bfloat16*>(k_new), static_cast<const __nv_bfloat16*>(v_new), tok, slots, s.hi_cap,
@@ -217,6 +219,8 @@ cudaError_t launch_gather(const mikv_shape& s, const mikv_cache& c, const void* 
                           const int32_t* src_tok, const float* src_scores, int n_src, const int32_t* rows,
                           int n_rows, cudaStream_t st) {
   if (n_rows == 0) return cudaSuccess;
+  if (hi_bits_of(s) != 16)
+    return launch_hi_quant(s, c, k_src, v_src, src_tok, src_scores, n_src, rows, n_rows, nullptr, 0, st);
   const dim3 grid((n_rows + 7) / 8, s.batch * s.heads_kv);
   gather_kernel<<<grid, 256, 0, st>>>(static_cast<__nv_bfloat16*>(c.k_hi), static_cast<__nv_bfloat16*>(c.v_hi),
                                       c.hi_tok, c.acc, static_cast<const __nv_bfloat16*>(k_src),

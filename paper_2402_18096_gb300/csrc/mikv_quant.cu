@@ -1,5 +1,5 @@
-// mikv_quant.cu — demotion of KV rows into the retained set (Eq. 1 with the Eq. 3 key balancer) and
-// the channel balancer itself (Eq. 2), arxiv 2402.18096.
+// mikv_quant.cu — demotion of KV rows into the retained set (Eq. 1 with the Eq. 3 key balancer), rows
+// entering a coded important set (Sec. 3.3), and the channel balancer itself (Eq. 2), arxiv 2402.18096.
 //
 // quantize_pack: one warp per (row, K or V) running quantize_row_warp (mikv_rows.cuh): each lane owns
 // 4 consecutive channels, group minima and maxima come from butterfly shuffles, scale and zero are
@@ -29,7 +29,7 @@ struct QPArgs {
 
 template <int BITS, int GROUP>
 __global__ void __launch_bounds__(256) quantize_pack_kernel(const QPArgs a) {
-  __shared__ uint32_t buf[8][16];
+  __shared__ uint32_t buf[8][32];
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int i = blockIdx.x * 4 + (w >> 1);
   const bool is_v = (w & 1) != 0;
@@ -54,6 +54,59 @@ cudaError_t qp_group(const QPArgs& a, int group, dim3 grid, cudaStream_t st) {
     default: return cudaErrorInvalidValue;
   }
   return cudaGetLastError();
+}
+
+// ------------------------------------------------------- coded important set (Sec. 3.3, Table 3)
+
+// Rows entering a coded important set, quantized like retained rows (Eq. 1 at hi_bits, groups of
+// kHiGroup; keys times the balancer first, Eq. 3). Two modes: insert (rows == nullptr: the new token of
+// every (b, h) into slot slots[b][h]) and gather (slot i < n_rows receives source row rows[b][h][i]).
+struct HiQArgs {
+  const __nv_bfloat16* k_src;
+  const __nv_bfloat16* v_src;
+  const int32_t* src_tok;
+  const float* src_scores;
+  const int32_t* rows;
+  const int32_t* slots;
+  const float* balancer;
+  uint8_t* k_hc;
+  uint8_t* v_hc;
+  __half2* k_hp;
+  __half2* v_hp;
+  int32_t* hi_tok;
+  float* acc;
+  int heads_kv, hi_cap, hi_stride, n_src, n_rows, tok;
+};
+
+template <int HB>
+__global__ void __launch_bounds__(256) hi_quant_kernel(const HiQArgs a) {
+  __shared__ uint32_t buf[8][32];
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int i = blockIdx.x * 4 + (w >> 1);
+  const bool is_v = (w & 1) != 0;
+  const int bh = blockIdx.y, h = bh % a.heads_kv;
+  int slot, r = 0;
+  const __nv_bfloat16* src;
+  if (a.rows) {
+    if (i >= a.n_rows) return;
+    r = a.rows[(size_t)bh * a.n_rows + i];
+    if (r < 0 || r >= a.n_src) return;  // out-of-range rows are skipped, as in quantize_pack
+    slot = i;
+    src = (is_v ? a.v_src : a.k_src) + ((size_t)bh * a.n_src + r) * kHeadDim;
+  } else {
+    if (i > 0) return;
+    slot = a.slots[bh];
+    if (slot < 0 || slot >= a.hi_cap) return;
+    src = (is_v ? a.v_src : a.k_src) + (size_t)bh * kHeadDim;
+  }
+  const size_t row = (size_t)bh * a.hi_stride + slot;
+  quantize_row_warp<HB, kHiGroup>(src, is_v ? nullptr : (a.balancer ? a.balancer + h * kHeadDim : nullptr),
+                                  (is_v ? a.v_hc : a.k_hc) + row * (16 * HB),
+                                  (is_v ? a.v_hp : a.k_hp) + row * (kHeadDim / kHiGroup), buf[w], lane);
+  if (!is_v && lane == 0) {
+    a.hi_tok[row] = a.rows ? (a.src_tok ? a.src_tok[(size_t)bh * a.n_src + r] : r) : a.tok;
+    a.acc[row] = a.rows && a.src_scores ? a.src_scores[(size_t)bh * a.n_src + r] : 0.f;
+  }
 }
 
 // ---------------------------------------------------------------------------- Eq. 2 balancer
@@ -112,6 +165,40 @@ cudaError_t launch_quantize_pack(const mikv_shape& s, const mikv_cache& c, const
     case 4: return qp_group<4>(a, s.group, grid, st);
   }
   return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_hi_quant(const mikv_shape& s, const mikv_cache& c, const void* k_src, const void* v_src,
+                            const int32_t* src_tok, const float* src_scores, int n_src, const int32_t* rows,
+                            int n_rows, const int32_t* slots, int tok, cudaStream_t st) {
+  HiQArgs a;
+  a.k_src = static_cast<const __nv_bfloat16*>(k_src);
+  a.v_src = static_cast<const __nv_bfloat16*>(v_src);
+  a.src_tok = src_tok;
+  a.src_scores = src_scores;
+  a.rows = rows;
+  a.slots = slots;
+  a.balancer = c.balancer;
+  a.k_hc = static_cast<uint8_t*>(c.k_hi);
+  a.v_hc = static_cast<uint8_t*>(c.v_hi);
+  a.k_hp = static_cast<__half2*>(c.k_hi_params);
+  a.v_hp = static_cast<__half2*>(c.v_hi_params);
+  a.hi_tok = c.hi_tok;
+  a.acc = c.acc;
+  a.heads_kv = s.heads_kv;
+  a.hi_cap = s.hi_cap;
+  a.hi_stride = s.hi_stride;
+  a.n_src = n_src;
+  a.n_rows = n_rows;
+  a.tok = tok;
+  const dim3 grid(rows ? (n_rows + 3) / 4 : 1, s.batch * s.heads_kv);
+  const int threads = rows ? 256 : 64;
+  switch (hi_bits_of(s)) {
+    case 8: hi_quant_kernel<8><<<grid, threads, 0, st>>>(a); break;
+    case 4: hi_quant_kernel<4><<<grid, threads, 0, st>>>(a); break;
+    case 2: hi_quant_kernel<2><<<grid, threads, 0, st>>>(a); break;
+    default: return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
 }
 
 cudaError_t launch_balancer(const mikv_shape& s, const void* q_pre, const void* k_pre, int T, float* out,

@@ -20,29 +20,19 @@ __device__ __forceinline__ void field_pos(int c, int f, int& unit, int& bit) {
   }
 }
 
-// Quantize one row (Eq. 1, Eq. 3) with one warp: lane l owns channels 4l..4l+3 of the bf16 row `src`;
-// keys pass `bal` (fp32 [128], or nullptr = 1). Writes 16 * BITS bytes of packed codes to `codes` and
-// 128 / GROUP (alpha, beta) fp16 pairs to `params`. `buf` is 16 words of this warp's shared memory.
-// Every rounding is explicit (fsub/fdiv round-to-nearest, fp16 round-down / round-up, round-half-even
-// to int), so codes and parameters are bit-identical to an IEEE fp32 evaluation.
+// Quantize one row (Eq. 1) held as fp32 values x[4] of channels 4 lane .. 4 lane + 3 of each lane, with
+// one warp. Writes 16 * BITS bytes of packed codes to `codes` and 128 / GROUP (alpha, beta) fp16 pairs to
+// `params`. `buf` is 32 words of this warp's shared memory. Every rounding is explicit (fsub/fdiv
+// round-to-nearest, fp16 round-down / round-up, round-half-even to int), so codes and parameters are
+// bit-identical to an IEEE fp32 evaluation. BITS in {2, 3, 4, 8}.
 template <int BITS, int GROUP>
-__device__ __forceinline__ void quantize_row_warp(const __nv_bfloat16* src, const float* bal, uint8_t* codes,
-                                                  __half2* params, uint32_t* buf, int lane) {
+__device__ __forceinline__ void quantize_values_warp(const float (&x)[4], uint8_t* codes, __half2* params,
+                                                     uint32_t* buf, int lane) {
   constexpr int QMAX = (1 << BITS) - 1;
   constexpr int LANES = GROUP / 4;  // lanes per quantization group
   constexpr int WORDS = 4 * BITS;   // 32-bit words of one packed row
-  if (lane < 16) buf[lane] = 0u;
+  if (lane < WORDS) buf[lane] = 0u;
   __syncwarp();
-  const uint2 raw = *reinterpret_cast<const uint2*>(src + 4 * lane);
-  float x[4] = {__uint_as_float(raw.x << 16), __uint_as_float(raw.x & 0xffff0000u),
-                __uint_as_float(raw.y << 16), __uint_as_float(raw.y & 0xffff0000u)};
-  if (bal) {  // Eq. 3: keys times the balancer before the quantizer
-    const float4 b = *reinterpret_cast<const float4*>(bal + 4 * lane);
-    x[0] = __fmul_rn(x[0], b.x);
-    x[1] = __fmul_rn(x[1], b.y);
-    x[2] = __fmul_rn(x[2], b.z);
-    x[3] = __fmul_rn(x[3], b.w);
-  }
   float mn = fminf(fminf(x[0], x[1]), fminf(x[2], x[3]));
   float mx = fmaxf(fmaxf(x[0], x[1]), fmaxf(x[2], x[3]));
 #pragma unroll
@@ -73,6 +63,42 @@ __device__ __forceinline__ void quantize_row_warp(const __nv_bfloat16* src, cons
   __syncwarp();
   if (lane < WORDS) reinterpret_cast<uint32_t*>(codes)[lane] = buf[lane];
   if ((lane & (LANES - 1)) == 0) params[(4 * lane) / GROUP] = __halves2half2(alpha16, beta16);
+}
+
+// Quantize one bf16 row (Eq. 1, Eq. 3): lane l owns channels 4l..4l+3 of `src`; keys pass `bal` (fp32
+// [128], or nullptr = 1), multiplied in before the quantizer.
+template <int BITS, int GROUP>
+__device__ __forceinline__ void quantize_row_warp(const __nv_bfloat16* src, const float* bal, uint8_t* codes,
+                                                  __half2* params, uint32_t* buf, int lane) {
+  const uint2 raw = *reinterpret_cast<const uint2*>(src + 4 * lane);
+  float x[4] = {__uint_as_float(raw.x << 16), __uint_as_float(raw.x & 0xffff0000u),
+                __uint_as_float(raw.y << 16), __uint_as_float(raw.y & 0xffff0000u)};
+  if (bal) {  // Eq. 3: keys times the balancer before the quantizer
+    const float4 b = *reinterpret_cast<const float4*>(bal + 4 * lane);
+    x[0] = __fmul_rn(x[0], b.x);
+    x[1] = __fmul_rn(x[1], b.y);
+    x[2] = __fmul_rn(x[2], b.z);
+    x[3] = __fmul_rn(x[3], b.w);
+  }
+  quantize_values_warp<BITS, GROUP>(x, codes, params, buf, lane);
+}
+
+// fp32 dequantization of channels 4 lane .. 4 lane + 3 of one packed row of `bits`-bit codes (bits in
+// {2, 4, 8}, one plane) with (alpha, beta) per group of `group` channels: x = alpha * code + beta, the
+// product exact in fp32 and the sum rounded once (one fma).
+__device__ __forceinline__ void dequantize_values_warp(const uint8_t* codes, const __half2* params, int bits,
+                                                       int group, int lane, float (&x)[4]) {
+  const uint16_t* units = reinterpret_cast<const uint16_t*>(codes);
+  const uint32_t mask = (1u << bits) - 1u;
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const int c = 4 * lane + e;
+    int unit, bit;
+    field_pos(c, bits, unit, bit);
+    const uint32_t code = ((uint32_t)units[unit] >> bit) & mask;
+    const float2 ab = __half22float2(params[c / group]);
+    x[e] = __fmaf_rn(ab.x, (float)code, ab.y);
+  }
 }
 
 // Total order of (score, id): ascending score, then ascending id. -0 is folded into +0.

@@ -25,7 +25,7 @@ __global__ void __launch_bounds__(kPostThreads) step_post_kernel(const StepPostA
   __shared__ unsigned long long s_best[kPostThreads / 32];
   __shared__ int s_slot[kPostThreads / 32];
   __shared__ int s_victim;
-  __shared__ uint32_t buf[2][16];
+  __shared__ uint32_t buf[2][32];
   const int bh = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int b = bh / a.heads_kv, h = bh - b * a.heads_kv;
 
@@ -114,16 +114,26 @@ __global__ void __launch_bounds__(kPostThreads) step_post_kernel(const StepPostA
   const int victim = s_victim;
   if (victim < 0) return;  // unreachable for valid scores (hi_cap >= 1, no NaN)
 
-  // 3. demote the victim: quantize its key (balanced, Eq. 3) and value rows into retained row n_lo
+  // 3. demote the victim: quantize its key (balanced, Eq. 3) and value rows into retained row n_lo; a
+  // coded important row is re-quantized from its fp32 dequantized values (already balanced, Sec. 3.3)
   if (warp < 2) {
     const bool is_v = warp == 1;
     const size_t pos = (size_t)bh * a.lo_cap + a.n_lo;
-    const __nv_bfloat16* src = static_cast<const __nv_bfloat16*>(is_v ? a.v_hi : a.k_hi) +
-                               ((size_t)bh * a.hi_stride + victim) * kHeadDim;
-    quantize_row_warp<BITS, GROUP>(src, is_v ? nullptr : (a.balancer ? a.balancer + h * kHeadDim : nullptr),
-                                   static_cast<uint8_t*>(is_v ? a.v_codes : a.k_codes) + pos * (16 * BITS),
-                                   static_cast<__half2*>(is_v ? a.v_params : a.k_params) + pos * (kHeadDim / GROUP),
-                                   buf[warp], lane);
+    const size_t hrow = (size_t)bh * a.hi_stride + victim;
+    uint8_t* codes = static_cast<uint8_t*>(is_v ? a.v_codes : a.k_codes) + pos * (16 * BITS);
+    __half2* params = static_cast<__half2*>(is_v ? a.v_params : a.k_params) + pos * (kHeadDim / GROUP);
+    if (a.hi_bits == 16) {
+      const __nv_bfloat16* src = static_cast<const __nv_bfloat16*>(is_v ? a.v_hi : a.k_hi) + hrow * kHeadDim;
+      quantize_row_warp<BITS, GROUP>(src, is_v ? nullptr : (a.balancer ? a.balancer + h * kHeadDim : nullptr),
+                                     codes, params, buf[warp], lane);
+    } else {
+      float x[4];
+      dequantize_values_warp(static_cast<const uint8_t*>(is_v ? a.v_hi : a.k_hi) + hrow * (16 * a.hi_bits),
+                             static_cast<const __half2*>(is_v ? a.v_hi_params : a.k_hi_params) +
+                                 hrow * (kHeadDim / kHiGroup),
+                             a.hi_bits, kHiGroup, lane, x);
+      quantize_values_warp<BITS, GROUP>(x, codes, params, buf[warp], lane);
+    }
     if (!is_v && lane == 0) {
       a.lo_tok[pos] = tok[victim];
       a.slots[bh] = victim;

@@ -3,7 +3,8 @@
 This is the flow a serving stack runs around the library (Fig. 4 of arxiv 2402.18096):
   prefill  -> channel balancer from prefill maxima (Eq. 2)
            -> choose the k most important tokens by accumulated attention (mikv_select_demote)
-           -> keep them in bf16 (mikv_gather_hi), quantize the rest into the retained set
+           -> keep them in high precision (mikv_gather_hi: bf16, or 8/4/2-bit codes for a reduced-
+              precision important set, Sec. 3.3), quantize the rest into the retained set
               (mikv_quantize_pack, Eq. 1 with Eq. 3 key balancing)
   decode   -> per token: insert, attend, update importance, demote the least important (mikv_decode_step)
 Every step runs in the library's kernels; this module only orders the calls and owns the buffers.

@@ -18,7 +18,7 @@ bits16 = mi.bf16_bits
 
 def make_shape(w: mi.Workload, steps: int = 4, batch: int = None) -> pkg.Shape:
     return pkg.Shape(w.batch if batch is None else batch, w.heads_q, w.heads_kv, w.bits, w.group, w.hi_cap,
-                     w.lo_cap_for(steps))
+                     w.lo_cap_for(steps), hi_bits=w.hi_bits)
 
 
 def raw_inputs(w: mi.Workload, layer: int = 0, device="cpu", balanced: bool = True):
@@ -52,8 +52,8 @@ def oracle_layer(w: mi.Workload, raw, lo_cap: int, heads=None):
         sc = scores[b:b + 1, h:h + 1].numpy()
         T = k.shape[2]
         dem, kept = oracle.select_demote(sc, T - w.budget)
-        c = oracle.empty_cache(1, 1, w.head_dim, w.bits, w.group, w.hi_cap, lo_cap)
-        oracle.gather_hi(c, ks, vs, kept, src_scores=sc)
+        c = oracle.empty_cache(1, 1, w.head_dim, w.bits, w.group, w.hi_cap, lo_cap, hi_bits=w.hi_bits)
+        oracle.gather_hi(c, ks, vs, kept, src_scores=sc, balancer_=bal)
         oracle.quantize_pack(c, ks, vs, dem, 0, balancer_=bal)
         out.append(dict(cache=c, balancer=bal, b=b, h=h, demoted=dem[0, 0], kept=kept[0, 0]))
     return out

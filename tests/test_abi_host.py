@@ -66,14 +66,15 @@ def test_row_bytes(lib):
 
 
 def _shape(**kw):
-    s = dict(batch=2, heads_q=8, heads_kv=2, head_dim=128, bits=2, group=32, hi_cap=20, hi_stride=32, lo_cap=64)
+    s = dict(batch=2, heads_q=8, heads_kv=2, head_dim=128, bits=2, group=32, hi_cap=20, hi_stride=32, lo_cap=64,
+             hi_bits=0, hi_group=64)
     s.update(kw)
     return pkg._Shape(*[s[n] for n, _ in pkg._Shape._fields_])
 
 
 def _fake_cache():
     # never dereferenced: validation rejects or the test stops before any launch
-    return pkg._Cache(*([0x10000] * 9 + [None]))
+    return pkg._Cache(*([0x10000] * 9 + [None, 0x10000, 0x10000]))
 
 
 def test_workspace_sizes_monotone(lib):
@@ -90,10 +91,15 @@ def test_workspace_sizes_monotone(lib):
     (dict(head_dim=64), 2), (dict(bits=5), 2), (dict(bits=8), 2), (dict(group=48), 2),
     (dict(heads_q=6, heads_kv=2), 2), (dict(heads_q=7), 1), (dict(hi_stride=24), 1),
     (dict(lo_cap=60), 1), (dict(batch=0), 1), (dict(hi_stride=16, hi_cap=20), 1),
+    (dict(hi_bits=3), 2), (dict(hi_bits=12), 2), (dict(hi_bits=8, hi_group=32), 2), (dict(hi_bits=4, hi_group=128), 2),
+    (dict(hi_bits=8), 0), (dict(hi_bits=4), 0), (dict(hi_bits=2), 0), (dict(hi_bits=16, hi_group=0), 0),
 ])
 def test_shape_validation(lib, kw, code):
     s = _shape(**kw)
     c = _fake_cache()
+    if code == 0:  # a valid shape: check it through the pure workspace query instead of launching
+        assert lib.mikv_workspace_bytes(ctypes.byref(s), 0, 16) > 0
+        return
     rc = lib.mikv_quantize_pack(ctypes.byref(s), ctypes.byref(c), 0x10000, 0x10000, None, 4, 0x10000, 1, 0, None)
     assert rc == code
 
@@ -105,8 +111,14 @@ def test_argument_validation_before_launch(lib):
     # retained capacity: lo_start + n_rows > lo_cap
     assert lib.mikv_quantize_pack(ctypes.byref(s), ctypes.byref(c), P, P, None, 4, P, 5, 60, None) == 3
     # null cache member
-    bad = pkg._Cache(*([P] * 8 + [None, None]))
+    bad = pkg._Cache(*([P] * 8 + [None, None, None, None]))
     assert lib.mikv_quantize_pack(ctypes.byref(s), ctypes.byref(bad), P, P, None, 4, P, 1, 0, None) == 1
+    # a coded important set needs its parameter arrays (16-byte aligned)
+    sq = _shape(hi_bits=8)
+    no_hp = pkg._Cache(*([P] * 9 + [None, None, None]))
+    assert lib.mikv_quantize_pack(ctypes.byref(sq), ctypes.byref(no_hp), P, P, None, 4, P, 1, 0, None) == 1
+    odd_hp = pkg._Cache(*([P] * 9 + [None, P + 8, P]))
+    assert lib.mikv_quantize_pack(ctypes.byref(sq), ctypes.byref(odd_hp), P, P, None, 4, P, 1, 0, None) == 1
     # attention: n_lo beyond capacity, bad output type, missing or misaligned workspace
     assert lib.mikv_decode_attention(ctypes.byref(s), ctypes.byref(c), 65, P, 1.0, P, 0, None, None, P, 1 << 20,
                                      None) == 3
