@@ -38,7 +38,8 @@ UNIT = "GB/s"
 DEFAULT_WORKLOAD = "mistral-7b"
 
 
-ATTN_SOURCES = ["mikv_attention.cu", "mikv_device.cuh", "mikv_internal.h", "mikv_rows.cuh"]
+ATTN_SOURCES = ["mikv_attention.cuh", "mikv_attention.cu", "mikv_attn_h16.cu", "mikv_device.cuh", "mikv_internal.h",
+                "mikv_rows.cuh"]
 TRAFFIC_SUMMARY = os.path.join(ROOT, "profiles", "attention_kernel_mistral7b_b4.md")
 
 
