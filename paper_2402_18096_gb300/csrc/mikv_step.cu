@@ -16,11 +16,55 @@
 namespace mikv {
 namespace {
 
-constexpr int kPostThreads = 1024;
-constexpr int kPostUnroll = 4;  // independent slots in flight per thread
+constexpr int kPostThreads = 256;
+
+// Four consecutive important slots of one (b, KV head): the G query heads' logits, the score and the
+// token id (hi_stride % 16 == 0 keeps every group 16-byte aligned).
+template <int G>
+struct SlotQuad {
+  float4 lg[G];
+  float4 ac;
+  int4 tk;
+};
+
+template <int G>
+__device__ __forceinline__ void load_quad(const float* logit, const float* acc, const int32_t* tok, int hi_stride,
+                                          int v, SlotQuad<G>& q) {
+#pragma unroll
+  for (int j = 0; j < G; ++j) q.lg[j] = reinterpret_cast<const float4*>(logit + (size_t)j * hi_stride)[v];
+  q.ac = reinterpret_cast<const float4*>(acc)[v];
+  q.tk = reinterpret_cast<const int4*>(tok)[v];
+}
+
+// Importance update of the slots of q below hi_cap (the arithmetic of update_importance_kernel: the
+// weights exp(s - m) / l of the G heads summed in head order, then added to the score), the updated
+// scores stored, and the running minimum of (score, id) advanced.
+template <int G>
+__device__ __forceinline__ void update_quad(float* acc, int hi_cap, int v, SlotQuad<G>& q, const float* s_m,
+                                            const float* s_l, unsigned long long& best, int& best_slot) {
+  float* ac = &q.ac.x;
+  const int32_t* tk = &q.tk.x;
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const int i = 4 * v + e;
+    if (i >= hi_cap) break;
+    float add = 0.f;
+#pragma unroll
+    for (int j = 0; j < G; ++j) add += expf((&q.lg[j].x)[e] - s_m[j]) / s_l[j];
+    ac[e] = ac[e] + add;
+    const unsigned long long k = order_key(ac[e], tk[e]);
+    if (k < best) {
+      best = k;
+      best_slot = i;
+    }
+  }
+  reinterpret_cast<float4*>(acc)[v] = q.ac;  // padding slots (>= hi_cap) are written back unchanged
+}
+
+static_assert(kPostThreads <= 1024, "the final argmin reduces at most one entry per lane of warp 0");
 
 template <int BITS, int GROUP, int G, int OUT_F32>
-__global__ void __launch_bounds__(kPostThreads) step_post_kernel(const StepPostArgs a) {
+__global__ void __launch_bounds__(kPostThreads, 2) step_post_kernel(const StepPostArgs a) {
   __shared__ float s_m[8], s_l[8];
   __shared__ unsigned long long s_best[kPostThreads / 32];
   __shared__ int s_slot[kPostThreads / 32];
@@ -28,6 +72,14 @@ __global__ void __launch_bounds__(kPostThreads) step_post_kernel(const StepPostA
   __shared__ uint32_t buf[2][32];
   const int bh = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int b = bh / a.heads_kv, h = bh - b * a.heads_kv;
+  float* acc = a.acc + (size_t)bh * a.hi_stride;
+  const int32_t* tok = a.hi_tok + (size_t)bh * a.hi_stride;
+  const float* logit = a.hi_logits + (size_t)(b * a.heads_q + h * G) * a.hi_stride;
+  const int nv = (a.hi_cap + 3) / 4;  // groups of four slots
+
+  // 0. this thread's first group of slots is loaded before the merge, which it does not depend on
+  SlotQuad<G> q0;
+  if (tid < nv) load_quad<G>(logit, acc, tok, a.hi_stride, tid, q0);
 
   // 1. combine the split partials of query heads h*G .. h*G+G-1 (one warp per query head)
   if (warp < G) {
@@ -53,38 +105,17 @@ __global__ void __launch_bounds__(kPostThreads) step_post_kernel(const StepPostA
   __syncthreads();
 
   // 2. importance update and the least important slot (keys are unique: ids are distinct)
-  float* acc = a.acc + (size_t)bh * a.hi_stride;
-  const int32_t* tok = a.hi_tok + (size_t)bh * a.hi_stride;
-  const float* logit = a.hi_logits + (size_t)(b * a.heads_q + h * G) * a.hi_stride;
   unsigned long long best = ~0ull;
   int best_slot = -1;
-  for (int i0 = tid; i0 < a.hi_cap; i0 += kPostThreads * kPostUnroll) {
-    float lg[kPostUnroll][G], ac[kPostUnroll];
-    int32_t tk[kPostUnroll];
-#pragma unroll
-    for (int r = 0; r < kPostUnroll; ++r) {  // issue every load of this round before using any
-      const int i = i0 + r * kPostThreads;
-      const bool ok = i < a.hi_cap;
-#pragma unroll
-      for (int j = 0; j < G; ++j) lg[r][j] = ok ? logit[(size_t)j * a.hi_stride + i] : 0.f;
-      ac[r] = ok ? acc[i] : 0.f;
-      tk[r] = ok ? tok[i] : 0;
-    }
-#pragma unroll
-    for (int r = 0; r < kPostUnroll; ++r) {
-      const int i = i0 + r * kPostThreads;
-      if (i >= a.hi_cap) continue;
-      float add = 0.f;
-#pragma unroll
-      for (int j = 0; j < G; ++j) add += expf(lg[r][j] - s_m[j]) / s_l[j];
-      const float v = ac[r] + add;
-      acc[i] = v;
-      const unsigned long long k = order_key(v, tk[r]);
-      if (k < best) {
-        best = k;
-        best_slot = i;
-      }
-    }
+  if (tid < nv) update_quad<G>(acc, a.hi_cap, tid, q0, s_m, s_l, best, best_slot);
+  constexpr int kInFlight = G <= 4 ? 2 : 1;  // groups loaded before any of them is used
+  for (int v = tid + kPostThreads; v < nv; v += kInFlight * kPostThreads) {
+    SlotQuad<G> q1, q2;
+    const bool two = kInFlight == 2 && v + kPostThreads < nv;
+    load_quad<G>(logit, acc, tok, a.hi_stride, v, q1);
+    if (two) load_quad<G>(logit, acc, tok, a.hi_stride, v + kPostThreads, q2);
+    update_quad<G>(acc, a.hi_cap, v, q1, s_m, s_l, best, best_slot);
+    if (two) update_quad<G>(acc, a.hi_cap, v + kPostThreads, q2, s_m, s_l, best, best_slot);
   }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) {
@@ -100,15 +131,19 @@ __global__ void __launch_bounds__(kPostThreads) step_post_kernel(const StepPostA
     s_slot[warp] = best_slot;
   }
   __syncthreads();
-  if (tid == 0) {
-    unsigned long long bb = s_best[0];
-    int bs = s_slot[0];
-    for (int w = 1; w < kPostThreads / 32; ++w)
-      if (s_best[w] < bb) {
-        bb = s_best[w];
-        bs = s_slot[w];
+  if (warp == 0) {  // minimum over the warps' minima (one per lane)
+    best = lane < kPostThreads / 32 ? s_best[lane] : ~0ull;
+    best_slot = lane < kPostThreads / 32 ? s_slot[lane] : -1;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      const unsigned long long o = __shfl_xor_sync(0xffffffffu, best, off);
+      const int os = __shfl_xor_sync(0xffffffffu, best_slot, off);
+      if (o < best) {
+        best = o;
+        best_slot = os;
       }
-    s_victim = bs;
+    }
+    if (lane == 0) s_victim = best_slot;
   }
   __syncthreads();
   const int victim = s_victim;
