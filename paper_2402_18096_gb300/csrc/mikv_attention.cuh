@@ -308,6 +308,12 @@ __device__ __forceinline__ void process_hi(uint32_t blk, int valid, int slot0, c
   softmax_blocks(s, st, o, ob, p);
   const uint32_t pb0 = movmatrix_t(pack_bf16(p[0][0], p[0][1]));
   const uint32_t pb1 = movmatrix_t(pack_bf16(p[0][2], p[0][3]));
+  {
+    // row 4 of the zero-row sums: the bf16 probabilities exactly as the PV MMA uses them (normaliser)
+    const uint32_t one = g == 4 ? 0x3F803F80u : 0u;
+    const uint32_t a[4] = {one, 0u, one, 0u};
+    mma_bf16(ob[0], a, pb0, pb1);
+  }
   uint32_t m01 = 0xffffffffu, m89 = 0xffffffffu;
   if (valid < 16) {
     m01 = (2 * t < valid ? 0x0000ffffu : 0u) | (2 * t + 1 < valid ? 0xffff0000u : 0u);
@@ -510,8 +516,12 @@ __device__ __forceinline__ void lo_values(uint32_t unit, int b, int valid, const
     if (t9 >= valid) bw9 = 0u;
   }
   {
-    const uint32_t a[4] = {prmt(bw0, bw1, 0x7632u), 0u, prmt(bw8, bw9, 0x7632u), 0u};
-    mma_f16(ob[0], a, pb0, pb1);  // ob[0][row r][heads 2t, 2t+1] += sum over tokens of p * beta
+    // rows 0..3: sum over tokens of p * beta per 32-channel slice; row 4: sum of the fp16 probabilities
+    // exactly as the code MMAs use them (the normaliser of the output)
+    uint32_t a0 = prmt(bw0, bw1, 0x7632u), a2 = prmt(bw8, bw9, 0x7632u);
+    if (g == 4) a0 = a2 = 0x3C003C00u;
+    const uint32_t a[4] = {a0, 0u, a2, 0u};
+    mma_f16(ob[0], a, pb0, pb1);
   }
   uint32_t pa0[NG], pa1[NG];  // p * alpha per group: B operand of the code MMAs
 #pragma unroll
@@ -599,9 +609,10 @@ __device__ __forceinline__ void process_coded(uint32_t unit, int b, int n_left, 
     lo_values<BITS, GROUP, NB, HI>(unit, b + k, min(16, n_left - 16 * k), p[k], o, ob, lane);
 }
 
-// Write this warp's partial for one head: output (plus the zero-row terms, minus the value-code offsets),
-// true max and sum. The running sums are at the reference max m; they are rescaled here to the largest
-// logit seen, so the partial's (max, sum) are the exact statistics of its tokens.
+// Write this warp's partial for one head: the output normalised by the sum of the rounded probabilities
+// the MMAs used (row 4 of the zero-row sums), so rounding the probabilities to bf16 / fp16 only perturbs
+// the weights of a convex combination; and the true max and fp32 sum of its tokens (the sum is kept at
+// the reference max m while streaming and rescaled here to the largest logit seen).
 template <int BITS, int GROUP, int G, int NB>
 __device__ __forceinline__ void write_partial(const AttnArgs& a, int slot, Softmax& st, const float (&o)[8][4],
                                               const float (&ob)[NB][4], int lane) {
@@ -623,6 +634,8 @@ __device__ __forceinline__ void write_partial(const AttnArgs& a, int slot, Softm
     bz0[r] = __shfl_sync(0xffffffffu, ob[0][0], r * 4 + t);
     bz1[r] = __shfl_sync(0xffffffffu, ob[0][1], r * 4 + t);
   }
+  const float inv[2] = {1.f / __shfl_sync(0xffffffffu, ob[0][0], 16 + t),   // row 4, lane 16 + t
+                        1.f / __shfl_sync(0xffffffffu, ob[0][1], 16 + t)};
 #pragma unroll
   for (int hd = 0; hd < 2; ++hd) {
     const int head = 2 * t + hd;
@@ -633,8 +646,8 @@ __device__ __forceinline__ void write_partial(const AttnArgs& a, int slot, Softm
         const int gi = (16 * mt) / GROUP;
         float z = hd ? bz1[mt >> 1] : bz0[mt >> 1];
         if (BITS != 3) z = fmaf(-voff<BITS>(mt), ob[1 + gi / 2][2 * (gi & 1) + hd], z);
-        po[16 * mt + g] = (o[mt][hd] + z) * c[hd];
-        po[16 * mt + 8 + g] = (o[mt][2 + hd] + z) * c[hd];
+        po[16 * mt + g] = (o[mt][hd] + z) * inv[hd];
+        po[16 * mt + 8 + g] = (o[mt][2 + hd] + z) * inv[hd];
       }
       if (g == 0) {
         a.part_ml[((size_t)slot * G + head) * 2] = st.mx[hd];

@@ -117,8 +117,9 @@ __device__ __forceinline__ int owner_warp(long long U, long long n_units, int n_
 }
 
 // One warp combines the split partials of query head jh of KV head bh (warps w0..w1 of the attention
-// kernel wrote slots w + bh): lane l returns the normalised output of channels 4l..4l+3, and every lane
-// returns (M, L) = (max logit, sum of exp(logit - M)). The per-slot statistics are read by all lanes at
+// kernel wrote slots w + bh; each partial is a normalised output with its (max, sum)): lane l returns
+// the output of channels 4l..4l+3, the partials weighted by exp(max - M) * sum, and every lane returns
+// (M, L) = (max logit, sum of exp(logit - M)). The per-slot statistics are read by all lanes at
 // once and broadcast with shuffles, so the merge costs a few dependent loads whatever the slot count.
 __device__ __forceinline__ void merge_head_warp(const float* part_o, const float* part_ml, int G, int bh, int jh,
                                                 int w0, int w1, int lane, float (&out)[4], float& M, float& L) {
@@ -140,8 +141,8 @@ __device__ __forceinline__ void merge_head_warp(const float* part_o, const float
       const size_t slot = (size_t)(w0 + i + bh);
       const float ms = part_ml[(slot * G + jh) * 2];
       if (ms != -INFINITY) {
-        wt = fast_exp2((ms - M) * kLog2e);
-        Lp += wt * part_ml[(slot * G + jh) * 2 + 1];
+        wt = fast_exp2((ms - M) * kLog2e) * part_ml[(slot * G + jh) * 2 + 1];
+        Lp += wt;
       }
     }
     const int cnt = min(32, n - c0);
