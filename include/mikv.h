@@ -62,8 +62,10 @@ typedef struct {
   int32_t heads_q;   /* Hq, query heads */
   int32_t heads_kv;  /* Hkv, KV heads; Hq / Hkv in {1, 2, 4, 8} */
   int32_t head_dim;  /* d, must be 128 */
-  int32_t bits;      /* N, retained-set code width: 2, 3 or 4 (Eq. 1) */
-  int32_t group;     /* g, channels per quantization group: 32, 64 or 128 (Sec. 3.2 uses d/2) */
+  int32_t bits;      /* N, retained-set code width: 2, 3 or 4 (Eq. 1); 0 = no retained set: demoted
+                        tokens are evicted (the importance-based eviction baseline, H2O, Sec. 2.2 /
+                        Fig. 2); the retained arrays are then unused and may be NULL, n_lo must be 0 */
+  int32_t group;     /* g, channels per quantization group: 32, 64 or 128 (Sec. 3.2 uses d/2); ignored when bits = 0 */
   int32_t hi_cap;    /* important slots attended per head: the budget k plus one staging slot */
   int32_t hi_stride; /* rows per head in the important-set arrays: multiple of 16, >= hi_cap */
   int32_t lo_cap;    /* rows per head in the retained-set arrays: multiple of 16 */
@@ -215,7 +217,8 @@ mikv_status mikv_gather_hi(const mikv_shape* shape, const mikv_cache* cache, con
  * update the importance scores (mikv_update_importance), choose the least important slot
  * (mikv_select_demote, n_demote = 1) and demote it to retained row n_lo (mikv_quantize_pack).
  * On return slots[b][h] holds the slot freed by the demotion (the next step's insertion slot);
- * the retained length becomes n_lo + 1. A coded important slot is demoted from its dequantized values:
+ * the retained length becomes n_lo + 1. With bits = 0 (eviction) nothing is demoted: the victim's slot
+ * is freed and the retained length stays 0. A coded important slot is demoted from its dequantized values:
  * per channel the fp32 value alpha * code + beta (rounded once), quantized at bits / group; keys are
  * already balanced and are not multiplied by the balancer again (Sec. 3.3).
  *   q, k_new, v_new   bf16 [B][Hq][d], [B][Hkv][d], [B][Hkv][d]

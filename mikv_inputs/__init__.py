@@ -32,7 +32,7 @@ class Workload:
     heads_kv: int
     context: int          # T, tokens in the cache before the first decode step
     layers: int
-    bits: int             # retained-set code width
+    bits: int             # retained-set code width (0: no retained set, the H2O eviction baseline)
     group: int            # channels per quantization group
     ratio: float          # fraction of tokens kept in bf16 (importance ratio)
     seed: int = 0
@@ -70,6 +70,10 @@ WORKLOADS = {
 }
 # Table 3 settings (INT2 retained, 20 % important, groups of 64) on the Mistral-7B shape, with the
 # important set itself at reduced precision (Sec. 3.3)
+# the importance-based eviction baseline (H2O) on the Mistral-7B shape: the same 20 % important set,
+# the other tokens dropped
+WORKLOADS["mistral-7b-h2o"] = Workload("mistral-7b-b32-l32-hq32-hkv8-t32768-h2o-r20", 32, 32, 8, 32768, 32, 0, 32,
+                                       0.20)
 for _hb in (16, 8, 4, 2):
     WORKLOADS[f"mistral-7b-t3-hi{_hb}"] = Workload(
         f"mistral-7b-b32-l32-hq32-hkv8-t32768-int2-g64-r20-hi{_hb}", 32, 32, 8, 32768, 32, 2, 64, 0.20,

@@ -159,10 +159,12 @@ class LayerCache:
             self.k_hi_params = self.v_hi_params = None
         self.hi_tok = torch.zeros(B, H, s.hi_stride, dtype=torch.int32, **z)
         self.acc = torch.zeros(B, H, s.hi_stride, dtype=torch.float32, **z)
+        # (bits = 0: eviction, no retained set; its arrays are empty)
         self.k_codes = torch.zeros(B, H, s.lo_cap, 16 * s.bits, dtype=torch.uint8, **z)
         self.v_codes = torch.zeros(B, H, s.lo_cap, 16 * s.bits, dtype=torch.uint8, **z)
-        self.k_params = torch.zeros(B, H, s.lo_cap, d // s.group, 2, dtype=torch.float16, **z)
-        self.v_params = torch.zeros(B, H, s.lo_cap, d // s.group, 2, dtype=torch.float16, **z)
+        npar = d // s.group if s.bits else 0
+        self.k_params = torch.zeros(B, H, s.lo_cap, npar, 2, dtype=torch.float16, **z)
+        self.v_params = torch.zeros(B, H, s.lo_cap, npar, 2, dtype=torch.float16, **z)
         self.lo_tok = torch.zeros(B, H, s.lo_cap, dtype=torch.int32, **z)
         self.balancer = balancer
         self.n_lo = 0

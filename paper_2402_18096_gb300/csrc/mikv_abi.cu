@@ -26,7 +26,8 @@ int num_sms() {
 
 bool shape_ok(const mikv_shape* s) {
   return s && s->batch > 0 && s->heads_q > 0 && s->heads_kv > 0 && s->heads_q % s->heads_kv == 0 &&
-         s->head_dim > 0 && s->bits > 0 && s->group > 0 && s->hi_cap >= 0 && s->hi_stride >= s->hi_cap &&
+         s->head_dim > 0 && s->bits >= 0 && (s->bits == 0 || s->group > 0) && s->hi_cap >= 0 &&
+         s->hi_stride >= s->hi_cap &&
          s->hi_stride % 16 == 0 && s->lo_cap >= 0 && s->lo_cap % 16 == 0;
 }
 
@@ -34,8 +35,10 @@ mikv_status shape_supported(const mikv_shape* s) {
   if (!shape_ok(s)) return MIKV_ERR_ARG;
   const int G = s->heads_q / s->heads_kv;
   if (s->head_dim != kHeadDim) return MIKV_ERR_UNSUPPORTED;
-  if (s->bits < 2 || s->bits > 4) return MIKV_ERR_UNSUPPORTED;
-  if (s->group != 32 && s->group != 64 && s->group != 128) return MIKV_ERR_UNSUPPORTED;
+  if (s->bits != 0) {  // bits == 0: eviction, no retained set (its group is ignored)
+    if (s->bits < 2 || s->bits > 4) return MIKV_ERR_UNSUPPORTED;
+    if (s->group != 32 && s->group != 64 && s->group != 128) return MIKV_ERR_UNSUPPORTED;
+  }
   if (G != 1 && G != 2 && G != 4 && G != 8) return MIKV_ERR_UNSUPPORTED;
   const int hb = s->hi_bits;
   if (hb != 0 && hb != 16 && hb != 8 && hb != 4 && hb != 2) return MIKV_ERR_UNSUPPORTED;
@@ -47,9 +50,8 @@ bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) %
 
 // The cache's arrays exist (and, for a coded important set, so do its parameter arrays, 16-byte aligned).
 bool cache_ok(const mikv_cache* c, const mikv_shape* s) {
-  if (!(c && c->k_hi && c->v_hi && c->hi_tok && c->acc && c->k_codes && c->v_codes && c->k_params &&
-        c->v_params && c->lo_tok))
-    return false;
+  if (!(c && c->k_hi && c->v_hi && c->hi_tok && c->acc)) return false;
+  if (!evicting(*s) && !(c->k_codes && c->v_codes && c->k_params && c->v_params && c->lo_tok)) return false;
   if (hi_bits_of(*s) != 16)
     return c->k_hi_params && c->v_hi_params && aligned(c->k_hi_params, 16) && aligned(c->v_hi_params, 16);
   return true;
@@ -131,6 +133,7 @@ mikv_status attention_args_ok(const mikv_shape* shape, const mikv_cache* cache, 
   if (!cache_ok(cache, shape) || !q || !out || n_lo < 0 || (out_dtype != MIKV_OUT_BF16 && out_dtype != MIKV_OUT_F32))
     return MIKV_ERR_ARG;
   if (n_lo > shape->lo_cap) return MIKV_ERR_CAPACITY;
+  if (evicting(*shape) && n_lo != 0) return MIKV_ERR_ARG;
   if (shape->hi_cap + n_lo < 1) return MIKV_ERR_ARG;
   if (!aligned(cache->k_hi, 16) || !aligned(cache->v_hi, 16) || !aligned(cache->k_codes, 16) ||
       !aligned(cache->v_codes, 16) || !aligned(cache->k_params, 16) || !aligned(cache->v_params, 16) ||
@@ -191,7 +194,7 @@ mikv_status attention_impl(const mikv_shape* s, const mikv_cache* c, int32_t n_l
          make_map(&a.map_v_hp, c->v_hi_params, CU_TENSOR_MAP_DATA_TYPE_UINT8, H.param_w, par_rows, H.param_w,
                   H.param_w, par_box, CU_TENSOR_MAP_SWIZZLE_NONE);
   }
-  if (ok && lo_rows > 0) {
+  if (ok && lo_rows > 0 && !evicting(*s)) {
     // retained arrays: each is viewed as rows of U.map_w (codes) or U.param_w (alpha, beta) bytes, and
     // one box covers a whole unit of 16 * U.blocks tokens (lo_cap % 16 == 0 keeps units row-aligned)
     const LoUnit U = lo_unit_layout(s->bits, s->group);
@@ -231,7 +234,7 @@ mikv_status attention_impl(const mikv_shape* s, const mikv_cache* c, int32_t n_l
   a.n_units = plan.n_units;
   a.n_warps = plan.n_warps;
   a.sm_scale = sm_scale;
-  cudaError_t e = launch_attention(a, s->bits, s->group, hb, G, plan.grid, st);
+  cudaError_t e = launch_attention(a, lo_bits_of(*s), lo_group_of(*s), hb, G, plan.grid, st);
   if (e != cudaSuccess) return MIKV_ERR_CUDA;
   if (args_out) *args_out = a;
   if (!merge) return MIKV_OK;
@@ -309,6 +312,7 @@ mikv_status mikv_quantize_pack(const mikv_shape* shape, const mikv_cache* cache,
                                int32_t n_rows, int32_t lo_start, void* stream) {
   mikv_status st = shape_supported(shape);
   if (st != MIKV_OK) return st;
+  if (evicting(*shape)) return MIKV_ERR_UNSUPPORTED;  // no retained set to write
   if (!cache_ok(cache, shape) || !k_src || !v_src || n_src <= 0 || n_rows < 0 || lo_start < 0 || (n_rows > 0 && !rows))
     return MIKV_ERR_ARG;
   if ((int64_t)lo_start + n_rows > shape->lo_cap) return MIKV_ERR_CAPACITY;
@@ -375,7 +379,7 @@ mikv_status mikv_decode_step(const mikv_shape* shape, const mikv_cache* cache, i
   if (st != MIKV_OK) return st;
   if (!cache_ok(cache, shape) || !q || !k_new || !v_new || !slots || !out || n_lo < 0) return MIKV_ERR_ARG;
   if (shape->hi_cap < 1) return MIKV_ERR_CAPACITY;
-  if ((int64_t)n_lo + 1 > shape->lo_cap) return MIKV_ERR_CAPACITY;
+  if (!evicting(*shape) && (int64_t)n_lo + 1 > shape->lo_cap) return MIKV_ERR_CAPACITY;
   if (!workspace || !aligned(workspace, 256)) return MIKV_ERR_WORKSPACE;
   const StepLayout L = step_layout(shape, n_lo);
   if (ws_bytes < L.total) return MIKV_ERR_WORKSPACE;
@@ -408,6 +412,7 @@ mikv_status mikv_decode_step(const mikv_shape* shape, const mikv_cache* cache, i
   p.k_hi_params = cache->k_hi_params;
   p.v_hi_params = cache->v_hi_params;
   p.hi_bits = hi_bits_of(*shape);
+  p.evict = evicting(*shape) ? 1 : 0;
   p.batch = shape->batch;
   p.heads_q = shape->heads_q;
   p.heads_kv = shape->heads_kv;
@@ -418,7 +423,7 @@ mikv_status mikv_decode_step(const mikv_shape* shape, const mikv_cache* cache, i
   p.n_u = a.n_u;
   p.n_units = a.n_units;
   p.n_warps = a.n_warps;
-  return cuda_status(launch_step_post(p, shape->bits, shape->group, shape->heads_q / shape->heads_kv,
+  return cuda_status(launch_step_post(p, lo_bits_of(*shape), lo_group_of(*shape), shape->heads_q / shape->heads_kv,
                                       out_dtype == MIKV_OUT_F32, static_cast<cudaStream_t>(stream)));
 }
 

@@ -43,7 +43,7 @@ AttnPlan plan_attention(const mikv_shape& s, int n_lo, int num_sms) {
   const int kh = hb == 16 ? 1 : lo_unit_layout(hb, kHiGroup).blocks;
   p.hi_units = (p.hi_blocks + kh - 1) / kh;
   p.lo_blocks = (n_lo + 15) / 16;
-  const int k = lo_unit_layout(s.bits, s.group).blocks;
+  const int k = evicting(s) ? 1 : lo_unit_layout(s.bits, s.group).blocks;
   p.lo_units = (p.lo_blocks + k - 1) / k;
   p.n_u = p.hi_units + p.lo_units;
   const long long bh = (long long)s.batch * s.heads_kv;

@@ -124,6 +124,7 @@ struct StepPostArgs {
   const void* k_hi_params;  // coded important set: (alpha, beta) of the important rows
   const void* v_hi_params;
   int hi_bits;              // 16 = bf16 important rows; 8, 4, 2 = coded (groups of kHiGroup)
+  int evict;                // no retained set: the victim's slot is freed, nothing is demoted
   int batch, heads_q, heads_kv, hi_cap, hi_stride, lo_cap, n_lo;
   int n_u, n_units, n_warps;
 };
@@ -140,6 +141,11 @@ cudaError_t launch_attention_h4(const AttnArgs& a, int bits, int group, int G, i
 cudaError_t launch_attention_h2(const AttnArgs& a, int bits, int group, int G, int grid, cudaStream_t st);
 // effective important-set precision of a shape: 16 for bf16 (hi_bits 0 or 16)
 inline int hi_bits_of(const mikv_shape& s) { return s.hi_bits == 0 ? 16 : s.hi_bits; }
+// bits == 0: no retained set, demoted tokens are evicted (the H2O baseline). The kernels then run with
+// any retained layout (none of its units exist); these give the one they are instantiated with.
+inline bool evicting(const mikv_shape& s) { return s.bits == 0; }
+inline int lo_bits_of(const mikv_shape& s) { return s.bits == 0 ? 2 : s.bits; }
+inline int lo_group_of(const mikv_shape& s) { return s.bits == 0 ? 32 : s.group; }
 cudaError_t launch_merge(const MergeArgs& a, int G, int out_f32, cudaStream_t st);
 
 cudaError_t launch_quantize_pack(const mikv_shape& s, const mikv_cache& c, const void* k_src,

@@ -151,7 +151,9 @@ __global__ void __launch_bounds__(kPostThreads, 2) step_post_kernel(const StepPo
 
   // 3. demote the victim: quantize its key (balanced, Eq. 3) and value rows into retained row n_lo; a
   // coded important row is re-quantized from its fp32 dequantized values (already balanced, Sec. 3.3)
-  if (warp < 2) {
+  if (a.evict) {  // eviction (no retained set): the victim's slot only becomes the next insertion slot
+    if (tid == 0) a.slots[bh] = victim;
+  } else if (warp < 2) {
     const bool is_v = warp == 1;
     const size_t pos = (size_t)bh * a.lo_cap + a.n_lo;
     const size_t hrow = (size_t)bh * a.hi_stride + victim;

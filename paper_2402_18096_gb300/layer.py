@@ -15,8 +15,8 @@ import math
 
 import torch
 
-from . import (LayerCache, Shape, WS_BALANCER, WS_STEP, mikv_compute_balancer, mikv_decode_step,
-               mikv_gather_hi, mikv_quantize_pack, mikv_select_demote, mikv_workspace_bytes)
+from . import (LayerCache, Shape, WS_BALANCER, WS_STEP, mikv_compute_balancer, mikv_decode_attention,
+               mikv_decode_step, mikv_gather_hi, mikv_quantize_pack, mikv_select_demote, mikv_workspace_bytes)
 
 
 def workspace(nbytes: int, device="cuda") -> torch.Tensor:
@@ -54,9 +54,9 @@ class MixedPrecisionLayer:
         mikv_select_demote(scores, T, n_demote, demoted, kept)
         if k_budget > 0:
             mikv_gather_hi(layer.cache, k, v, kept, src_scores=scores)
-        if n_demote > 0:
+        if n_demote > 0 and shape.bits:
             mikv_quantize_pack(layer.cache, k, v, demoted, 0)
-        layer.n_lo = n_demote
+        layer.n_lo = n_demote if shape.bits else 0  # bits = 0: eviction, the demoted tokens are dropped
         layer.pos = T
         layer.slots.fill_(k_budget)  # the staging slot receives the first decoded token
         return layer
@@ -65,5 +65,44 @@ class MixedPrecisionLayer:
         """One decode step: the new token enters, attention runs, the least important slot is demoted."""
         mikv_decode_step(self.cache, self.n_lo, q, k_new, v_new, self.pos, self.slots, self.sm_scale, out,
                          self.ws)
-        self.n_lo += 1
+        if self.shape.bits:
+            self.n_lo += 1
         self.pos += 1
+
+
+def oracle_eviction_attention(k, v, q, budget: int, sm_scale: float, out, device="cuda"):
+    """Oracle eviction (Sec. 2.2, Fig. 2), the comparison baseline: attention computed over the full bf16
+    cache k, v [B, Hkv, T, d] for q [B, Hq, d], then top-k sparsity imposed on the attention map. Reading:
+    each query head keeps its `budget` largest attention weights (ties: the smaller token index) and the
+    output is the softmax over the logits of those tokens (the kept weights renormalised). Built from the
+    library's entry points only: full attention with its logits, selection of the T - budget smallest
+    logits (mikv_select_demote) whose complement is kept, gather of the kept rows, and attention over them; query heads of a KV head are handled one by one
+    because each keeps its own tokens. Writes out [B, Hq, d]; returns the kept token indices [B, Hq, budget]."""
+    B, H, T, d = k.shape
+    Hq = q.shape[1]
+    G = Hq // H
+    full = Shape(B, H, H, 2, 32, T, 16)  # one query head per KV head at a time; bf16 important set of T rows
+    cache = LayerCache(full, device=device)
+    rows = torch.arange(T, dtype=torch.int32, device=device).expand(B, H, T).contiguous()
+    mikv_gather_hi(cache, k, v, rows)
+    kept_all = torch.empty(B, Hq, budget, dtype=torch.int32, device=device)
+    small = Shape(B, H, H, 2, 32, budget, 16)
+    ws = workspace(max(mikv_workspace_bytes(full, 0, 0), mikv_workspace_bytes(small, 0, 0)), device)
+    # ids T-1-t: among equal logits the larger token index is dropped first, so the smaller one is kept
+    ids = torch.arange(T - 1, -1, -1, dtype=torch.int32, device=device).expand(B, H, T).contiguous()
+    ids = torch.nn.functional.pad(ids, (0, full.hi_stride - T))
+    for j in range(G):
+        qj = q[:, j::G].contiguous()
+        logits = torch.empty(B, H, full.hi_stride, dtype=torch.float32, device=device)
+        tmp = torch.empty(B, H, d, dtype=torch.float32, device=device)
+        mikv_decode_attention(cache, 0, qj, sm_scale, tmp, ws, hi_logits=logits)
+        kept = torch.empty(B, H, budget, dtype=torch.int32, device=device)
+        dropped = torch.empty(B, H, T - budget, dtype=torch.int32, device=device)
+        mikv_select_demote(logits, T, T - budget, dropped, kept=kept, ids=ids)
+        sel = LayerCache(small, device=device)
+        mikv_gather_hi(sel, k, v, kept)
+        oj = torch.empty(B, H, d, dtype=out.dtype, device=device)
+        mikv_decode_attention(sel, 0, qj, sm_scale, oj, ws)
+        out[:, j::G] = oj
+        kept_all[:, j::G] = kept
+    return kept_all

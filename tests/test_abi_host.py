@@ -93,6 +93,7 @@ def test_workspace_sizes_monotone(lib):
     (dict(lo_cap=60), 1), (dict(batch=0), 1), (dict(hi_stride=16, hi_cap=20), 1),
     (dict(hi_bits=3), 2), (dict(hi_bits=12), 2), (dict(hi_bits=8, hi_group=32), 2), (dict(hi_bits=4, hi_group=128), 2),
     (dict(hi_bits=8), 0), (dict(hi_bits=4), 0), (dict(hi_bits=2), 0), (dict(hi_bits=16, hi_group=0), 0),
+    (dict(bits=0, group=7), 0), (dict(bits=-1), 1),
 ])
 def test_shape_validation(lib, kw, code):
     s = _shape(**kw)
@@ -119,6 +120,12 @@ def test_argument_validation_before_launch(lib):
     assert lib.mikv_quantize_pack(ctypes.byref(sq), ctypes.byref(no_hp), P, P, None, 4, P, 1, 0, None) == 1
     odd_hp = pkg._Cache(*([P] * 9 + [None, P + 8, P]))
     assert lib.mikv_quantize_pack(ctypes.byref(sq), ctypes.byref(odd_hp), P, P, None, 4, P, 1, 0, None) == 1
+    # eviction (bits = 0): there is no retained set to write, and attention takes no retained rows
+    se = _shape(bits=0, lo_cap=0)
+    no_lo = pkg._Cache(*([P] * 4 + [None] * 8))
+    assert lib.mikv_quantize_pack(ctypes.byref(se), ctypes.byref(no_lo), P, P, None, 4, P, 1, 0, None) == 2
+    assert lib.mikv_decode_attention(ctypes.byref(se), ctypes.byref(no_lo), 1, P, ctypes.c_float(1.0), P, 0, None, None,
+                                     P, 1 << 20, None) == 3
     # attention: n_lo beyond capacity, bad output type, missing or misaligned workspace
     assert lib.mikv_decode_attention(ctypes.byref(s), ctypes.byref(c), 65, P, 1.0, P, 0, None, None, P, 1 << 20,
                                      None) == 3
