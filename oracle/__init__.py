@@ -74,6 +74,7 @@ def _load():
                 "mikv_ref_gather_hi": (I, [I, I, I, I, P, P, P, P, I, P, I, P, P, P, P]),
                 "mikv_ref_cache_fraction": (D, [I, I, D, I]),
                 "mikv_ref_dequantize_row_f32": (I, [P, P, I, I, I, P]),
+                "mikv_ref_prefill_scores": (I, [I, I, I, I, I, P, P, D, P]),
                 "mikv_ref_gather_hi_q": (I, [I, I, I, I, I, I, P, P, P, P, I, P, I, P, P, P, P, P, P, P]),
                 "mikv_ref_insert_token_q": (I, [I, I, I, I, I, I, P, P, I, P, P, P, P, P, P, P, P]),
                 "mikv_ref_decode_attention_q": (I, [I, I, I, I, I, I, I, I, I, I, I, P, P, P, P, P, P, P, P,
@@ -345,6 +346,19 @@ def dequantize_row_f32(packed, params, bits: int, g: int, d: int = 128):
     params = _arr(params, np.uint16)
     out = np.zeros(d, np.float32)
     _check(_load().mikv_ref_dequantize_row_f32(_p(packed), _p(params), d, bits, g, _p(out)), "dequantize_row_f32")
+    return out
+
+
+def prefill_scores(q_pre, k_pre, sm_scale: float):
+    """Initial importance from the prefill's causal attention: q_pre uint16 [B, Hq, T, d], k_pre uint16
+    [B, Hkv, T, d] (bf16 bits) -> fp64 [B, Hkv, T]."""
+    q_pre = _arr(q_pre, np.uint16)
+    k_pre = _arr(k_pre, np.uint16)
+    B, Hq, T, d = q_pre.shape
+    Hkv = k_pre.shape[1]
+    out = np.zeros((B, Hkv, T), np.float64)
+    _check(_load().mikv_ref_prefill_scores(B, Hq, Hkv, T, d, _p(q_pre), _p(k_pre), float(sm_scale), _p(out)),
+           "prefill_scores")
     return out
 
 

@@ -637,6 +637,46 @@ int mikv_ref_demote_hi_q(int B, int Hkv, int d, int hi_cap, int hi_bits, int hg,
   return 0;
 }
 
+/* ---------------------------------------------------------------- prefill importance */
+
+/*
+ * Initial importance of every prefill token: the accumulated attention it receives from the prefill's
+ * causal attention (H2O's heavy-hitter score, the policy MiKV plugs in, Fig. 4 / Sec. 3): for KV head h,
+ * scores[t] = sum over the G query heads j of h and over queries i >= t of the causal softmax weight
+ * softmax_{t' <= i}(sm_scale * q_i . k_t') at t' = t. Reading: the same accumulation as the decode-time
+ * update (R9) applied to the prefill queries; fp64 throughout.
+ * q_pre bf16 [B][Hq][T][d], k_pre bf16 [B][Hkv][T][d], scores fp64 [B][Hkv][T].
+ */
+int mikv_ref_prefill_scores(int B, int Hq, int Hkv, int T, int d, const uint16_t* q_pre, const uint16_t* k_pre,
+                            double sm_scale, double* scores) {
+  if (B <= 0 || Hkv <= 0 || Hq % Hkv || T <= 0 || d <= 0) return -1;
+  int G = Hq / Hkv;
+  double* s = (double*)malloc(sizeof(double) * (size_t)T);
+  if (!s) return -1;
+  for (size_t x = 0; x < (size_t)B * Hkv * T; ++x) scores[x] = 0.0;
+  for (int b = 0; b < B; ++b)
+    for (int hq = 0; hq < Hq; ++hq) {
+      int h = hq / G;
+      const uint16_t* qh = q_pre + ((size_t)b * Hq + hq) * T * d;
+      const uint16_t* kh = k_pre + ((size_t)b * Hkv + h) * T * d;
+      double* out = scores + ((size_t)b * Hkv + h) * T;
+      for (int i = 0; i < T; ++i) {
+        double m = -INFINITY;
+        for (int t = 0; t <= i; ++t) {
+          double acc = 0.0;
+          for (int c = 0; c < d; ++c) acc += (double)bf16_to_f32(qh[(size_t)i * d + c]) * bf16_to_f32(kh[(size_t)t * d + c]);
+          s[t] = sm_scale * acc;
+          if (s[t] > m) m = s[t];
+        }
+        double l = 0.0;
+        for (int t = 0; t <= i; ++t) l += exp(s[t] - m);
+        for (int t = 0; t <= i; ++t) out[t] += exp(s[t] - m) / l;
+      }
+    }
+  free(s);
+  return 0;
+}
+
 /* ---------------------------------------------------------------- memory accounting */
 
 /*

@@ -136,6 +136,12 @@ int mikv_ref_demote_hi_q(int B, int Hkv, int d, int hi_cap, int hi_bits, int hg,
                          const uint16_t* k_hp, const uint16_t* v_hp, const int32_t* hi_tok, uint8_t* k_codes,
                          uint8_t* v_codes, uint16_t* k_params, uint16_t* v_params, int32_t* lo_tok);
 
+/* Prefill importance (the initial accumulated-attention score of every token): scores[b][h][t] = sum over
+ * the G query heads of KV head h and the queries i >= t of the causal softmax weight of key t in row i,
+ * s = sm_scale * q . k. q_pre bf16 [B][Hq][T][d], k_pre bf16 [B][Hkv][T][d], scores fp64 [B][Hkv][T]. */
+int mikv_ref_prefill_scores(int B, int Hq, int Hkv, int T, int d, const uint16_t* q_pre, const uint16_t* k_pre,
+                            double sm_scale, double* scores);
+
 /* Closed-form KV-cache size as a fraction of an all-fp16 cache: ratio r of tokens at hi_bits
  * (16 = fp16, else hi_bits-bit codes with fp16 alpha/beta per group g) plus (1 - r) at bits-bit codes
  * with fp16 alpha/beta per group g. */
