@@ -95,13 +95,13 @@ typedef struct {
 enum { MIKV_OUT_BF16 = 0, MIKV_OUT_F32 = 1 };
 
 /* Which operation a workspace is sized for (mikv_workspace_bytes). */
-enum { MIKV_WS_ATTENTION = 0, MIKV_WS_BALANCER = 1, MIKV_WS_STEP = 2 };
+enum { MIKV_WS_ATTENTION = 0, MIKV_WS_BALANCER = 1, MIKV_WS_STEP = 2, MIKV_WS_PREFILL = 3 };
 
 /* Human-readable name of a status code (static string). */
 const char* mikv_status_string(mikv_status s);
 
 /* Bytes of workspace `op` needs for `shape` with up to `n_lo_max` retained rows per head (the
- * attention split count depends on it). Returns 0 for an invalid shape. The workspace must be
+ * attention split count depends on it; for MIKV_WS_PREFILL the third argument is the prefill length T). Returns 0 for an invalid shape. The workspace must be
  * 256-byte aligned; its first 16 bytes hold a status word that kernels set on an internal failure. */
 size_t mikv_workspace_bytes(const mikv_shape* shape, int32_t op, int32_t n_lo_max);
 
@@ -145,6 +145,24 @@ mikv_status mikv_compute_balancer(const mikv_shape* shape, const void* q_pre, co
 mikv_status mikv_quantize_pack(const mikv_shape* shape, const mikv_cache* cache, const void* k_src,
                                const void* v_src, const int32_t* src_tok, int32_t n_src,
                                const int32_t* rows, int32_t n_rows, int32_t lo_start, void* stream);
+
+/*
+ * Initial importance of the prefill tokens: the accumulated attention each key receives from the prefill's
+ * causal attention (the heavy-hitter score of Fig. 4 / Sec. 3, here taken over the prefill queries):
+ *   scores[b][h][t] = sum over the G query heads j of KV head h and the queries i >= t of
+ *                     exp(s_it - m_i) / l_i,  s_it = sm_scale * q_pre[b][hG+j][i] . k_pre[b][h][t],
+ *   m_i = max_{t' <= i} s_it', l_i = sum_{t' <= i} exp(s_it' - m_i)  (the causal softmax of row i).
+ * These are the scores mikv_select_demote / mikv_gather_hi take to build the cache. Two tensor-core
+ * passes over the causal triangle (row statistics, then column sums), fp32 accumulation.
+ *   q_pre      bf16 [B][Hq][T][d], 16-byte aligned (prefill queries after the positional embedding)
+ *   k_pre      bf16 [B][Hkv][T][d], 16-byte aligned
+ *   scores     fp32 [B][Hkv][T]
+ *   workspace  >= mikv_workspace_bytes(shape, MIKV_WS_PREFILL, T) bytes, 256-byte aligned (the row
+ *              statistics; its status word reports an internal failure as in the other entry points)
+ * Only batch, heads_q, heads_kv and head_dim of `shape` are used. Requires B * Hq * T < 2^31.
+ */
+mikv_status mikv_prefill_scores(const mikv_shape* shape, const void* q_pre, const void* k_pre, int32_t T,
+                                float sm_scale, float* scores, void* workspace, size_t ws_bytes, void* stream);
 
 /*
  * Single-token decode attention over the mixed-precision cache (Eq. 3-4; Sec. 3.4):

@@ -8,6 +8,7 @@ library is not built or no GPU is present, calls raise.
 from __future__ import annotations
 
 import ctypes
+import math
 import os
 import threading
 from dataclasses import dataclass
@@ -21,13 +22,13 @@ __all__ = [
     "mikv_workspace_reset", "mikv_workspace_check", "mikv_compute_balancer", "mikv_quantize_pack",
     "mikv_decode_attention", "mikv_update_importance", "mikv_select_demote", "mikv_insert_token",
     "mikv_gather_hi", "mikv_decode_step", "mikv_cache_fraction", "mikv_retained_row_bytes",
-    "mikv_decode_attention_noalloc", "NOALLOC_SCRATCH_BYTES",
-    "WS_ATTENTION", "WS_BALANCER", "WS_STEP", "OUT_BF16", "OUT_F32", "HEAD_DIM",
+    "mikv_decode_attention_noalloc", "NOALLOC_SCRATCH_BYTES", "mikv_prefill_scores",
+    "WS_ATTENTION", "WS_BALANCER", "WS_STEP", "WS_PREFILL", "OUT_BF16", "OUT_F32", "HEAD_DIM",
 ]
 
 HEAD_DIM = 128
 OUT_BF16, OUT_F32 = 0, 1
-WS_ATTENTION, WS_BALANCER, WS_STEP = 0, 1, 2
+WS_ATTENTION, WS_BALANCER, WS_STEP, WS_PREFILL = 0, 1, 2, 3
 STATUS = {0: "MIKV_OK", 1: "MIKV_ERR_ARG", 2: "MIKV_ERR_UNSUPPORTED", 3: "MIKV_ERR_CAPACITY",
           4: "MIKV_ERR_CUDA", 5: "MIKV_ERR_WORKSPACE", 6: "MIKV_ERR_DEVICE", 7: "MIKV_ERR_SCRATCH"}
 NOALLOC_SCRATCH_BYTES = 8 << 20
@@ -83,6 +84,7 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
                 "mikv_gather_hi": (I, [SP, CP, P, P, P, P, I, P, I, P]),
                 "mikv_decode_step": (I, [SP, CP, I, P, P, P, I, P, F, P, I, P, Z, P]),
                 "mikv_decode_attention_noalloc": (I, [SP, CP, I, P, F, P, I, P, P, P]),
+                "mikv_prefill_scores": (I, [SP, P, P, I, F, P, P, Z, P]),
                 "mikv_cache_fraction": (ctypes.c_double, [I, I, ctypes.c_double, I]),
                 "mikv_retained_row_bytes": (Z, [I, I, I]),
             }
@@ -261,6 +263,16 @@ def mikv_decode_step(cache: LayerCache, n_lo: int, q, k_new, v_new, tok: int, sl
     _check("mikv_decode_step", load().mikv_decode_step(
         ctypes.byref(cache.shape.c()), ctypes.byref(cache.c()), n_lo, _ptr(q), _ptr(k_new), _ptr(v_new), tok,
         _ptr(slots), float(sm_scale), _ptr(out), out_dtype, _ptr(workspace), workspace.numel(), _stream(stream)))
+
+
+def mikv_prefill_scores(shape: Shape, q_pre, k_pre, scores, workspace, sm_scale: float = None, stream=None):
+    """Initial importance of the prefill tokens into scores [B, Hkv, T] (fp32) from q_pre [B, Hq, T, d] and
+    k_pre [B, Hkv, T, d] (bf16); workspace of mikv_workspace_bytes(shape, WS_PREFILL, T) bytes."""
+    T = k_pre.shape[2]
+    scale = 1.0 / math.sqrt(shape.head_dim) if sm_scale is None else sm_scale
+    _check("mikv_prefill_scores", load().mikv_prefill_scores(
+        ctypes.byref(shape.c()), _ptr(q_pre), _ptr(k_pre), T, float(scale), _ptr(scores), _ptr(workspace),
+        workspace.numel(), _stream(stream)))
 
 
 def mikv_cache_fraction(bits: int, group: int, ratio: float, hi_bits: int = 16) -> float:

@@ -10,6 +10,7 @@
 
 #include "mikv_device.cuh"
 #include "mikv_internal.h"
+#include "mikv_prefill.h"
 
 using namespace mikv;
 
@@ -277,6 +278,7 @@ size_t mikv_workspace_bytes(const mikv_shape* shape, int32_t op, int32_t n_lo_ma
     case MIKV_WS_ATTENTION: return attention_workspace_bytes(*shape, n_lo_max, num_sms());
     case MIKV_WS_BALANCER: return kWsHeader + 2 * (size_t)shape->heads_kv * kHeadDim * sizeof(uint32_t);
     case MIKV_WS_STEP: return step_layout(shape, n_lo_max).total;
+    case MIKV_WS_PREFILL: return prefill_workspace_bytes(shape->batch, shape->heads_q, n_lo_max);
   }
   return 0;
 }
@@ -320,6 +322,37 @@ mikv_status mikv_quantize_pack(const mikv_shape* shape, const mikv_cache* cache,
     return MIKV_ERR_UNSUPPORTED;
   return cuda_status(launch_quantize_pack(*shape, *cache, k_src, v_src, src_tok, n_src, rows, n_rows, lo_start,
                                           static_cast<cudaStream_t>(stream)));
+}
+
+mikv_status mikv_prefill_scores(const mikv_shape* shape, const void* q_pre, const void* k_pre, int32_t T,
+                                float sm_scale, float* scores, void* workspace, size_t ws_bytes, void* stream) {
+  mikv_status st = shape_supported(shape);
+  if (st != MIKV_OK) return st;
+  if (!q_pre || !k_pre || !scores || T <= 0) return MIKV_ERR_ARG;
+  if (!aligned(q_pre, 16) || !aligned(k_pre, 16) || !aligned(scores, 4)) return MIKV_ERR_ARG;
+  if ((int64_t)shape->batch * shape->heads_q * T + kPfTile >= 2147483647LL ||
+      (int64_t)shape->batch * shape->heads_q > 65535)
+    return MIKV_ERR_UNSUPPORTED;
+  if (!workspace || !aligned(workspace, 256) || ws_bytes < prefill_workspace_bytes(shape->batch, shape->heads_q, T))
+    return MIKV_ERR_WORKSPACE;
+  PrefillArgs a;
+  memset(&a, 0, sizeof a);
+  const uint64_t qrows = (uint64_t)shape->batch * shape->heads_q * T;
+  const uint64_t krows = (uint64_t)shape->batch * shape->heads_kv * T;
+  if (!make_map(&a.map_q, q_pre, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, kHeadDim, qrows, 2 * kHeadDim, 64, kPfTile,
+                CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !make_map(&a.map_k, k_pre, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, kHeadDim, krows, 2 * kHeadDim, 64, kPfTile,
+                CU_TENSOR_MAP_SWIZZLE_128B))
+    return MIKV_ERR_CUDA;
+  char* wsb = static_cast<char*>(workspace);
+  a.status = reinterpret_cast<int*>(wsb);
+  a.stats = reinterpret_cast<float2*>(wsb + kWsHeader);
+  a.scores = scores;
+  a.heads_q = shape->heads_q;
+  a.heads_kv = shape->heads_kv;
+  a.T = T;
+  a.scale_log2 = sm_scale * 1.4426950408889634f;
+  return cuda_status(launch_prefill(a, shape->batch, static_cast<cudaStream_t>(stream)));
 }
 
 mikv_status mikv_decode_attention(const mikv_shape* shape, const mikv_cache* cache, int32_t n_lo, const void* q,

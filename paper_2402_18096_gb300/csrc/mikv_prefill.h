@@ -1,0 +1,33 @@
+// mikv_prefill.h — arguments of the prefill-importance kernels (mikv_prefill.cu).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include "mikv_device.cuh"
+#include "mikv_internal.h"
+
+namespace mikv {
+
+// Tiles of 64 tokens x 128 channels (bf16) stream through shared memory by TMA.
+constexpr int kPfTile = 64;
+
+struct PrefillArgs {
+  CUtensorMap map_q;  // q_pre rows [B * Hq * T][128] bf16, box 64 channels x 64 rows, 128B swizzle
+  CUtensorMap map_k;  // k_pre rows [B * Hkv * T][128] bf16, same boxes
+  float2* stats;      // [B * Hq][T]: (row max of the logits in log2 units, 1 / row sum)
+  float* scores;      // [B * Hkv][T]
+  int* status;        // workspace status word
+  int heads_q, heads_kv, T;
+  float scale_log2;   // sm_scale * log2(e)
+};
+
+// Workspace of mikv_prefill_scores: the status header plus the per-query row statistics.
+inline size_t prefill_workspace_bytes(int batch, int heads_q, int T) {
+  const size_t stats = (size_t)batch * heads_q * T * sizeof(float2);
+  return kWsHeader + (stats + 255) / 256 * 256;
+}
+
+cudaError_t launch_prefill(const PrefillArgs& a, int batch, cudaStream_t st);
+
+}  // namespace mikv

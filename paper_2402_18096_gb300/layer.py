@@ -15,8 +15,9 @@ import math
 
 import torch
 
-from . import (LayerCache, Shape, WS_BALANCER, WS_STEP, mikv_compute_balancer, mikv_decode_attention,
-               mikv_decode_step, mikv_gather_hi, mikv_quantize_pack, mikv_select_demote, mikv_workspace_bytes)
+from . import (LayerCache, Shape, WS_BALANCER, WS_PREFILL, WS_STEP, mikv_compute_balancer, mikv_decode_attention,
+               mikv_decode_step, mikv_gather_hi, mikv_prefill_scores, mikv_quantize_pack, mikv_select_demote,
+               mikv_workspace_bytes)
 
 
 def workspace(nbytes: int, device="cuda") -> torch.Tensor:
@@ -39,8 +40,16 @@ class MixedPrecisionLayer:
     @classmethod
     def from_prefill(cls, shape: Shape, k, v, scores, q_pre=None, budget: int = None, device="cuda"):
         """Build the cache from prefill K, V [B, Hkv, T, d] (bf16) and importance scores [B, Hkv, T].
-        With q_pre [B, Hq, T, d] the channel balancer is computed (Eq. 2); without it, b = 1."""
+        With q_pre [B, Hq, T, d] the channel balancer is computed (Eq. 2); without it, b = 1. With scores
+        None the importance is the prefill's accumulated causal attention (mikv_prefill_scores, q_pre
+        required)."""
         B, H, T, _ = k.shape
+        if scores is None:
+            if q_pre is None:
+                raise ValueError("prefill scores need the prefill queries")
+            scores = torch.empty(B, H, T, dtype=torch.float32, device=device)
+            ws = workspace(mikv_workspace_bytes(shape, WS_PREFILL, T), device)
+            mikv_prefill_scores(shape, q_pre, k, scores, ws)
         k_budget = shape.hi_cap - 1 if budget is None else budget
         bal = None
         if q_pre is not None:
