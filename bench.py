@@ -484,6 +484,56 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+def run_prefill(args):
+    """Prefill importance (mikv_prefill_scores) for one layer of the workload: the accumulated causal
+    attention of every prefill token; tensor-core roofline against the measured bf16 peak."""
+    import paper_2402_18096_gb300 as pkg
+    from paper_2402_18096_gb300.layer import workspace
+    w = mi.WORKLOADS[args.workload]
+    if args.batch:
+        w = mi.scaled(w, batch=args.batch)
+    dev = torch.device("cuda")
+    pkg.load()
+    k, _ = mi.prefill_kv(w, 0, dev)
+    q = mi.prefill_queries(w, 0, dev)
+    shape = pkg.Shape(w.batch, w.heads_q, w.heads_kv, 2, 32, 1, 16)
+    out = torch.empty(w.batch, w.heads_kv, w.context, device=dev)
+    ws = workspace(pkg.mikv_workspace_bytes(shape, pkg.WS_PREFILL, w.context), dev)
+    for _ in range(args.warmup):
+        pkg.mikv_prefill_scores(shape, q, k, out, ws)
+    torch.cuda.synchronize()
+    sampler = ClockSampler(torch.cuda.current_device())
+    sampler.start()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(args.steps):
+        pkg.mikv_prefill_scores(shape, q, k, out, ws)
+    e1.record()
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    pkg.mikv_workspace_check(ws)
+    ms = e0.elapsed_time(e1) / args.steps
+    T = w.context
+    # algorithmic work: two passes (row statistics, column sums) over the causal triangle of Q K^T
+    flops = 2.0 * w.batch * w.heads_q * (T * (T + 1) / 2) * 2 * w.head_dim
+    tflops = flops / ms / 1e9
+    peak, kind = None, "fallback"
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            peak, kind = float(json.load(f)["bf16_tflops"]), "measured"
+    if peak is None:
+        peak = 1900.0
+    print(json.dumps({
+        "metric": "prefill importance (accumulated causal attention) TFLOP/s", "value": round(tflops, 1),
+        "unit": "TFLOP/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_layer": round(ms, 3),
+        "higher_is_better": True, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": w.name, "batch": w.batch, "heads_q": w.heads_q, "heads_kv": w.heads_kv, "context": T},
+        "roofline": {"kernel": "prefill_rows_kernel + prefill_cols_kernel", "bound": "tensor", "achieved": round(tflops, 1),
+                     "peak": peak, "peak_kind": kind + " bf16 burst", "unit": "TFLOP/s", "frac": round(tflops / peak, 3)},
+        "clocks": clocks}))
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -496,6 +546,7 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--sweep", action="store_true", help="the batch-64 bits x ratio x group sweep (one layer)")
+    ap.add_argument("--prefill", action="store_true", help="prefill importance scores of one layer")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "mikv" and not (args.batch or args.layers):
         ap.error("--warmup must be >= 3")
@@ -503,6 +554,8 @@ def main():
         run_reference(args)
     elif args.sweep:
         run_sweep(args)
+    elif args.prefill:
+        run_prefill(args)
     else:
         run_mikv(args)
 
