@@ -473,7 +473,7 @@ def run_reference(args):
     value = sum(nbytes) / sum(times) / 1e9
     ms = 1e3 * sum(times) / K
     line = {
-        "impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": UNIT, "n_gpus": 0,
+        "impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": UNIT, "n_gpus": args.gpus,
         "steps": K, "warmup": W, "ms_per_step": round(ms, 3), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64 attention, f32 quantizer", "data": "synthetic",
         "config": {"workload": w.name, "sample": "one KV head (batch row 0, head 0) of layer 0 per step"},

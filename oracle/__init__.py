@@ -75,6 +75,10 @@ def _load():
                 "mikv_ref_cache_fraction": (D, [I, I, D, I]),
                 "mikv_ref_dequantize_row_f32": (I, [P, P, I, I, I, P]),
                 "mikv_ref_prefill_scores": (I, [I, I, I, I, I, P, P, D, P]),
+                "mikv_ref_quantize_channel_group": (I, [P, I, I, P, P]),
+                "mikv_ref_append_retained_kch": (I, [I, I, I, I, I, I, I, I, I, P, P, P, I, P, I, P, P, P, P, P, P, P,
+                                                     P]),
+                "mikv_ref_decode_attention_kch": (I, [I, I, I, I, I, I, I, I, I, I, P, P, P, P, P, P, P, D, P, P, P]),
                 "mikv_ref_gather_hi_q": (I, [I, I, I, I, I, I, P, P, P, P, I, P, I, P, P, P, P, P, P, P]),
                 "mikv_ref_insert_token_q": (I, [I, I, I, I, I, I, P, P, I, P, P, P, P, P, P, P, P]),
                 "mikv_ref_decode_attention_q": (I, [I, I, I, I, I, I, I, I, I, I, I, P, P, P, P, P, P, P, P,
@@ -208,6 +212,8 @@ def decode_attention(cache: dict, q, n_lo: int, sm_scale: float, balancer_=None)
     q: uint16 bf16 bits [B, Hq, d]."""
     if cache.get("hi_bits", 16) < 16:
         return _decode_attention_q(cache, q, n_lo, sm_scale, balancer_)
+    if cache.get("kch"):
+        return _decode_attention_kch(cache, q, n_lo, sm_scale)
     q = _arr(q, np.uint16)
     B, Hq, d = q.shape
     k_hi = _arr(cache["k_hi"], np.uint16)
@@ -250,6 +256,58 @@ def _decode_attention_q(cache: dict, q, n_lo: int, sm_scale: float, balancer_=No
         B, Hq, Hkv, d, hb, hg, bits, g, hi_cap, lo_cap, n_lo, _p(khc), _p(vhc), _p(khp), _p(vhp), _p(kc),
         _p(vc), _p(kp), _p(vp), _p(bal), _p(q), float(sm_scale), _p(out), _p(hl), _p(ml)), "decode_attention_q")
     return out, hl, ml
+
+
+def _decode_attention_kch(cache: dict, q, n_lo: int, sm_scale: float):
+    """Per-channel retained keys: the important set plus the n_lo mod 64 staged tokens in bf16, the rest of
+    the retained set in quantized groups. hi_logits covers the important slots and the staged rows."""
+    q = _arr(q, np.uint16)
+    B, Hq, d = q.shape
+    k_hi = _arr(cache["k_hi"], np.uint16)
+    v_hi = _arr(cache["v_hi"], np.uint16)
+    Hkv, hi_rows = k_hi.shape[1], k_hi.shape[2]
+    n_stage = n_lo % 64
+    n_hi, n_lo_q = cache["hi_cap"] + n_stage, n_lo - n_stage
+    kc = _arr(cache["k_codes"], np.uint8)
+    vc = _arr(cache["v_codes"], np.uint8)
+    kp = _arr(cache["k_params"], np.uint16)
+    vp = _arr(cache["v_params"], np.uint16)
+    lo_cap, bits = kc.shape[2], kc.shape[3] // 16
+    g = d // vp.shape[3]
+    out = np.zeros((B, Hq, d), np.float64)
+    hl = np.zeros((B, Hq, n_hi), np.float64)
+    ml = np.zeros((B, Hq, 2), np.float64)
+    _check(_load().mikv_ref_decode_attention_kch(
+        B, Hq, Hkv, d, bits, g, hi_rows, n_hi, lo_cap, n_lo_q, _p(k_hi), _p(v_hi), _p(kc), _p(vc), _p(kp), _p(vp),
+        _p(q), float(sm_scale), _p(out), _p(hl), _p(ml)), "decode_attention_kch")
+    return out, hl, ml
+
+
+def quantize_channel_group(x, bits: int):
+    """Per-channel quantization of 64 token rows (App. C): x fp32 [64, 128] -> (packed uint8 [64, 16*bits],
+    params uint16 [128, 2] = (alpha16, beta16) per channel)."""
+    x = _arr(x, np.float32)
+    packed = np.zeros((64, 16 * bits), np.uint8)
+    params = np.zeros((128, 2), np.uint16)
+    _check(_load().mikv_ref_quantize_channel_group(_p(x), 128, bits, _p(packed), _p(params)), "quantize_channel_group")
+    return packed, params
+
+
+def append_retained(cache: dict, k_src, v_src, rows, n_lo: int, src_tok=None):
+    """Per-channel-key cache: append rows rows[b, h, :] of k_src/v_src (uint16 [B, Hkv, n_src, d]) at retained
+    positions n_lo.. (staged in bf16; quantized per group of 64 when a group completes)."""
+    k_src = _arr(k_src, np.uint16)
+    v_src = _arr(v_src, np.uint16)
+    rows = _arr(rows, np.int32)
+    src_tok = _arr(src_tok, np.int32)
+    B, Hkv, n_src, d = k_src.shape
+    kc = cache["k_codes"]
+    lo_cap, bits = kc.shape[2], kc.shape[3] // 16
+    g = d // cache["v_params"].shape[3]
+    _check(_load().mikv_ref_append_retained_kch(
+        B, Hkv, d, bits, g, cache["hi_cap"], cache["k_hi"].shape[2], lo_cap, n_lo, _p(k_src), _p(v_src), _p(src_tok),
+        n_src, _p(rows), rows.shape[2], _p(cache["k_hi"]), _p(cache["v_hi"]), _p(cache["hi_tok"]), _p(cache["k_codes"]),
+        _p(cache["v_codes"]), _p(cache["k_params"]), _p(cache["v_params"]), _p(cache["lo_tok"])), "append_retained_kch")
 
 
 def update_importance(acc, hi_logits, ml, Hq: int):
@@ -367,9 +425,15 @@ def cache_fraction(bits: int, g: int, ratio: float, hi_bits: int = 16) -> float:
 
 
 def empty_cache(B: int, Hkv: int, d: int, bits: int, g: int, hi_cap: int, lo_cap: int, hi_bits: int = 16,
-                hi_group: int = 64) -> dict:
+                hi_group: int = 64, k_channel: bool = False) -> dict:
     """Zero-initialised numpy arrays in the oracle's (dense) layout. With hi_bits < 16 the important set
-    holds codes (k_hi, v_hi uint8 [B, Hkv, hi_cap, d*hi_bits/8]) and parameters (k_hp, v_hp)."""
+    holds codes (k_hi, v_hi uint8 [B, Hkv, hi_cap, d*hi_bits/8]) and parameters (k_hp, v_hp). With
+    k_channel the retained keys are per channel (App. C): the important arrays carry 64 staging rows
+    after the hi_cap slots, and k_params is [B, Hkv, lo_cap/64, d, 2]."""
+    if k_channel:
+        c = empty_cache(B, Hkv, d, bits, g, hi_cap + 64, lo_cap)
+        c.update({"kch": True, "hi_cap": hi_cap, "k_params": np.zeros((B, Hkv, lo_cap // 64, d, 2), np.uint16)})
+        return c
     if hi_bits < 16:
         c = empty_cache(B, Hkv, d, bits, g, hi_cap, lo_cap)
         c.update({

@@ -637,6 +637,156 @@ int mikv_ref_demote_hi_q(int B, int Hkv, int d, int hi_cap, int hi_bits, int hg,
   return 0;
 }
 
+/* ---------------------------------------------------------------- per-channel keys (App. C) */
+
+/*
+ * App. C ("Experiments on Per-Channel Quantization of Keys"): keys quantized per channel, over groups of
+ * 64 consecutive retained tokens, with incoming tokens buffered until a group is complete. Readings:
+ *  - Eq. 1 with its rounding rules (R2, R3) applied to each channel's 64 values of a token group: one
+ *    (alpha16, beta16) per (group, channel); each token's codes are packed in the usual row layout;
+ *  - no balancer on per-channel keys (per-channel scales isolate the outlier channels themselves);
+ *    values stay per-token (Eq. 1 with group g);
+ *  - demoted tokens wait in bf16 in a staging buffer, which here is important-set rows hi_cap ..
+ *    hi_cap + 63 (attended like important rows, never scored); when a group of 64 completes it is
+ *    quantized into retained rows 64 j .. 64 j + 63 and the buffer starts over.
+ * Key parameters: k_params fp16 [B][Hkv][lo_cap / 64][d][2].
+ */
+#define MIKV_REF_KCH_GROUP 64
+
+int mikv_ref_quantize_channel_group(const float* x, int d, int bits, uint8_t* packed, uint16_t* params) {
+  const int n = MIKV_REF_KCH_GROUP;
+  if (!valid_bits(bits) || d != 128) return -1;
+  float* col = (float*)malloc(sizeof(float) * n);
+  int32_t* codes = (int32_t*)malloc(sizeof(int32_t) * (size_t)n * d);
+  int32_t* ccol = (int32_t*)malloc(sizeof(int32_t) * n);
+  if (!col || !codes || !ccol) { free(col); free(codes); free(ccol); return -1; }
+  for (int c = 0; c < d; ++c) {
+    for (int t = 0; t < n; ++t) col[t] = x[(size_t)t * d + c];
+    mikv_ref_quantize_group(col, n, bits, ccol, &params[2 * c], &params[2 * c + 1]);
+    for (int t = 0; t < n; ++t) codes[(size_t)t * d + c] = ccol[t];
+  }
+  for (int t = 0; t < n; ++t) mikv_ref_pack_row(codes + (size_t)t * d, d, bits, packed + (size_t)t * d * bits / 8);
+  free(col); free(codes); free(ccol);
+  return 0;
+}
+
+/*
+ * Append n_rows source rows (k_src/v_src bf16 [B][Hkv][n_src][d], rows [B][Hkv][n_rows], token ids src_tok or
+ * the row index) to the retained set at positions n_lo .. n_lo + n_rows - 1 of every (b, h): a position
+ * whose group completes is quantized with its group (keys per channel from the staged rows and the new
+ * ones, values per token at group g), the others go to staging row hi_cap + (position mod 64) of the
+ * important arrays (k_hi/v_hi bf16 [B][Hkv][hi_rows][d], hi_tok [B][Hkv][hi_rows], hi_rows >= hi_cap + 64).
+ */
+int mikv_ref_append_retained_kch(int B, int Hkv, int d, int bits, int g, int hi_cap, int hi_rows, int lo_cap,
+                                 int n_lo, const uint16_t* k_src, const uint16_t* v_src, const int32_t* src_tok,
+                                 int n_src, const int32_t* rows, int n_rows, uint16_t* k_hi, uint16_t* v_hi,
+                                 int32_t* hi_tok, uint8_t* k_codes, uint8_t* v_codes, uint16_t* k_params,
+                                 uint16_t* v_params, int32_t* lo_tok) {
+  const int n = MIKV_REF_KCH_GROUP;
+  if (!valid_bits(bits) || g <= 0 || d % g || d != 128 || hi_rows < hi_cap + n || lo_cap % n || n_lo < 0 ||
+      n_rows < 0 || n_lo + n_rows > lo_cap)
+    return -1;
+  size_t rb = (size_t)d * bits / 8, np = (size_t)(d / g) * 2;
+  float* x = (float*)malloc(sizeof(float) * (size_t)n * d);
+  float* xr = (float*)malloc(sizeof(float) * (size_t)d);
+  if (!x || !xr) { free(x); free(xr); return -1; }
+  for (int b = 0; b < B; ++b)
+    for (int h = 0; h < Hkv; ++h) {
+      size_t bh = (size_t)b * Hkv + h;
+      for (int i = 0; i < n_rows; ++i) {
+        int r = rows[bh * n_rows + i];
+        if (r < 0 || r >= n_src) { free(x); free(xr); return -1; }
+        int p = n_lo + i, slot = hi_cap + p % n;
+        /* stage the row (bf16 copy, unbalanced key) */
+        memcpy(k_hi + (bh * hi_rows + slot) * d, k_src + (bh * n_src + r) * d, sizeof(uint16_t) * (size_t)d);
+        memcpy(v_hi + (bh * hi_rows + slot) * d, v_src + (bh * n_src + r) * d, sizeof(uint16_t) * (size_t)d);
+        hi_tok[bh * hi_rows + slot] = src_tok ? src_tok[bh * n_src + r] : r;
+        if (p % n != n - 1) continue;
+        /* the group of positions p - 63 .. p is complete: quantize it from the staging rows */
+        int grp = p / n;
+        for (int t = 0; t < n; ++t)
+          for (int c = 0; c < d; ++c) x[(size_t)t * d + c] = bf16_to_f32(k_hi[(bh * hi_rows + hi_cap + t) * d + c]);
+        mikv_ref_quantize_channel_group(x, d, bits, k_codes + (bh * lo_cap + (size_t)grp * n) * rb,
+                                        k_params + ((bh * (lo_cap / n)) + grp) * (size_t)d * 2);
+        for (int t = 0; t < n; ++t) {
+          size_t pos = bh * lo_cap + (size_t)grp * n + t;
+          for (int c = 0; c < d; ++c) xr[c] = bf16_to_f32(v_hi[(bh * hi_rows + hi_cap + t) * d + c]);
+          mikv_ref_quantize_row(xr, d, bits, g, v_codes + pos * rb, v_params + pos * np);
+          lo_tok[pos] = hi_tok[bh * hi_rows + hi_cap + t];
+        }
+      }
+    }
+  free(x); free(xr);
+  return 0;
+}
+
+/*
+ * Decode attention with per-channel retained keys: like mikv_ref_decode_attention, except that the
+ * important set holds n_hi bf16 rows (hi_cap slots plus the staged retained tokens) of arrays with
+ * hi_rows rows per head, the retained rows are the n_lo_q = 64 * complete-group rows, and a retained key
+ * is alpha16[group][c] * code + beta16[group][c] attended with the plain query (no balancer).
+ */
+int mikv_ref_decode_attention_kch(int B, int Hq, int Hkv, int d, int bits, int g, int hi_rows, int n_hi, int lo_cap,
+                                  int n_lo_q, const uint16_t* k_hi, const uint16_t* v_hi, const uint8_t* k_codes,
+                                  const uint8_t* v_codes, const uint16_t* k_params, const uint16_t* v_params,
+                                  const uint16_t* q, double sm_scale, double* out, double* hi_logits, double* ml) {
+  const int n = MIKV_REF_KCH_GROUP;
+  if (B <= 0 || Hkv <= 0 || Hq % Hkv || !valid_bits(bits) || g <= 0 || d % g || d != 128 || n_hi < 0 ||
+      n_hi > hi_rows || n_lo_q < 0 || n_lo_q % n || n_lo_q > lo_cap || n_hi + n_lo_q == 0)
+    return -1;
+  int G = Hq / Hkv, tot = n_hi + n_lo_q;
+  size_t rb = (size_t)d * bits / 8, np = (size_t)(d / g) * 2;
+  double* s = (double*)malloc(sizeof(double) * (size_t)tot);
+  double* qv = (double*)malloc(sizeof(double) * (size_t)d);
+  double* xr = (double*)malloc(sizeof(double) * (size_t)d);
+  int32_t* codes = (int32_t*)malloc(sizeof(int32_t) * (size_t)d);
+  if (!s || !qv || !xr || !codes) { free(s); free(qv); free(xr); free(codes); return -1; }
+  for (int b = 0; b < B; ++b)
+    for (int hq = 0; hq < Hq; ++hq) {
+      int h = hq / G;
+      size_t bh = (size_t)b * Hkv + h, bq = (size_t)b * Hq + hq;
+      for (int c = 0; c < d; ++c) qv[c] = bf16_to_f32(q[bq * d + c]);
+      for (int i = 0; i < tot; ++i) {
+        double acc = 0.0;
+        if (i < n_hi) {
+          for (int c = 0; c < d; ++c) acc += qv[c] * bf16_to_f32(k_hi[(bh * hi_rows + i) * d + c]);
+        } else {
+          int t = i - n_hi;
+          const uint16_t* kp = k_params + ((bh * (lo_cap / n)) + t / n) * (size_t)d * 2;
+          mikv_ref_unpack_row(k_codes + (bh * lo_cap + t) * rb, d, bits, codes);
+          for (int c = 0; c < d; ++c)
+            acc += qv[c] * (mikv_ref_f16_to_f64(kp[2 * c]) * codes[c] + mikv_ref_f16_to_f64(kp[2 * c + 1]));
+        }
+        s[i] = sm_scale * acc;
+      }
+      double m = -INFINITY;
+      for (int i = 0; i < tot; ++i)
+        if (s[i] > m) m = s[i];
+      double l = 0.0;
+      for (int i = 0; i < tot; ++i) l += exp(s[i] - m);
+      double* o = out + bq * d;
+      for (int c = 0; c < d; ++c) o[c] = 0.0;
+      for (int i = 0; i < tot; ++i) {
+        double p = exp(s[i] - m) / l;
+        if (i < n_hi) {
+          for (int c = 0; c < d; ++c) o[c] += p * bf16_to_f32(v_hi[(bh * hi_rows + i) * d + c]);
+        } else {
+          size_t pos = bh * lo_cap + (i - n_hi);
+          mikv_ref_dequantize_row(v_codes + pos * rb, v_params + pos * np, d, bits, g, xr);
+          for (int c = 0; c < d; ++c) o[c] += p * xr[c];
+        }
+      }
+      if (hi_logits)
+        for (int i = 0; i < n_hi; ++i) hi_logits[bq * n_hi + i] = s[i];
+      if (ml) {
+        ml[2 * bq] = m;
+        ml[2 * bq + 1] = l;
+      }
+    }
+  free(s); free(qv); free(xr); free(codes);
+  return 0;
+}
+
 /* ---------------------------------------------------------------- prefill importance */
 
 /*

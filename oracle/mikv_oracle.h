@@ -136,6 +136,23 @@ int mikv_ref_demote_hi_q(int B, int Hkv, int d, int hi_cap, int hi_bits, int hg,
                          const uint16_t* k_hp, const uint16_t* v_hp, const int32_t* hi_tok, uint8_t* k_codes,
                          uint8_t* v_codes, uint16_t* k_params, uint16_t* v_params, int32_t* lo_tok);
 
+/* Per-channel retained keys (App. C): keys quantized per channel over groups of 64 retained tokens (one
+ * fp16 (alpha, beta) per group and channel, no balancer), values per token; retained tokens wait in bf16
+ * in staging rows hi_cap .. hi_cap + 63 of the important arrays until their group is complete.
+ * quantize_channel_group: x fp32 [64][d] -> packed [64][d*bits/8] (per-token row layout), params [d][2].
+ * append_retained_kch: appends rows at retained positions n_lo.. (staging, then group quantization).
+ * decode_attention_kch: attention over n_hi bf16 rows (important + staged) and n_lo_q quantized rows. */
+int mikv_ref_quantize_channel_group(const float* x, int d, int bits, uint8_t* packed, uint16_t* params);
+int mikv_ref_append_retained_kch(int B, int Hkv, int d, int bits, int g, int hi_cap, int hi_rows, int lo_cap,
+                                 int n_lo, const uint16_t* k_src, const uint16_t* v_src, const int32_t* src_tok,
+                                 int n_src, const int32_t* rows, int n_rows, uint16_t* k_hi, uint16_t* v_hi,
+                                 int32_t* hi_tok, uint8_t* k_codes, uint8_t* v_codes, uint16_t* k_params,
+                                 uint16_t* v_params, int32_t* lo_tok);
+int mikv_ref_decode_attention_kch(int B, int Hq, int Hkv, int d, int bits, int g, int hi_rows, int n_hi, int lo_cap,
+                                  int n_lo_q, const uint16_t* k_hi, const uint16_t* v_hi, const uint8_t* k_codes,
+                                  const uint8_t* v_codes, const uint16_t* k_params, const uint16_t* v_params,
+                                  const uint16_t* q, double sm_scale, double* out, double* hi_logits, double* ml);
+
 /* Prefill importance (the initial accumulated-attention score of every token): scores[b][h][t] = sum over
  * the G query heads of KV head h and the queries i >= t of the causal softmax weight of key t in row i,
  * s = sm_scale * q . k. q_pre bf16 [B][Hq][T][d], k_pre bf16 [B][Hkv][T][d], scores fp64 [B][Hkv][T]. */
