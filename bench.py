@@ -164,7 +164,7 @@ def build_model(w, steps_cap: int, dev, rank: int):
     import paper_2402_18096_gb300 as pkg
     from paper_2402_18096_gb300.layer import MixedPrecisionLayer
     shape = pkg.Shape(w.batch, w.heads_q, w.heads_kv, w.bits, w.group, w.hi_cap, w.lo_cap_for(steps_cap),
-                      hi_bits=w.hi_bits)
+                      hi_bits=w.hi_bits, k_channel_group=64 if w.k_channel else 0)
     wr = rank_workload(w, rank)  # each rank owns a different batch
     layers = []
     for li in range(w.layers):
@@ -207,16 +207,13 @@ def run_mikv(args):
             q, kn, vn = inputs[s][li]
             layer.step(q, kn, vn, out)
 
-    def compressed_bytes():
-        return sum(layer.cache.nbytes_attended(layer.n_lo) for layer in layers)
-
     for s in range(W):
         step(s)
     torch.cuda.synchronize()
     for layer in layers:
         pkg.mikv_workspace_check(layer.ws)
 
-    bytes_before = compressed_bytes()
+    n_lo_before = [layer.n_lo for layer in layers]
     clocks = ClockSampler(torch.cuda.current_device()) if rank == 0 else None
     if clocks:
         clocks.start()
@@ -232,10 +229,12 @@ def run_mikv(args):
     if dist:
         dist.barrier()
     clk = clocks.stop() if clocks else None
-    bytes_after = compressed_bytes()
-    # bytes attended over the K steps: n_lo grows by one per step per layer
-    bytes_per_step = (bytes_before + bytes_after) / 2 - sum(
-        layer.cache.nbytes_attended(1) - layer.cache.nbytes_attended(0) for layer in layers) / 2
+    # bytes attended over the K steps (the attention of step s reads n_lo + s retained rows per layer)
+    grow = 1 if w.bits else 0
+    bytes_per_step = sum(layer.cache.nbytes_attended(n0 + grow * s) for layer, n0 in zip(layers, n_lo_before)
+                         for s in range(K)) / K
+    # per-channel keys: a step whose demotion completes a group of 64 adds one quantization launch per layer
+    kch_launches = sum(1 for n0 in n_lo_before for s in range(K) if w.k_channel and (n0 + s) % 64 == 63)
     ms = e0.elapsed_time(e1) / K
     ms = max_over_ranks(dist, ms)
     for layer in layers:
@@ -311,7 +310,7 @@ def run_mikv(args):
                      "traffic": traffic, "bytes_per_launch": int(attn_bytes), "avg_launch_us": round(attn_ms * 1e3, 2)},
         "e2e": {"value": round(world * bytes_per_step / (e2e_ms * 1e-3) / 1e9, 1), "unit": UNIT,
                 "ms_per_step": round(e2e_ms, 4), "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-        "gpu_launches": K * L * 3,  # per layer step: insert, attention, fused tail
+        "gpu_launches": K * L * 3 + kch_launches,  # per layer step: insert, attention, fused tail
     }
     if clk:
         line["clocks"] = clk
@@ -336,14 +335,20 @@ def _oracle_head(w, b, h, steps_cap):
     k, v = mi.prefill_kv(w, 0, gen_dev, heads=[h])
     scores = mi.initial_scores(w, 0, gen_dev, rows=[b], heads=[h]).cpu()
     q_pre = mi.prefill_queries(w, 0, gen_dev, heads=list(range(h * G, (h + 1) * G)))
-    bal = oracle.balancer(mi.bf16_bits(q_pre), mi.bf16_bits(k))
+    bal = None if w.k_channel else oracle.balancer(mi.bf16_bits(q_pre), mi.bf16_bits(k))
     ks, vs = mi.bf16_bits(k[b:b + 1]), mi.bf16_bits(v[b:b + 1])
     sc = scores.numpy()
     del k, v, q_pre
     dem, kept = oracle.select_demote(sc, w.context - w.budget)
-    c = oracle.empty_cache(1, 1, w.head_dim, w.bits, w.group, w.hi_cap, w.lo_cap_for(steps_cap), hi_bits=w.hi_bits)
-    oracle.gather_hi(c, ks, vs, kept, src_scores=sc, balancer_=bal)
-    oracle.quantize_pack(c, ks, vs, dem, 0, balancer_=bal)
+    if w.k_channel:  # per-channel retained keys: no balancer, the last incomplete group staged in bf16
+        c = oracle.empty_cache(1, 1, w.head_dim, w.bits, w.group, w.hi_cap, w.lo_cap_for(steps_cap), k_channel=True)
+        oracle.gather_hi(c, ks, vs, kept, src_scores=sc)
+        oracle.append_retained(c, ks, vs, dem, 0)
+    else:
+        c = oracle.empty_cache(1, 1, w.head_dim, w.bits, w.group, w.hi_cap, w.lo_cap_for(steps_cap),
+                               hi_bits=w.hi_bits)
+        oracle.gather_hi(c, ks, vs, kept, src_scores=sc, balancer_=bal)
+        oracle.quantize_pack(c, ks, vs, dem, 0, balancer_=bal)
     return c, bal, np.array([[w.budget]], np.int32)
 
 
@@ -354,14 +359,22 @@ def _oracle_step(w, c, bal, slots, n_lo, pos, q, kn, vn):
     G = w.heads_q // w.heads_kv
     oracle.insert_token(c, kn, vn, pos, slots, balancer_=bal)
     _, hl, ml = oracle.decode_attention(c, q, n_lo, 1 / math.sqrt(w.head_dim), balancer_=bal)
-    c["acc"] = oracle.update_importance(c["acc"], hl.astype(np.float32), ml.astype(np.float32), G)
-    dem, _ = oracle.select_demote(c["acc"], 1, c["hi_tok"], want_kept=False)
-    oracle.demote_hi(c, dem[:, :, 0], n_lo, balancer_=bal)
+    hc = w.hi_cap
+    acc = oracle.update_importance(c["acc"][:, :, :hc], hl[:, :, :hc].astype(np.float32), ml.astype(np.float32), G)
+    c["acc"][:, :, :hc] = acc
+    dem, _ = oracle.select_demote(acc, 1, c["hi_tok"][:, :, :hc], want_kept=False)
+    if w.k_channel:
+        oracle.append_retained(c, c["k_hi"], c["v_hi"], dem, n_lo, src_tok=c["hi_tok"])
+    else:
+        oracle.demote_hi(c, dem[:, :, 0], n_lo, balancer_=bal)
     return dem[0]
 
 
 def _head_bytes(w, n_lo):
     lo = 2 * (w.head_dim * w.bits // 8 + 4 * (w.head_dim // w.group))
+    if w.k_channel:  # keys: codes per token, (alpha, beta) per channel and 64 tokens; staged rows in bf16
+        lo = 2 * w.head_dim * w.bits // 8 + 4 * (w.head_dim // w.group) + 4 * w.head_dim // 64
+        return w.hi_cap * 4 * w.head_dim + (n_lo // 64 * 64) * lo + (n_lo % 64) * 4 * w.head_dim
     hi = 4 * w.head_dim if w.hi_bits >= 16 else 2 * (w.head_dim * w.hi_bits // 8 + 4 * (w.head_dim // 64))
     return w.hi_cap * hi + n_lo * lo
 

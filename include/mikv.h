@@ -71,6 +71,14 @@ typedef struct {
   int32_t lo_cap;    /* rows per head in the retained-set arrays: multiple of 16 */
   int32_t hi_bits;   /* important-set precision: 0 or 16 = bf16; 8, 4 or 2 = codes (Sec. 3.3, Table 3) */
   int32_t hi_group;  /* channels per group of a coded important set: 64 (ignored for bf16) */
+  int32_t k_channel_group; /* 0: retained keys per token (Eq. 1, groups of `group` channels, balanced).
+                              64: retained keys per CHANNEL over groups of 64 consecutive retained tokens
+                              (App. C): one fp16 (alpha, beta) per (token group, channel), no balancer;
+                              values stay per token. Retained tokens wait in bf16 in staging rows
+                              hi_cap .. hi_cap + 63 of the important arrays until their group of 64 is
+                              complete: of n_lo retained tokens, n_lo mod 64 are staged (in order) and
+                              the rest quantized. Requires a bf16 important set, hi_stride >= hi_cap + 64
+                              and lo_cap % 64 == 0; k_params is then fp16 [B][Hkv][lo_cap / 64][d][2]. */
 } mikv_shape;
 
 /* Device arrays of one layer's cache. Rows >= hi_cap of the important arrays are padding and are
@@ -142,6 +150,10 @@ mikv_status mikv_compute_balancer(const mikv_shape* shape, const void* q_pre, co
  * Errors: MIKV_ERR_CAPACITY if lo_start + n_rows > lo_cap. Rows outside [0, n_src) are skipped by the
  * kernel. Codes and parameters are bit-exact with an IEEE fp32 evaluation of the formulas above.
  */
+/* With per-channel keys (k_channel_group = 64), mikv_quantize_pack APPENDS the rows at retained positions
+ * lo_start .. lo_start + n_rows - 1, lo_start being the current retained length: a position whose group of
+ * 64 completes is quantized with its group (keys per channel from the staged rows and the new ones, values
+ * per token), the others are copied into the staging rows (bf16, keys unbalanced) with their token ids. */
 mikv_status mikv_quantize_pack(const mikv_shape* shape, const mikv_cache* cache, const void* k_src,
                                const void* v_src, const int32_t* src_tok, int32_t n_src,
                                const int32_t* rows, int32_t n_rows, int32_t lo_start, void* stream);

@@ -38,6 +38,7 @@ class Workload:
     seed: int = 0
     head_dim: int = HEAD_DIM
     hi_bits: int = 16     # important-set precision: 16 = bf16, or 8 / 4 / 2-bit codes in groups of 64
+    k_channel: bool = False  # retained keys per channel over groups of 64 tokens (App. C)
 
     @property
     def budget(self) -> int:
@@ -58,7 +59,8 @@ class Workload:
         return self.context - self.budget
 
     def lo_cap_for(self, steps: int) -> int:
-        return max(16, (self.n_lo0 + steps + 15) // 16 * 16)
+        q = 64 if self.k_channel else 16
+        return max(q, (self.n_lo0 + steps + q - 1) // q * q)
 
 
 WORKLOADS = {
@@ -78,6 +80,12 @@ for _hb in (16, 8, 4, 2):
     WORKLOADS[f"mistral-7b-t3-hi{_hb}"] = Workload(
         f"mistral-7b-b32-l32-hq32-hkv8-t32768-int2-g64-r20-hi{_hb}", 32, 32, 8, 32768, 32, 2, 64, 0.20,
         hi_bits=_hb)
+# per-channel retained keys (App. C, Table 8 settings): INT2 / INT3 retained, 20 % important, keys quantized
+# per channel over groups of 64 retained tokens, values per token in groups of 64 channels
+for _b in (2, 3):
+    WORKLOADS[f"mistral-7b-kch-int{_b}"] = Workload(
+        f"mistral-7b-b32-l32-hq32-hkv8-t32768-int{_b}-g64-r20-kch64", 32, 32, 8, 32768, 32, _b, 64, 0.20,
+        k_channel=True)
 
 
 def sweep_workloads() -> List[Workload]:

@@ -44,7 +44,7 @@ class MikvError(RuntimeError):
 class _Shape(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in
                 ("batch", "heads_q", "heads_kv", "head_dim", "bits", "group", "hi_cap", "hi_stride", "lo_cap",
-                 "hi_bits", "hi_group")]
+                 "hi_bits", "hi_group", "k_channel_group")]
 
 
 class _Cache(ctypes.Structure):
@@ -128,10 +128,12 @@ class Shape:
     head_dim: int = HEAD_DIM
     hi_bits: int = 16   # important-set precision: 16 = bf16; 8, 4, 2 = codes (Sec. 3.3, Table 3)
     hi_group: int = 64  # channels per group of a coded important set
+    k_channel_group: int = 0  # 64: retained keys per channel over groups of 64 tokens (App. C)
 
     @property
     def hi_stride(self) -> int:
-        return (self.hi_cap + 15) // 16 * 16
+        # per-channel keys: 64 staging rows of retained tokens follow the important slots
+        return (self.hi_cap + (64 if self.k_channel_group else 0) + 15) // 16 * 16
 
     @property
     def hi_coded(self) -> bool:
@@ -139,7 +141,7 @@ class Shape:
 
     def c(self) -> _Shape:
         return _Shape(self.batch, self.heads_q, self.heads_kv, self.head_dim, self.bits, self.group,
-                      self.hi_cap, self.hi_stride, self.lo_cap, self.hi_bits, self.hi_group)
+                      self.hi_cap, self.hi_stride, self.lo_cap, self.hi_bits, self.hi_group, self.k_channel_group)
 
 
 class LayerCache:
@@ -165,7 +167,10 @@ class LayerCache:
         self.k_codes = torch.zeros(B, H, s.lo_cap, 16 * s.bits, dtype=torch.uint8, **z)
         self.v_codes = torch.zeros(B, H, s.lo_cap, 16 * s.bits, dtype=torch.uint8, **z)
         npar = d // s.group if s.bits else 0
-        self.k_params = torch.zeros(B, H, s.lo_cap, npar, 2, dtype=torch.float16, **z)
+        if s.k_channel_group:  # one (alpha, beta) per channel and group of 64 retained tokens
+            self.k_params = torch.zeros(B, H, s.lo_cap // s.k_channel_group, d, 2, dtype=torch.float16, **z)
+        else:
+            self.k_params = torch.zeros(B, H, s.lo_cap, npar, 2, dtype=torch.float16, **z)
         self.v_params = torch.zeros(B, H, s.lo_cap, npar, 2, dtype=torch.float16, **z)
         self.lo_tok = torch.zeros(B, H, s.lo_cap, dtype=torch.int32, **z)
         self.balancer = balancer
@@ -181,6 +186,10 @@ class LayerCache:
         s = self.shape
         row_lo = 2 * mikv_retained_row_bytes(s.bits, s.group, s.head_dim)
         row_hi = 2 * mikv_retained_row_bytes(s.hi_bits, s.hi_group, s.head_dim) if s.hi_coded else 4 * s.head_dim
+        if s.k_channel_group:  # keys: codes per token plus 4 bytes per channel per 64 tokens; staged rows bf16
+            g = s.k_channel_group
+            row_lo = 2 * s.head_dim * s.bits // 8 + 4 * s.head_dim // s.group + 4 * s.head_dim // g
+            return s.batch * s.heads_kv * (s.hi_cap * row_hi + n_lo // g * g * row_lo + n_lo % g * row_hi)
         return s.batch * s.heads_kv * (s.hi_cap * row_hi + n_lo * row_lo)
 
 

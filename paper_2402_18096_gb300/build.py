@@ -15,7 +15,8 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 OUT_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(OUT_DIR, "libmikv.so")
-SOURCES = ["mikv_attn_h16.cu", "mikv_attn_h8.cu", "mikv_attn_h4.cu", "mikv_attn_h2.cu", "mikv_attention.cu",
+SOURCES = ["mikv_attn_h16.cu", "mikv_attn_h8.cu", "mikv_attn_h4.cu", "mikv_attn_h2.cu", "mikv_attn_kch.cu",
+           "mikv_attention.cu",
            "mikv_quant.cu", "mikv_policy.cu", "mikv_step.cu", "mikv_prefill.cu", "mikv_abi.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr"]

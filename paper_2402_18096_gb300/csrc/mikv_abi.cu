@@ -44,6 +44,10 @@ mikv_status shape_supported(const mikv_shape* s) {
   const int hb = s->hi_bits;
   if (hb != 0 && hb != 16 && hb != 8 && hb != 4 && hb != 2) return MIKV_ERR_UNSUPPORTED;
   if (hb != 0 && hb != 16 && s->hi_group != kHiGroup) return MIKV_ERR_UNSUPPORTED;
+  if (s->k_channel_group != 0) {  // per-channel retained keys (App. C)
+    if (s->k_channel_group != kKchGroup || (hb != 0 && hb != 16) || s->bits == 0) return MIKV_ERR_UNSUPPORTED;
+    if (s->hi_stride < s->hi_cap + kKchGroup || s->lo_cap % kKchGroup) return MIKV_ERR_ARG;
+  }
   return MIKV_OK;
 }
 
@@ -162,8 +166,14 @@ mikv_status attention_impl(const mikv_shape* s, const mikv_cache* c, int32_t n_l
                            void* out, int32_t out_dtype, float* hi_logits, float* ml, void* ws, size_t ws_bytes,
                            cudaStream_t st, bool merge = true, AttnArgs* args_out = nullptr) {
   const int sms = num_sms();
-  const AttnPlan plan = plan_attention(*s, n_lo, sms);
-  if (ws_bytes < attention_workspace_bytes(*s, n_lo, sms)) return MIKV_ERR_WORKSPACE;
+  // per-channel keys: the n_lo mod 64 staged retained tokens are attended as important rows hi_cap ..
+  const bool kch = kch_of(*s);
+  const int n_stage = kch ? n_lo % kKchGroup : 0;
+  mikv_shape se = *s;
+  se.hi_cap += n_stage;
+  n_lo -= n_stage;
+  const AttnPlan plan = plan_attention(se, n_lo, sms);
+  if (ws_bytes < attention_workspace_bytes(*s, n_lo + n_stage, sms)) return MIKV_ERR_WORKSPACE;
   if ((long long)s->batch * s->heads_kv * plan.n_u > 2000000000LL) return MIKV_ERR_UNSUPPORTED;
   const int G = s->heads_q / s->heads_kv;
   AttnArgs a;
@@ -198,7 +208,7 @@ mikv_status attention_impl(const mikv_shape* s, const mikv_cache* c, int32_t n_l
   if (ok && lo_rows > 0 && !evicting(*s)) {
     // retained arrays: each is viewed as rows of U.map_w (codes) or U.param_w (alpha, beta) bytes, and
     // one box covers a whole unit of 16 * U.blocks tokens (lo_cap % 16 == 0 keeps units row-aligned)
-    const LoUnit U = lo_unit_layout(s->bits, s->group);
+    const LoUnit U = kch ? lo_unit_layout_kch(s->bits, s->group) : lo_unit_layout(s->bits, s->group);
     const uint64_t code_rows = lo_rows * U.pitch / U.map_w;
     const uint32_t code_box = 16u * U.blocks * U.pitch / U.map_w;
     const CUtensorMapSwizzle swz = s->bits == 3 ? CU_TENSOR_MAP_SWIZZLE_NONE : CU_TENSOR_MAP_SWIZZLE_64B;
@@ -208,8 +218,10 @@ mikv_status attention_impl(const mikv_shape* s, const mikv_cache* c, int32_t n_l
                   code_box, swz) &&
          make_map(&a.map_v_lo, c->v_codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, U.map_w, code_rows, U.map_w, U.map_w,
                   code_box, swz) &&
-         make_map(&a.map_k_par, c->k_params, CU_TENSOR_MAP_DATA_TYPE_UINT8, U.param_w, par_rows, U.param_w,
-                  U.param_w, par_box, CU_TENSOR_MAP_SWIZZLE_NONE) &&
+         (kch ? make_map(&a.map_k_par, c->k_params, CU_TENSOR_MAP_DATA_TYPE_UINT8, 128,
+                         lo_rows / kKchGroup * 4, 128, 128, 4, CU_TENSOR_MAP_SWIZZLE_NONE)  // 512 B per group
+              : make_map(&a.map_k_par, c->k_params, CU_TENSOR_MAP_DATA_TYPE_UINT8, U.param_w, par_rows, U.param_w,
+                         U.param_w, par_box, CU_TENSOR_MAP_SWIZZLE_NONE)) &&
          make_map(&a.map_v_par, c->v_params, CU_TENSOR_MAP_DATA_TYPE_UINT8, U.param_w, par_rows, U.param_w,
                   U.param_w, par_box, CU_TENSOR_MAP_SWIZZLE_NONE);
   }
@@ -224,7 +236,7 @@ mikv_status attention_impl(const mikv_shape* s, const mikv_cache* c, int32_t n_l
   a.batch = s->batch;
   a.heads_q = s->heads_q;
   a.heads_kv = s->heads_kv;
-  a.hi_cap = s->hi_cap;
+  a.hi_cap = se.hi_cap;
   a.hi_stride = s->hi_stride;
   a.lo_cap = s->lo_cap;
   a.n_lo = n_lo;
@@ -235,7 +247,7 @@ mikv_status attention_impl(const mikv_shape* s, const mikv_cache* c, int32_t n_l
   a.n_units = plan.n_units;
   a.n_warps = plan.n_warps;
   a.sm_scale = sm_scale;
-  cudaError_t e = launch_attention(a, lo_bits_of(*s), lo_group_of(*s), hb, G, plan.grid, st);
+  cudaError_t e = launch_attention(a, lo_bits_of(*s), lo_group_of(*s), hb, G, plan.grid, st, kch);
   if (e != cudaSuccess) return MIKV_ERR_CUDA;
   if (args_out) *args_out = a;
   if (!merge) return MIKV_OK;
@@ -320,6 +332,12 @@ mikv_status mikv_quantize_pack(const mikv_shape* shape, const mikv_cache* cache,
   if ((int64_t)lo_start + n_rows > shape->lo_cap) return MIKV_ERR_CAPACITY;
   if ((int64_t)(n_rows + 3) / 4 > 2147483647 || (int64_t)shape->batch * shape->heads_kv > 65535)
     return MIKV_ERR_UNSUPPORTED;
+  if (kch_of(*shape)) {  // append: complete groups quantized per channel, the rest staged
+    if (n_rows == 0) return MIKV_OK;
+    if (!rows) return MIKV_ERR_ARG;
+    return cuda_status(launch_kch_append(*shape, *cache, k_src, v_src, src_tok, n_src, rows, n_rows, lo_start,
+                                         static_cast<cudaStream_t>(stream)));
+  }
   return cuda_status(launch_quantize_pack(*shape, *cache, k_src, v_src, src_tok, n_src, rows, n_rows, lo_start,
                                           static_cast<cudaStream_t>(stream)));
 }
@@ -446,6 +464,7 @@ mikv_status mikv_decode_step(const mikv_shape* shape, const mikv_cache* cache, i
   p.v_hi_params = cache->v_hi_params;
   p.hi_bits = hi_bits_of(*shape);
   p.evict = evicting(*shape) ? 1 : 0;
+  p.kch = kch_of(*shape) ? 1 : 0;
   p.batch = shape->batch;
   p.heads_q = shape->heads_q;
   p.heads_kv = shape->heads_kv;
@@ -456,8 +475,12 @@ mikv_status mikv_decode_step(const mikv_shape* shape, const mikv_cache* cache, i
   p.n_u = a.n_u;
   p.n_units = a.n_units;
   p.n_warps = a.n_warps;
-  return cuda_status(launch_step_post(p, lo_bits_of(*shape), lo_group_of(*shape), shape->heads_q / shape->heads_kv,
-                                      out_dtype == MIKV_OUT_F32, static_cast<cudaStream_t>(stream)));
+  cudaError_t e = launch_step_post(p, lo_bits_of(*shape), lo_group_of(*shape), shape->heads_q / shape->heads_kv,
+                                   out_dtype == MIKV_OUT_F32, static_cast<cudaStream_t>(stream));
+  if (e == cudaSuccess && p.kch && n_lo % kKchGroup == kKchGroup - 1)  // the victim completed a group
+    e = launch_kch_append(*shape, *cache, nullptr, nullptr, nullptr, 0, nullptr, 0, n_lo + 1,
+                          static_cast<cudaStream_t>(stream));
+  return cuda_status(e);
 }
 
 double mikv_cache_fraction(int32_t bits, int32_t group, double ratio, int32_t hi_bits) {

@@ -43,7 +43,8 @@ AttnPlan plan_attention(const mikv_shape& s, int n_lo, int num_sms) {
   const int kh = hb == 16 ? 1 : lo_unit_layout(hb, kHiGroup).blocks;
   p.hi_units = (p.hi_blocks + kh - 1) / kh;
   p.lo_blocks = (n_lo + 15) / 16;
-  const int k = evicting(s) ? 1 : lo_unit_layout(s.bits, s.group).blocks;
+  const int k = evicting(s) ? 1 : kch_of(s) ? lo_unit_layout_kch(s.bits, s.group).blocks
+                                          : lo_unit_layout(s.bits, s.group).blocks;
   p.lo_units = (p.lo_blocks + k - 1) / k;
   p.n_u = p.hi_units + p.lo_units;
   const long long bh = (long long)s.batch * s.heads_kv;
@@ -69,7 +70,9 @@ size_t attention_workspace_bytes(const mikv_shape& s, int n_lo_max, int num_sms)
   return kWsHeader + (part + 255) / 256 * 256;
 }
 
-cudaError_t launch_attention(const AttnArgs& a, int bits, int group, int hi_bits, int G, int grid, cudaStream_t st) {
+cudaError_t launch_attention(const AttnArgs& a, int bits, int group, int hi_bits, int G, int grid, cudaStream_t st,
+                             bool kch) {
+  if (kch) return hi_bits == 16 ? launch_attention_kch(a, bits, group, G, grid, st) : cudaErrorInvalidValue;
   switch (hi_bits) {
     case 16: return launch_attention_h16(a, bits, group, G, grid, st);
     case 8: return launch_attention_h8(a, bits, group, G, grid, st);

@@ -339,11 +339,14 @@ __device__ __forceinline__ void process_hi(uint32_t blk, int valid, int slot0, c
 
 // Key side of coded block b of a unit (retained, or coded important with logit_base set): scaled
 // logits s, -inf past valid; important-set logits are also stored at logit_base[head][slot0 + token].
-template <int BITS, int GROUP, int G, int QACC>
+// KCH (per-channel retained keys, App. C): qh holds the query scaled by the group's per-channel alpha,
+// the codes enter the MMA as exact integers, and kbias[hd] (sum over channels of q * beta for heads 2t,
+// 2t+1) is added to the dot products; no per-token key parameters.
+template <int BITS, int GROUP, int G, int QACC, bool KCH = false>
 __device__ __forceinline__ void lo_logits(uint32_t unit, int b, int valid, const uint32_t (&qh)[8][2], float scale,
                                           float (&s)[4], int lane, float* logit_base = nullptr, int hi_stride = 0,
-                                          int slot0 = 0) {
-  constexpr LoUnit U = lo_unit_layout(BITS, GROUP);
+                                          int slot0 = 0, const float* kbias = nullptr) {
+  constexpr LoUnit U = KCH ? lo_unit_layout_kch(BITS, GROUP) : lo_unit_layout(BITS, GROUP);
   constexpr int NG = kHeadDim / GROUP;
   constexpr int PR = U.param_row;
   // this block's rows inside the unit's sections
@@ -353,8 +356,10 @@ __device__ __forceinline__ void lo_logits(uint32_t unit, int b, int valid, const
   const int g = lane >> 2, t = lane & 3, r8 = lane & 7, j = lane >> 3;
 
   uint32_t pk0[NG], pk1[NG];
-  lds_vec<NG>(kp + g * PR, pk0);
-  lds_vec<NG>(kp + (g + 8) * PR, pk1);
+  if constexpr (!KCH) {
+    lds_vec<NG>(kp + g * PR, pk0);
+    lds_vec<NG>(kp + (g + 8) * PR, pk1);
+  }
   float accs[QACC][4];
 #pragma unroll
   for (int q = 0; q < QACC; ++q) accs[q][0] = accs[q][1] = accs[q][2] = accs[q][3] = 0.f;
@@ -416,9 +421,6 @@ __device__ __forceinline__ void lo_logits(uint32_t unit, int b, int valid, const
   for (int ks = 0; ks < 8; ++ks) {
     const int gi = (16 * ks) / GROUP;
     // (alpha, alpha) and (beta, beta) of tokens g and g + 8: half-broadcasts the HFMA2 operand selectors absorb
-    const __half2 p0 = u32_as_h2(pk0[gi]), p1 = u32_as_h2(pk1[gi]);
-    const uint32_t al0 = h2_as_u32(__low2half2(p0)), be0 = h2_as_u32(__high2half2(p0));
-    const uint32_t al1 = h2_as_u32(__low2half2(p1)), be1 = h2_as_u32(__high2half2(p1));
     uint32_t c[4];
     if (BITS == 4) {
       const int ri = (ks >> 2) * 4, p = ks & 3;
@@ -433,24 +435,59 @@ __device__ __forceinline__ void lo_logits(uint32_t unit, int b, int valid, const
       c[2] = code3(kr[2], kb0, ks, 8 + ks);
       c[3] = code3(kr[3], kb1, ks, 8 + ks);
     }
-    const uint32_t a[4] = {h2_as_u32(__hfma2(u32_as_h2(c[0]), u32_as_h2(al0), u32_as_h2(be0))),
-                           h2_as_u32(__hfma2(u32_as_h2(c[1]), u32_as_h2(al1), u32_as_h2(be1))),
-                           h2_as_u32(__hfma2(u32_as_h2(c[2]), u32_as_h2(al0), u32_as_h2(be0))),
-                           h2_as_u32(__hfma2(u32_as_h2(c[3]), u32_as_h2(al1), u32_as_h2(be1)))};
-    mma_f16(accs[ks % QACC], a, qh[ks][0], qh[ks][1]);
+    if constexpr (KCH) {
+      mma_f16(accs[ks % QACC], c, qh[ks][0], qh[ks][1]);
+    } else {
+      const __half2 p0 = u32_as_h2(pk0[gi]), p1 = u32_as_h2(pk1[gi]);
+      const __half2 al0 = __low2half2(p0), be0 = __high2half2(p0);
+      const __half2 al1 = __low2half2(p1), be1 = __high2half2(p1);
+      const uint32_t a[4] = {h2_as_u32(__hfma2(u32_as_h2(c[0]), al0, be0)), h2_as_u32(__hfma2(u32_as_h2(c[1]), al1, be1)),
+                             h2_as_u32(__hfma2(u32_as_h2(c[2]), al0, be0)), h2_as_u32(__hfma2(u32_as_h2(c[3]), al1, be1))};
+      mma_f16(accs[ks % QACC], a, qh[ks][0], qh[ks][1]);
+    }
   }
   float acc[4];
   sum_acc(accs, acc);
+  if constexpr (KCH) {
+    acc[0] += kbias[0];
+    acc[1] += kbias[1];
+    acc[2] += kbias[0];
+    acc[3] += kbias[1];
+  }
   finish_logits<G>(acc, scale, valid, g, t, logit_base, hi_stride, slot0, s);
+}
+
+// Per-channel keys (App. C): from the group's (alpha, beta) pairs of the key channels (512 bytes at kp),
+// the query fragments scaled per channel, qk = q * alpha, and the per-head bias sum_c q_c beta_c (one MMA
+// per k-step whose row 0 holds beta; lanes 4 t .. 4 t + 3 all receive heads 2t, 2t+1).
+__device__ __forceinline__ void kch_prepare(uint32_t kp, const uint32_t (&qh)[8][2], uint32_t (&qk)[8][2],
+                                            float (&kbias)[2], int lane) {
+  const int g = lane >> 2, t = lane & 3;
+  float cb[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int ks = 0; ks < 8; ++ks) {
+    uint32_t be[2];
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      const int c = 16 * ks + 8 * r + 2 * t;  // channels c, c + 1 of this fragment
+      const uint32_t p0 = lds32(kp + 4 * c), p1 = lds32(kp + 4 * c + 4);
+      qk[ks][r] = h2_as_u32(__hmul2(u32_as_h2(qh[ks][r]), u32_as_h2(prmt(p0, p1, 0x5410u))));
+      be[r] = prmt(p0, p1, 0x7632u);
+    }
+    const uint32_t a[4] = {g == 0 ? be[0] : 0u, 0u, g == 0 ? be[1] : 0u, 0u};
+    mma_f16(cb, a, qh[ks][0], qh[ks][1]);
+  }
+  kbias[0] = __shfl_sync(0xffffffffu, cb[0], t);
+  kbias[1] = __shfl_sync(0xffffffffu, cb[1], t);
 }
 
 // Value side of coded block b: o, ob += P (this block's probabilities p) times the block's values.
 // EXACT (coded important blocks): codes enter the MMA as exact integers, so the block adds nothing to
 // the alpha sums that remove the retained set's code offsets.
-template <int BITS, int GROUP, int NB, bool EXACT>
+template <int BITS, int GROUP, int NB, bool EXACT, bool KCH = false>
 __device__ __forceinline__ void lo_values(uint32_t unit, int b, int valid, const float (&p)[4], float (&o)[8][4],
                                           float (&ob)[NB][4], int lane) {
-  constexpr LoUnit U = lo_unit_layout(BITS, GROUP);
+  constexpr LoUnit U = KCH ? lo_unit_layout_kch(BITS, GROUP) : lo_unit_layout(BITS, GROUP);
   constexpr int NG = kHeadDim / GROUP;
   constexpr int PR = U.param_row;
   const uint32_t va = unit + U.v_a + b * 16 * U.pitch;
@@ -593,20 +630,21 @@ __device__ __forceinline__ void lo_values(uint32_t unit, int b, int valid, const
 // least 16 (NK - 1) + 1): the key sides first, one softmax update over all NK blocks, then the value
 // sides, so the dependency chains of the blocks overlap. HI: blocks of a coded important set (logits
 // stored for the importance update, exact value codes); slot0 = important slot of block b's first row.
-template <int BITS, int GROUP, int G, int NB, int NK, bool HI>
+template <int BITS, int GROUP, int G, int NB, int NK, bool HI, bool KCH = false>
 __device__ __forceinline__ void process_coded(uint32_t unit, int b, int n_left, const uint32_t (&qh)[8][2],
                                               float scale, Softmax& st, float (&o)[8][4], float (&ob)[NB][4],
                                               int lane, float* logit_base = nullptr, int hi_stride = 0,
-                                              int slot0 = 0) {
+                                              int slot0 = 0, const float* kbias = nullptr) {
   float s[NK][4], p[NK][4];
 #pragma unroll
   for (int k = 0; k < NK; ++k)
-    lo_logits<BITS, GROUP, G, NK == 1 ? kQkAcc : kPairAcc>(unit, b + k, min(16, n_left - 16 * k), qh, scale, s[k],
-                                                           lane, HI ? logit_base : nullptr, hi_stride, slot0 + 16 * k);
+    lo_logits<BITS, GROUP, G, NK == 1 ? kQkAcc : kPairAcc, KCH>(unit, b + k, min(16, n_left - 16 * k), qh, scale,
+                                                                s[k], lane, HI ? logit_base : nullptr, hi_stride,
+                                                                slot0 + 16 * k, kbias);
   softmax_blocks(s, st, o, ob, p);
 #pragma unroll
   for (int k = 0; k < NK; ++k)
-    lo_values<BITS, GROUP, NB, HI>(unit, b + k, min(16, n_left - 16 * k), p[k], o, ob, lane);
+    lo_values<BITS, GROUP, NB, HI, KCH>(unit, b + k, min(16, n_left - 16 * k), p[k], o, ob, lane);
 }
 
 // Write this warp's partial for one head: the output normalised by the sum of the rounded probabilities
@@ -657,9 +695,9 @@ __device__ __forceinline__ void write_partial(const AttnArgs& a, int slot, Softm
   }
 }
 
-template <int BITS, int GROUP, int HB>
+template <int BITS, int GROUP, int HB, bool KCH>
 __device__ __forceinline__ void issue_unit(const AttnArgs& a, const Cursor& c, uint32_t dst, uint32_t bar) {
-  constexpr LoUnit U = lo_unit_layout(BITS, GROUP);
+  constexpr LoUnit U = KCH ? lo_unit_layout_kch(BITS, GROUP) : lo_unit_layout(BITS, GROUP);
   const UnitKind k = cursor_kind(c, a.hi_units, a.n_u);
   if constexpr (HB != 16) {
     if (k.hi) {
@@ -689,7 +727,12 @@ __device__ __forceinline__ void issue_unit(const AttnArgs& a, const Cursor& c, u
     const int crow = (int)(row * U.pitch / U.map_w), prow = (int)(row * U.param_row / U.param_w);
     tma_load_2d(dst + U.k_a, &a.map_k_lo, 0, crow, bar);
     tma_load_2d(dst + U.v_a, &a.map_v_lo, 0, crow, bar);
-    tma_load_2d(dst + U.k_p, &a.map_k_par, 0, prow, bar);
+    if constexpr (KCH) {  // the group's key (alpha, beta) pairs: four 128-byte rows per group of 64 tokens
+      const long long grp = (long long)c.bh * (a.lo_cap / kKchGroup) + (16 * U.blocks * k.index) / kKchGroup;
+      tma_load_2d(dst + U.k_p, &a.map_k_par, 0, (int)(4 * grp), bar);
+    } else {
+      tma_load_2d(dst + U.k_p, &a.map_k_par, 0, prow, bar);
+    }
     tma_load_2d(dst + U.v_p, &a.map_v_par, 0, prow, bar);
   }
 }
@@ -698,11 +741,12 @@ __device__ __forceinline__ void fence_proxy_async() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
-template <int BITS, int GROUP, int HB, int G>
+template <int BITS, int GROUP, int HB, int G, bool KCH = false>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const __grid_constant__ AttnArgs a) {
-  constexpr LoUnit U = lo_unit_layout(BITS, GROUP);
+  constexpr LoUnit U = KCH ? lo_unit_layout_kch(BITS, GROUP) : lo_unit_layout(BITS, GROUP);
   constexpr LoUnit H = lo_unit_layout(HB == 16 ? 2 : HB, kHiGroup);
   static_assert(U.total <= kStageBytes && H.total <= kStageBytes, "unit too large for a stage");
+  static_assert(!KCH || HB == 16, "per-channel retained keys need a bf16 important set");
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -731,7 +775,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
       prefetch_tensormap(&a.map_v_par);
     }
     for (int k = 0; k < kNS && u0 + k < u1; ++k) {
-      issue_unit<BITS, GROUP, HB>(a, ci, ring + k * kStageBytes, bars + 8 * k);
+      issue_unit<BITS, GROUP, HB, KCH>(a, ci, ring + k * kStageBytes, bars + 8 * k);
       cursor_next(ci, hu, n_u);
     }
   }
@@ -764,9 +808,13 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
             const uint32_t w = *reinterpret_cast<const uint32_t*>(qp + c);
             qb[ks][r] = w;
             const float q0 = __uint_as_float(w << 16), q1 = __uint_as_float(w & 0xffff0000u);
-            const float b0 = a.balancer ? a.balancer[h * kHeadDim + c] : 1.f;
-            const float b1 = a.balancer ? a.balancer[h * kHeadDim + c + 1] : 1.f;
-            qh[ks][r] = pack_f16(__fdiv_rn(q0, b0), __fdiv_rn(q1, b1));  // Eq. 4
+            if constexpr (KCH) {  // per-channel retained keys are not balanced
+              qh[ks][r] = pack_f16(q0, q1);
+            } else {
+              const float b0 = a.balancer ? a.balancer[h * kHeadDim + c] : 1.f;
+              const float b1 = a.balancer ? a.balancer[h * kHeadDim + c + 1] : 1.f;
+              qh[ks][r] = pack_f16(__fdiv_rn(q0, b0), __fdiv_rn(q1, b1));  // Eq. 4
+            }
           }
       } else {
 #pragma unroll
@@ -810,19 +858,28 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
       const int first = k.index * U.blocks;
       const int nb = min(U.blocks, a.lo_blocks - first);
       int b = 0;
-      if (kLoPair)
+      if constexpr (KCH) {
+        uint32_t qk[8][2];
+        float kbias[2];
+        kch_prepare(stage + U.k_p, qh, qk, kbias, lane);
         for (; b + 1 < nb; b += 2)
-          process_coded<BITS, GROUP, G, NB, 2, false>(stage, b, a.n_lo - 16 * (first + b), qh, a.sm_scale, st, o,
+          process_coded<BITS, GROUP, G, NB, 2, false, true>(stage, b, a.n_lo - 16 * (first + b), qk, a.sm_scale, st,
+                                                            o, ob, lane, nullptr, 0, 0, kbias);
+      } else {
+        if (kLoPair)
+          for (; b + 1 < nb; b += 2)
+            process_coded<BITS, GROUP, G, NB, 2, false>(stage, b, a.n_lo - 16 * (first + b), qh, a.sm_scale, st, o,
+                                                        ob, lane);
+        for (; b < nb; ++b)
+          process_coded<BITS, GROUP, G, NB, 1, false>(stage, b, a.n_lo - 16 * (first + b), qh, a.sm_scale, st, o,
                                                       ob, lane);
-      for (; b < nb; ++b)
-        process_coded<BITS, GROUP, G, NB, 1, false>(stage, b, a.n_lo - 16 * (first + b), qh, a.sm_scale, st, o, ob,
-                                                    lane);
+      }
     }
     cursor_next(cc, hu, n_u);
     __syncwarp();
     if (lane == 0 && u + kNS < u1) {
       fence_proxy_async();  // our generic reads of this stage precede the next asynchronous write
-      issue_unit<BITS, GROUP, HB>(a, ci, stage, bars + 8 * s);
+      issue_unit<BITS, GROUP, HB, KCH>(a, ci, stage, bars + 8 * s);
       cursor_next(ci, hu, n_u);
     }
   }
@@ -838,9 +895,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
   if (cur >= 0) write_partial<BITS, GROUP, G, NB>(a, wg + cur, st, o, ob, lane);
 }
 
-template <int BITS, int GROUP, int HB, int G>
+template <int BITS, int GROUP, int HB, int G, bool KCH = false>
 cudaError_t launch_kernel(const AttnArgs& a, int grid, cudaStream_t st) {
-  auto kern = attention_kernel<BITS, GROUP, HB, G>;
+  auto kern = attention_kernel<BITS, GROUP, HB, G, KCH>;
   static bool configured = false;
   const int smem = smem_bytes();
   if (!configured) {
@@ -852,34 +909,35 @@ cudaError_t launch_kernel(const AttnArgs& a, int grid, cudaStream_t st) {
   return cudaGetLastError();
 }
 
-template <int BITS, int GROUP, int HB>
+template <int BITS, int GROUP, int HB, bool KCH>
 cudaError_t dispatch_g(const AttnArgs& a, int G, int grid, cudaStream_t st) {
   switch (G) {
-    case 1: return launch_kernel<BITS, GROUP, HB, 1>(a, grid, st);
-    case 2: return launch_kernel<BITS, GROUP, HB, 2>(a, grid, st);
-    case 4: return launch_kernel<BITS, GROUP, HB, 4>(a, grid, st);
-    case 8: return launch_kernel<BITS, GROUP, HB, 8>(a, grid, st);
+    case 1: return launch_kernel<BITS, GROUP, HB, 1, KCH>(a, grid, st);
+    case 2: return launch_kernel<BITS, GROUP, HB, 2, KCH>(a, grid, st);
+    case 4: return launch_kernel<BITS, GROUP, HB, 4, KCH>(a, grid, st);
+    case 8: return launch_kernel<BITS, GROUP, HB, 8, KCH>(a, grid, st);
   }
   return cudaErrorInvalidValue;
 }
 
-template <int BITS, int HB>
+template <int BITS, int HB, bool KCH>
 cudaError_t dispatch_group(const AttnArgs& a, int group, int G, int grid, cudaStream_t st) {
   switch (group) {
-    case 32: return dispatch_g<BITS, 32, HB>(a, G, grid, st);
-    case 64: return dispatch_g<BITS, 64, HB>(a, G, grid, st);
-    case 128: return dispatch_g<BITS, 128, HB>(a, G, grid, st);
+    case 32: return dispatch_g<BITS, 32, HB, KCH>(a, G, grid, st);
+    case 64: return dispatch_g<BITS, 64, HB, KCH>(a, G, grid, st);
+    case 128: return dispatch_g<BITS, 128, HB, KCH>(a, G, grid, st);
   }
   return cudaErrorInvalidValue;
 }
 
-// Every (retained bits, group, G) kernel for one important-set precision HB (16 = bf16).
-template <int HB>
+// Every (retained bits, group, G) kernel for one important-set precision HB (16 = bf16), with per-token
+// or (KCH) per-channel retained keys.
+template <int HB, bool KCH = false>
 cudaError_t launch_attention_hb(const AttnArgs& a, int bits, int group, int G, int grid, cudaStream_t st) {
   switch (bits) {
-    case 2: return dispatch_group<2, HB>(a, group, G, grid, st);
-    case 3: return dispatch_group<3, HB>(a, group, G, grid, st);
-    case 4: return dispatch_group<4, HB>(a, group, G, grid, st);
+    case 2: return dispatch_group<2, HB, KCH>(a, group, G, grid, st);
+    case 3: return dispatch_group<3, HB, KCH>(a, group, G, grid, st);
+    case 4: return dispatch_group<4, HB, KCH>(a, group, G, grid, st);
   }
   return cudaErrorInvalidValue;
 }

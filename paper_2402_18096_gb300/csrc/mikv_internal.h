@@ -28,6 +28,7 @@ struct LoUnit {
 };
 
 constexpr int kUnitBytes = 8192;
+constexpr int kHeadDimH = 128;  // head dimension (host-side copy)
 
 __host__ __device__ constexpr int align_up(int x, int a) { return (x + a - 1) / a * a; }
 
@@ -53,6 +54,24 @@ __host__ __device__ constexpr LoUnit lo_unit_layout_n(int bits, int group, int n
   u.v_p = align_up(u.k_p + rows * u.param_row, 128);
   u.total = u.v_p + rows * u.param_row;
   u.tx = 2 * rows * u.pitch + 2 * rows * u.param_row;
+  return u;
+}
+
+// Per-channel retained keys (App. C): tokens are grouped by 64; a retained unit is one group (N = 2, 3) or
+// half of one (N = 4: two blocks), carrying the group's 128 (alpha, beta) key pairs (512 bytes) in place of
+// per-token key parameters; values keep their per-token layout.
+constexpr int kKchGroup = 64;
+
+__host__ __device__ constexpr LoUnit lo_unit_layout_kch(int bits, int group) {
+  LoUnit u = lo_unit_layout_n(bits, group, bits == 4 ? 2 : 4);
+  const int rows = 16 * u.blocks;
+  const int code_align = bits == 3 ? 128 : 512;
+  u.k_a = 0;
+  u.v_a = align_up(rows * u.pitch, code_align);
+  u.k_p = align_up(u.v_a + rows * u.pitch, 128);
+  u.v_p = align_up(u.k_p + 4 * kHeadDimH, 128);
+  u.total = u.v_p + rows * u.param_row;
+  u.tx = 2 * rows * u.pitch + 4 * kHeadDimH + rows * u.param_row;
   return u;
 }
 
@@ -111,9 +130,9 @@ struct StepPostArgs {
   void* out;
   const float* hi_logits;
   float* acc;
-  const int32_t* hi_tok;
-  const void* k_hi;
-  const void* v_hi;
+  int32_t* hi_tok;  // written only for per-channel keys (staging)
+  void* k_hi;
+  void* v_hi;
   const float* balancer;
   void* k_codes;
   void* v_codes;
@@ -125,6 +144,7 @@ struct StepPostArgs {
   const void* v_hi_params;
   int hi_bits;              // 16 = bf16 important rows; 8, 4, 2 = coded (groups of kHiGroup)
   int evict;                // no retained set: the victim's slot is freed, nothing is demoted
+  int kch;                  // per-channel retained keys: the victim is staged at important row hi_cap + n_lo % 64
   int batch, heads_q, heads_kv, hi_cap, hi_stride, lo_cap, n_lo;
   int n_u, n_units, n_warps;
 };
@@ -133,7 +153,10 @@ cudaError_t launch_step_post(const StepPostArgs& a, int bits, int group, int G, 
 
 AttnPlan plan_attention(const mikv_shape& s, int n_lo, int num_sms);
 size_t attention_workspace_bytes(const mikv_shape& s, int n_lo_max, int num_sms);
-cudaError_t launch_attention(const AttnArgs& a, int bits, int group, int hi_bits, int G, int grid, cudaStream_t st);
+cudaError_t launch_attention(const AttnArgs& a, int bits, int group, int hi_bits, int G, int grid, cudaStream_t st,
+                             bool kch = false);
+// per-channel retained keys, bf16 important set (mikv_attn_kch.cu)
+cudaError_t launch_attention_kch(const AttnArgs& a, int bits, int group, int G, int grid, cudaStream_t st);
 // one translation unit per important-set precision (mikv_attn_h*.cu)
 cudaError_t launch_attention_h16(const AttnArgs& a, int bits, int group, int G, int grid, cudaStream_t st);
 cudaError_t launch_attention_h8(const AttnArgs& a, int bits, int group, int G, int grid, cudaStream_t st);
@@ -144,6 +167,8 @@ inline int hi_bits_of(const mikv_shape& s) { return s.hi_bits == 0 ? 16 : s.hi_b
 // bits == 0: no retained set, demoted tokens are evicted (the H2O baseline). The kernels then run with
 // any retained layout (none of its units exist); these give the one they are instantiated with.
 inline bool evicting(const mikv_shape& s) { return s.bits == 0; }
+// per-channel retained keys (App. C), groups of kKchGroup tokens
+inline bool kch_of(const mikv_shape& s) { return s.k_channel_group == kKchGroup; }
 inline int lo_bits_of(const mikv_shape& s) { return s.bits == 0 ? 2 : s.bits; }
 inline int lo_group_of(const mikv_shape& s) { return s.bits == 0 ? 32 : s.group; }
 cudaError_t launch_merge(const MergeArgs& a, int G, int out_f32, cudaStream_t st);
@@ -151,6 +176,13 @@ cudaError_t launch_merge(const MergeArgs& a, int G, int out_f32, cudaStream_t st
 cudaError_t launch_quantize_pack(const mikv_shape& s, const mikv_cache& c, const void* k_src,
                                  const void* v_src, const int32_t* src_tok, int n_src,
                                  const int32_t* rows, int n_rows, int lo_start, cudaStream_t st);
+
+// Per-channel retained keys (App. C): append rows at retained positions p0 .. p0 + n_rows - 1 (quantizing
+// every group of 64 that completes, staging the rest in important rows hi_cap ..); with n_rows == 0 and
+// p0 = 64 (j + 1), quantize group j from its staged rows.
+cudaError_t launch_kch_append(const mikv_shape& s, const mikv_cache& c, const void* k_src, const void* v_src,
+                              const int32_t* src_tok, int n_src, const int32_t* rows, int n_rows, int p0,
+                              cudaStream_t st);
 
 // insert (rows == nullptr, slots/tok used) or gather (rows/n_rows) into a coded important set
 cudaError_t launch_hi_quant(const mikv_shape& s, const mikv_cache& c, const void* k_src, const void* v_src,

@@ -109,6 +109,135 @@ __global__ void __launch_bounds__(256) hi_quant_kernel(const HiQArgs a) {
   }
 }
 
+// ------------------------------------------------------------- per-channel retained keys (App. C)
+
+// Rows of the retained set with per-channel keys: position p of (b, h) belongs to token group p / 64. New
+// rows (source rows rows[b][h][p - p0]) and staged rows (important rows hi_cap + p % 64, positions < p0)
+// feed the group kernel; the stage kernel copies the rows of an incomplete last group into staging.
+struct KchArgs {
+  const __nv_bfloat16* k_src;
+  const __nv_bfloat16* v_src;
+  const int32_t* src_tok;
+  const int32_t* rows;
+  __nv_bfloat16* k_hi;
+  __nv_bfloat16* v_hi;
+  int32_t* hi_tok;
+  uint8_t* k_codes;
+  uint8_t* v_codes;
+  __half2* k_params;  // [B][Hkv][lo_cap / 64][128]
+  __half2* v_params;
+  int32_t* lo_tok;
+  int heads_kv, hi_cap, hi_stride, lo_cap, n_src, n_rows, p0, p_end, g0;
+};
+
+constexpr int kKchThreads = 256;
+
+// Source of position p of head bh: the staged row (p < p0) or the new source row; token id in *tok.
+// A source row outside [0, n_src) reads as zeros (the host passes rows from mikv_select_demote).
+__device__ __forceinline__ const __nv_bfloat16* kch_row(const KchArgs& a, int bh, int p, bool key, int32_t* tok) {
+  if (p < a.p0) {
+    const size_t r = (size_t)bh * a.hi_stride + a.hi_cap + (p % kKchGroup);
+    if (tok) *tok = a.hi_tok[r];
+    return (key ? a.k_hi : a.v_hi) + r * kHeadDim;
+  }
+  const int r = a.rows[(size_t)bh * a.n_rows + (p - a.p0)];
+  if (tok) *tok = (r >= 0 && r < a.n_src) ? (a.src_tok ? a.src_tok[(size_t)bh * a.n_src + r] : r) : -1;
+  if (r < 0 || r >= a.n_src) return nullptr;
+  return (key ? a.k_src : a.v_src) + ((size_t)bh * a.n_src + r) * kHeadDim;
+}
+
+// Group g0 + blockIdx.x of (b, h) = blockIdx.y, complete: keys quantized per channel over its 64 tokens
+// (Eq. 1 with the same explicitly rounded fp32 steps as the per-token quantizer), values per token.
+template <int BITS, int GROUP>
+__global__ void __launch_bounds__(kKchThreads) kch_group_kernel(const KchArgs a) {
+  __shared__ __align__(16) __nv_bfloat16 sk[kKchGroup][kHeadDim];
+  __shared__ __align__(16) __nv_bfloat16 sv[kKchGroup][kHeadDim];
+  __shared__ uint32_t cbuf[kKchGroup][4 * BITS];
+  __shared__ uint32_t wbuf[kKchThreads / 32][32];
+  __shared__ int32_t stok[kKchGroup];
+  constexpr int QMAX = (1 << BITS) - 1;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int j = a.g0 + blockIdx.x, bh = blockIdx.y;
+  // 1. the group's 64 key and value rows (16-byte chunks) into shared memory; code rows cleared
+  for (int i = tid; i < kKchGroup * 16; i += kKchThreads) {
+    const int t = i >> 4, ch = i & 15;
+    const int p = kKchGroup * j + t;
+    int32_t tk = -1;
+    const __nv_bfloat16* kr = kch_row(a, bh, p, true, &tk);
+    const __nv_bfloat16* vr = kch_row(a, bh, p, false, nullptr);
+    const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+    reinterpret_cast<uint4*>(&sk[t][0])[ch] = kr ? reinterpret_cast<const uint4*>(kr)[ch] : z;
+    reinterpret_cast<uint4*>(&sv[t][0])[ch] = vr ? reinterpret_cast<const uint4*>(vr)[ch] : z;
+    if (ch == 0) stok[t] = tk;
+  }
+  for (int i = tid; i < kKchGroup * 4 * BITS; i += kKchThreads) (&cbuf[0][0])[i] = 0u;
+  __syncthreads();
+  // 2. keys: one thread per channel
+  if (tid < kHeadDim) {
+    const int c = tid;
+    float mn = INFINITY, mx = -INFINITY;
+    for (int t = 0; t < kKchGroup; ++t) {
+      const float x = __bfloat162float(sk[t][c]);
+      mn = fminf(mn, x);
+      mx = fmaxf(mx, x);
+    }
+    const __half beta16 = __float2half_rd(mn);
+    const float beta = __half2float(beta16);
+    const float span = __fsub_rn(mx, beta);
+    const __half alpha16 = span == 0.f ? __float2half_rn(1.f) : __float2half_ru(__fdiv_rn(span, (float)QMAX));
+    const float alpha = __half2float(alpha16);
+    a.k_params[((size_t)bh * (a.lo_cap / kKchGroup) + j) * kHeadDim + c] = __halves2half2(alpha16, beta16);
+    int unit, bit, unit1 = 0, bit1 = 0;
+    field_pos(c, BITS == 3 ? 2 : BITS, unit, bit);
+    if (BITS == 3) field_pos(c, 1, unit1, bit1);
+    for (int t = 0; t < kKchGroup; ++t) {
+      int code = __float2int_rn(__fdiv_rn(__fsub_rn(__bfloat162float(sk[t][c]), beta), alpha));
+      code = code < 0 ? 0 : (code > QMAX ? QMAX : code);
+      const uint32_t fmask = BITS == 3 ? 3u : (uint32_t)QMAX;
+      atomicOr(&cbuf[t][unit >> 1], (((uint32_t)code & fmask) << bit) << (16 * (unit & 1)));
+      if (BITS == 3) atomicOr(&cbuf[t][8 + (unit1 >> 1)], (((uint32_t)code >> 2) << bit1) << (16 * (unit1 & 1)));
+    }
+  }
+  __syncthreads();
+  const size_t pos0 = (size_t)bh * a.lo_cap + (size_t)kKchGroup * j;
+  for (int i = tid; i < kKchGroup * 4 * BITS; i += kKchThreads)
+    reinterpret_cast<uint32_t*>(a.k_codes + pos0 * (16 * BITS))[i] = (&cbuf[0][0])[i];
+  // 3. values per token (8 rows per warp) and token ids
+  for (int t = warp; t < kKchGroup; t += kKchThreads / 32) {
+    quantize_row_warp<BITS, GROUP>(&sv[t][0], nullptr, a.v_codes + (pos0 + t) * (16 * BITS),
+                                   a.v_params + (pos0 + t) * (kHeadDim / GROUP), wbuf[warp], lane);
+    if (lane == 0) a.lo_tok[pos0 + t] = stok[t];
+  }
+}
+
+// Rows of the incomplete last group (positions max(p0, 64 * floor(p_end / 64)) .. p_end - 1) into staging.
+__global__ void __launch_bounds__(kKchThreads) kch_stage_kernel(const KchArgs a) {
+  const int bh = blockIdx.x;
+  const int first = max(a.p0, a.p_end / kKchGroup * kKchGroup);
+  for (int i = threadIdx.x; i < (a.p_end - first) * 16; i += kKchThreads) {
+    const int p = first + (i >> 4), ch = i & 15;
+    int32_t tk = -1;
+    const __nv_bfloat16* kr = kch_row(a, bh, p, true, &tk);
+    const __nv_bfloat16* vr = kch_row(a, bh, p, false, nullptr);
+    const size_t r = (size_t)bh * a.hi_stride + a.hi_cap + (p % kKchGroup);
+    const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+    reinterpret_cast<uint4*>(a.k_hi + r * kHeadDim)[ch] = kr ? reinterpret_cast<const uint4*>(kr)[ch] : z;
+    reinterpret_cast<uint4*>(a.v_hi + r * kHeadDim)[ch] = vr ? reinterpret_cast<const uint4*>(vr)[ch] : z;
+    if (ch == 0) a.hi_tok[r] = tk;
+  }
+}
+
+template <int BITS>
+cudaError_t kch_group_launch(const KchArgs& a, int group, dim3 grid, cudaStream_t st) {
+  switch (group) {
+    case 32: kch_group_kernel<BITS, 32><<<grid, kKchThreads, 0, st>>>(a); break;
+    case 64: kch_group_kernel<BITS, 64><<<grid, kKchThreads, 0, st>>>(a); break;
+    case 128: kch_group_kernel<BITS, 128><<<grid, kKchThreads, 0, st>>>(a); break;
+    default: return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
 // ---------------------------------------------------------------------------- Eq. 2 balancer
 
 // Per (token chunk, batch row, head): column maxima of |x| folded into ws with atomicMax on the bit
@@ -199,6 +328,54 @@ cudaError_t launch_hi_quant(const mikv_shape& s, const mikv_cache& c, const void
     default: return cudaErrorInvalidValue;
   }
   return cudaGetLastError();
+}
+
+cudaError_t launch_kch_append(const mikv_shape& s, const mikv_cache& c, const void* k_src, const void* v_src,
+                              const int32_t* src_tok, int n_src, const int32_t* rows, int n_rows, int p0,
+                              cudaStream_t st) {
+  KchArgs a;
+  a.k_src = static_cast<const __nv_bfloat16*>(k_src);
+  a.v_src = static_cast<const __nv_bfloat16*>(v_src);
+  a.src_tok = src_tok;
+  a.rows = rows;
+  a.k_hi = static_cast<__nv_bfloat16*>(c.k_hi);
+  a.v_hi = static_cast<__nv_bfloat16*>(c.v_hi);
+  a.hi_tok = c.hi_tok;
+  a.k_codes = static_cast<uint8_t*>(c.k_codes);
+  a.v_codes = static_cast<uint8_t*>(c.v_codes);
+  a.k_params = static_cast<__half2*>(c.k_params);
+  a.v_params = static_cast<__half2*>(c.v_params);
+  a.lo_tok = c.lo_tok;
+  a.heads_kv = s.heads_kv;
+  a.hi_cap = s.hi_cap;
+  a.hi_stride = s.hi_stride;
+  a.lo_cap = s.lo_cap;
+  a.n_src = n_src;
+  a.n_rows = n_rows;
+  a.p0 = p0;  // positions < p0 come from staging
+  a.p_end = p0 + n_rows;
+  const int bh = s.batch * s.heads_kv;
+  // groups completed by this append: j0 = first group touched .. (p_end / 64) - 1; with no new rows, the
+  // caller asks for the group that ends at p0 (all of it staged)
+  const int j0 = n_rows > 0 ? p0 / kKchGroup : p0 / kKchGroup - 1;
+  const int j1 = n_rows > 0 ? a.p_end / kKchGroup : p0 / kKchGroup;
+  a.g0 = j0;
+  if (j1 > j0) {
+    cudaError_t e;
+    const dim3 grid(j1 - j0, bh);
+    switch (s.bits) {
+      case 2: e = kch_group_launch<2>(a, s.group, grid, st); break;
+      case 3: e = kch_group_launch<3>(a, s.group, grid, st); break;
+      case 4: e = kch_group_launch<4>(a, s.group, grid, st); break;
+      default: return cudaErrorInvalidValue;
+    }
+    if (e != cudaSuccess) return e;
+  }
+  if (n_rows > 0 && a.p_end % kKchGroup != 0) {  // the incomplete last group waits in staging
+    kch_stage_kernel<<<bh, kKchThreads, 0, st>>>(a);
+    return cudaGetLastError();
+  }
+  return cudaSuccess;
 }
 
 cudaError_t launch_balancer(const mikv_shape& s, const void* q_pre, const void* k_pre, int T, float* out,

@@ -153,6 +153,19 @@ __global__ void __launch_bounds__(kPostThreads, 2) step_post_kernel(const StepPo
   // coded important row is re-quantized from its fp32 dequantized values (already balanced, Sec. 3.3)
   if (a.evict) {  // eviction (no retained set): the victim's slot only becomes the next insertion slot
     if (tid == 0) a.slots[bh] = victim;
+  } else if (a.kch) {  // per-channel keys: the victim waits in bf16 in staging row hi_cap + n_lo % 64
+    const size_t src = (size_t)bh * a.hi_stride + victim;
+    const size_t dst = (size_t)bh * a.hi_stride + a.hi_cap + (a.n_lo % kKchGroup);
+    __nv_bfloat16* k = static_cast<__nv_bfloat16*>(a.k_hi);
+    __nv_bfloat16* v = static_cast<__nv_bfloat16*>(a.v_hi);
+    if (tid < 32) {
+      reinterpret_cast<uint2*>(k + dst * kHeadDim)[tid] = reinterpret_cast<const uint2*>(k + src * kHeadDim)[tid];
+    } else if (tid < 64) {
+      reinterpret_cast<uint2*>(v + dst * kHeadDim)[tid - 32] = reinterpret_cast<const uint2*>(v + src * kHeadDim)[tid - 32];
+    } else if (tid == 64) {
+      a.hi_tok[dst] = tok[victim];
+      a.slots[bh] = victim;
+    }
   } else if (warp < 2) {
     const bool is_v = warp == 1;
     const size_t pos = (size_t)bh * a.lo_cap + a.n_lo;

@@ -40,7 +40,8 @@ class MixedPrecisionLayer:
     @classmethod
     def from_prefill(cls, shape: Shape, k, v, scores, q_pre=None, budget: int = None, device="cuda"):
         """Build the cache from prefill K, V [B, Hkv, T, d] (bf16) and importance scores [B, Hkv, T].
-        With q_pre [B, Hq, T, d] the channel balancer is computed (Eq. 2); without it, b = 1. With scores
+        With q_pre [B, Hq, T, d] the channel balancer is computed (Eq. 2; not for per-channel keys, which
+        need none); without it, b = 1. With scores
         None the importance is the prefill's accumulated causal attention (mikv_prefill_scores, q_pre
         required)."""
         B, H, T, _ = k.shape
@@ -52,7 +53,7 @@ class MixedPrecisionLayer:
             mikv_prefill_scores(shape, q_pre, k, scores, ws)
         k_budget = shape.hi_cap - 1 if budget is None else budget
         bal = None
-        if q_pre is not None:
+        if q_pre is not None and not shape.k_channel_group:
             bal = torch.empty(H, shape.head_dim, dtype=torch.float32, device=device)
             ws = workspace(mikv_workspace_bytes(shape, WS_BALANCER, 0), device)
             mikv_compute_balancer(shape, q_pre, k, bal, ws)

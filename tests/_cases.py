@@ -18,7 +18,7 @@ bits16 = mi.bf16_bits
 
 def make_shape(w: mi.Workload, steps: int = 4, batch: int = None) -> pkg.Shape:
     return pkg.Shape(w.batch if batch is None else batch, w.heads_q, w.heads_kv, w.bits, w.group, w.hi_cap,
-                     w.lo_cap_for(steps), hi_bits=w.hi_bits)
+                     w.lo_cap_for(steps), hi_bits=w.hi_bits, k_channel_group=64 if w.k_channel else 0)
 
 
 def raw_inputs(w: mi.Workload, layer: int = 0, device="cpu", balanced: bool = True):
@@ -52,9 +52,14 @@ def oracle_layer(w: mi.Workload, raw, lo_cap: int, heads=None):
         sc = scores[b:b + 1, h:h + 1].numpy()
         T = k.shape[2]
         dem, kept = oracle.select_demote(sc, T - w.budget)
-        c = oracle.empty_cache(1, 1, w.head_dim, w.bits, w.group, w.hi_cap, lo_cap, hi_bits=w.hi_bits)
-        oracle.gather_hi(c, ks, vs, kept, src_scores=sc, balancer_=bal)
-        oracle.quantize_pack(c, ks, vs, dem, 0, balancer_=bal)
+        if w.k_channel:  # per-channel retained keys (App. C): no balancer, staging for the last group
+            c = oracle.empty_cache(1, 1, w.head_dim, w.bits, w.group, w.hi_cap, lo_cap, k_channel=True)
+            oracle.gather_hi(c, ks, vs, kept, src_scores=sc)
+            oracle.append_retained(c, ks, vs, dem, 0)
+        else:
+            c = oracle.empty_cache(1, 1, w.head_dim, w.bits, w.group, w.hi_cap, lo_cap, hi_bits=w.hi_bits)
+            oracle.gather_hi(c, ks, vs, kept, src_scores=sc, balancer_=bal)
+            oracle.quantize_pack(c, ks, vs, dem, 0, balancer_=bal)
         out.append(dict(cache=c, balancer=bal, b=b, h=h, demoted=dem[0, 0], kept=kept[0, 0]))
     return out
 

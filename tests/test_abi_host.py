@@ -67,7 +67,7 @@ def test_row_bytes(lib):
 
 def _shape(**kw):
     s = dict(batch=2, heads_q=8, heads_kv=2, head_dim=128, bits=2, group=32, hi_cap=20, hi_stride=32, lo_cap=64,
-             hi_bits=0, hi_group=64)
+             hi_bits=0, hi_group=64, k_channel_group=0)
     s.update(kw)
     return pkg._Shape(*[s[n] for n, _ in pkg._Shape._fields_])
 
@@ -94,6 +94,10 @@ def test_workspace_sizes_monotone(lib):
     (dict(hi_bits=3), 2), (dict(hi_bits=12), 2), (dict(hi_bits=8, hi_group=32), 2), (dict(hi_bits=4, hi_group=128), 2),
     (dict(hi_bits=8), 0), (dict(hi_bits=4), 0), (dict(hi_bits=2), 0), (dict(hi_bits=16, hi_group=0), 0),
     (dict(bits=0, group=7), 0), (dict(bits=-1), 1),
+    # per-channel keys: groups of 64 tokens, 64 staging rows after the important slots, bf16 important set
+    (dict(k_channel_group=64, hi_stride=96), 0), (dict(k_channel_group=32, hi_stride=96), 2),
+    (dict(k_channel_group=64, hi_stride=80), 1), (dict(k_channel_group=64, hi_stride=96, lo_cap=96), 1),
+    (dict(k_channel_group=64, hi_stride=96, hi_bits=8), 2), (dict(k_channel_group=64, hi_stride=96, bits=0), 2),
 ])
 def test_shape_validation(lib, kw, code):
     s = _shape(**kw)
