@@ -11,6 +11,8 @@ template <int OUT_F32>
 __global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a, int G) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int bq = blockIdx.x * 4 + warp;
+  grid_dependency_wait();
+  allow_dependent_launch();
   if (bq >= a.batch * a.heads_q) return;
   const int b = bq / a.heads_q, hq = bq - b * a.heads_q;
   const int h = hq / G, jh = hq - h * G;
@@ -18,7 +20,8 @@ __global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a, int G) {
   const int w0 = owner_warp((long long)bh * a.n_u, a.n_units, a.n_warps);
   const int w1 = owner_warp((long long)(bh + 1) * a.n_u - 1, a.n_units, a.n_warps);
   float r[4], M, L;
-  merge_head_warp(a.part_o, a.part_ml, G, bh, jh, w0, w1, lane, r, M, L);
+  merge_stats_warp(a.part_ml, G, bh, jh, w0, w1, lane, M, L);
+  merge_output_warp(a.part_o, a.part_ml, G, bh, jh, w0, w1, lane, M, L, r);
   if (OUT_F32) {
     reinterpret_cast<float4*>(static_cast<float*>(a.out) + (size_t)bq * kHeadDim)[lane] = make_float4(r[0], r[1], r[2], r[3]);
   } else {
@@ -84,11 +87,7 @@ cudaError_t launch_attention(const AttnArgs& a, int bits, int group, int hi_bits
 
 cudaError_t launch_merge(const MergeArgs& a, int G, int out_f32, cudaStream_t st) {
   const int grid = (a.batch * a.heads_q + 3) / 4;
-  if (out_f32)
-    merge_kernel<1><<<grid, 128, 0, st>>>(a, G);
-  else
-    merge_kernel<0><<<grid, 128, 0, st>>>(a, G);
-  return cudaGetLastError();
+  return launch_chained(out_f32 ? merge_kernel<1> : merge_kernel<0>, dim3(grid), dim3(128), 0, st, a, G);
 }
 
 }  // namespace mikv

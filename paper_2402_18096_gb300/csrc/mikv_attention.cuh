@@ -774,6 +774,10 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
       prefetch_tensormap(&a.map_k_par);
       prefetch_tensormap(&a.map_v_par);
     }
+  }
+  grid_dependency_wait();  // the cache and the query come from the kernels before this one
+  allow_dependent_launch();
+  if (lane == 0) {
     for (int k = 0; k < kNS && u0 + k < u1; ++k) {
       issue_unit<BITS, GROUP, HB, KCH>(a, ci, ring + k * kStageBytes, bars + 8 * k);
       cursor_next(ci, hu, n_u);
@@ -905,8 +909,7 @@ cudaError_t launch_kernel(const AttnArgs& a, int grid, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  kern<<<grid, kThreads, smem, st>>>(a);
-  return cudaGetLastError();
+  return launch_chained(kern, dim3(grid), dim3(kThreads), smem, st, a);
 }
 
 template <int BITS, int GROUP, int HB, bool KCH>

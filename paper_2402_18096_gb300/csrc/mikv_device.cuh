@@ -211,4 +211,12 @@ __device__ __forceinline__ void record_error(int* status, int code) {
   if (status) atomicCAS(status, 0, code);
 }
 
+// Programmatic dependent launch (kernels of one decode step launched by launch_chained): a chained
+// kernel may be scheduled while its predecessor in the stream is still running, so it waits here for
+// the predecessor to complete (and its writes to be visible) before touching global memory that another
+// kernel writes or reads; outside such a launch both instructions do nothing.
+__device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+// Lets the next chained kernel be scheduled once every CTA of this grid has reached this point (or exited).
+__device__ __forceinline__ void allow_dependent_launch() { asm volatile("griddepcontrol.launch_dependents;" :::); }
+
 }  // namespace mikv

@@ -205,4 +205,22 @@ cudaError_t launch_gather(const mikv_shape& s, const mikv_cache& c, const void* 
                           const int32_t* src_tok, const float* src_scores, int n_src,
                           const int32_t* rows, int n_rows, cudaStream_t st);
 
+// Launch of a kernel on the decode-step path with programmatic dependent launch allowed: the kernel may be
+// scheduled while the previous kernel of the stream finishes (hiding the launch gap), and executes
+// grid_dependency_wait() before its first access to memory that other kernels write or read.
+template <typename... P, typename... A>
+cudaError_t launch_chained(void (*kernel)(P...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, A&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<A&&>(args)...);
+}
+
 }  // namespace mikv

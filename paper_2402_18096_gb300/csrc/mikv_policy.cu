@@ -19,7 +19,7 @@ __global__ void __launch_bounds__(128) update_importance_kernel(float* acc, cons
   float add = 0.f;
   for (int j = 0; j < G; ++j) {
     const int bq = b * Hq + h * G + j;
-    add += expf(hi_logits[(size_t)bq * hi_stride + i] - ml[2 * bq]) / ml[2 * bq + 1];
+    add += importance_weight(hi_logits[(size_t)bq * hi_stride + i], ml[2 * bq], 1.f / ml[2 * bq + 1]);
   }
   acc[(size_t)bh * hi_stride + i] += add;
 }
@@ -153,6 +153,8 @@ __global__ void __launch_bounds__(64) insert_kernel(__nv_bfloat16* k_hi, __nv_bf
                                                     const __nv_bfloat16* v_new, int tok, const int32_t* slots,
                                                     int hi_cap, int hi_stride) {
   const int bh = blockIdx.x, tid = threadIdx.x;
+  grid_dependency_wait();  // the slot comes from the previous step's tail
+  allow_dependent_launch();
   const int s = slots[bh];
   if (s < 0 || s >= hi_cap) return;
   const size_t row = (size_t)bh * hi_stride + s;
@@ -208,11 +210,10 @@ cudaError_t launch_insert(const mikv_shape& s, const mikv_cache& c, const void* 
                           int tok, const int32_t* slots, cudaStream_t st) {
   if (hi_bits_of(s) != 16)
     return launch_hi_quant(s, c, k_new, v_new, nullptr, nullptr, 0, nullptr, 0, slots, tok, st);
-  insert_kernel<<<s.batch * s.heads_kv, 64, 0, st>>>(
-      static_cast<__nv_bfloat16*>(c.k_hi), static_cast<__nv_bfloat16*>(c.v_hi), c.hi_tok, c.acc,
-      static_cast<const __nv_bfloat16*>(k_new), static_cast<const __nv_bfloat16*>(v_new), tok, slots, s.hi_cap,
-      s.hi_stride);
-  return cudaGetLastError();
+  return launch_chained(insert_kernel, dim3(s.batch * s.heads_kv), dim3(64), 0, st,
+                        static_cast<__nv_bfloat16*>(c.k_hi), static_cast<__nv_bfloat16*>(c.v_hi), c.hi_tok, c.acc,
+                        static_cast<const __nv_bfloat16*>(k_new), static_cast<const __nv_bfloat16*>(v_new), tok, slots,
+                        s.hi_cap, s.hi_stride);
 }
 
 cudaError_t launch_gather(const mikv_shape& s, const mikv_cache& c, const void* k_src, const void* v_src,

@@ -82,6 +82,8 @@ template <int HB>
 __global__ void __launch_bounds__(256) hi_quant_kernel(const HiQArgs a) {
   __shared__ uint32_t buf[8][32];
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  grid_dependency_wait();  // insertion: the slot comes from the previous step's tail
+  allow_dependent_launch();
   const int i = blockIdx.x * 4 + (w >> 1);
   const bool is_v = (w & 1) != 0;
   const int bh = blockIdx.y, h = bh % a.heads_kv;
@@ -158,6 +160,8 @@ __global__ void __launch_bounds__(kKchThreads) kch_group_kernel(const KchArgs a)
   constexpr int QMAX = (1 << BITS) - 1;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int j = a.g0 + blockIdx.x, bh = blockIdx.y;
+  grid_dependency_wait();  // the group's last row is staged by the step tail before this kernel
+  allow_dependent_launch();
   // 1. the group's 64 key and value rows (16-byte chunks) into shared memory; code rows cleared
   for (int i = tid; i < kKchGroup * 16; i += kKchThreads) {
     const int t = i >> 4, ch = i & 15;
@@ -230,12 +234,11 @@ __global__ void __launch_bounds__(kKchThreads) kch_stage_kernel(const KchArgs a)
 template <int BITS>
 cudaError_t kch_group_launch(const KchArgs& a, int group, dim3 grid, cudaStream_t st) {
   switch (group) {
-    case 32: kch_group_kernel<BITS, 32><<<grid, kKchThreads, 0, st>>>(a); break;
-    case 64: kch_group_kernel<BITS, 64><<<grid, kKchThreads, 0, st>>>(a); break;
-    case 128: kch_group_kernel<BITS, 128><<<grid, kKchThreads, 0, st>>>(a); break;
-    default: return cudaErrorInvalidValue;
+    case 32: return launch_chained(kch_group_kernel<BITS, 32>, grid, dim3(kKchThreads), 0, st, a);
+    case 64: return launch_chained(kch_group_kernel<BITS, 64>, grid, dim3(kKchThreads), 0, st, a);
+    case 128: return launch_chained(kch_group_kernel<BITS, 128>, grid, dim3(kKchThreads), 0, st, a);
   }
-  return cudaGetLastError();
+  return cudaErrorInvalidValue;
 }
 
 // ---------------------------------------------------------------------------- Eq. 2 balancer
@@ -322,12 +325,11 @@ cudaError_t launch_hi_quant(const mikv_shape& s, const mikv_cache& c, const void
   const dim3 grid(rows ? (n_rows + 3) / 4 : 1, s.batch * s.heads_kv);
   const int threads = rows ? 256 : 64;
   switch (hi_bits_of(s)) {
-    case 8: hi_quant_kernel<8><<<grid, threads, 0, st>>>(a); break;
-    case 4: hi_quant_kernel<4><<<grid, threads, 0, st>>>(a); break;
-    case 2: hi_quant_kernel<2><<<grid, threads, 0, st>>>(a); break;
-    default: return cudaErrorInvalidValue;
+    case 8: return launch_chained(hi_quant_kernel<8>, grid, dim3(threads), 0, st, a);
+    case 4: return launch_chained(hi_quant_kernel<4>, grid, dim3(threads), 0, st, a);
+    case 2: return launch_chained(hi_quant_kernel<2>, grid, dim3(threads), 0, st, a);
   }
-  return cudaGetLastError();
+  return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_kch_append(const mikv_shape& s, const mikv_cache& c, const void* k_src, const void* v_src,

@@ -116,14 +116,20 @@ __device__ __forceinline__ int owner_warp(long long U, long long n_units, int n_
   return w;
 }
 
-// One warp combines the split partials of query head jh of KV head bh (warps w0..w1 of the attention
-// kernel wrote slots w + bh; each partial is a normalised output with its (max, sum)): lane l returns
-// the output of channels 4l..4l+3, the partials weighted by exp(max - M) * sum, and every lane returns
-// (M, L) = (max logit, sum of exp(logit - M)). The per-slot statistics are read by all lanes at
-// once and broadcast with shuffles, so the merge costs a few dependent loads whatever the slot count.
-__device__ __forceinline__ void merge_head_warp(const float* part_o, const float* part_ml, int G, int bh, int jh,
-                                                int w0, int w1, int lane, float (&out)[4], float& M, float& L) {
+// The split partials of query head jh of KV head bh: warps w0..w1 of the attention kernel wrote slots
+// w + bh, each a normalised output with its (max, sum). merge_stats_warp gives every lane (M, L) = (max
+// logit, sum of exp(logit - M)); merge_output_warp gives lane l the output of channels 4l..4l+3, the
+// partials weighted by exp(max - M) * sum, over L. The per-slot statistics are read by all lanes at once
+// and broadcast with shuffles, so a merge costs a few dependent loads whatever the slot count.
+__device__ __forceinline__ float merge_weight(const float* part_ml, int G, int bh, int jh, int w0, int i, float M) {
   constexpr float kLog2e = 1.4426950408889634f;
+  const size_t slot = (size_t)(w0 + i + bh);
+  const float ms = part_ml[(slot * G + jh) * 2];
+  return ms == -INFINITY ? 0.f : fast_exp2((ms - M) * kLog2e) * part_ml[(slot * G + jh) * 2 + 1];
+}
+
+__device__ __forceinline__ void merge_stats_warp(const float* part_ml, int G, int bh, int jh, int w0, int w1, int lane,
+                                                 float& M, float& L) {
   const int n = w1 - w0 + 1;
   M = -INFINITY;
   for (int c0 = 0; c0 < n; c0 += 32) {
@@ -132,24 +138,38 @@ __device__ __forceinline__ void merge_head_warp(const float* part_o, const float
   }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
-  float O[4] = {0.f, 0.f, 0.f, 0.f};
   float Lp = 0.f;
+  for (int c0 = lane; c0 < n; c0 += 32) Lp += merge_weight(part_ml, G, bh, jh, w0, c0, M);
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) Lp += __shfl_xor_sync(0xffffffffu, Lp, off);
+  L = Lp;
+}
+
+__device__ __forceinline__ void merge_output_warp(const float* part_o, const float* part_ml, int G, int bh, int jh,
+                                                  int w0, int w1, int lane, float M, float L, float (&out)[4]) {
+  const int n = w1 - w0 + 1;
+  float O[4] = {0.f, 0.f, 0.f, 0.f};
   for (int c0 = 0; c0 < n; c0 += 32) {
-    const int i = c0 + lane;
-    float wt = 0.f;
-    if (i < n) {
-      const size_t slot = (size_t)(w0 + i + bh);
-      const float ms = part_ml[(slot * G + jh) * 2];
-      if (ms != -INFINITY) {
-        wt = fast_exp2((ms - M) * kLog2e) * part_ml[(slot * G + jh) * 2 + 1];
-        Lp += wt;
+    const float wt = c0 + lane < n ? merge_weight(part_ml, G, bh, jh, w0, c0 + lane, M) : 0.f;
+    const int cnt = min(32, n - c0);
+    int k = 0;
+    for (; k + 4 <= cnt; k += 4) {  // four partials' loads in flight, summed in slot order
+      float4 po[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        po[u] = reinterpret_cast<const float4*>(part_o + ((size_t)(w0 + c0 + k + u + bh) * G + jh) * kHeadDim)[lane];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const float ws = __shfl_sync(0xffffffffu, wt, k + u);
+        O[0] += ws * po[u].x;
+        O[1] += ws * po[u].y;
+        O[2] += ws * po[u].z;
+        O[3] += ws * po[u].w;
       }
     }
-    const int cnt = min(32, n - c0);
-    for (int k = 0; k < cnt; ++k) {
+    for (; k < cnt; ++k) {
       const float ws = __shfl_sync(0xffffffffu, wt, k);
-      const size_t slot = (size_t)(w0 + c0 + k + bh);
-      const float4 po = reinterpret_cast<const float4*>(part_o + (slot * G + jh) * kHeadDim)[lane];
+      const float4 po = reinterpret_cast<const float4*>(part_o + ((size_t)(w0 + c0 + k + bh) * G + jh) * kHeadDim)[lane];
       O[0] += ws * po.x;
       O[1] += ws * po.y;
       O[2] += ws * po.z;
@@ -157,10 +177,14 @@ __device__ __forceinline__ void merge_head_warp(const float* part_o, const float
     }
   }
 #pragma unroll
-  for (int off = 16; off > 0; off >>= 1) Lp += __shfl_xor_sync(0xffffffffu, Lp, off);
-  L = Lp;
-#pragma unroll
   for (int i = 0; i < 4; ++i) out[i] = O[i] / L;
+}
+
+// Importance weight of one slot for one query head: exp(s - M) / L, as exp2((s - M) log2 e) times the
+// reciprocal of L (the same arithmetic in the fused step tail and in mikv_update_importance).
+__device__ __forceinline__ float importance_weight(float s, float M, float inv_L) {
+  constexpr float kLog2e = 1.4426950408889634f;
+  return fast_exp2((s - M) * kLog2e) * inv_L;
 }
 
 }  // namespace mikv

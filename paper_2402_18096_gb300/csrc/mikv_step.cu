@@ -41,7 +41,7 @@ __device__ __forceinline__ void load_quad(const float* logit, const float* acc, 
 // scores stored, and the running minimum of (score, id) advanced.
 template <int G>
 __device__ __forceinline__ void update_quad(float* acc, int hi_cap, int v, SlotQuad<G>& q, const float* s_m,
-                                            const float* s_l, unsigned long long& best, int& best_slot) {
+                                            const float* s_il, unsigned long long& best, int& best_slot) {
   float* ac = &q.ac.x;
   const int32_t* tk = &q.tk.x;
 #pragma unroll
@@ -50,7 +50,7 @@ __device__ __forceinline__ void update_quad(float* acc, int hi_cap, int v, SlotQ
     if (i >= hi_cap) break;
     float add = 0.f;
 #pragma unroll
-    for (int j = 0; j < G; ++j) add += expf((&q.lg[j].x)[e] - s_m[j]) / s_l[j];
+    for (int j = 0; j < G; ++j) add += importance_weight((&q.lg[j].x)[e], s_m[j], s_il[j]);
     ac[e] = ac[e] + add;
     const unsigned long long k = order_key(ac[e], tk[e]);
     if (k < best) {
@@ -61,17 +61,19 @@ __device__ __forceinline__ void update_quad(float* acc, int hi_cap, int v, SlotQ
   reinterpret_cast<float4*>(acc)[v] = q.ac;  // padding slots (>= hi_cap) are written back unchanged
 }
 
-static_assert(kPostThreads <= 1024, "the final argmin reduces at most one entry per lane of warp 0");
+static_assert(kPostThreads == 256, "eight warps: one per query head for the merge, one argmin entry per warp");
 
 template <int BITS, int GROUP, int G, int OUT_F32>
 __global__ void __launch_bounds__(kPostThreads, 2) step_post_kernel(const StepPostArgs a) {
-  __shared__ float s_m[8], s_l[8];
+  __shared__ float s_m[8], s_l[8], s_il[8];
   __shared__ unsigned long long s_best[kPostThreads / 32];
   __shared__ int s_slot[kPostThreads / 32];
   __shared__ int s_victim;
   __shared__ uint32_t buf[2][32];
   const int bh = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int b = bh / a.heads_kv, h = bh - b * a.heads_kv;
+  grid_dependency_wait();  // logits and partials come from the attention kernel
+  allow_dependent_launch();
   float* acc = a.acc + (size_t)bh * a.hi_stride;
   const int32_t* tok = a.hi_tok + (size_t)bh * a.hi_stride;
   const float* logit = a.hi_logits + (size_t)(b * a.heads_q + h * G) * a.hi_stride;
@@ -81,25 +83,16 @@ __global__ void __launch_bounds__(kPostThreads, 2) step_post_kernel(const StepPo
   SlotQuad<G> q0;
   if (tid < nv) load_quad<G>(logit, acc, tok, a.hi_stride, tid, q0);
 
-  // 1. combine the split partials of query heads h*G .. h*G+G-1 (one warp per query head)
+  // 1. softmax statistics (M, L) of query heads h*G .. h*G+G-1 from the split partials (one warp per head)
+  const int w0 = owner_warp((long long)bh * a.n_u, a.n_units, a.n_warps);
+  const int w1 = owner_warp((long long)(bh + 1) * a.n_u - 1, a.n_units, a.n_warps);
   if (warp < G) {
-    const int w0 = owner_warp((long long)bh * a.n_u, a.n_units, a.n_warps);
-    const int w1 = owner_warp((long long)(bh + 1) * a.n_u - 1, a.n_units, a.n_warps);
-    float r[4], M, L;
-    merge_head_warp(a.part_o, a.part_ml, G, bh, warp, w0, w1, lane, r, M, L);
-    const size_t bq = (size_t)b * a.heads_q + h * G + warp;
-    if (OUT_F32) {
-      reinterpret_cast<float4*>(static_cast<float*>(a.out) + bq * kHeadDim)[lane] = make_float4(r[0], r[1], r[2], r[3]);
-    } else {
-      __nv_bfloat162 v0 = __floats2bfloat162_rn(r[0], r[1]), v1 = __floats2bfloat162_rn(r[2], r[3]);
-      uint2 u;
-      u.x = *reinterpret_cast<uint32_t*>(&v0);
-      u.y = *reinterpret_cast<uint32_t*>(&v1);
-      reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(a.out) + bq * kHeadDim)[lane] = u;
-    }
+    float M, L;
+    merge_stats_warp(a.part_ml, G, bh, warp, w0, w1, lane, M, L);
     if (lane == 0) {
       s_m[warp] = M;
       s_l[warp] = L;
+      s_il[warp] = 1.f / L;
     }
   }
   __syncthreads();
@@ -107,15 +100,15 @@ __global__ void __launch_bounds__(kPostThreads, 2) step_post_kernel(const StepPo
   // 2. importance update and the least important slot (keys are unique: ids are distinct)
   unsigned long long best = ~0ull;
   int best_slot = -1;
-  if (tid < nv) update_quad<G>(acc, a.hi_cap, tid, q0, s_m, s_l, best, best_slot);
+  if (tid < nv) update_quad<G>(acc, a.hi_cap, tid, q0, s_m, s_il, best, best_slot);
   constexpr int kInFlight = G <= 4 ? 2 : 1;  // groups loaded before any of them is used
   for (int v = tid + kPostThreads; v < nv; v += kInFlight * kPostThreads) {
     SlotQuad<G> q1, q2;
     const bool two = kInFlight == 2 && v + kPostThreads < nv;
     load_quad<G>(logit, acc, tok, a.hi_stride, v, q1);
     if (two) load_quad<G>(logit, acc, tok, a.hi_stride, v + kPostThreads, q2);
-    update_quad<G>(acc, a.hi_cap, v, q1, s_m, s_l, best, best_slot);
-    if (two) update_quad<G>(acc, a.hi_cap, v + kPostThreads, q2, s_m, s_l, best, best_slot);
+    update_quad<G>(acc, a.hi_cap, v, q1, s_m, s_il, best, best_slot);
+    if (two) update_quad<G>(acc, a.hi_cap, v + kPostThreads, q2, s_m, s_il, best, best_slot);
   }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) {
@@ -146,10 +139,27 @@ __global__ void __launch_bounds__(kPostThreads, 2) step_post_kernel(const StepPo
     if (lane == 0) s_victim = best_slot;
   }
   __syncthreads();
+
+  // 3. the attention output of each query head (warps 2, 3, ... so that warps 0 and 1 demote meanwhile)
+  const int jm = (warp + 6) & 7;
+  if (jm < G) {
+    float r[4];
+    merge_output_warp(a.part_o, a.part_ml, G, bh, jm, w0, w1, lane, s_m[jm], s_l[jm], r);
+    const size_t bq = (size_t)b * a.heads_q + h * G + jm;
+    if (OUT_F32) {
+      reinterpret_cast<float4*>(static_cast<float*>(a.out) + bq * kHeadDim)[lane] = make_float4(r[0], r[1], r[2], r[3]);
+    } else {
+      __nv_bfloat162 v0 = __floats2bfloat162_rn(r[0], r[1]), v1 = __floats2bfloat162_rn(r[2], r[3]);
+      uint2 u;
+      u.x = *reinterpret_cast<uint32_t*>(&v0);
+      u.y = *reinterpret_cast<uint32_t*>(&v1);
+      reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(a.out) + bq * kHeadDim)[lane] = u;
+    }
+  }
   const int victim = s_victim;
   if (victim < 0) return;  // unreachable for valid scores (hi_cap >= 1, no NaN)
 
-  // 3. demote the victim: quantize its key (balanced, Eq. 3) and value rows into retained row n_lo; a
+  // 4. demote the victim: quantize its key (balanced, Eq. 3) and value rows into retained row n_lo; a
   // coded important row is re-quantized from its fp32 dequantized values (already balanced, Sec. 3.3)
   if (a.evict) {  // eviction (no retained set): the victim's slot only becomes the next insertion slot
     if (tid == 0) a.slots[bh] = victim;
@@ -194,11 +204,8 @@ __global__ void __launch_bounds__(kPostThreads, 2) step_post_kernel(const StepPo
 template <int BITS, int GROUP, int G>
 cudaError_t post_out(const StepPostArgs& a, int out_f32, cudaStream_t st) {
   const int grid = a.batch * a.heads_kv;
-  if (out_f32)
-    step_post_kernel<BITS, GROUP, G, 1><<<grid, kPostThreads, 0, st>>>(a);
-  else
-    step_post_kernel<BITS, GROUP, G, 0><<<grid, kPostThreads, 0, st>>>(a);
-  return cudaGetLastError();
+  return launch_chained(out_f32 ? step_post_kernel<BITS, GROUP, G, 1> : step_post_kernel<BITS, GROUP, G, 0>, dim3(grid),
+                        dim3(kPostThreads), 0, st, a);
 }
 
 template <int BITS, int GROUP>
