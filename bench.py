@@ -256,21 +256,24 @@ def run_mikv(args):
     attn_bytes = sum(layer.cache.nbytes_attended(layer.n_lo) for layer in layers) / L
 
     # ---- end to end through the C ABI with host buffers: H2D inputs, D2H outputs, every step
+    # every layer's (q, k_new, v_new) of a step sit in one pinned host buffer and arrive in one copy
     per_in = [inputs[0][li] for li in range(L)]
-    host_in = [[t.cpu().pin_memory() for t in trip] for trip in per_in]
+    sizes = [t.numel() for trip in per_in for t in trip]
+    host_flat = torch.cat([t.reshape(-1).cpu() for trip in per_in for t in trip]).pin_memory()
+    dev_flat = torch.empty_like(host_flat, device=dev)
+    views = list(torch.split(dev_flat, sizes))
+    dev_in = [[views[3 * li + j].view(per_in[li][j].shape) for j in range(3)] for li in range(L)]
     host_out = torch.empty(L, w.batch, w.heads_q, w.head_dim, dtype=torch.bfloat16).pin_memory()
-    dev_in = [[torch.empty_like(t) for t in trip] for trip in per_in]
     dev_out = torch.empty(L, w.batch, w.heads_q, w.head_dim, dtype=torch.bfloat16, device=dev)
-    h2d = sum(t.numel() * t.element_size() for trip in host_in for t in trip)
+    h2d = host_flat.numel() * host_flat.element_size()
     d2h = host_out.numel() * host_out.element_size()
     torch.cuda.synchronize()
     if dist:
         dist.barrier()
     t0 = time.perf_counter()
     for s in range(e2e_steps):
+        dev_flat.copy_(host_flat, non_blocking=True)
         for li, layer in enumerate(layers):
-            for d, h in zip(dev_in[li], host_in[li]):
-                d.copy_(h, non_blocking=True)
             layer.step(dev_in[li][0], dev_in[li][1], dev_in[li][2], dev_out[li])
         host_out.copy_(dev_out, non_blocking=True)
         torch.cuda.current_stream().synchronize()
