@@ -696,7 +696,7 @@ __device__ __forceinline__ void write_partial(const AttnArgs& a, int slot, Softm
 }
 
 template <int BITS, int GROUP, int HB, bool KCH>
-__device__ __forceinline__ void issue_unit(const AttnArgs& a, const Cursor& c, uint32_t dst, uint32_t bar) {
+__device__ __forceinline__ void issue_unit(const AttnArgs& a, const Cursor& c, uint32_t dst, uint32_t bar, uint64_t pol) {
   constexpr LoUnit U = KCH ? lo_unit_layout_kch(BITS, GROUP) : lo_unit_layout(BITS, GROUP);
   const UnitKind k = cursor_kind(c, a.hi_units, a.n_u);
   if constexpr (HB != 16) {
@@ -705,35 +705,35 @@ __device__ __forceinline__ void issue_unit(const AttnArgs& a, const Cursor& c, u
       const long long row = (long long)c.bh * a.hi_stride + 16 * H.blocks * k.index;  // first slot
       mbar_arrive_expect_tx(bar, H.tx);
       const int crow = (int)(row * H.pitch / H.map_w), prow = (int)(row * H.param_row / H.param_w);
-      tma_load_2d(dst + H.k_a, &a.map_k_hi, 0, crow, bar);
-      tma_load_2d(dst + H.v_a, &a.map_v_hi, 0, crow, bar);
-      tma_load_2d(dst + H.k_p, &a.map_k_hp, 0, prow, bar);
-      tma_load_2d(dst + H.v_p, &a.map_v_hp, 0, prow, bar);
+      tma_load_2d(dst + H.k_a, &a.map_k_hi, 0, crow, bar, pol);
+      tma_load_2d(dst + H.v_a, &a.map_v_hi, 0, crow, bar, pol);
+      tma_load_2d(dst + H.k_p, &a.map_k_hp, 0, prow, bar, pol);
+      tma_load_2d(dst + H.v_p, &a.map_v_hp, 0, prow, bar, pol);
       return;
     }
   }
   if (k.hi) {
     const int row = c.bh * a.hi_stride + 16 * k.index;
     mbar_arrive_expect_tx(bar, kHiBlockBytes);
-    tma_load_2d(dst, &a.map_k_hi, 0, row, bar);
-    tma_load_2d(dst + 2048, &a.map_k_hi, 64, row, bar);
-    tma_load_2d(dst + 4096, &a.map_v_hi, 0, row, bar);
-    tma_load_2d(dst + 6144, &a.map_v_hi, 64, row, bar);
+    tma_load_2d(dst, &a.map_k_hi, 0, row, bar, pol);
+    tma_load_2d(dst + 2048, &a.map_k_hi, 64, row, bar, pol);
+    tma_load_2d(dst + 4096, &a.map_v_hi, 0, row, bar, pol);
+    tma_load_2d(dst + 6144, &a.map_v_hi, 64, row, bar, pol);
   } else {
     // one box per array covers the whole unit (U.blocks blocks of 16 rows); rows past this head's
     // retained length are masked by the consumer, rows past the array are zero-filled by TMA
     const long long row = (long long)c.bh * a.lo_cap + 16 * U.blocks * k.index;  // first token row
     mbar_arrive_expect_tx(bar, U.tx);
     const int crow = (int)(row * U.pitch / U.map_w), prow = (int)(row * U.param_row / U.param_w);
-    tma_load_2d(dst + U.k_a, &a.map_k_lo, 0, crow, bar);
-    tma_load_2d(dst + U.v_a, &a.map_v_lo, 0, crow, bar);
+    tma_load_2d(dst + U.k_a, &a.map_k_lo, 0, crow, bar, pol);
+    tma_load_2d(dst + U.v_a, &a.map_v_lo, 0, crow, bar, pol);
     if constexpr (KCH) {  // the group's key (alpha, beta) pairs: four 128-byte rows per group of 64 tokens
       const long long grp = (long long)c.bh * (a.lo_cap / kKchGroup) + (16 * U.blocks * k.index) / kKchGroup;
-      tma_load_2d(dst + U.k_p, &a.map_k_par, 0, (int)(4 * grp), bar);
+      tma_load_2d(dst + U.k_p, &a.map_k_par, 0, (int)(4 * grp), bar, pol);
     } else {
-      tma_load_2d(dst + U.k_p, &a.map_k_par, 0, prow, bar);
+      tma_load_2d(dst + U.k_p, &a.map_k_par, 0, prow, bar, pol);
     }
-    tma_load_2d(dst + U.v_p, &a.map_v_par, 0, prow, bar);
+    tma_load_2d(dst + U.v_p, &a.map_v_par, 0, prow, bar, pol);
   }
 }
 
@@ -759,6 +759,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
   const int u1 = (int)((long long)(wg + 1) * a.n_units / a.n_warps);
   const int hu = a.hi_units, n_u = a.n_u;
   Cursor ci = cursor_at(u0, hu, n_u);  // next unit to issue (lane 0)
+  const uint64_t pol = l2_evict_first();  // the cache is streamed once per launch
   if (lane == 0) {
     for (int s = 0; s < kNS; ++s) mbar_init(bars + 8 * s, 1);
     fence_mbar_init();
@@ -779,7 +780,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
   allow_dependent_launch();
   if (lane == 0) {
     for (int k = 0; k < kNS && u0 + k < u1; ++k) {
-      issue_unit<BITS, GROUP, HB, KCH>(a, ci, ring + k * kStageBytes, bars + 8 * k);
+      issue_unit<BITS, GROUP, HB, KCH>(a, ci, ring + k * kStageBytes, bars + 8 * k, pol);
       cursor_next(ci, hu, n_u);
     }
   }
@@ -883,7 +884,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
     __syncwarp();
     if (lane == 0 && u + kNS < u1) {
       fence_proxy_async();  // our generic reads of this stage precede the next asynchronous write
-      issue_unit<BITS, GROUP, HB, KCH>(a, ci, stage, bars + 8 * s);
+      issue_unit<BITS, GROUP, HB, KCH>(a, ci, stage, bars + 8 * s, pol);
       cursor_next(ci, hu, n_u);
     }
   }
