@@ -9,11 +9,11 @@
 
 namespace mikv {
 
-// Tiles of 64 tokens x 128 channels (bf16) stream through shared memory by TMA.
-constexpr int kPfTile = 64;
+// Tiles of 128 tokens x 128 channels (bf16) stream through shared memory by TMA.
+constexpr int kPfTile = 128;
 
 struct PrefillArgs {
-  CUtensorMap map_q;  // q_pre rows [B * Hq * T][128] bf16, box 64 channels x 64 rows, 128B swizzle
+  CUtensorMap map_q;  // q_pre rows [B * Hq * T][128] bf16, box 64 channels x 128 rows, 128B swizzle
   CUtensorMap map_k;  // k_pre rows [B * Hkv * T][128] bf16, same boxes
   float2* stats;      // [B * Hq][T]: (row max of the logits in log2 units, 1 / row sum)
   float* scores;      // [B * Hkv][T]
