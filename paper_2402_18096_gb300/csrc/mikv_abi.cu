@@ -364,11 +364,12 @@ mikv_status mikv_prefill_scores(const mikv_shape* shape, const void* q_pre, cons
     return MIKV_ERR_CUDA;
   char* wsb = static_cast<char*>(workspace);
   a.status = reinterpret_cast<int*>(wsb);
-  a.stats = reinterpret_cast<float2*>(wsb + kWsHeader);
+  a.stats = reinterpret_cast<float*>(wsb + kWsHeader);
   a.scores = scores;
   a.heads_q = shape->heads_q;
   a.heads_kv = shape->heads_kv;
   a.T = T;
+  a.T_pad = prefill_padded(T);
   a.scale_log2 = sm_scale * 1.4426950408889634f;
   return cuda_status(launch_prefill(a, shape->batch, static_cast<cudaStream_t>(stream)));
 }

@@ -5,9 +5,9 @@
 //
 // Two passes over the causal score matrix S = sm_scale * Q K^T, each a tiled bf16 contraction on the
 // fifth-generation tensor cores (tcgen05.mma, M = N = 128, fp32 accumulators in tensor memory) fed by TMA:
-//   1. rows:    per query i, m_i = max_{t <= i} s_it and l_i = sum_{t <= i} exp(s_it - m_i)  (online, as in
-//               flash attention, without values);
-//   2. columns: per key t, sum over the G query heads and the queries i >= t of exp(s_it - m_i) / l_i.
+//   1. rows:    per query i, the log2 of its softmax normaliser, c_i = log2 sum_{t <= i} 2^(s_it log2 e)
+//               (accumulated online against a reference, as in flash attention, without values);
+//   2. columns: per key t, sum over the G query heads and the queries i >= t of 2^(s_it log2 e - c_i).
 // A CTA of four warps owns one 128-token tile of its fixed operand (queries in pass 1, keys in pass 2: the M
 // side, so that thread r of the CTA owns accumulator row r = TMEM lane r) and streams the 128-token tiles of
 // the other operand through a two-stage shared-memory ring (128B-swizzled TMA boxes). One thread issues the
@@ -170,7 +170,36 @@ __device__ __forceinline__ bool pf_tiles(const PrefillArgs& a, const CUtensorMap
   return !failed;
 }
 
+// Exact maximum of a row of the tile (four independent chains).
+__device__ __forceinline__ float pf_row_max(const float (&v)[kPfTile]) {
+  float mx[4] = {v[0], v[1], v[2], v[3]};
+#pragma unroll
+  for (int j = 4; j < kPfTile; ++j) mx[j & 3] = fmaxf(mx[j & 3], v[j]);
+  return fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+}
+
+// sum_j 2^(v_j * scale - ref): the exponent formed two columns at a time, four independent partial sums.
+__device__ __forceinline__ float pf_exp_sum(const float (&v)[kPfTile], float scale, float ref) {
+  const uint64_t s2 = f32x2(scale, scale), r2 = f32x2(-ref, -ref);
+  uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
+#pragma unroll
+  for (int j = 0; j < kPfTile / 2; ++j) {
+    float x0, x1;
+    f32x2_split(fma_f32x2(f32x2(v[2 * j], v[2 * j + 1]), s2, r2), x0, x1);
+    acc[j & 3] = add_f32x2(acc[j & 3], f32x2(fast_exp2(x0), fast_exp2(x1)));
+  }
+  float t[8];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) f32x2_split(acc[k], t[2 * k], t[2 * k + 1]);
+  return ((t[0] + t[1]) + (t[2] + t[3])) + ((t[4] + t[5]) + (t[6] + t[7]));
+}
+
 // ------------------------------------------------------------------------------- pass 1: row statistics
+//
+// Per query row the softmax normaliser is accumulated against a reference r (log2 units): the exact maximum
+// of the row's first tile, raised only when a later tile's sum would leave the fp32 range (a logit more than
+// 64 above r, rare), so most tiles need no maximum at all. The pair (r, sum_t 2^(s_t - r)) defines the same
+// normaliser as the true maximum; the kernel stores its log2, r + log2(sum).
 
 __global__ void __launch_bounds__(kPfThreads, 2) prefill_rows_kernel(const __grid_constant__ PrefillArgs a) {
   const int tid = threadIdx.x;
@@ -181,7 +210,7 @@ __global__ void __launch_bounds__(kPfThreads, 2) prefill_rows_kernel(const __gri
   const int b = bq / a.heads_q, h = (bq - b * a.heads_q) / G;
   const int krow0 = (b * a.heads_kv + h) * a.T;
   const int q = kPfTile * qt + tid;  // this thread's query
-  float m = -INFINITY, l = 0.f;
+  float r = -INFINITY, l = 0.f;
   const bool ok = pf_tiles(
       a, &a.map_q, bq * a.T + kPfTile * qt, &a.map_k, qt + 1, [&](int n) { return krow0 + kPfTile * n; },
       [&](int n, float (&v)[kPfTile]) {
@@ -191,24 +220,27 @@ __global__ void __launch_bounds__(kPfThreads, 2) prefill_rows_kernel(const __gri
           for (int j = 0; j < kPfTile; ++j)
             if (k0 + j > q || k0 + j >= a.T) v[j] = -INFINITY;
         }
-        float mx = v[0];
-#pragma unroll
-        for (int j = 1; j < kPfTile; ++j) mx = fmaxf(mx, v[j]);
-        const float mn = fmaxf(m, mx * a.scale_log2);
-        if (mn == -INFINITY) return;  // no key of this row yet
-        float sum = 0.f;
-#pragma unroll
-        for (int j = 0; j < kPfTile; ++j) sum += fast_exp2(fmaf(v[j], a.scale_log2, -mn));
-        l = l * fast_exp2(m - mn) + sum;
-        m = mn;
+        if (r == -INFINITY) {  // the row's first tile fixes the reference
+          const float mx = pf_row_max(v);
+          if (mx == -INFINITY) return;
+          r = mx * a.scale_log2;
+        }
+        float sum = pf_exp_sum(v, a.scale_log2, r);
+        if (!(sum <= 0x1p64f)) {  // a logit far above the reference: move the reference to this tile's maximum
+          const float rn = fmaxf(r, pf_row_max(v) * a.scale_log2);
+          sum = pf_exp_sum(v, a.scale_log2, rn);
+          l *= fast_exp2(r - rn);
+          r = rn;
+        }
+        l += sum;
       });
-  if (ok && q < a.T) a.stats[(size_t)bq * a.T + q] = make_float2(m, 1.f / l);
+  if (ok) a.stats[(size_t)bq * a.T_pad + q] = q < a.T ? r + log2f(l) : INFINITY;
 }
 
 // ------------------------------------------------------------------------------ pass 2: column sums
 
 __global__ void __launch_bounds__(kPfThreads, 2) prefill_cols_kernel(const __grid_constant__ PrefillArgs a) {
-  __shared__ float2 s_stat[2][kPfTile];  // (m, 1 / l) of the queries of the tile being summed and the next
+  __shared__ __align__(16) float s_nc[2][kPfTile];  // minus the log2 normalisers of the current and next tile
   const int tid = threadIdx.x;
   const int nq = (a.T + kPfTile - 1) / kPfTile;
   const int kt = blockIdx.x;  // the keys with the most queries first
@@ -217,36 +249,41 @@ __global__ void __launch_bounds__(kPfThreads, 2) prefill_cols_kernel(const __gri
   const int b = bh / a.heads_kv, h = bh - b * a.heads_kv;
   const int per_head = nq - kt;  // query tiles kt .. nq - 1 of each query head
   const int n_tiles = G * per_head;
-  // query tile n: head j = n / per_head, tile qt = kt + n % per_head; its first row in the q map and stats
-  auto qrow = [&](int n) {
-    const int j = n / per_head, qt = kt + (n - j * per_head);
-    return ((b * a.heads_q + h * G + j) * a.T) + kPfTile * qt;
-  };
+  // query tile n: head j = n / per_head, tile qt = kt + n % per_head
+  auto qhead = [&](int n) { return b * a.heads_q + h * G + n / per_head; };
   auto qfirst = [&](int n) { return kPfTile * (kt + (n % per_head)); };
-  // statistics of tile n's query tid; queries past the prefill weigh nothing (m = +inf, 1 / l = 0)
-  auto stat = [&](int n) {
-    const int qi = qfirst(n) + tid;
-    return qi < a.T ? a.stats[(size_t)qrow(n) + tid] : make_float2(INFINITY, 0.f);
-  };
-  s_stat[0][tid] = stat(0);  // visible after the first barrier inside pf_tiles
+  auto qrow = [&](int n) { return qhead(n) * a.T + qfirst(n); };  // first row in the q map
+  // tile n's query tid (padding queries carry +inf: they weigh nothing)
+  auto neg_norm = [&](int n) { return -a.stats[(size_t)qhead(n) * a.T_pad + qfirst(n) + tid]; };
+  s_nc[0][tid] = neg_norm(0);  // visible after the first barrier inside pf_tiles
   const int key = kPfTile * kt + tid;  // this thread's key
   float cs = 0.f;
   const bool ok = pf_tiles(
       a, &a.map_k, bh * a.T + kPfTile * kt, &a.map_q, n_tiles, qrow, [&](int n, float (&v)[kPfTile]) {
-        const float2 next = n + 1 < n_tiles ? stat(n + 1) : make_float2(INFINITY, 0.f);
-        const float2* st = s_stat[n & 1];
+        const float next = n + 1 < n_tiles ? neg_norm(n + 1) : 0.f;
         const int q0 = qfirst(n);
         if (q0 == kPfTile * kt) {  // the diagonal tile: queries before the key do not attend to it
 #pragma unroll
-          for (int j = 0; j < kPfTile; ++j) {
-            const float p = fast_exp2(fmaf(v[j], a.scale_log2, -st[j].x)) * st[j].y;
-            cs += q0 + j >= key ? p : 0.f;
-          }
-        } else {
-#pragma unroll
-          for (int j = 0; j < kPfTile; ++j) cs = fmaf(fast_exp2(fmaf(v[j], a.scale_log2, -st[j].x)), st[j].y, cs);
+          for (int j = 0; j < kPfTile; ++j)
+            if (q0 + j < key) v[j] = -INFINITY;
         }
-        s_stat[(n + 1) & 1][tid] = next;  // read after the barrier that ends this tile
+        const float4* nc = reinterpret_cast<const float4*>(s_nc[n & 1]);
+        const uint64_t s2 = f32x2(a.scale_log2, a.scale_log2);
+        uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
+#pragma unroll
+        for (int j = 0; j < kPfTile / 4; ++j) {
+          const float4 c = nc[j];
+          float x0, x1, x2, x3;
+          f32x2_split(fma_f32x2(f32x2(v[4 * j], v[4 * j + 1]), s2, f32x2(c.x, c.y)), x0, x1);
+          f32x2_split(fma_f32x2(f32x2(v[4 * j + 2], v[4 * j + 3]), s2, f32x2(c.z, c.w)), x2, x3);
+          acc[(2 * j) & 3] = add_f32x2(acc[(2 * j) & 3], f32x2(fast_exp2(x0), fast_exp2(x1)));
+          acc[(2 * j + 1) & 3] = add_f32x2(acc[(2 * j + 1) & 3], f32x2(fast_exp2(x2), fast_exp2(x3)));
+        }
+        float t[8];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) f32x2_split(acc[k], t[2 * k], t[2 * k + 1]);
+        cs += ((t[0] + t[1]) + (t[2] + t[3])) + ((t[4] + t[5]) + (t[6] + t[7]));
+        s_nc[(n + 1) & 1][tid] = next;  // read after the barrier that ends this tile
       });
   if (ok && key < a.T) a.scores[(size_t)bh * a.T + key] = cs;
 }

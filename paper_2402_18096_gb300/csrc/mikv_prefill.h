@@ -15,16 +15,19 @@ constexpr int kPfTile = 128;
 struct PrefillArgs {
   CUtensorMap map_q;  // q_pre rows [B * Hq * T][128] bf16, box 64 channels x 128 rows, 128B swizzle
   CUtensorMap map_k;  // k_pre rows [B * Hkv * T][128] bf16, same boxes
-  float2* stats;      // [B * Hq][T]: (row max of the logits in log2 units, 1 / row sum)
+  float* stats;       // [B * Hq][T_pad]: log2 of each query's softmax normaliser, log2 sum_t 2^(s_it log2 e);
+                      // +inf for the padding queries T .. T_pad - 1
   float* scores;      // [B * Hkv][T]
   int* status;        // workspace status word
-  int heads_q, heads_kv, T;
+  int heads_q, heads_kv, T, T_pad;  // T_pad = T rounded up to a whole tile
   float scale_log2;   // sm_scale * log2(e)
 };
 
-// Workspace of mikv_prefill_scores: the status header plus the per-query row statistics.
+// Workspace of mikv_prefill_scores: the status header plus the per-query normalisers (rows padded to whole
+// tiles).
+inline int prefill_padded(int T) { return (T + kPfTile - 1) / kPfTile * kPfTile; }
 inline size_t prefill_workspace_bytes(int batch, int heads_q, int T) {
-  const size_t stats = (size_t)batch * heads_q * T * sizeof(float2);
+  const size_t stats = (size_t)batch * heads_q * prefill_padded(T) * sizeof(float);
   return kWsHeader + (stats + 255) / 256 * 256;
 }
 
