@@ -360,6 +360,10 @@ mikv_status mikv_prefill_scores(const mikv_shape* shape, const void* q_pre, cons
   if (!make_map(&a.map_q, q_pre, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, kHeadDim, qrows, 2 * kHeadDim, 64, kPfTile,
                 CU_TENSOR_MAP_SWIZZLE_128B) ||
       !make_map(&a.map_k, k_pre, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, kHeadDim, krows, 2 * kHeadDim, 64, kPfTile,
+                CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !make_map(&a.map_q_str, q_pre, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, kHeadDim, qrows, 2 * kHeadDim, 64, kPfTile / 2,
+                CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !make_map(&a.map_k_str, k_pre, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, kHeadDim, krows, 2 * kHeadDim, 64, kPfTile / 2,
                 CU_TENSOR_MAP_SWIZZLE_128B))
     return MIKV_ERR_CUDA;
   char* wsb = static_cast<char*>(workspace);

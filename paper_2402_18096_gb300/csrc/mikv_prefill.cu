@@ -8,12 +8,13 @@
 //   1. rows:    per query i, the log2 of its softmax normaliser, c_i = log2 sum_{t <= i} 2^(s_it log2 e)
 //               (accumulated online against a reference, as in flash attention, without values);
 //   2. columns: per key t, sum over the G query heads and the queries i >= t of 2^(s_it log2 e - c_i).
-// A CTA of four warps owns one 128-token tile of its fixed operand (queries in pass 1, keys in pass 2: the M
-// side, so that thread r of the CTA owns accumulator row r = TMEM lane r) and streams the 128-token tiles of
-// the other operand through a two-stage shared-memory ring (128B-swizzled TMA boxes). One thread issues the
-// eight K = 16 MMAs of a tile into one of two TMEM accumulators while all four warps read the other one with
-// tcgen05.ld and do the softmax arithmetic (the exponentials, one per score, bound the kernel). Only the
-// causal triangle is visited; every wait is bounded in time.
+// A CTA owns one 128-token tile of its fixed operand (queries in pass 1, keys in pass 2: the M side, so that
+// epilogue thread r owns accumulator row r = TMEM lane r) and streams 64-token tiles of the other operand.
+// Its warps specialise: warp 4 issues the TMA copies (the fixed tile, then a four-stage ring of 128B-swizzled
+// streamed tiles), warp 5 issues the eight K = 16 MMAs of each tile (M = 128, N = 64) into one of four TMEM
+// accumulators, and warps 0-3 read each accumulator row with tcgen05.ld, release it, and do the softmax
+// arithmetic (an exponential per score). The roles hand tiles over through mbarriers only; every wait is
+// bounded in time and gives up when another role has failed. Only the causal triangle is visited.
 #include <math.h>
 
 #include "mikv_device.cuh"
@@ -23,19 +24,28 @@
 namespace mikv {
 namespace {
 
-constexpr int kPfThreads = 128;                       // thread r <-> accumulator row r (TMEM lane r)
-constexpr int kPfHalf = kPfTile * 128;                // bytes of one 64-channel box (128 rows x 128 B)
-constexpr int kPfTileBytes = 2 * kPfHalf;             // 32 KB: one 128 x 128 bf16 tile
-constexpr int kPfStages = 2;
-constexpr int kPfTmemCols = 2 * kPfTile;              // two fp32 accumulators of 128 columns
-constexpr int kPfSmem = (1 + kPfStages) * kPfTileBytes + 64 + 1024;  // tiles, barriers, alignment
-static_assert(kPfTile == 128, "one accumulator row per thread");
+constexpr int kPfN = 64;                                // tokens of a streamed tile (the MMA's N)
+constexpr int kPfThreads = 192;                         // warps 0-3 epilogue, 4 copies, 5 MMAs
+constexpr int kPfFixBytes = kPfTile * kHeadDim * 2;     // 32 KB: the fixed 128 x 128 bf16 tile
+constexpr int kPfFixHalf = kPfTile * 128;               // one 64-channel box of it
+constexpr int kPfStrBytes = kPfN * kHeadDim * 2;        // 16 KB: a streamed 64 x 128 tile
+constexpr int kPfStrHalf = kPfN * 128;
+constexpr int kPfStages = 4;                            // streamed tiles in flight
+constexpr int kPfAcc = 4;                               // TMEM accumulators of kPfN columns
+constexpr int kPfTmemCols = kPfAcc * kPfN;
+constexpr int kPfBars = 1 + 4 * kPfStages + 1;          // fixed, full/free/acc-full/acc-empty x 4, drain
+constexpr int kPfSmem = kPfFixBytes + kPfStages * kPfStrBytes + 8 * kPfBars + 1024;
+static_assert(kPfTile == 128 && kPfStages == kPfAcc, "one accumulator row per epilogue thread; shared indices");
 
 struct PfSmem {
-  uint32_t fixed, stage0, bar_fixed, bar_full0, bar_mma0;
-  __device__ uint32_t stage(int s) const { return stage0 + s * kPfTileBytes; }
-  __device__ uint32_t full(int s) const { return bar_full0 + 8 * s; }
-  __device__ uint32_t mma(int d) const { return bar_mma0 + 8 * d; }
+  uint32_t fixed, stage0, bars;
+  __device__ uint32_t stage(int s) const { return stage0 + s * kPfStrBytes; }
+  __device__ uint32_t bar_fixed() const { return bars; }
+  __device__ uint32_t full(int s) const { return bars + 8 * (1 + s); }                 // copy landed
+  __device__ uint32_t sfree(int s) const { return bars + 8 * (1 + kPfStages + s); }    // MMAs read it
+  __device__ uint32_t tfull(int d) const { return bars + 8 * (1 + 2 * kPfStages + d); }  // accumulator ready
+  __device__ uint32_t tempty(int d) const { return bars + 8 * (1 + 3 * kPfStages + d); } // accumulator read
+  __device__ uint32_t drain() const { return bars + 8 * (1 + 4 * kPfStages); }
 };
 
 __device__ __forceinline__ PfSmem pf_smem() {
@@ -43,126 +53,130 @@ __device__ __forceinline__ PfSmem pf_smem() {
   const uint32_t base = (smem_u32(smem_raw) + 1023u) & ~1023u;
   PfSmem r;
   r.fixed = base;
-  r.stage0 = base + kPfTileBytes;
-  r.bar_fixed = base + (1 + kPfStages) * kPfTileBytes;
-  r.bar_full0 = r.bar_fixed + 8;
-  r.bar_mma0 = r.bar_full0 + 8 * kPfStages;
+  r.stage0 = base + kPfFixBytes;
+  r.bars = r.stage0 + kPfStages * kPfStrBytes;
   return r;
 }
 
-// One 128 x 128 tile (rows row0 .. row0 + 127 of a map) into dst: two 64-channel boxes.
-__device__ __forceinline__ void pf_issue(const CUtensorMap* map, int row0, uint32_t dst, uint32_t bar) {
-  mbar_arrive_expect_tx(bar, kPfTileBytes);
-  tma_load_2d(dst, map, 0, row0, bar);
-  tma_load_2d(dst + kPfHalf, map, 64, row0, bar);
+// Bounded wait that also gives up as soon as another role of the CTA has failed.
+__device__ __forceinline__ bool pf_wait(uint32_t bar, uint32_t parity, volatile int* fail) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_timer_ns();
+  for (uint32_t i = 1;; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((i & 63u) == 0 && (*fail || global_timer_ns() - t0 > kWaitLimitNs)) {
+      *fail = 1;
+      return false;
+    }
+  }
 }
 
-// The eight K = 16 MMAs of one tile: D = A (fixed tile) x B (staged tile)^T over the 128 channels.
-__device__ __forceinline__ void pf_mma_tile(uint32_t d_tmem, uint32_t a_tile, uint32_t b_tile) {
-  constexpr uint32_t idesc = umma_idesc_bf16_f32(kPfTile, kPfTile);
+// The eight K = 16 MMAs of one tile: D (128 x 64) = fixed tile x streamed tile^T over the 128 channels.
+__device__ __forceinline__ void pf_mma_tile(uint32_t d_tmem, uint32_t fix, uint32_t str) {
+  constexpr uint32_t idesc = umma_idesc_bf16_f32(kPfTile, kPfN);
 #pragma unroll
   for (int ks = 0; ks < 8; ++ks) {
-    const uint32_t off = (ks >> 2) * kPfHalf + (ks & 3) * 32;  // channels 16 ks .. 16 ks + 15
-    umma_bf16(d_tmem, umma_desc_sw128(a_tile + off), umma_desc_sw128(b_tile + off), idesc, ks > 0 ? 1u : 0u);
+    const uint32_t k = (ks & 3) * 32;  // channels 16 ks .. 16 ks + 15 inside their 64-channel box
+    umma_bf16(d_tmem, umma_desc_sw128(fix + (ks >> 2) * kPfFixHalf + k),
+              umma_desc_sw128(str + (ks >> 2) * kPfStrHalf + k), idesc, ks > 0 ? 1u : 0u);
   }
 }
 
-// This thread's accumulator row (128 fp32 columns) of buffer d.
-__device__ __forceinline__ void pf_load_row(uint32_t tmem, int d, int warp, float (&v)[kPfTile]) {
-  const uint32_t t = tmem + (uint32_t)(d * kPfTile) + ((uint32_t)(32 * warp) << 16);
-  tmem_ld32(t, v);
-  tmem_ld32(t + 32, v + 32);
-  tmem_ld32(t + 64, v + 64);
-  tmem_ld32(t + 96, v + 96);
-  tmem_wait_ld(v);
-  reg_fence(v + 32);
-  reg_fence(v + 64);
-  reg_fence(v + 96);
-}
-
-// The tile loop shared by both passes. Tile n's operand rows come from b_row(n); its accumulator, once the
-// MMAs are done, goes to epi(n, v). Returns false when a wait timed out (after draining what is in flight).
-template <class BRow, class Epi>
-__device__ __forceinline__ bool pf_tiles(const PrefillArgs& a, const CUtensorMap* map_a, int a_row,
-                                         const CUtensorMap* map_b, int n_tiles, BRow b_row, Epi epi) {
+// The pipeline shared by both passes: warp 4 streams the n_tiles tiles (rows str_row(n) of map_str) behind
+// the fixed tile (rows fix_row .. + 127 of map_fix), warp 5 multiplies each into one of four TMEM
+// accumulators, and warps 0-3 hand accumulator rows (thread r: row r) to epi(n, v). Returns false when a
+// wait timed out (after draining what was in flight); every role leaves through the final barrier.
+template <class StrRow, class Epi>
+__device__ __forceinline__ bool pf_pipeline(const PrefillArgs& a, const CUtensorMap* map_fix, int fix_row,
+                                            const CUtensorMap* map_str, int n_tiles, StrRow str_row, Epi epi) {
   __shared__ uint32_t s_tmem;
   __shared__ int s_fail;
+  volatile int* fail = &s_fail;
   const PfSmem sm = pf_smem();
-  const int tid = threadIdx.x, warp = tid >> 5;
-  int issued_tma = 0, issued_mma = 0;  // tiles whose copies / MMAs were issued (thread 0)
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   if (tid == 0) {
     s_fail = 0;
-    mbar_init(sm.bar_fixed, 1);
-    for (int s = 0; s < kPfStages; ++s) mbar_init(sm.full(s), 1);
-    for (int d = 0; d < 2; ++d) mbar_init(sm.mma(d), 1);
+    mbar_init(sm.bar_fixed(), 1);
+    for (int s = 0; s < kPfStages; ++s) {
+      mbar_init(sm.full(s), 1);
+      mbar_init(sm.sfree(s), 1);
+      mbar_init(sm.tfull(s), 1);
+      mbar_init(sm.tempty(s), 4);  // one arrival per epilogue warp
+    }
+    mbar_init(sm.drain(), 1);
     fence_mbar_init();
-    pf_issue(map_a, a_row, sm.fixed, sm.bar_fixed);
-    for (; issued_tma < kPfStages && issued_tma < n_tiles; ++issued_tma)
-      pf_issue(map_b, b_row(issued_tma), sm.stage(issued_tma), sm.full(issued_tma));
   }
-  __syncwarp();
-  if (warp == 0) tmem_alloc(smem_u32(&s_tmem), kPfTmemCols);
+  if (warp == 5) tmem_alloc(smem_u32(&s_tmem), kPfTmemCols);
   tcgen05_before_sync();
   __syncthreads();
   tcgen05_after_sync();
   const uint32_t tmem = s_tmem;
-  bool fixed_ok = true;
-  if (tid == 0) {
-    fixed_ok = mbar_wait(sm.bar_fixed, 0);
-    if (fixed_ok && mbar_wait(sm.full(0), 0)) {
-      pf_mma_tile(tmem, sm.fixed, sm.stage(0));
-      umma_commit(sm.mma(0));
-      issued_mma = 1;
-    } else {
-      s_fail = 1;
-    }
-  }
-  __syncthreads();
-  int n = 0;
-  for (; n < n_tiles && !s_fail; ++n) {
-    const int d = n & 1;
-    // the next tile's MMAs into the other accumulator (its last reader finished before the barrier below)
-    if (tid == 0 && n + 1 < n_tiles) {
-      const int s1 = (n + 1) % kPfStages;
-      if (mbar_wait(sm.full(s1), ((n + 1) / kPfStages) & 1)) {
-        tcgen05_after_sync();
-        pf_mma_tile(tmem + (uint32_t)((d ^ 1) * kPfTile), sm.fixed, sm.stage(s1));
-        umma_commit(sm.mma(d ^ 1));
-        issued_mma = n + 2;
-      } else {
-        s_fail = 1;
+
+  if (warp == 4) {
+    if (lane == 0) {  // copies: the fixed tile, then the streamed tiles as stages free up
+      int last[kPfStages];
+      for (int s = 0; s < kPfStages; ++s) last[s] = -1;
+      mbar_arrive_expect_tx(sm.bar_fixed(), kPfFixBytes);
+      tma_load_2d(sm.fixed, map_fix, 0, fix_row, sm.bar_fixed());
+      tma_load_2d(sm.fixed + kPfFixHalf, map_fix, 64, fix_row, sm.bar_fixed());
+      for (int t = 0; t < n_tiles; ++t) {
+        const int s = t % kPfStages;
+        if (t >= kPfStages && !pf_wait(sm.sfree(s), ((t / kPfStages) & 1) ^ 1, fail)) break;
+        const int row = str_row(t);
+        mbar_arrive_expect_tx(sm.full(s), kPfStrBytes);
+        tma_load_2d(sm.stage(s), map_str, 0, row, sm.full(s));
+        tma_load_2d(sm.stage(s) + kPfStrHalf, map_str, 64, row, sm.full(s));
+        last[s] = t;
+      }
+      if (*fail) {  // no copy may outlive the CTA
+        if (!mbar_wait(sm.bar_fixed(), 0)) record_error(a.status, kErrDrainTimeout);
+        for (int s = 0; s < kPfStages; ++s)
+          if (last[s] >= 0 && !mbar_wait(sm.full(s), (last[s] / kPfStages) & 1))
+            record_error(a.status, kErrDrainTimeout);
       }
     }
-    // warp-uniform, so that the warp-wide TMEM loads below run converged
-    if (!__all_sync(0xffffffffu, mbar_wait(sm.mma(d), (n >> 1) & 1))) {
-      s_fail = 1;
-    } else {
+  } else if (warp == 5) {
+    if (lane == 0) {  // MMAs: tile n into accumulator n % 4 once its copy landed and its last reader is done
+      if (pf_wait(sm.bar_fixed(), 0, fail)) {
+        for (int n = 0; n < n_tiles; ++n) {
+          const int s = n % kPfStages;
+          const uint32_t ph = (n / kPfStages) & 1;
+          if (!pf_wait(sm.full(s), ph, fail) || !pf_wait(sm.tempty(s), ph ^ 1, fail)) break;
+          tcgen05_after_sync();
+          pf_mma_tile(tmem + (uint32_t)(s * kPfN), sm.fixed, sm.stage(s));
+          umma_commit(sm.sfree(s));
+          umma_commit(sm.tfull(s));
+        }
+      }
+      umma_commit(sm.drain());  // every MMA issued has completed once this arrives
+      if (!mbar_wait(sm.drain(), 0)) record_error(a.status, kErrDrainTimeout);
+    }
+  } else {  // epilogue warps 0-3: accumulator lanes 32 w .. 32 w + 31
+    for (int n = 0; n < n_tiles; ++n) {
+      const int d = n % kPfAcc;
+      const bool ok = pf_wait(sm.tfull(d), (n / kPfAcc) & 1, fail);
+      if (!__all_sync(0xffffffffu, ok)) {
+        *fail = 1;
+        break;
+      }
       tcgen05_after_sync();
-      // tile n's stage is free again (its MMAs have completed): tile n + kPfStages goes there
-      if (tid == 0 && issued_tma < n_tiles && issued_tma == n + kPfStages) {
-        pf_issue(map_b, b_row(issued_tma), sm.stage(n % kPfStages), sm.full(n % kPfStages));
-        ++issued_tma;
-      }
-      float v[kPfTile];
-      pf_load_row(tmem, d, warp, v);
+      float v[kPfN];
+      const uint32_t t = tmem + (uint32_t)(d * kPfN) + ((uint32_t)(32 * warp) << 16);
+      tmem_ld32(t, v);
+      tmem_ld32(t + 32, v + 32);
+      tmem_wait_ld(v);
+      reg_fence(v + 32);
+      tcgen05_before_sync();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(sm.tempty(d));
       epi(n, v);
     }
-    tcgen05_before_sync();
-    __syncthreads();
-  }
-  const bool failed = s_fail != 0;
-  if (failed && tid == 0) {
-    record_error(a.status, kErrFullTimeout);
-    // no copy and no MMA may outlive the CTA: wait (bounded) for those still in flight
-    if (!fixed_ok && !mbar_wait(sm.bar_fixed, 0)) record_error(a.status, kErrDrainTimeout);
-    for (int t = issued_mma; t < issued_tma; ++t)
-      if (!mbar_wait(sm.full(t % kPfStages), (t / kPfStages) & 1)) record_error(a.status, kErrDrainTimeout);
-    for (int t = n; t < issued_mma; ++t)
-      if (!mbar_wait(sm.mma(t & 1), (t >> 1) & 1)) record_error(a.status, kErrDrainTimeout);
   }
   tcgen05_before_sync();
   __syncthreads();
-  if (warp == 0) {
+  const bool failed = s_fail != 0;
+  if (failed && tid == 0) record_error(a.status, kErrFullTimeout);
+  if (warp == 5) {
     __syncwarp();
     tcgen05_after_sync();
     tmem_dealloc(tmem, kPfTmemCols);
@@ -171,19 +185,19 @@ __device__ __forceinline__ bool pf_tiles(const PrefillArgs& a, const CUtensorMap
 }
 
 // Exact maximum of a row of the tile (four independent chains).
-__device__ __forceinline__ float pf_row_max(const float (&v)[kPfTile]) {
+__device__ __forceinline__ float pf_row_max(const float (&v)[kPfN]) {
   float mx[4] = {v[0], v[1], v[2], v[3]};
 #pragma unroll
-  for (int j = 4; j < kPfTile; ++j) mx[j & 3] = fmaxf(mx[j & 3], v[j]);
+  for (int j = 4; j < kPfN; ++j) mx[j & 3] = fmaxf(mx[j & 3], v[j]);
   return fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
 }
 
 // sum_j 2^(v_j * scale - ref): the exponent formed two columns at a time, four independent partial sums.
-__device__ __forceinline__ float pf_exp_sum(const float (&v)[kPfTile], float scale, float ref) {
+__device__ __forceinline__ float pf_exp_sum(const float (&v)[kPfN], float scale, float ref) {
   const uint64_t s2 = f32x2(scale, scale), r2 = f32x2(-ref, -ref);
   uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
-  for (int j = 0; j < kPfTile / 2; ++j) {
+  for (int j = 0; j < kPfN / 2; ++j) {
     float x0, x1;
     f32x2_split(fma_f32x2(f32x2(v[2 * j], v[2 * j + 1]), s2, r2), x0, x1);
     acc[j & 3] = add_f32x2(acc[j & 3], f32x2(fast_exp2(x0), fast_exp2(x1)));
@@ -209,15 +223,17 @@ __global__ void __launch_bounds__(kPfThreads, 2) prefill_rows_kernel(const __gri
   const int G = a.heads_q / a.heads_kv;
   const int b = bq / a.heads_q, h = (bq - b * a.heads_q) / G;
   const int krow0 = (b * a.heads_kv + h) * a.T;
-  const int q = kPfTile * qt + tid;  // this thread's query
+  const int q = kPfTile * qt + tid;  // an epilogue thread's query
+  const int kend = min(kPfTile * (qt + 1), a.T);  // keys 0 .. kend - 1 can reach this tile's queries
   float r = -INFINITY, l = 0.f;
-  const bool ok = pf_tiles(
-      a, &a.map_q, bq * a.T + kPfTile * qt, &a.map_k, qt + 1, [&](int n) { return krow0 + kPfTile * n; },
-      [&](int n, float (&v)[kPfTile]) {
-        const int k0 = kPfTile * n;
-        if (n == qt || k0 + kPfTile > a.T) {  // keys after the query, or past the prefill, do not count
+  const bool ok = pf_pipeline(
+      a, &a.map_q, bq * a.T + kPfTile * qt, &a.map_k_str, (kend + kPfN - 1) / kPfN,
+      [&](int n) { return krow0 + kPfN * n; },
+      [&](int n, float (&v)[kPfN]) {
+        const int k0 = kPfN * n;
+        if (k0 + kPfN > kPfTile * qt) {  // keys after the query, or past the prefill, do not count
 #pragma unroll
-          for (int j = 0; j < kPfTile; ++j)
+          for (int j = 0; j < kPfN; ++j)
             if (k0 + j > q || k0 + j >= a.T) v[j] = -INFINITY;
         }
         if (r == -INFINITY) {  // the row's first tile fixes the reference
@@ -234,48 +250,43 @@ __global__ void __launch_bounds__(kPfThreads, 2) prefill_rows_kernel(const __gri
         }
         l += sum;
       });
-  if (ok) a.stats[(size_t)bq * a.T_pad + q] = q < a.T ? r + log2f(l) : INFINITY;
+  if (ok && tid < kPfTile) a.stats[(size_t)bq * a.T_pad + q] = q < a.T ? r + log2f(l) : INFINITY;
 }
 
 // ------------------------------------------------------------------------------ pass 2: column sums
 
 __global__ void __launch_bounds__(kPfThreads, 2) prefill_cols_kernel(const __grid_constant__ PrefillArgs a) {
-  __shared__ __align__(16) float s_nc[2][kPfTile];  // minus the log2 normalisers of the current and next tile
   const int tid = threadIdx.x;
-  const int nq = (a.T + kPfTile - 1) / kPfTile;
   const int kt = blockIdx.x;  // the keys with the most queries first
   const int bh = blockIdx.y;  // b * Hkv + KV head
   const int G = a.heads_q / a.heads_kv;
   const int b = bh / a.heads_kv, h = bh - b * a.heads_kv;
-  const int per_head = nq - kt;  // query tiles kt .. nq - 1 of each query head
-  const int n_tiles = G * per_head;
-  // query tile n: head j = n / per_head, tile qt = kt + n % per_head
+  const int per_head = (a.T - kPfTile * kt + kPfN - 1) / kPfN;  // query tiles of each head reaching the keys
+  // query tile n: head j = n / per_head, first query kPfTile kt + kPfN (n % per_head)
   auto qhead = [&](int n) { return b * a.heads_q + h * G + n / per_head; };
-  auto qfirst = [&](int n) { return kPfTile * (kt + (n % per_head)); };
-  auto qrow = [&](int n) { return qhead(n) * a.T + qfirst(n); };  // first row in the q map
-  // tile n's query tid (padding queries carry +inf: they weigh nothing)
-  auto neg_norm = [&](int n) { return -a.stats[(size_t)qhead(n) * a.T_pad + qfirst(n) + tid]; };
-  s_nc[0][tid] = neg_norm(0);  // visible after the first barrier inside pf_tiles
-  const int key = kPfTile * kt + tid;  // this thread's key
+  auto qfirst = [&](int n) { return kPfTile * kt + kPfN * (n % per_head); };
+  const int key = kPfTile * kt + tid;  // an epilogue thread's key
   float cs = 0.f;
-  const bool ok = pf_tiles(
-      a, &a.map_k, bh * a.T + kPfTile * kt, &a.map_q, n_tiles, qrow, [&](int n, float (&v)[kPfTile]) {
-        const float next = n + 1 < n_tiles ? neg_norm(n + 1) : 0.f;
+  const bool ok = pf_pipeline(
+      a, &a.map_k, bh * a.T + kPfTile * kt, &a.map_q_str, G * per_head,
+      [&](int n) { return qhead(n) * a.T + qfirst(n); },
+      [&](int n, float (&v)[kPfN]) {
         const int q0 = qfirst(n);
-        if (q0 == kPfTile * kt) {  // the diagonal tile: queries before the key do not attend to it
+        // minus the log2 normalisers of the tile's queries (+inf for padding queries: they weigh nothing)
+        const float4* nc = reinterpret_cast<const float4*>(a.stats + (size_t)qhead(n) * a.T_pad + q0);
+        if (q0 < kPfTile * (kt + 1)) {  // the diagonal: queries before the key do not attend to it
 #pragma unroll
-          for (int j = 0; j < kPfTile; ++j)
+          for (int j = 0; j < kPfN; ++j)
             if (q0 + j < key) v[j] = -INFINITY;
         }
-        const float4* nc = reinterpret_cast<const float4*>(s_nc[n & 1]);
         const uint64_t s2 = f32x2(a.scale_log2, a.scale_log2);
         uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
-        for (int j = 0; j < kPfTile / 4; ++j) {
-          const float4 c = nc[j];
+        for (int j = 0; j < kPfN / 4; ++j) {
+          const float4 c = __ldg(nc + j);
           float x0, x1, x2, x3;
-          f32x2_split(fma_f32x2(f32x2(v[4 * j], v[4 * j + 1]), s2, f32x2(c.x, c.y)), x0, x1);
-          f32x2_split(fma_f32x2(f32x2(v[4 * j + 2], v[4 * j + 3]), s2, f32x2(c.z, c.w)), x2, x3);
+          f32x2_split(fma_f32x2(f32x2(v[4 * j], v[4 * j + 1]), s2, f32x2(-c.x, -c.y)), x0, x1);
+          f32x2_split(fma_f32x2(f32x2(v[4 * j + 2], v[4 * j + 3]), s2, f32x2(-c.z, -c.w)), x2, x3);
           acc[(2 * j) & 3] = add_f32x2(acc[(2 * j) & 3], f32x2(fast_exp2(x0), fast_exp2(x1)));
           acc[(2 * j + 1) & 3] = add_f32x2(acc[(2 * j + 1) & 3], f32x2(fast_exp2(x2), fast_exp2(x3)));
         }
@@ -283,9 +294,8 @@ __global__ void __launch_bounds__(kPfThreads, 2) prefill_cols_kernel(const __gri
 #pragma unroll
         for (int k = 0; k < 4; ++k) f32x2_split(acc[k], t[2 * k], t[2 * k + 1]);
         cs += ((t[0] + t[1]) + (t[2] + t[3])) + ((t[4] + t[5]) + (t[6] + t[7]));
-        s_nc[(n + 1) & 1][tid] = next;  // read after the barrier that ends this tile
       });
-  if (ok && key < a.T) a.scores[(size_t)bh * a.T + key] = cs;
+  if (ok && tid < kPfTile && key < a.T) a.scores[(size_t)bh * a.T + key] = cs;
 }
 
 }  // namespace

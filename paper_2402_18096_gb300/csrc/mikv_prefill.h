@@ -13,8 +13,10 @@ namespace mikv {
 constexpr int kPfTile = 128;
 
 struct PrefillArgs {
-  CUtensorMap map_q;  // q_pre rows [B * Hq * T][128] bf16, box 64 channels x 128 rows, 128B swizzle
-  CUtensorMap map_k;  // k_pre rows [B * Hkv * T][128] bf16, same boxes
+  CUtensorMap map_q;      // q_pre rows [B * Hq * T][128] bf16, box 64 channels x 128 rows, 128B swizzle
+  CUtensorMap map_k;      // k_pre rows [B * Hkv * T][128] bf16, same boxes
+  CUtensorMap map_q_str;  // the same arrays in boxes of 64 channels x 64 rows (streamed tiles)
+  CUtensorMap map_k_str;
   float* stats;       // [B * Hq][T_pad]: log2 of each query's softmax normaliser, log2 sum_t 2^(s_it log2 e);
                       // +inf for the padding queries T .. T_pad - 1
   float* scores;      // [B * Hkv][T]
