@@ -737,6 +737,46 @@ __device__ __forceinline__ void issue_unit(const AttnArgs& a, const Cursor& c, u
   }
 }
 
+// The copies of issue_unit as L2 prefetches (issued before the kernel may read the cache).
+template <int BITS, int GROUP, int HB, bool KCH>
+__device__ __forceinline__ void prefetch_unit(const AttnArgs& a, const Cursor& c) {
+  constexpr LoUnit U = KCH ? lo_unit_layout_kch(BITS, GROUP) : lo_unit_layout(BITS, GROUP);
+  const UnitKind k = cursor_kind(c, a.hi_units, a.n_u);
+  if constexpr (HB != 16) {
+    if (k.hi) {
+      constexpr LoUnit H = lo_unit_layout(HB, kHiGroup);
+      const long long row = (long long)c.bh * a.hi_stride + 16 * H.blocks * k.index;  // first slot
+      const int crow = (int)(row * H.pitch / H.map_w), prow = (int)(row * H.param_row / H.param_w);
+      tma_prefetch_2d(&a.map_k_hi, 0, crow);
+      tma_prefetch_2d(&a.map_v_hi, 0, crow);
+      tma_prefetch_2d(&a.map_k_hp, 0, prow);
+      tma_prefetch_2d(&a.map_v_hp, 0, prow);
+      return;
+    }
+  }
+  if (k.hi) {
+    const int row = c.bh * a.hi_stride + 16 * k.index;
+    tma_prefetch_2d(&a.map_k_hi, 0, row);
+    tma_prefetch_2d(&a.map_k_hi, 64, row);
+    tma_prefetch_2d(&a.map_v_hi, 0, row);
+    tma_prefetch_2d(&a.map_v_hi, 64, row);
+  } else {
+    // one box per array covers the whole unit (U.blocks blocks of 16 rows); rows past this head's
+    // retained length are masked by the consumer, rows past the array are zero-filled by TMA
+    const long long row = (long long)c.bh * a.lo_cap + 16 * U.blocks * k.index;  // first token row
+    const int crow = (int)(row * U.pitch / U.map_w), prow = (int)(row * U.param_row / U.param_w);
+    tma_prefetch_2d(&a.map_k_lo, 0, crow);
+    tma_prefetch_2d(&a.map_v_lo, 0, crow);
+    if constexpr (KCH) {  // the group's key (alpha, beta) pairs: four 128-byte rows per group of 64 tokens
+      const long long grp = (long long)c.bh * (a.lo_cap / kKchGroup) + (16 * U.blocks * k.index) / kKchGroup;
+      tma_prefetch_2d(&a.map_k_par, 0, (int)(4 * grp));
+    } else {
+      tma_prefetch_2d(&a.map_k_par, 0, prow);
+    }
+    tma_prefetch_2d(&a.map_v_par, 0, prow);
+  }
+}
+
 __device__ __forceinline__ void fence_proxy_async() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
@@ -776,6 +816,11 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
       prefetch_tensormap(&a.map_v_par);
     }
   }
+  if (lane == 0)  // warm L2 with this warp's first units while the previous kernel drains (reads only)
+    for (int k = 0; k < kNS && u0 + k < u1; ++k) {
+      Cursor cp = cursor_at(u0 + k, hu, n_u);
+      prefetch_unit<BITS, GROUP, HB, KCH>(a, cp);
+    }
   grid_dependency_wait();  // the cache and the query come from the kernels before this one
   allow_dependent_launch();
   if (lane == 0) {

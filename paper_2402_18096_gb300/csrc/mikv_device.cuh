@@ -89,6 +89,13 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       : "memory");
 }
 
+// Prefetch of the same tile into L2 only (no shared memory, no completion to wait for).
+__device__ __forceinline__ void tma_prefetch_2d(const CUtensorMap* map, int x, int y) {
+  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y)
+               : "memory");
+}
+
 // L2 policy for data a kernel streams through once: its lines are evicted before others, so what the
 // kernel writes for the next one (logits, split partials) stays in L2 across the stream.
 __device__ __forceinline__ uint64_t l2_evict_first() {
