@@ -25,7 +25,10 @@ namespace mikv {
 namespace {
 
 constexpr int kPfN = 64;                                // tokens of a streamed tile (the MMA's N)
-constexpr int kPfThreads = 192;                         // warps 0-3 epilogue, 4 copies, 5 MMAs
+constexpr int kPfEpiWarps = 8;                          // two per accumulator lane quarter: one per column half
+constexpr int kPfCols = kPfN / 2;                       // accumulator columns of one epilogue thread
+constexpr int kPfThreads = 32 * (kPfEpiWarps + 2);      // warps 0-7 epilogue, 8 copies, 9 MMAs
+constexpr int kPfCopyWarp = kPfEpiWarps, kPfMmaWarp = kPfEpiWarps + 1;
 constexpr int kPfFixBytes = kPfTile * kHeadDim * 2;     // 32 KB: the fixed 128 x 128 bf16 tile
 constexpr int kPfFixHalf = kPfTile * 128;               // one 64-channel box of it
 constexpr int kPfStrBytes = kPfN * kHeadDim * 2;        // 16 KB: a streamed 64 x 128 tile
@@ -82,10 +85,11 @@ __device__ __forceinline__ void pf_mma_tile(uint32_t d_tmem, uint32_t fix, uint3
   }
 }
 
-// The pipeline shared by both passes: warp 4 streams the n_tiles tiles (rows str_row(n) of map_str) behind
-// the fixed tile (rows fix_row .. + 127 of map_fix), warp 5 multiplies each into one of four TMEM
-// accumulators, and warps 0-3 hand accumulator rows (thread r: row r) to epi(n, v). Returns false when a
-// wait timed out (after draining what was in flight); every role leaves through the final barrier.
+// The pipeline shared by both passes: warp 8 streams the n_tiles tiles (rows str_row(n) of map_str) behind
+// the fixed tile (rows fix_row .. + 127 of map_fix), warp 9 multiplies each into one of four TMEM
+// accumulators, and warps 0-7 hand accumulator row halves to epi(n, col0, v): warp w gets row 32 (w % 4) +
+// lane, columns col0 = 32 (w / 4) .. col0 + 31. Returns false when a wait timed out (after draining what was
+// in flight); every role leaves through the final barrier.
 template <class StrRow, class Epi>
 __device__ __forceinline__ bool pf_pipeline(const PrefillArgs& a, const CUtensorMap* map_fix, int fix_row,
                                             const CUtensorMap* map_str, int n_tiles, StrRow str_row, Epi epi) {
@@ -101,18 +105,18 @@ __device__ __forceinline__ bool pf_pipeline(const PrefillArgs& a, const CUtensor
       mbar_init(sm.full(s), 1);
       mbar_init(sm.sfree(s), 1);
       mbar_init(sm.tfull(s), 1);
-      mbar_init(sm.tempty(s), 4);  // one arrival per epilogue warp
+      mbar_init(sm.tempty(s), kPfEpiWarps);  // one arrival per epilogue warp
     }
     mbar_init(sm.drain(), 1);
     fence_mbar_init();
   }
-  if (warp == 5) tmem_alloc(smem_u32(&s_tmem), kPfTmemCols);
+  if (warp == kPfMmaWarp) tmem_alloc(smem_u32(&s_tmem), kPfTmemCols);
   tcgen05_before_sync();
   __syncthreads();
   tcgen05_after_sync();
   const uint32_t tmem = s_tmem;
 
-  if (warp == 4) {
+  if (warp == kPfCopyWarp) {
     if (lane == 0) {  // copies: the fixed tile, then the streamed tiles as stages free up
       int last[kPfStages];
       for (int s = 0; s < kPfStages; ++s) last[s] = -1;
@@ -135,7 +139,7 @@ __device__ __forceinline__ bool pf_pipeline(const PrefillArgs& a, const CUtensor
             record_error(a.status, kErrDrainTimeout);
       }
     }
-  } else if (warp == 5) {
+  } else if (warp == kPfMmaWarp) {
     if (lane == 0) {  // MMAs: tile n into accumulator n % 4 once its copy landed and its last reader is done
       if (pf_wait(sm.bar_fixed(), 0, fail)) {
         for (int n = 0; n < n_tiles; ++n) {
@@ -151,7 +155,8 @@ __device__ __forceinline__ bool pf_pipeline(const PrefillArgs& a, const CUtensor
       umma_commit(sm.drain());  // every MMA issued has completed once this arrives
       if (!mbar_wait(sm.drain(), 0)) record_error(a.status, kErrDrainTimeout);
     }
-  } else {  // epilogue warps 0-3: accumulator lanes 32 w .. 32 w + 31
+  } else {  // epilogue warps: accumulator lanes 32 (w % 4) .., columns kPfCols (w / 4) ..
+    const int half = warp / 4;
     for (int n = 0; n < n_tiles; ++n) {
       const int d = n % kPfAcc;
       const bool ok = pf_wait(sm.tfull(d), (n / kPfAcc) & 1, fail);
@@ -160,23 +165,20 @@ __device__ __forceinline__ bool pf_pipeline(const PrefillArgs& a, const CUtensor
         break;
       }
       tcgen05_after_sync();
-      float v[kPfN];
-      const uint32_t t = tmem + (uint32_t)(d * kPfN) + ((uint32_t)(32 * warp) << 16);
-      tmem_ld32(t, v);
-      tmem_ld32(t + 32, v + 32);
+      float v[kPfCols];
+      tmem_ld32(tmem + (uint32_t)(d * kPfN + kPfCols * half) + ((uint32_t)(32 * (warp & 3)) << 16), v);
       tmem_wait_ld(v);
-      reg_fence(v + 32);
       tcgen05_before_sync();
       __syncwarp();
       if (lane == 0) mbar_arrive(sm.tempty(d));
-      epi(n, v);
+      epi(n, kPfCols * half, v);
     }
   }
   tcgen05_before_sync();
   __syncthreads();
   const bool failed = s_fail != 0;
   if (failed && tid == 0) record_error(a.status, kErrFullTimeout);
-  if (warp == 5) {
+  if (warp == kPfMmaWarp) {
     __syncwarp();
     tcgen05_after_sync();
     tmem_dealloc(tmem, kPfTmemCols);
@@ -185,19 +187,19 @@ __device__ __forceinline__ bool pf_pipeline(const PrefillArgs& a, const CUtensor
 }
 
 // Exact maximum of a row of the tile (four independent chains).
-__device__ __forceinline__ float pf_row_max(const float (&v)[kPfN]) {
+__device__ __forceinline__ float pf_row_max(const float (&v)[kPfCols]) {
   float mx[4] = {v[0], v[1], v[2], v[3]};
 #pragma unroll
-  for (int j = 4; j < kPfN; ++j) mx[j & 3] = fmaxf(mx[j & 3], v[j]);
+  for (int j = 4; j < kPfCols; ++j) mx[j & 3] = fmaxf(mx[j & 3], v[j]);
   return fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
 }
 
 // sum_j 2^(v_j * scale - ref): the exponent formed two columns at a time, four independent partial sums.
-__device__ __forceinline__ float pf_exp_sum(const float (&v)[kPfN], float scale, float ref) {
+__device__ __forceinline__ float pf_exp_sum(const float (&v)[kPfCols], float scale, float ref) {
   const uint64_t s2 = f32x2(scale, scale), r2 = f32x2(-ref, -ref);
   uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
-  for (int j = 0; j < kPfN / 2; ++j) {
+  for (int j = 0; j < kPfCols / 2; ++j) {
     float x0, x1;
     f32x2_split(fma_f32x2(f32x2(v[2 * j], v[2 * j + 1]), s2, r2), x0, x1);
     acc[j & 3] = add_f32x2(acc[j & 3], f32x2(fast_exp2(x0), fast_exp2(x1)));
@@ -223,17 +225,19 @@ __global__ void __launch_bounds__(kPfThreads, 2) prefill_rows_kernel(const __gri
   const int G = a.heads_q / a.heads_kv;
   const int b = bq / a.heads_q, h = (bq - b * a.heads_q) / G;
   const int krow0 = (b * a.heads_kv + h) * a.T;
-  const int q = kPfTile * qt + tid;  // an epilogue thread's query
+  __shared__ float s_r[kPfTile], s_l[kPfTile];  // the second column half's partial of each row
+  const int row = tid & (kPfTile - 1);
+  const int q = kPfTile * qt + row;  // an epilogue thread's query
   const int kend = min(kPfTile * (qt + 1), a.T);  // keys 0 .. kend - 1 can reach this tile's queries
-  float r = -INFINITY, l = 0.f;
+  float r = -INFINITY, l = 0.f;  // over this thread's column half of every tile
   const bool ok = pf_pipeline(
       a, &a.map_q, bq * a.T + kPfTile * qt, &a.map_k_str, (kend + kPfN - 1) / kPfN,
       [&](int n) { return krow0 + kPfN * n; },
-      [&](int n, float (&v)[kPfN]) {
-        const int k0 = kPfN * n;
-        if (k0 + kPfN > kPfTile * qt) {  // keys after the query, or past the prefill, do not count
+      [&](int n, int col0, float (&v)[kPfCols]) {
+        const int k0 = kPfN * n + col0;
+        if (k0 + kPfCols > kPfTile * qt) {  // keys after the query, or past the prefill, do not count
 #pragma unroll
-          for (int j = 0; j < kPfN; ++j)
+          for (int j = 0; j < kPfCols; ++j)
             if (k0 + j > q || k0 + j >= a.T) v[j] = -INFINITY;
         }
         if (r == -INFINITY) {  // the row's first tile fixes the reference
@@ -250,7 +254,16 @@ __global__ void __launch_bounds__(kPfThreads, 2) prefill_rows_kernel(const __gri
         }
         l += sum;
       });
-  if (ok && tid < kPfTile) a.stats[(size_t)bq * a.T_pad + q] = q < a.T ? r + log2f(l) : INFINITY;
+  if (tid >= kPfTile && tid < 2 * kPfTile) {
+    s_r[row] = r;
+    s_l[row] = l;
+  }
+  __syncthreads();
+  if (ok && tid < kPfTile) {  // both halves against the larger reference
+    const float r2 = s_r[row], rm = fmaxf(r, r2);
+    const float lt = (r == -INFINITY ? 0.f : l * fast_exp2(r - rm)) + (r2 == -INFINITY ? 0.f : s_l[row] * fast_exp2(r2 - rm));
+    a.stats[(size_t)bq * a.T_pad + q] = q < a.T ? rm + log2f(lt) : INFINITY;
+  }
 }
 
 // ------------------------------------------------------------------------------ pass 2: column sums
@@ -265,24 +278,26 @@ __global__ void __launch_bounds__(kPfThreads, 2) prefill_cols_kernel(const __gri
   // query tile n: head j = n / per_head, first query kPfTile kt + kPfN (n % per_head)
   auto qhead = [&](int n) { return b * a.heads_q + h * G + n / per_head; };
   auto qfirst = [&](int n) { return kPfTile * kt + kPfN * (n % per_head); };
-  const int key = kPfTile * kt + tid;  // an epilogue thread's key
+  __shared__ float s_cs[kPfTile];  // the second column half's sum of each row
+  const int row = tid & (kPfTile - 1);
+  const int key = kPfTile * kt + row;  // an epilogue thread's key
   float cs = 0.f;
   const bool ok = pf_pipeline(
       a, &a.map_k, bh * a.T + kPfTile * kt, &a.map_q_str, G * per_head,
       [&](int n) { return qhead(n) * a.T + qfirst(n); },
-      [&](int n, float (&v)[kPfN]) {
-        const int q0 = qfirst(n);
-        // minus the log2 normalisers of the tile's queries (+inf for padding queries: they weigh nothing)
+      [&](int n, int col0, float (&v)[kPfCols]) {
+        const int q0 = qfirst(n) + col0;
+        // minus the log2 normalisers of these queries (+inf for padding queries: they weigh nothing)
         const float4* nc = reinterpret_cast<const float4*>(a.stats + (size_t)qhead(n) * a.T_pad + q0);
         if (q0 < kPfTile * (kt + 1)) {  // the diagonal: queries before the key do not attend to it
 #pragma unroll
-          for (int j = 0; j < kPfN; ++j)
+          for (int j = 0; j < kPfCols; ++j)
             if (q0 + j < key) v[j] = -INFINITY;
         }
         const uint64_t s2 = f32x2(a.scale_log2, a.scale_log2);
         uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
-        for (int j = 0; j < kPfN / 4; ++j) {
+        for (int j = 0; j < kPfCols / 4; ++j) {
           const float4 c = __ldg(nc + j);
           float x0, x1, x2, x3;
           f32x2_split(fma_f32x2(f32x2(v[4 * j], v[4 * j + 1]), s2, f32x2(-c.x, -c.y)), x0, x1);
@@ -295,7 +310,9 @@ __global__ void __launch_bounds__(kPfThreads, 2) prefill_cols_kernel(const __gri
         for (int k = 0; k < 4; ++k) f32x2_split(acc[k], t[2 * k], t[2 * k + 1]);
         cs += ((t[0] + t[1]) + (t[2] + t[3])) + ((t[4] + t[5]) + (t[6] + t[7]));
       });
-  if (ok && tid < kPfTile && key < a.T) a.scores[(size_t)bh * a.T + key] = cs;
+  if (tid >= kPfTile && tid < 2 * kPfTile) s_cs[row] = cs;
+  __syncthreads();
+  if (ok && tid < kPfTile && key < a.T) a.scores[(size_t)bh * a.T + key] = cs + s_cs[row];
 }
 
 }  // namespace
