@@ -313,7 +313,9 @@ def run_mikv(args):
                      "traffic": traffic, "bytes_per_launch": int(attn_bytes), "avg_launch_us": round(attn_ms * 1e3, 2)},
         "e2e": {"value": round(world * bytes_per_step / (e2e_ms * 1e-3) / 1e9, 1), "unit": UNIT,
                 "ms_per_step": round(e2e_ms, 4), "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-        "gpu_launches": K * L * 3 + kch_launches,  # per layer step: insert, attention, fused tail
+        # per layer step: attention (with the new token's insertion) and the fused tail; a coded important set
+        # quantizes the new token in a kernel of its own
+        "gpu_launches": K * L * (2 if w.hi_bits >= 16 else 3) + kch_launches,
     }
     if clk:
         line["clocks"] = clk

@@ -164,7 +164,9 @@ StepLayout step_layout(const mikv_shape* s, int n_lo_max) {
 // With `merge` unset the partials stay in the workspace and *args_out describes them.
 mikv_status attention_impl(const mikv_shape* s, const mikv_cache* c, int32_t n_lo, const void* q, float sm_scale,
                            void* out, int32_t out_dtype, float* hi_logits, float* ml, void* ws, size_t ws_bytes,
-                           cudaStream_t st, bool merge = true, AttnArgs* args_out = nullptr) {
+                           cudaStream_t st, bool merge = true, AttnArgs* args_out = nullptr,
+                           const int32_t* ins_slots = nullptr, const void* ins_k = nullptr,
+                           const void* ins_v = nullptr, int32_t ins_tok = 0) {
   const int sms = num_sms();
   // per-channel keys: the n_lo mod 64 staged retained tokens are attended as important rows hi_cap ..
   const bool kch = kch_of(*s);
@@ -247,6 +249,16 @@ mikv_status attention_impl(const mikv_shape* s, const mikv_cache* c, int32_t n_l
   a.n_units = plan.n_units;
   a.n_warps = plan.n_warps;
   a.sm_scale = sm_scale;
+  if (ins_slots) {
+    a.ins_slots = ins_slots;
+    a.ins_k = static_cast<const __nv_bfloat16*>(ins_k);
+    a.ins_v = static_cast<const __nv_bfloat16*>(ins_v);
+    a.ins_k_hi = static_cast<__nv_bfloat16*>(c->k_hi);
+    a.ins_v_hi = static_cast<__nv_bfloat16*>(c->v_hi);
+    a.ins_hi_tok = c->hi_tok;
+    a.ins_acc = c->acc;
+    a.ins_tok = ins_tok;
+  }
   cudaError_t e = launch_attention(a, lo_bits_of(*s), lo_group_of(*s), hb, G, plan.grid, st, kch);
   if (e != cudaSuccess) return MIKV_ERR_CUDA;
   if (args_out) *args_out = a;
@@ -443,11 +455,15 @@ mikv_status mikv_decode_step(const mikv_shape* shape, const mikv_cache* cache, i
   float* logits = reinterpret_cast<float*>(wsb + L.logits);
   if ((st = attention_args_ok(shape, cache, n_lo, q, out, out_dtype)) != MIKV_OK) return st;
   if (!aligned(k_new, 8) || !aligned(v_new, 8)) return MIKV_ERR_ARG;
-  if ((st = mikv_insert_token(shape, cache, k_new, v_new, tok, slots, stream)) != MIKV_OK) return st;
+  // a bf16 important set takes the new token inside the attention kernel; a coded one quantizes it first
+  const bool fused_insert = hi_bits_of(*shape) == 16;
+  if (!fused_insert && (st = mikv_insert_token(shape, cache, k_new, v_new, tok, slots, stream)) != MIKV_OK)
+    return st;
   // attention without its separate merge: the fused tail below merges, updates, selects and demotes
   AttnArgs a;
   if ((st = attention_impl(shape, cache, n_lo, q, sm_scale, out, out_dtype, logits, nullptr, workspace, L.attn,
-                           static_cast<cudaStream_t>(stream), false, &a)) != MIKV_OK)
+                           static_cast<cudaStream_t>(stream), false, &a, fused_insert ? slots : nullptr, k_new,
+                           v_new, tok)) != MIKV_OK)
     return st;
   StepPostArgs p;
   p.part_o = a.part_o;

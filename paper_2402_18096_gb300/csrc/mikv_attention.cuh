@@ -777,6 +777,27 @@ __device__ __forceinline__ void prefetch_unit(const AttnArgs& a, const Cursor& c
   }
 }
 
+// The step's new token for important slot `slot` of head bh (fused insertion, bf16 important set): its key and
+// value rows replace row slot % 16 of the staged 16-token unit (the 128B-swizzled boxes of 64 channels x 16
+// rows, keys at +0 / +2048, values at +4096 / +6144) and are written to the cache with its id and a zero score.
+// Lane l carries channels 4 l .. 4 l + 3 of both rows.
+__device__ __forceinline__ void insert_row(const AttnArgs& a, int bh, int slot, uint32_t stage, int lane) {
+  const uint2 kw = reinterpret_cast<const uint2*>(a.ins_k + (size_t)bh * kHeadDim)[lane];
+  const uint2 vw = reinterpret_cast<const uint2*>(a.ins_v + (size_t)bh * kHeadDim)[lane];
+  const int r = slot & 15, box = lane >> 4, chunk = (lane & 15) >> 1;
+  const uint32_t off = box * 2048 + r * 128 + ((chunk ^ (r & 7)) << 4) + (lane & 1) * 8;
+  asm volatile("st.shared.v2.u32 [%0], {%1, %2};" ::"r"(stage + off), "r"(kw.x), "r"(kw.y) : "memory");
+  asm volatile("st.shared.v2.u32 [%0], {%1, %2};" ::"r"(stage + 4096 + off), "r"(vw.x), "r"(vw.y) : "memory");
+  const size_t row = (size_t)bh * a.hi_stride + slot;
+  reinterpret_cast<uint2*>(a.ins_k_hi + row * kHeadDim)[lane] = kw;
+  reinterpret_cast<uint2*>(a.ins_v_hi + row * kHeadDim)[lane] = vw;
+  if (lane == 0) {
+    a.ins_hi_tok[row] = a.ins_tok;
+    a.ins_acc[row] = 0.f;
+  }
+  __syncwarp();
+}
+
 __device__ __forceinline__ void fence_proxy_async() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
@@ -836,6 +857,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
   constexpr int NB = 1 + (BITS == 3 ? 0 : (kHeadDim / GROUP + 1) / 2);  // beta rows + alpha-sum pairs
   Softmax st;
   float o[8][4], ob[NB][4];
+  __shared__ int s_ins[kWarps];  // each warp's insertion slot of its current head (fused insertion; kept out of
+                                 // the register file)
+  if (lane == 0) s_ins[warp] = -1;
   float* logit_base = nullptr;
   Cursor cc = cursor_at(u0, hu, n_u);  // unit being consumed
   int cur = -1;
@@ -871,6 +895,14 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
         for (int ks = 0; ks < 8; ++ks) qb[ks][0] = qb[ks][1] = qh[ks][0] = qh[ks][1] = 0u;
       }
       logit_base = a.hi_logits ? a.hi_logits + (size_t)(b * a.heads_q + h * G) * a.hi_stride : nullptr;
+      if (HB == 16 && a.ins_slots) {
+        __syncwarp();
+        if (lane == 0) {
+          const int sl = a.ins_slots[cur];
+          s_ins[warp] = sl < a.hi_cap ? sl : -1;
+        }
+        __syncwarp();
+      }
       st.m[0] = st.m[1] = -INFINITY;
       st.l[0] = st.l[1] = 0.f;
       st.mx[0] = st.mx[1] = -INFINITY;
@@ -890,6 +922,10 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
     const UnitKind k = cursor_kind(cc, hu, n_u);
     if (k.hi) {
       if constexpr (HB == 16) {
+        if (a.ins_slots) {
+          const int sl = s_ins[warp];
+          if (sl >= 0 && (sl >> 4) == k.index) insert_row(a, cur, sl, stage, lane);
+        }
         process_hi<G, NB>(stage, min(16, a.hi_cap - 16 * k.index), 16 * k.index, qb, a.sm_scale, logit_base,
                           a.hi_stride, st, o, ob, lane);
       } else {

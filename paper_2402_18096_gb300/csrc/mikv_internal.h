@@ -112,6 +112,17 @@ struct AttnArgs {
   int batch, heads_q, heads_kv, hi_cap, hi_stride, lo_cap, n_lo;
   int hi_blocks, hi_units, lo_blocks, n_u, n_units, n_warps;
   float sm_scale;
+  // insertion of a decode step's new token, fused into the attention of a bf16 important set: the unit
+  // holding slot ins_slots[b, h] takes the new rows in shared memory, and its warp writes them (and the
+  // token id, a zero score) into the cache. ins_slots == nullptr: no insertion.
+  const int32_t* ins_slots;
+  const __nv_bfloat16* ins_k;  // [B][Hkv][128]
+  const __nv_bfloat16* ins_v;
+  __nv_bfloat16* ins_k_hi;
+  __nv_bfloat16* ins_v_hi;
+  int32_t* ins_hi_tok;
+  float* ins_acc;
+  int ins_tok;
 };
 
 struct MergeArgs {
