@@ -44,13 +44,13 @@ namespace {
 
 // Launch shape (compile-time tuning knobs; the defaults are the measured best on GB300).
 #ifndef MIKV_ATTN_WARPS
-#define MIKV_ATTN_WARPS 6
+#define MIKV_ATTN_WARPS 12
 #endif
 #ifndef MIKV_ATTN_STAGES
 #define MIKV_ATTN_STAGES 2
 #endif
 #ifndef MIKV_ATTN_CTAS
-#define MIKV_ATTN_CTAS 2
+#define MIKV_ATTN_CTAS 1
 #endif
 #ifndef MIKV_QK_ACC
 #define MIKV_QK_ACC 2
