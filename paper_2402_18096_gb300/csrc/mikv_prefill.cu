@@ -36,19 +36,24 @@ constexpr int kPfStrHalf = kPfN * 128;
 constexpr int kPfStages = 4;                            // streamed tiles in flight
 constexpr int kPfAcc = 4;                               // TMEM accumulators of kPfN columns
 constexpr int kPfTmemCols = kPfAcc * kPfN;
-constexpr int kPfBars = 1 + 4 * kPfStages + 1;          // fixed, full/free/acc-full/acc-empty x 4, drain
-constexpr int kPfSmem = kPfFixBytes + kPfStages * kPfStrBytes + 8 * kPfBars + 1024;
+constexpr int kPfStatBytes = kPfN * 4;                 // pass 2: the streamed queries' log2 normalisers
+constexpr int kPfBars = 1 + 5 * kPfStages + 1;          // fixed, full/free/acc-full/acc-empty/stats x 4, drain
+constexpr int kPfSmem = kPfFixBytes + kPfStages * (kPfStrBytes + kPfStatBytes) + 8 * kPfBars + 1024;
 static_assert(kPfTile == 128 && kPfStages == kPfAcc, "one accumulator row per epilogue thread; shared indices");
 
 struct PfSmem {
-  uint32_t fixed, stage0, bars;
+  uint32_t fixed, stage0, stat0, bars;
+  const uint8_t* gbase;  // generic address of `fixed`
   __device__ uint32_t stage(int s) const { return stage0 + s * kPfStrBytes; }
+  __device__ uint32_t stat(int s) const { return stat0 + s * kPfStatBytes; }
+  __device__ const float* stat_ptr(int s) const { return reinterpret_cast<const float*>(gbase + (stat(s) - fixed)); }
   __device__ uint32_t bar_fixed() const { return bars; }
   __device__ uint32_t full(int s) const { return bars + 8 * (1 + s); }                 // copy landed
   __device__ uint32_t sfree(int s) const { return bars + 8 * (1 + kPfStages + s); }    // MMAs read it
   __device__ uint32_t tfull(int d) const { return bars + 8 * (1 + 2 * kPfStages + d); }  // accumulator ready
   __device__ uint32_t tempty(int d) const { return bars + 8 * (1 + 3 * kPfStages + d); } // accumulator read
-  __device__ uint32_t drain() const { return bars + 8 * (1 + 4 * kPfStages); }
+  __device__ uint32_t sdone(int s) const { return bars + 8 * (1 + 4 * kPfStages + s); }   // stats read
+  __device__ uint32_t drain() const { return bars + 8 * (1 + 5 * kPfStages); }
 };
 
 __device__ __forceinline__ PfSmem pf_smem() {
@@ -56,8 +61,10 @@ __device__ __forceinline__ PfSmem pf_smem() {
   const uint32_t base = (smem_u32(smem_raw) + 1023u) & ~1023u;
   PfSmem r;
   r.fixed = base;
+  r.gbase = smem_raw + (base - smem_u32(smem_raw));
   r.stage0 = base + kPfFixBytes;
-  r.bars = r.stage0 + kPfStages * kPfStrBytes;
+  r.stat0 = r.stage0 + kPfStages * kPfStrBytes;
+  r.bars = r.stat0 + kPfStages * kPfStatBytes;
   return r;
 }
 
@@ -90,9 +97,12 @@ __device__ __forceinline__ void pf_mma_tile(uint32_t d_tmem, uint32_t fix, uint3
 // accumulators, and warps 0-7 hand accumulator row halves to epi(n, col0, v): warp w gets row 32 (w % 4) +
 // lane, columns col0 = 32 (w / 4) .. col0 + 31. Returns false when a wait timed out (after draining what was
 // in flight); every role leaves through the final barrier.
-template <class StrRow, class Epi>
+// STATS (pass 2): the copy warp also stages each streamed tile's kPfN query normalisers (stats + stat_off(n),
+// 16-byte aligned in the padded rows) with the tile; the epilogue warps release them through sdone.
+template <bool STATS, class StrRow, class StatOff, class Epi>
 __device__ __forceinline__ bool pf_pipeline(const PrefillArgs& a, const CUtensorMap* map_fix, int fix_row,
-                                            const CUtensorMap* map_str, int n_tiles, StrRow str_row, Epi epi) {
+                                            const CUtensorMap* map_str, int n_tiles, StrRow str_row,
+                                            StatOff stat_off, Epi epi) {
   __shared__ uint32_t s_tmem;
   __shared__ int s_fail;
   volatile int* fail = &s_fail;
@@ -106,6 +116,7 @@ __device__ __forceinline__ bool pf_pipeline(const PrefillArgs& a, const CUtensor
       mbar_init(sm.sfree(s), 1);
       mbar_init(sm.tfull(s), 1);
       mbar_init(sm.tempty(s), kPfEpiWarps);  // one arrival per epilogue warp
+      mbar_init(sm.sdone(s), kPfEpiWarps);
     }
     mbar_init(sm.drain(), 1);
     fence_mbar_init();
@@ -125,11 +136,14 @@ __device__ __forceinline__ bool pf_pipeline(const PrefillArgs& a, const CUtensor
       tma_load_2d(sm.fixed + kPfFixHalf, map_fix, 64, fix_row, sm.bar_fixed());
       for (int t = 0; t < n_tiles; ++t) {
         const int s = t % kPfStages;
-        if (t >= kPfStages && !pf_wait(sm.sfree(s), ((t / kPfStages) & 1) ^ 1, fail)) break;
+        const uint32_t ph = ((t / kPfStages) & 1) ^ 1;
+        if (t >= kPfStages && !pf_wait(sm.sfree(s), ph, fail)) break;
+        if (STATS && t >= kPfStages && !pf_wait(sm.sdone(s), ph, fail)) break;
         const int row = str_row(t);
-        mbar_arrive_expect_tx(sm.full(s), kPfStrBytes);
+        mbar_arrive_expect_tx(sm.full(s), kPfStrBytes + (STATS ? kPfStatBytes : 0));
         tma_load_2d(sm.stage(s), map_str, 0, row, sm.full(s));
         tma_load_2d(sm.stage(s) + kPfStrHalf, map_str, 64, row, sm.full(s));
+        if (STATS) bulk_load(sm.stat(s), a.stats + stat_off(t), kPfStatBytes, sm.full(s));
         last[s] = t;
       }
       if (*fail) {  // no copy may outlive the CTA
@@ -171,7 +185,17 @@ __device__ __forceinline__ bool pf_pipeline(const PrefillArgs& a, const CUtensor
       tcgen05_before_sync();
       __syncwarp();
       if (lane == 0) mbar_arrive(sm.tempty(d));
-      epi(n, kPfCols * half, v);
+      // the staged normalisers: observe their copy's completion directly (it has completed: the MMAs
+      // that produced this accumulator waited for it, and the stage is not refilled before sdone)
+      if (STATS && !__all_sync(0xffffffffu, pf_wait(sm.full(d), (n / kPfStages) & 1, fail))) {
+        *fail = 1;
+        break;
+      }
+      epi(n, kPfCols * half, v, sm.stat_ptr(d) + kPfCols * half);
+      if (STATS) {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(sm.sdone(d));
+      }
     }
   }
   tcgen05_before_sync();
@@ -230,10 +254,10 @@ __global__ void __launch_bounds__(kPfThreads, 2) prefill_rows_kernel(const __gri
   const int q = kPfTile * qt + row;  // an epilogue thread's query
   const int kend = min(kPfTile * (qt + 1), a.T);  // keys 0 .. kend - 1 can reach this tile's queries
   float r = -INFINITY, l = 0.f;  // over this thread's column half of every tile
-  const bool ok = pf_pipeline(
+  const bool ok = pf_pipeline<false>(
       a, &a.map_q, bq * a.T + kPfTile * qt, &a.map_k_str, (kend + kPfN - 1) / kPfN,
-      [&](int n) { return krow0 + kPfN * n; },
-      [&](int n, int col0, float (&v)[kPfCols]) {
+      [&](int n) { return krow0 + kPfN * n; }, [](int) { return (size_t)0; },
+      [&](int n, int col0, float (&v)[kPfCols], const float*) {
         const int k0 = kPfN * n + col0;
         if (k0 + kPfCols > kPfTile * qt) {  // keys after the query, or past the prefill, do not count
 #pragma unroll
@@ -282,13 +306,14 @@ __global__ void __launch_bounds__(kPfThreads, 2) prefill_cols_kernel(const __gri
   const int row = tid & (kPfTile - 1);
   const int key = kPfTile * kt + row;  // an epilogue thread's key
   float cs = 0.f;
-  const bool ok = pf_pipeline(
+  const bool ok = pf_pipeline<true>(
       a, &a.map_k, bh * a.T + kPfTile * kt, &a.map_q_str, G * per_head,
       [&](int n) { return qhead(n) * a.T + qfirst(n); },
-      [&](int n, int col0, float (&v)[kPfCols]) {
+      [&](int n) { return (size_t)qhead(n) * a.T_pad + qfirst(n); },
+      [&](int n, int col0, float (&v)[kPfCols], const float* stat) {
         const int q0 = qfirst(n) + col0;
-        // minus the log2 normalisers of these queries (+inf for padding queries: they weigh nothing)
-        const float4* nc = reinterpret_cast<const float4*>(a.stats + (size_t)qhead(n) * a.T_pad + q0);
+        // the log2 normalisers of these queries, staged with the tile (+inf for padding: they weigh nothing)
+        const float4* nc = reinterpret_cast<const float4*>(stat);
         if (q0 < kPfTile * (kt + 1)) {  // the diagonal: queries before the key do not attend to it
 #pragma unroll
           for (int j = 0; j < kPfCols; ++j)
@@ -298,7 +323,7 @@ __global__ void __launch_bounds__(kPfThreads, 2) prefill_cols_kernel(const __gri
         uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
         for (int j = 0; j < kPfCols / 4; ++j) {
-          const float4 c = __ldg(nc + j);
+          const float4 c = nc[j];
           float x0, x1, x2, x3;
           f32x2_split(fma_f32x2(f32x2(v[4 * j], v[4 * j + 1]), s2, f32x2(-c.x, -c.y)), x0, x1);
           f32x2_split(fma_f32x2(f32x2(v[4 * j + 2], v[4 * j + 3]), s2, f32x2(-c.z, -c.w)), x2, x3);
