@@ -4,17 +4,18 @@
 // arxiv 2402.18096).
 //
 // Two passes over the causal score matrix S = sm_scale * Q K^T, each a tiled bf16 contraction on the
-// fifth-generation tensor cores (tcgen05.mma, M = N = 128, fp32 accumulators in tensor memory) fed by TMA:
+// fifth-generation tensor cores (tcgen05.mma, M = 128, N = 64, fp32 accumulators in tensor memory) fed by TMA:
 //   1. rows:    per query i, the log2 of its softmax normaliser, c_i = log2 sum_{t <= i} 2^(s_it log2 e)
 //               (accumulated online against a reference, as in flash attention, without values);
 //   2. columns: per key t, sum over the G query heads and the queries i >= t of 2^(s_it log2 e - c_i).
 // A CTA owns one 128-token tile of its fixed operand (queries in pass 1, keys in pass 2: the M side, so that
 // epilogue thread r owns accumulator row r = TMEM lane r) and streams 64-token tiles of the other operand.
-// Its warps specialise: warp 4 issues the TMA copies (the fixed tile, then a four-stage ring of 128B-swizzled
-// streamed tiles), warp 5 issues the eight K = 16 MMAs of each tile (M = 128, N = 64) into one of four TMEM
-// accumulators, and warps 0-3 read each accumulator row with tcgen05.ld, release it, and do the softmax
-// arithmetic (an exponential per score). The roles hand tiles over through mbarriers only; every wait is
-// bounded in time and gives up when another role has failed. Only the causal triangle is visited.
+// Its warps specialise: warp 8 issues the TMA copies (the fixed tile, then a four-stage ring of 128B-swizzled
+// streamed tiles, with pass 2's query normalisers), warp 9 issues the eight K = 16 MMAs of each tile into one
+// of four TMEM accumulators, and warps 0-7 (two per accumulator lane quarter, one per column half) read
+// their accumulator rows with tcgen05.ld, release them, and do the softmax arithmetic (an exponential per
+// score). The roles hand tiles over through mbarriers only; every wait is bounded in time and gives up when
+// another role has failed. Only the causal triangle is visited.
 #include <math.h>
 
 #include "mikv_device.cuh"
