@@ -79,9 +79,12 @@ __global__ void __launch_bounds__(kPostThreads, 2) step_post_kernel(const StepPo
   const float* logit = a.hi_logits + (size_t)(b * a.heads_q + h * G) * a.hi_stride;
   const int nv = (a.hi_cap + 3) / 4;  // groups of four slots
 
-  // 0. this thread's first group of slots is loaded before the merge, which it does not depend on
-  SlotQuad<G> q0;
+  // 0. this thread's first groups of slots are loaded before the statistics, which they do not depend on
+  // (two groups each where registers allow: those loads overlap the statistics' loads below)
+  constexpr int kPre = G <= 4 ? 2 : 1;
+  SlotQuad<G> q0, qp;
   if (tid < nv) load_quad<G>(logit, acc, tok, a.hi_stride, tid, q0);
+  if (kPre == 2 && tid + kPostThreads < nv) load_quad<G>(logit, acc, tok, a.hi_stride, tid + kPostThreads, qp);
 
   // 1. softmax statistics (M, L) of query heads h*G .. h*G+G-1 from the split partials (one warp per head)
   const int w0 = owner_warp((long long)bh * a.n_u, a.n_units, a.n_warps);
@@ -101,8 +104,9 @@ __global__ void __launch_bounds__(kPostThreads, 2) step_post_kernel(const StepPo
   unsigned long long best = ~0ull;
   int best_slot = -1;
   if (tid < nv) update_quad<G>(acc, a.hi_cap, tid, q0, s_m, s_il, best, best_slot);
+  if (kPre == 2 && tid + kPostThreads < nv) update_quad<G>(acc, a.hi_cap, tid + kPostThreads, qp, s_m, s_il, best, best_slot);
   constexpr int kInFlight = G <= 4 ? 2 : 1;  // groups loaded before any of them is used
-  for (int v = tid + kPostThreads; v < nv; v += kInFlight * kPostThreads) {
+  for (int v = tid + kPre * kPostThreads; v < nv; v += kInFlight * kPostThreads) {
     SlotQuad<G> q1, q2;
     const bool two = kInFlight == 2 && v + kPostThreads < nv;
     load_quad<G>(logit, acc, tok, a.hi_stride, v, q1);
