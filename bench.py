@@ -166,16 +166,28 @@ def build_model(w, steps_cap: int, dev, rank: int):
     shape = pkg.Shape(w.batch, w.heads_q, w.heads_kv, w.bits, w.group, w.hi_cap, w.lo_cap_for(steps_cap),
                       hi_bits=w.hi_bits, k_channel_group=64 if w.k_channel else 0)
     wr = rank_workload(w, rank)  # each rank owns a different batch
-    layers = []
+    layers, ms, in_bytes = [], [], 0
     for li in range(w.layers):
         k, v = mi.prefill_kv(wr, li, dev)
         scores = mi.initial_scores(wr, li, dev)
         q_pre = mi.prefill_queries(wr, li, dev)
+        in_bytes = sum(x.numel() * x.element_size() for x in (k, v, scores, q_pre))
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+        ev[0].record()
         layers.append(MixedPrecisionLayer.from_prefill(shape, k, v, scores, q_pre, device=dev))
+        ev[1].record()
+        ev[1].synchronize()
+        ms.append(ev[0].elapsed_time(ev[1]))
         del k, v, scores, q_pre
     torch.cuda.synchronize()
     torch.cuda.empty_cache()
-    return shape, layers
+    # cache build (balancer, selection, gather of the important rows, quantize/pack of the rest) per layer;
+    # the first layer also pays one-time costs and is left out when there are others
+    t = statistics.median(ms[1:] if len(ms) > 1 else ms)
+    build = {"ms_per_layer": round(t, 3), "input_bytes_per_layer": in_bytes,
+             "input_gbs": round(in_bytes / (t * 1e-3) / 1e9, 1),
+             "inputs": "prefill q, k, v (bf16) and importance scores (fp32), each read once"}
+    return shape, layers, build
 
 
 def run_mikv(args):
@@ -193,7 +205,7 @@ def run_mikv(args):
     e2e_steps = max(2, K // 2)
     attn_reps = 2
     steps_cap = W + K + W + e2e_steps + 4
-    shape, layers = build_model(w, steps_cap, dev, rank)
+    shape, layers, build = build_model(w, steps_cap, dev, rank)
     L = len(layers)
     # per-step decode inputs, resident on the device
     n_in = W + K
@@ -316,6 +328,7 @@ def run_mikv(args):
         # per layer step: attention (with the new token's insertion) and the fused tail; a coded important set
         # quantizes the new token in a kernel of its own
         "gpu_launches": K * L * (2 if w.hi_bits >= 16 else 3) + kch_launches,
+        "cache_build": build,
     }
     if clk:
         line["clocks"] = clk

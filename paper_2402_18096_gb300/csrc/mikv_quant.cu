@@ -1,14 +1,14 @@
 // mikv_quant.cu — demotion of KV rows into the retained set (Eq. 1 with the Eq. 3 key balancer), rows
 // entering a coded important set (Sec. 3.3), and the channel balancer itself (Eq. 2), arxiv 2402.18096.
 //
-// quantize_pack: one warp per (row, K or V) running quantize_row_warp (mikv_rows.cuh): each lane owns
-// 4 consecutive channels, group minima and maxima come from butterfly shuffles, scale and zero are
-// rounded to fp16 outward so the stored grid covers the group's range, codes are round-half-even of
-// the IEEE fp32 quotient (x - beta) / alpha, OR-ed into the packed layout in shared memory and written
-// out as whole words.
+// quantize_pack: each warp quantizes four rows of K or of V (their loads issued together) with
+// quantize_values_warp (mikv_rows.cuh): each lane owns 4 consecutive channels, group minima and maxima
+// come from butterfly shuffles, scale and zero are rounded to fp16 outward so the stored grid covers the
+// group's range, codes are round-half-even of the IEEE fp32 quotient (x - beta) / alpha, and the packed
+// words are assembled by an OR butterfly across the lanes that share them and stored 8 bytes at a time.
 #include "mikv_device.cuh"
 #include "mikv_internal.h"
-#include "mikv_rows.cuh"
+#include "mikv_quant_rows.cuh"
 
 namespace mikv {
 namespace {
@@ -27,22 +27,39 @@ struct QPArgs {
   int heads_kv, n_src, n_rows, lo_start, lo_cap;
 };
 
+// Rows each warp of quantize_pack_kernel quantizes; their loads are issued together (1 KB per warp in
+// flight) before any of them is quantized.
+constexpr int kQpRows = 4;
+
 template <int BITS, int GROUP>
 __global__ void __launch_bounds__(256) quantize_pack_kernel(const QPArgs a) {
-  __shared__ uint32_t buf[8][32];
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int i = blockIdx.x * 4 + (w >> 1);
   const bool is_v = (w & 1) != 0;
   const int bh = blockIdx.y, h = bh % a.heads_kv;
-  if (i >= a.n_rows) return;
-  const int r = a.rows[(size_t)bh * a.n_rows + i];
-  if (r < 0 || r >= a.n_src) return;  // out-of-range rows are skipped (documented in the ABI)
-  const size_t pos = (size_t)bh * a.lo_cap + a.lo_start + i;
-  const __nv_bfloat16* src = (is_v ? a.v_src : a.k_src) + ((size_t)bh * a.n_src + r) * kHeadDim;
-  quantize_row_warp<BITS, GROUP>(src, is_v ? nullptr : (a.balancer ? a.balancer + h * kHeadDim : nullptr),
-                                 (is_v ? a.v_codes : a.k_codes) + pos * (16 * BITS),
-                                 (is_v ? a.v_params : a.k_params) + pos * (kHeadDim / GROUP), buf[w], lane);
-  if (!is_v && lane == 0) a.lo_tok[pos] = a.src_tok ? a.src_tok[(size_t)bh * a.n_src + r] : r;
+  const int i0 = (blockIdx.x * 4 + (w >> 1)) * kQpRows;
+  const __nv_bfloat16* src = (is_v ? a.v_src : a.k_src) + (size_t)bh * a.n_src * kHeadDim + 4 * lane;
+  int r[kQpRows];
+  uint2 raw[kQpRows];
+#pragma unroll
+  for (int k = 0; k < kQpRows; ++k) {
+    const int i = i0 + k;
+    r[k] = i < a.n_rows ? a.rows[(size_t)bh * a.n_rows + i] : -1;
+    if (r[k] >= a.n_src) r[k] = -1;  // out-of-range rows are skipped (documented in the ABI)
+  }
+#pragma unroll
+  for (int k = 0; k < kQpRows; ++k)
+    if (r[k] >= 0) raw[k] = *reinterpret_cast<const uint2*>(src + (size_t)r[k] * kHeadDim);
+  const float* bal = is_v ? nullptr : (a.balancer ? a.balancer + h * kHeadDim : nullptr);
+#pragma unroll
+  for (int k = 0; k < kQpRows; ++k) {
+    if (r[k] < 0) continue;  // warp-uniform
+    const size_t pos = (size_t)bh * a.lo_cap + a.lo_start + i0 + k;
+    float x[4];
+    row_values(raw[k], bal, lane, x);
+    quantize_values_warp<BITS, GROUP>(x, (is_v ? a.v_codes : a.k_codes) + pos * (16 * BITS),
+                                      (is_v ? a.v_params : a.k_params) + pos * (kHeadDim / GROUP), lane);
+    if (!is_v && lane == 0) a.lo_tok[pos] = a.src_tok ? a.src_tok[(size_t)bh * a.n_src + r[k]] : r[k];
+  }
 }
 
 template <int BITS>
@@ -80,7 +97,6 @@ struct HiQArgs {
 
 template <int HB>
 __global__ void __launch_bounds__(256) hi_quant_kernel(const HiQArgs a) {
-  __shared__ uint32_t buf[8][32];
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
   grid_dependency_wait();  // insertion: the slot comes from the previous step's tail
   allow_dependent_launch();
@@ -104,7 +120,7 @@ __global__ void __launch_bounds__(256) hi_quant_kernel(const HiQArgs a) {
   const size_t row = (size_t)bh * a.hi_stride + slot;
   quantize_row_warp<HB, kHiGroup>(src, is_v ? nullptr : (a.balancer ? a.balancer + h * kHeadDim : nullptr),
                                   (is_v ? a.v_hc : a.k_hc) + row * (16 * HB),
-                                  (is_v ? a.v_hp : a.k_hp) + row * (kHeadDim / kHiGroup), buf[w], lane);
+                                  (is_v ? a.v_hp : a.k_hp) + row * (kHeadDim / kHiGroup), lane);
   if (!is_v && lane == 0) {
     a.hi_tok[row] = a.rows ? (a.src_tok ? a.src_tok[(size_t)bh * a.n_src + r] : r) : a.tok;
     a.acc[row] = a.rows && a.src_scores ? a.src_scores[(size_t)bh * a.n_src + r] : 0.f;
@@ -155,7 +171,6 @@ __global__ void __launch_bounds__(kKchThreads) kch_group_kernel(const KchArgs a)
   __shared__ __align__(16) __nv_bfloat16 sk[kKchGroup][kHeadDim];
   __shared__ __align__(16) __nv_bfloat16 sv[kKchGroup][kHeadDim];
   __shared__ uint32_t cbuf[kKchGroup][4 * BITS];
-  __shared__ uint32_t wbuf[kKchThreads / 32][32];
   __shared__ int32_t stok[kKchGroup];
   constexpr int QMAX = (1 << BITS) - 1;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -209,7 +224,7 @@ __global__ void __launch_bounds__(kKchThreads) kch_group_kernel(const KchArgs a)
   // 3. values per token (8 rows per warp) and token ids
   for (int t = warp; t < kKchGroup; t += kKchThreads / 32) {
     quantize_row_warp<BITS, GROUP>(&sv[t][0], nullptr, a.v_codes + (pos0 + t) * (16 * BITS),
-                                   a.v_params + (pos0 + t) * (kHeadDim / GROUP), wbuf[warp], lane);
+                                   a.v_params + (pos0 + t) * (kHeadDim / GROUP), lane);
     if (lane == 0) a.lo_tok[pos0 + t] = stok[t];
   }
 }
@@ -290,7 +305,7 @@ cudaError_t launch_quantize_pack(const mikv_shape& s, const mikv_cache& c, const
   a.n_rows = n_rows;
   a.lo_start = lo_start;
   a.lo_cap = s.lo_cap;
-  const dim3 grid((n_rows + 3) / 4, s.batch * s.heads_kv);
+  const dim3 grid((n_rows + 4 * kQpRows - 1) / (4 * kQpRows), s.batch * s.heads_kv);
   switch (s.bits) {
     case 2: return qp_group<2>(a, s.group, grid, st);
     case 3: return qp_group<3>(a, s.group, grid, st);

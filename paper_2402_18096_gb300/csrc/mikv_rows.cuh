@@ -1,105 +1,11 @@
 // mikv_rows.cuh — warp-level building blocks shared by the standalone kernels and the fused step
-// kernel: Eq. 1 quantization of one 128-channel row into the packed layout, the (score, id) demotion
-// order, and the combination of split-attention partials.
+// kernel: the (score, id) demotion order, the combination of split-attention partials and the
+// importance weight of a slot.
 #pragma once
 
 #include "mikv_device.cuh"
 
 namespace mikv {
-
-// Bit position of channel c (= 16 m + u) in a plane of f-bit fields: 16-bit unit and bit offset.
-__device__ __forceinline__ void field_pos(int c, int f, int& unit, int& bit) {
-  const int u = c & 15, m = c >> 4;
-  if (f == 1) {
-    unit = u & 7;
-    bit = 8 * (u >> 3) + m;
-  } else {
-    const int P = 16 / f;
-    unit = 8 * (2 * (m / P) + (u >> 3)) + (u & 7);
-    bit = f * (m % P);
-  }
-}
-
-// Quantize one row (Eq. 1) held as fp32 values x[4] of channels 4 lane .. 4 lane + 3 of each lane, with
-// one warp. Writes 16 * BITS bytes of packed codes to `codes` and 128 / GROUP (alpha, beta) fp16 pairs to
-// `params`. `buf` is 32 words of this warp's shared memory. Every rounding is explicit (fsub/fdiv
-// round-to-nearest, fp16 round-down / round-up, round-half-even to int), so codes and parameters are
-// bit-identical to an IEEE fp32 evaluation. BITS in {2, 3, 4, 8}.
-template <int BITS, int GROUP>
-__device__ __forceinline__ void quantize_values_warp(const float (&x)[4], uint8_t* codes, __half2* params,
-                                                     uint32_t* buf, int lane) {
-  constexpr int QMAX = (1 << BITS) - 1;
-  constexpr int LANES = GROUP / 4;  // lanes per quantization group
-  constexpr int WORDS = 4 * BITS;   // 32-bit words of one packed row
-  if (lane < WORDS) buf[lane] = 0u;
-  __syncwarp();
-  float mn = fminf(fminf(x[0], x[1]), fminf(x[2], x[3]));
-  float mx = fmaxf(fmaxf(x[0], x[1]), fmaxf(x[2], x[3]));
-#pragma unroll
-  for (int off = 1; off < LANES; off <<= 1) {
-    mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, off));
-    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-  }
-  // Eq. 1: beta = min, alpha = (max - min) / (2^N - 1), stored in fp16 with outward rounding.
-  const __half beta16 = __float2half_rd(mn);
-  const float beta = __half2float(beta16);
-  const float span = __fsub_rn(mx, beta);
-  const __half alpha16 = span == 0.f ? __float2half_rn(1.f) : __float2half_ru(__fdiv_rn(span, (float)QMAX));
-  const float alpha = __half2float(alpha16);
-#pragma unroll
-  for (int e = 0; e < 4; ++e) {
-    int code = __float2int_rn(__fdiv_rn(__fsub_rn(x[e], beta), alpha));
-    code = code < 0 ? 0 : (code > QMAX ? QMAX : code);
-    const int c = 4 * lane + e;
-    int unit, bit;
-    field_pos(c, BITS == 3 ? 2 : BITS, unit, bit);
-    const uint32_t fmask = BITS == 3 ? 3u : (uint32_t)QMAX;
-    atomicOr(&buf[unit >> 1], (((uint32_t)code & fmask) << bit) << (16 * (unit & 1)));
-    if (BITS == 3) {
-      field_pos(c, 1, unit, bit);
-      atomicOr(&buf[8 + (unit >> 1)], (((uint32_t)code >> 2) << bit) << (16 * (unit & 1)));
-    }
-  }
-  __syncwarp();
-  if (lane < WORDS) reinterpret_cast<uint32_t*>(codes)[lane] = buf[lane];
-  if ((lane & (LANES - 1)) == 0) params[(4 * lane) / GROUP] = __halves2half2(alpha16, beta16);
-}
-
-// Quantize one bf16 row (Eq. 1, Eq. 3): lane l owns channels 4l..4l+3 of `src`; keys pass `bal` (fp32
-// [128], or nullptr = 1), multiplied in before the quantizer.
-template <int BITS, int GROUP>
-__device__ __forceinline__ void quantize_row_warp(const __nv_bfloat16* src, const float* bal, uint8_t* codes,
-                                                  __half2* params, uint32_t* buf, int lane) {
-  const uint2 raw = *reinterpret_cast<const uint2*>(src + 4 * lane);
-  float x[4] = {__uint_as_float(raw.x << 16), __uint_as_float(raw.x & 0xffff0000u),
-                __uint_as_float(raw.y << 16), __uint_as_float(raw.y & 0xffff0000u)};
-  if (bal) {  // Eq. 3: keys times the balancer before the quantizer
-    const float4 b = *reinterpret_cast<const float4*>(bal + 4 * lane);
-    x[0] = __fmul_rn(x[0], b.x);
-    x[1] = __fmul_rn(x[1], b.y);
-    x[2] = __fmul_rn(x[2], b.z);
-    x[3] = __fmul_rn(x[3], b.w);
-  }
-  quantize_values_warp<BITS, GROUP>(x, codes, params, buf, lane);
-}
-
-// fp32 dequantization of channels 4 lane .. 4 lane + 3 of one packed row of `bits`-bit codes (bits in
-// {2, 4, 8}, one plane) with (alpha, beta) per group of `group` channels: x = alpha * code + beta, the
-// product exact in fp32 and the sum rounded once (one fma).
-__device__ __forceinline__ void dequantize_values_warp(const uint8_t* codes, const __half2* params, int bits,
-                                                       int group, int lane, float (&x)[4]) {
-  const uint16_t* units = reinterpret_cast<const uint16_t*>(codes);
-  const uint32_t mask = (1u << bits) - 1u;
-#pragma unroll
-  for (int e = 0; e < 4; ++e) {
-    const int c = 4 * lane + e;
-    int unit, bit;
-    field_pos(c, bits, unit, bit);
-    const uint32_t code = ((uint32_t)units[unit] >> bit) & mask;
-    const float2 ab = __half22float2(params[c / group]);
-    x[e] = __fmaf_rn(ab.x, (float)code, ab.y);
-  }
-}
 
 // Total order of (score, id): ascending score, then ascending id. -0 is folded into +0.
 __device__ __forceinline__ unsigned long long order_key(float s, int32_t id) {

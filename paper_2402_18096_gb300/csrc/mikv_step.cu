@@ -11,6 +11,7 @@
 
 #include "mikv_device.cuh"
 #include "mikv_internal.h"
+#include "mikv_quant_rows.cuh"
 #include "mikv_rows.cuh"
 
 namespace mikv {
@@ -69,7 +70,6 @@ __global__ void __launch_bounds__(kPostThreads, 2) step_post_kernel(const StepPo
   __shared__ unsigned long long s_best[kPostThreads / 32];
   __shared__ int s_slot[kPostThreads / 32];
   __shared__ int s_victim;
-  __shared__ uint32_t buf[2][32];
   const int bh = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int b = bh / a.heads_kv, h = bh - b * a.heads_kv;
   grid_dependency_wait();  // logits and partials come from the attention kernel
@@ -189,14 +189,14 @@ __global__ void __launch_bounds__(kPostThreads, 2) step_post_kernel(const StepPo
     if (a.hi_bits == 16) {
       const __nv_bfloat16* src = static_cast<const __nv_bfloat16*>(is_v ? a.v_hi : a.k_hi) + hrow * kHeadDim;
       quantize_row_warp<BITS, GROUP>(src, is_v ? nullptr : (a.balancer ? a.balancer + h * kHeadDim : nullptr),
-                                     codes, params, buf[warp], lane);
+                                     codes, params, lane);
     } else {
       float x[4];
       dequantize_values_warp(static_cast<const uint8_t*>(is_v ? a.v_hi : a.k_hi) + hrow * (16 * a.hi_bits),
                              static_cast<const __half2*>(is_v ? a.v_hi_params : a.k_hi_params) +
                                  hrow * (kHeadDim / kHiGroup),
                              a.hi_bits, kHiGroup, lane, x);
-      quantize_values_warp<BITS, GROUP>(x, codes, params, buf[warp], lane);
+      quantize_values_warp<BITS, GROUP>(x, codes, params, lane);
     }
     if (!is_v && lane == 0) {
       a.lo_tok[pos] = tok[victim];

@@ -55,6 +55,42 @@ def test_quantize_pack_bit_exact(bits, group):
     assert int(cache.k_codes[:, :, :lo_start].abs().sum()) == 0
 
 
+@pytest.mark.parametrize("bits", [2, 3, 4])
+@pytest.mark.parametrize("group", [32, 128])
+def test_quantize_pack_exact_ties(bits, group):
+    """Every quotient (x - beta) / alpha an exact half-integer (beta = -s, alpha = s / 4 with s a power of
+    two, x = beta + alpha (m + 1/2)): the codes must round half to even exactly as the IEEE quotient does,
+    which the kernel's reciprocal product only decides after falling back to the division."""
+    qmax = (1 << bits) - 1
+    B, Hkv, n_src = 1, 2, 24
+    shape = pkg.Shape(B, 2, Hkv, bits, group, hi_cap=1, lo_cap=32)
+    rows_ = []
+    for r in range(B * Hkv * n_src):
+        s = 2.0 ** ((r % 7) - 3)
+        beta, alpha = -s, s / 4
+        m = np.arange(D) % group
+        x = beta + alpha * ((m * 5 + r) % qmax + 0.5)
+        x[m == 0] = beta                   # the group's minimum
+        x[m == 1] = beta + alpha * qmax    # and maximum: alpha = span / qmax exactly
+        rows_.append(x)
+    kv = torch.tensor(np.array(rows_), dtype=torch.float32).reshape(B, Hkv, n_src, D).to(torch.bfloat16)
+    assert torch.equal(kv.float().reshape(-1, D), torch.tensor(np.array(rows_), dtype=torch.float32))  # exact
+    k, v = kv, kv.flip(2).contiguous()
+    rows = torch.arange(n_src, dtype=torch.int32).expand(B, Hkv, n_src).contiguous()[..., :20].contiguous()
+    dev = torch.device("cuda")
+    cache = pkg.LayerCache(shape, device=dev)
+    pkg.mikv_quantize_pack(cache, k.to(dev), v.to(dev), rows.to(dev), 0)
+    torch.cuda.synchronize()
+    ref = oracle.empty_cache(B, Hkv, D, bits, group, 1, 32)
+    oracle.quantize_pack(ref, bits16(k), bits16(v), rows.numpy(), 0)
+    for name in ("k_codes", "v_codes"):
+        np.testing.assert_array_equal(getattr(cache, name)[:, :, :20].cpu().numpy(), ref[name][:, :, :20],
+                                      err_msg=name)
+    for name in ("k_params", "v_params"):
+        got = getattr(cache, name)[:, :, :20].cpu().view(torch.int16).numpy().view(np.uint16)
+        np.testing.assert_array_equal(got, ref[name][:, :, :20], err_msg=name)
+
+
 def test_quantize_pack_without_balancer_and_skips_bad_rows():
     gen = torch.Generator().manual_seed(3)
     B, Hkv, n_src = 1, 2, 8
