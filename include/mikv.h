@@ -144,11 +144,11 @@ mikv_status mikv_compute_balancer(const mikv_shape* shape, const void* q_pre, co
  *   toward +inf of fp32((max(x) - beta16) / (2^N - 1)) (1.0 when max(x) == beta16); code = clamp(
  *   round-half-even(fp32((x - beta16) / alpha16)), 0, 2^N - 1). Codes are packed as in the header.
  *   lo_tok[b][h][lo_start + i] = src_tok ? src_tok[b][h][r] : r.
- *   k_src, v_src  bf16 [B][Hkv][n_src][d]   (e.g. the important arrays with n_src = hi_stride)
+ *   k_src, v_src  bf16 [B][Hkv][n_src][d], 16-byte aligned (e.g. the important arrays, n_src = hi_stride)
  *   src_tok       int32 [B][Hkv][n_src] or NULL
  *   rows          int32 [B][Hkv][n_rows]   (device; e.g. the output of mikv_select_demote)
- * Errors: MIKV_ERR_CAPACITY if lo_start + n_rows > lo_cap. Rows outside [0, n_src) are skipped by the
- * kernel. Codes and parameters are bit-exact with an IEEE fp32 evaluation of the formulas above.
+ * Errors: MIKV_ERR_ARG if k_src or v_src is not 16-byte aligned; MIKV_ERR_CAPACITY if lo_start + n_rows >
+ * lo_cap. Rows outside [0, n_src) are skipped by the kernel. Codes and parameters are bit-exact with an IEEE fp32 evaluation of the formulas above.
  */
 /* With per-channel keys (k_channel_group = 64), mikv_quantize_pack APPENDS the rows at retained positions
  * lo_start .. lo_start + n_rows - 1, lo_start being the current retained length: a position whose group of

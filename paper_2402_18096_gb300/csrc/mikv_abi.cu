@@ -341,8 +341,9 @@ mikv_status mikv_quantize_pack(const mikv_shape* shape, const mikv_cache* cache,
   if (evicting(*shape)) return MIKV_ERR_UNSUPPORTED;  // no retained set to write
   if (!cache_ok(cache, shape) || !k_src || !v_src || n_src <= 0 || n_rows < 0 || lo_start < 0 || (n_rows > 0 && !rows))
     return MIKV_ERR_ARG;
+  if (!aligned(k_src, 16) || !aligned(v_src, 16)) return MIKV_ERR_ARG;  // rows are read in 16-byte pieces
   if ((int64_t)lo_start + n_rows > shape->lo_cap) return MIKV_ERR_CAPACITY;
-  if ((int64_t)(n_rows + 3) / 4 > 2147483647 || (int64_t)shape->batch * shape->heads_kv > 65535)
+  if ((int64_t)shape->batch * shape->heads_kv > 65535)
     return MIKV_ERR_UNSUPPORTED;
   if (kch_of(*shape)) {  // append: complete groups quantized per channel, the rest staged
     if (n_rows == 0) return MIKV_OK;

@@ -1,11 +1,12 @@
 // mikv_quant.cu — demotion of KV rows into the retained set (Eq. 1 with the Eq. 3 key balancer), rows
 // entering a coded important set (Sec. 3.3), and the channel balancer itself (Eq. 2), arxiv 2402.18096.
 //
-// quantize_pack: each warp quantizes four rows of K or of V (their loads issued together) with
-// quantize_values_warp (mikv_rows.cuh): each lane owns 4 consecutive channels, group minima and maxima
-// come from butterfly shuffles, scale and zero are rounded to fp16 outward so the stored grid covers the
-// group's range, codes are round-half-even of the IEEE fp32 quotient (x - beta) / alpha, and the packed
-// words are assembled by an OR butterfly across the lanes that share them and stored 8 bytes at a time.
+// quantize_pack: each warp quantizes four rows of K or of V, eight lanes per row and 16 channels per lane;
+// group minima and maxima come from the lane's channels and butterfly shuffles, scale and zero are
+// rounded to fp16 outward so the stored grid covers the group's range, codes are round-half-even of the
+// IEEE fp32 quotient (x - beta) / alpha (the Eq. 1 helpers of mikv_quant_rows.cuh, shared with the
+// one-row quantizer of the step tail), and the packed words are assembled by a reduce-scatter over the
+// lanes that share them.
 #include "mikv_device.cuh"
 #include "mikv_internal.h"
 #include "mikv_quant_rows.cuh"
@@ -27,39 +28,146 @@ struct QPArgs {
   int heads_kv, n_src, n_rows, lo_start, lo_cap;
 };
 
-// Rows each warp of quantize_pack_kernel quantizes; their loads are issued together (1 KB per warp in
-// flight) before any of them is quantized.
-constexpr int kQpRows = 4;
+// Bulk quantize/pack (Eq. 1): eight lanes per row and four rows per warp. Lane l8 = lane & 7 of a row owns
+// channels 16 l8 .. 16 l8 + 15 (two 16-byte loads), so a group's scale and zero are computed by GROUP / 16
+// lanes, and in the packed layout every channel of the lane sits at field index m = l8 of its 16-bit unit:
+// the lane's codes form partial words at fixed positions, which a reduce-scatter over the lanes that share
+// them turns into whole words, one or two per lane.
+constexpr int kQpRowsPerWarp = 4;
+
+// Reduce-scatter of N partial words over lane bits OFF, OFF / 2, ...: in each round a lane keeps the half
+// of its words selected by its lane bit and ORs in the partner's copy of that half. After log2(N) rounds
+// lane l8 holds the whole word index (bits of l8 from OFF down), as a single value.
+template <int N, int OFF>
+__device__ __forceinline__ uint32_t reduce_scatter(const uint32_t (&w)[N], int l8) {
+  constexpr int H = N / 2;
+  const bool up = (l8 & OFF) != 0;
+  uint32_t k[H];
+#pragma unroll
+  for (int i = 0; i < H; ++i) {
+    const uint32_t send = up ? w[i] : w[i + H];
+    k[i] = (up ? w[i + H] : w[i]) | __shfl_xor_sync(0xffffffffu, send, OFF);
+  }
+  if constexpr (H == 1) {
+    return k[0];
+  } else {
+    return reduce_scatter<H, OFF / 2>(k, l8);
+  }
+}
 
 template <int BITS, int GROUP>
 __global__ void __launch_bounds__(256) quantize_pack_kernel(const QPArgs a) {
-  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  constexpr int QMAX = (1 << BITS) - 1;
+  constexpr int GL = GROUP / 16;  // lanes per quantization group
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31, l8 = lane & 7;
   const bool is_v = (w & 1) != 0;
   const int bh = blockIdx.y, h = bh % a.heads_kv;
-  const int i0 = (blockIdx.x * 4 + (w >> 1)) * kQpRows;
-  const __nv_bfloat16* src = (is_v ? a.v_src : a.k_src) + (size_t)bh * a.n_src * kHeadDim + 4 * lane;
-  int r[kQpRows];
-  uint2 raw[kQpRows];
+  const int i = (blockIdx.x * 4 + (w >> 1)) * kQpRowsPerWarp + (lane >> 3);
+  const int r = i < a.n_rows ? a.rows[(size_t)bh * a.n_rows + i] : -1;
+  const bool valid = r >= 0 && r < a.n_src;  // out-of-range rows are skipped (documented in the ABI)
+  // invalid rows run the arithmetic on zeros (every lane takes part in the shuffles) and store nothing
+  uint4 raw[2] = {make_uint4(0u, 0u, 0u, 0u), make_uint4(0u, 0u, 0u, 0u)};
+  if (valid) {
+    const uint4* src = reinterpret_cast<const uint4*>((is_v ? a.v_src : a.k_src) +
+                                                      ((size_t)bh * a.n_src + r) * kHeadDim + 16 * l8);
+    raw[0] = src[0];
+    raw[1] = src[1];
+  }
+  float x[16];
 #pragma unroll
-  for (int k = 0; k < kQpRows; ++k) {
-    const int i = i0 + k;
-    r[k] = i < a.n_rows ? a.rows[(size_t)bh * a.n_rows + i] : -1;
-    if (r[k] >= a.n_src) r[k] = -1;  // out-of-range rows are skipped (documented in the ABI)
+  for (int k = 0; k < 2; ++k) {
+    const uint32_t wd[4] = {raw[k].x, raw[k].y, raw[k].z, raw[k].w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      x[8 * k + 2 * j] = __uint_as_float(wd[j] << 16);
+      x[8 * k + 2 * j + 1] = __uint_as_float(wd[j] & 0xffff0000u);
+    }
+  }
+  if (!is_v && a.balancer) {  // Eq. 3: keys times the balancer before the quantizer (warp-uniform)
+    const float4* bal = reinterpret_cast<const float4*>(a.balancer + h * kHeadDim + 16 * l8);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const float4 b = bal[k];
+      x[4 * k] = __fmul_rn(x[4 * k], b.x);
+      x[4 * k + 1] = __fmul_rn(x[4 * k + 1], b.y);
+      x[4 * k + 2] = __fmul_rn(x[4 * k + 2], b.z);
+      x[4 * k + 3] = __fmul_rn(x[4 * k + 3], b.w);
+    }
+  }
+  float mn = x[0], mx = x[0];
+#pragma unroll
+  for (int e = 1; e < 16; ++e) {
+    mn = fminf(mn, x[e]);
+    mx = fmaxf(mx, x[e]);
   }
 #pragma unroll
-  for (int k = 0; k < kQpRows; ++k)
-    if (r[k] >= 0) raw[k] = *reinterpret_cast<const uint2*>(src + (size_t)r[k] * kHeadDim);
-  const float* bal = is_v ? nullptr : (a.balancer ? a.balancer + h * kHeadDim : nullptr);
-#pragma unroll
-  for (int k = 0; k < kQpRows; ++k) {
-    if (r[k] < 0) continue;  // warp-uniform
-    const size_t pos = (size_t)bh * a.lo_cap + a.lo_start + i0 + k;
-    float x[4];
-    row_values(raw[k], bal, lane, x);
-    quantize_values_warp<BITS, GROUP>(x, (is_v ? a.v_codes : a.k_codes) + pos * (16 * BITS),
-                                      (is_v ? a.v_params : a.k_params) + pos * (kHeadDim / GROUP), lane);
-    if (!is_v && lane == 0) a.lo_tok[pos] = a.src_tok ? a.src_tok[(size_t)bh * a.n_src + r[k]] : r[k];
+  for (int off = 1; off < GL; off <<= 1) {
+    mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, off));
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
   }
+  const Eq1Params p = eq1_params<QMAX>(mn, mx);
+  uint32_t code[16];
+  bool redo = false;
+#pragma unroll
+  for (int e = 0; e < 16; ++e) code[e] = eq1_code_fast<QMAX>(x[e], p, redo);
+  if (redo) {
+#pragma unroll
+    for (int e = 0; e < 16; ++e) code[e] = eq1_code_exact<QMAX>(x[e], p);
+  }
+
+  const size_t pos = (size_t)bh * a.lo_cap + a.lo_start + i;
+  uint32_t* row = reinterpret_cast<uint32_t*>((is_v ? a.v_codes : a.k_codes) + pos * (16 * BITS));
+  if constexpr (BITS == 4) {
+    // channel 16 l8 + u: unit 16 (l8 >> 2) + u, bits 4 (l8 & 3); the lanes with equal l8 >> 2 share
+    // words 8 (l8 >> 2) .. + 7, and lane l8 ends with words 2 l8, 2 l8 + 1
+    const int sh = 4 * (l8 & 3);
+    uint32_t L[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) L[k] = (code[2 * k] << sh) | (code[2 * k + 1] << (16 + sh));
+    uint32_t K[2][4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const bool up = (l8 & 2) != 0;
+      K[0][k] = (up ? L[k + 4] : L[k]) | __shfl_xor_sync(0xffffffffu, up ? L[k] : L[k + 4], 2);
+    }
+    uint32_t out[2];
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+      const bool up = (l8 & 1) != 0;
+      out[k] = (up ? K[0][k + 2] : K[0][k]) | __shfl_xor_sync(0xffffffffu, up ? K[0][k] : K[0][k + 2], 1);
+    }
+    if (valid) *reinterpret_cast<uint2*>(row + 2 * l8) = make_uint2(out[0], out[1]);
+  } else {
+    // two-bit fields (INT2, and the low bits of INT3): channel 16 l8 + u sits in unit u at bits 2 l8;
+    // all eight lanes share words 0..7, and lane l8 ends with word l8
+    const int sh = 2 * l8;
+    uint32_t L[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) L[k] = ((code[2 * k] & 3u) << sh) | ((code[2 * k + 1] & 3u) << (16 + sh));
+    const uint32_t wd = reduce_scatter<8, 4>(L, l8);
+    if (valid) row[l8] = wd;
+    if constexpr (BITS == 3) {
+      // high bits: channel 16 l8 + u sits in unit u & 7 at bit 8 (u >> 3) + l8 (words 8..11 of the row);
+      // after two rounds a lane pair holds one word, and the pair's even lane stores it
+      uint32_t H[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+      for (int u = 0; u < 16; ++u) H[(u & 7) >> 1] |= (code[u] >> 2) << (16 * (u & 1) + 8 * (u >> 3) + l8);
+      uint32_t K[2];
+#pragma unroll
+      for (int k = 0; k < 2; ++k) {
+        const bool up = (l8 & 4) != 0;
+        K[k] = (up ? H[k + 2] : H[k]) | __shfl_xor_sync(0xffffffffu, up ? H[k] : H[k + 2], 4);
+      }
+      const bool up = (l8 & 2) != 0;
+      uint32_t hw = (up ? K[1] : K[0]) | __shfl_xor_sync(0xffffffffu, up ? K[0] : K[1], 2);
+      hw |= __shfl_xor_sync(0xffffffffu, hw, 1);
+      if (valid && (l8 & 1) == 0) row[8 + (l8 >> 1)] = hw;
+    }
+  }
+  if (valid && l8 % GL == 0)
+    ((is_v ? a.v_params : a.k_params) + pos * (kHeadDim / GROUP))[(16 * l8) / GROUP] =
+        __halves2half2(p.alpha16, p.beta16);
+  if (valid && !is_v && l8 == 0) a.lo_tok[pos] = a.src_tok ? a.src_tok[(size_t)bh * a.n_src + r] : r;
 }
 
 template <int BITS>
@@ -305,7 +413,7 @@ cudaError_t launch_quantize_pack(const mikv_shape& s, const mikv_cache& c, const
   a.n_rows = n_rows;
   a.lo_start = lo_start;
   a.lo_cap = s.lo_cap;
-  const dim3 grid((n_rows + 4 * kQpRows - 1) / (4 * kQpRows), s.batch * s.heads_kv);
+  const dim3 grid((n_rows + 4 * kQpRowsPerWarp - 1) / (4 * kQpRowsPerWarp), s.batch * s.heads_kv);
   switch (s.bits) {
     case 2: return qp_group<2>(a, s.group, grid, st);
     case 3: return qp_group<3>(a, s.group, grid, st);

@@ -52,6 +52,48 @@ __device__ __forceinline__ void pack_fields(const uint32_t (&code)[4], uint32_t*
   if ((lane & R) == 0) *reinterpret_cast<uint2*>(row + word0) = make_uint2(w0, w1);
 }
 
+// Eq. 1 scale and zero of a group with minimum mn and maximum mx: beta = min, alpha = (max - min) /
+// (2^N - 1), stored in fp16 with outward rounding (beta down, alpha up) so the stored grid covers the
+// group; a group with zero span gets alpha = 1 (every code 0). Also the fp32 values of the stored pair
+// and the IEEE reciprocal of alpha.
+struct Eq1Params {
+  __half alpha16, beta16;
+  float alpha, beta, ralpha;
+};
+
+template <int QMAX>
+__device__ __forceinline__ Eq1Params eq1_params(float mn, float mx) {
+  Eq1Params p;
+  p.beta16 = __float2half_rd(mn);
+  p.beta = __half2float(p.beta16);
+  const float span = __fsub_rn(mx, p.beta);
+  p.alpha16 = span == 0.f ? __float2half_rn(1.f) : __float2half_ru(__fdiv_rn(span, (float)QMAX));
+  p.alpha = __half2float(p.alpha16);
+  p.ralpha = __frcp_rn(p.alpha);
+  return p;
+}
+
+// Eq. 1 code of x: round-half-even of the IEEE quotient (x - beta) / alpha, clamped to [0, QMAX].
+// eq1_code_fast takes the product (x - beta) * (1 / alpha) (both factors IEEE-rounded), which lies within
+// 2^-15 of the true quotient for quotients below 256 while the IEEE quotient lies within 2^-17 of it, and
+// rounds it half to even by adding 2^23 (the fp32 sum is an integer; its low mantissa bits are the code).
+// The two agree unless the product is within 2^-13 of a half-integer (or not finite): such elements set
+// `redo`, and eq1_code_exact decides them with the division.
+template <int QMAX>
+__device__ __forceinline__ uint32_t eq1_code_fast(float x, const Eq1Params& p, bool& redo) {
+  const float q = __fmul_rn(__fsub_rn(x, p.beta), p.ralpha);
+  const float y = __fadd_rn(q, 8388608.f);
+  const float fr = __fsub_rn(q, __fsub_rn(y, 8388608.f));  // q - rint(q), exact
+  redo |= !(fabsf(fr) < 0.5f - 0x1p-13f);
+  return min(__float_as_uint(y) - 0x4B000000u, (uint32_t)QMAX);
+}
+
+template <int QMAX>
+__device__ __forceinline__ uint32_t eq1_code_exact(float x, const Eq1Params& p) {
+  const int c = __float2int_rn(__fdiv_rn(__fsub_rn(x, p.beta), p.alpha));
+  return (uint32_t)(c < 0 ? 0 : (c > QMAX ? QMAX : c));
+}
+
 // Quantize one row (Eq. 1) held as fp32 values x[4] of channels 4 lane .. 4 lane + 3 of each lane, with
 // one warp. Writes 16 * BITS bytes of packed codes to `codes` (8-byte aligned) and 128 / GROUP
 // (alpha, beta) fp16 pairs to `params`. Every rounding is explicit (fsub/fdiv round-to-nearest, fp16
@@ -69,26 +111,14 @@ __device__ __forceinline__ void quantize_values_warp(const float (&x)[4], uint8_
     mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, off));
     mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
   }
-  // Eq. 1: beta = min, alpha = (max - min) / (2^N - 1), stored in fp16 with outward rounding.
-  const __half beta16 = __float2half_rd(mn);
-  const float beta = __half2float(beta16);
-  const float span = __fsub_rn(mx, beta);
-  const __half alpha16 = span == 0.f ? __float2half_rn(1.f) : __float2half_ru(__fdiv_rn(span, (float)QMAX));
-  const float alpha = __half2float(alpha16);
-  // Codes: round-half-even of the IEEE quotient d / alpha, d = x - beta (>= 0, below about 256 alpha).
-  // The product d * (1 / alpha), both factors IEEE-rounded, lies within 2^-15 of d / alpha and the IEEE
-  // quotient within 2^-17 of it, so the two round to the same integer unless the product is within
-  // 2^-13 of a half-integer; only those (rare) elements take the division. Infinities and NaN pass the
-  // product through as the division would give them.
-  const float ralpha = __frcp_rn(alpha);
+  const Eq1Params p = eq1_params<QMAX>(mn, mx);
   uint32_t code[4];
+  bool redo = false;
 #pragma unroll
-  for (int e = 0; e < 4; ++e) {
-    const float d = __fsub_rn(x[e], beta);
-    float q = __fmul_rn(d, ralpha);
-    if (fabsf(fabsf(q - rintf(q)) - 0.5f) < 0x1p-13f) q = __fdiv_rn(d, alpha);
-    const int c = __float2int_rn(q);
-    code[e] = (uint32_t)(c < 0 ? 0 : (c > QMAX ? QMAX : c));
+  for (int e = 0; e < 4; ++e) code[e] = eq1_code_fast<QMAX>(x[e], p, redo);
+  if (redo) {
+#pragma unroll
+    for (int e = 0; e < 4; ++e) code[e] = eq1_code_exact<QMAX>(x[e], p);
   }
   uint32_t* row = reinterpret_cast<uint32_t*>(codes);
   if constexpr (BITS == 3) {
@@ -99,7 +129,7 @@ __device__ __forceinline__ void quantize_values_warp(const float (&x)[4], uint8_
   } else {
     pack_fields<BITS>(code, row, lane);
   }
-  if ((lane & (LANES - 1)) == 0) params[(4 * lane) / GROUP] = __halves2half2(alpha16, beta16);
+  if ((lane & (LANES - 1)) == 0) params[(4 * lane) / GROUP] = __halves2half2(p.alpha16, p.beta16);
 }
 
 // Channels 4 lane .. 4 lane + 3 of a bf16 row (8 bytes, `raw`) as fp32, times the key balancer `bal`

@@ -115,6 +115,9 @@ def test_argument_validation_before_launch(lib):
     P = 0x10000
     # retained capacity: lo_start + n_rows > lo_cap
     assert lib.mikv_quantize_pack(ctypes.byref(s), ctypes.byref(c), P, P, None, 4, P, 5, 60, None) == 3
+    # source rows are read in 16-byte pieces: both sources 16-byte aligned
+    assert lib.mikv_quantize_pack(ctypes.byref(s), ctypes.byref(c), P + 8, P, None, 4, P, 1, 0, None) == 1
+    assert lib.mikv_quantize_pack(ctypes.byref(s), ctypes.byref(c), P, P + 8, None, 4, P, 1, 0, None) == 1
     # null cache member
     bad = pkg._Cache(*([P] * 8 + [None, None, None, None]))
     assert lib.mikv_quantize_pack(ctypes.byref(s), ctypes.byref(bad), P, P, None, 4, P, 1, 0, None) == 1
