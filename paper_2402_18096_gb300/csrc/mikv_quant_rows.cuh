@@ -1,7 +1,8 @@
-// mikv_quant_rows.cuh — Eq. 1 quantization of one 128-channel row into the packed retained layout
-// (group-wise asymmetric codes with fp16 scale and zero, keys times the Eq. 3 balancer), and the fp32
-// dequantization of a coded important row (Sec. 3.3), one warp per row: shared by the standalone
-// quantize kernels and the fused step tail, so both produce the same bits.
+// mikv_quant_rows.cuh — Eq. 1 quantization into the packed retained layout (group-wise asymmetric codes
+// with fp16 scale and zero, keys times the Eq. 3 balancer): the scale / zero / code helpers every
+// quantizer uses (so the bulk kernel, the fused step tail and the coded important set produce the same
+// bits), the one-warp-per-row quantizer of a single 128-channel row, and the fp32 dequantization of a
+// coded important row (Sec. 3.3).
 #pragma once
 
 #include "mikv_device.cuh"
