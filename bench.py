@@ -332,7 +332,7 @@ def run_mikv(args):
     }
     if clk:
         line["clocks"] = clk
-    if rank == 0 and not args.no_cpu_baseline:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:  # the host baseline is an N = 1 figure
         line["cpu_baseline"] = cpu_baseline(w, seconds=args.cpu_seconds)
     if rank == 0:
         print(json.dumps(line), flush=True)
@@ -397,12 +397,10 @@ def _head_bytes(w, n_lo):
     return w.hi_cap * hi + n_lo * lo
 
 
-def cpu_baseline(w, seconds: float = 15.0, steps=None):
-    """The oracle, as it stands, on a bounded sample: whole decode steps of single KV heads."""
-    import oracle
-    oracle.build()
+def _oracle_steps(w, c, bal, slots, seconds: float, steps=None):
+    """Whole decode steps of one KV head on the oracle until `seconds` of oracle time (or `steps` steps)
+    have passed; returns (compressed bytes attended, oracle seconds, steps). Input generation is untimed."""
     G = w.heads_q // w.heads_kv
-    c, bal, slots = _oracle_head(w, 0, 0, 64)
     n_lo = w.n_lo0
     done_bytes, elapsed, n = 0, 0.0, 0
     while (steps is None and elapsed < seconds) or (steps is not None and n < steps):
@@ -417,10 +415,92 @@ def cpu_baseline(w, seconds: float = 15.0, steps=None):
         n += 1
         if n_lo >= c["k_codes"].shape[2]:
             break
-    return {"value": round(done_bytes / elapsed / 1e9, 4), "unit": UNIT, "cores": 1, "kind": "oracle",
+    return done_bytes, elapsed, n
+
+
+def _oracle_core(w, c, bal, slots, seconds, ready, start, out):
+    """One host core of the all-cores sample: the single-core sample's steps on its own copy of the head."""
+    torch.set_num_threads(1)
+    try:
+        import oracle  # noqa: F401  (built by the parent)
+        ready.put(os.getpid())
+        if not start.wait(timeout=600):
+            out.put(None)
+            return
+        out.put(_oracle_steps(w, c, bal, slots, seconds))
+    except Exception as e:  # reported to the parent, which then leaves the all-cores figure out
+        out.put(repr(e))
+
+
+def _all_cores(w, c, bal, slots, seconds: float):
+    """The same single-head decode steps on every host core at once (one spawned process per core, each on
+    its own copy of the head's cache, started together): the sum of the per-core rates, or None with the
+    reason if the processes cannot be run."""
+    import multiprocessing as mp
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else (os.cpu_count() or 1)
+    if cores < 2:
+        return None, "one host core"
+    ctx = mp.get_context("spawn")  # a fresh interpreter per core: nothing inherited from the CUDA parent
+    ready, out, start = ctx.Queue(), ctx.Queue(), ctx.Event()
+    procs = [ctx.Process(target=_oracle_core, args=(w, c, bal, slots, seconds, ready, start, out), daemon=True)
+             for _ in range(cores)]
+    def collect(q, n, deadline):  # n items from q, giving up at the deadline or when a process died
+        got = []
+        while len(got) < n:
+            if time.time() > deadline:
+                raise TimeoutError("host-core processes did not answer in time")
+            try:
+                got.append(q.get(timeout=1.0))
+            except Exception:
+                if any(p.exitcode not in (None, 0) for p in procs):
+                    raise RuntimeError("a host-core process exited early")
+        return got
+
+    try:
+        for p in procs:
+            p.start()
+        collect(ready, len(procs), time.time() + 180)
+        start.set()
+        res = collect(out, len(procs), time.time() + seconds + 120)
+    except Exception as e:
+        return None, repr(e)
+    finally:
+        for p in procs:
+            p.join(timeout=30)
+            if p.is_alive():
+                p.kill()
+    bad = [r for r in res if not isinstance(r, tuple)]
+    if bad:
+        return None, str(bad[0])
+    rate = sum(b / t for b, t, _ in res if t > 0)
+    return {"value": round(rate / 1e9, 4), "cores": cores, "steps": sum(n for _, _, n in res)}, None
+
+
+def cpu_baseline(w, seconds: float = 15.0, steps=None, all_cores: bool = True):
+    """The oracle, as it stands, on a bounded sample: whole decode steps of single KV heads, first on one
+    core, then on every host core at once (one process per core). `value` is the all-cores rate when it
+    could be measured, else the single-core rate."""
+    import oracle
+    oracle.build()
+    c, bal, slots = _oracle_head(w, 0, 0, 64)
+    c0 = {k: a.copy() for k, a in c.items()}  # the single-core run advances its copy of the cache
+    s0 = slots.copy()
+    done_bytes, elapsed, n = _oracle_steps(w, c, bal, slots, seconds, steps)
+    single = done_bytes / elapsed / 1e9
+    line = {"value": round(single, 4), "unit": UNIT, "cores": 1, "kind": "oracle",
             "sample": f"{n} whole decode steps of one KV head (batch row 0, head 0, layer 0) of {w.name}; "
                       f"single-threaded C, fp64 attention; bytes = that head's compressed KV",
-            "ms_per_head_step": round(1e3 * elapsed / n, 3)}
+            "ms_per_head_step": round(1e3 * elapsed / n, 3), "single_core_value": round(single, 4)}
+    if all_cores:
+        par, why = _all_cores(w, c0, bal, s0, seconds / 2)
+        if par:
+            line.update(value=par["value"], cores=par["cores"])
+            line["sample"] = (f"the same single-head decode steps on {par['cores']} host cores at once (one "
+                              f"process per core, {par['steps']} steps in all, about {seconds / 2:.0f} s of oracle "
+                              f"time each; sum of the per-core rates), after {n} steps on one core")
+        else:
+            line["all_cores_unavailable"] = why
+    return line
 
 
 def run_sweep(args):
