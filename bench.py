@@ -36,11 +36,13 @@ import mikv_inputs as mi  # noqa: E402
 METRIC = "decode-attn compressed-KV GB/s and % of GB300 HBM peak; us per decode step"
 UNIT = "GB/s"
 DEFAULT_WORKLOAD = "mistral-7b"
+L2_BYTES = 129 * 10 ** 6          # GB300 L2
+L2_FLUSH_BYTES = 512 << 20        # a write this large evicts every cache line of L2
 
 
 ATTN_SOURCES = ["mikv_attention.cuh", "mikv_attention.cu", "mikv_attn_h16.cu", "mikv_device.cuh", "mikv_internal.h",
                 "mikv_rows.cuh"]
-TRAFFIC_SUMMARY = os.path.join(ROOT, "profiles", "attention_kernel_mistral7b_b4.md")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "attention_traffic.json")
 
 
 def attention_source_sha256() -> str:
@@ -52,23 +54,33 @@ def attention_source_sha256() -> str:
     return h.hexdigest()
 
 
-def profiled_traffic_ratio():
-    """DRAM bytes per algorithmic byte of the attention kernel, from the committed ncu summary, if it was
-    taken on the current kernel sources (else None: counters of another kernel do not apply)."""
-    if not os.path.exists(TRAFFIC_SUMMARY):
+def profiled_traffic_ratio(workload: str):
+    """DRAM bytes (read + write) per algorithmic byte of the attention kernel on `workload`, from the
+    committed ncu figures (profiles/attention_traffic.json), if they were taken on this workload and on the
+    current kernel sources; else None (counters of another kernel or shape do not apply)."""
+    if not os.path.exists(TRAFFIC_FILE):
         return None
-    vals = {}
-    with open(TRAFFIC_SUMMARY) as f:
-        for line in f:
-            if ":" in line and line.strip().startswith("- `"):
-                k, v = line.strip()[3:].split("`", 1)
-                vals[k] = v.split(":", 1)[1].strip()
     try:
-        if vals.get("kernel_source_sha256") != attention_source_sha256():
+        with open(TRAFFIC_FILE) as f:
+            d = json.load(f)
+        if d.get("kernel_source_sha256") != attention_source_sha256() or workload not in d.get("workloads", []):
             return None
-        return float(vals["dram_bytes_per_algorithmic_byte"])
-    except (KeyError, ValueError):
+        return float(d["dram_bytes_per_algorithmic_byte"])
+    except (OSError, KeyError, ValueError, TypeError):
         return None
+
+
+def timed_with_flush(fn, n: int, scrub: torch.Tensor, stream) -> float:
+    """Milliseconds of n calls fn(i), each timed alone with CUDA events on `stream` after a write of
+    `scrub` (larger than L2) has evicted whatever the previous call left in L2."""
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
+    for i in range(n):
+        scrub.add_(1)
+        evs[i][0].record(stream)
+        fn(i)
+        evs[i][1].record(stream)
+    torch.cuda.synchronize()
+    return sum(a.elapsed_time(b) for a, b in evs)
 
 
 def _peaks():
@@ -163,8 +175,8 @@ def build_model(w, steps_cap: int, dev, rank: int):
     """All layers' caches, built from seeded prefill tensors with the library's own kernels."""
     import paper_2402_18096_gb300 as pkg
     from paper_2402_18096_gb300.layer import MixedPrecisionLayer
-    shape = pkg.Shape(w.batch, w.heads_q, w.heads_kv, w.bits, w.group, w.hi_cap, w.lo_cap_for(steps_cap),
-                      hi_bits=w.hi_bits, k_channel_group=64 if w.k_channel else 0)
+    shape = pkg.shape_for_context(w.batch, w.heads_q, w.heads_kv, w.bits, w.group, w.context, w.ratio, steps_cap,
+                                  hi_bits=w.hi_bits, k_channel_group=64 if w.k_channel else 0)
     wr = rank_workload(w, rank)  # each rank owns a different batch
     layers, ms, in_bytes = [], [], 0
     for li in range(w.layers):
@@ -226,18 +238,25 @@ def run_mikv(args):
         pkg.mikv_workspace_check(layer.ws)
 
     n_lo_before = [layer.n_lo for layer in layers]
+    # a cache that L2 would hold between steps is timed step by step after an L2 flush
+    cache_total = sum(layer.cache.nbytes_attended(layer.n_lo) for layer in layers)
+    scrub = torch.zeros(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev) if cache_total < 2 * L2_BYTES else None
     clocks = ClockSampler(torch.cuda.current_device()) if rank == 0 else None
     if clocks:
         clocks.start()
     if dist:
         dist.barrier()
     torch.cuda.synchronize()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for s in range(K):
-        step(W + s)
-    e1.record(stream)
-    torch.cuda.synchronize()
+    if scrub is None:
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for s in range(K):
+            step(W + s)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        step_ms = e0.elapsed_time(e1)
+    else:  # a cache that fits in L2: every timed step starts from a flushed L2 (the flush is not timed)
+        step_ms = timed_with_flush(lambda s: step(W + s), K, scrub, stream)
     if dist:
         dist.barrier()
     clk = clocks.stop() if clocks else None
@@ -247,7 +266,7 @@ def run_mikv(args):
                          for s in range(K)) / K
     # per-channel keys: a step whose demotion completes a group of 64 adds one quantization launch per layer
     kch_launches = sum(1 for n0 in n_lo_before for s in range(K) if w.k_channel and (n0 + s) % 64 == 63)
-    ms = e0.elapsed_time(e1) / K
+    ms = step_ms / K
     ms = max_over_ranks(dist, ms)
     for layer in layers:
         pkg.mikv_workspace_check(layer.ws)
@@ -256,15 +275,21 @@ def run_mikv(args):
     ws_attn = [torch.zeros(pkg.mikv_workspace_bytes(shape, pkg.WS_ATTENTION, layer.n_lo) + 256, dtype=torch.uint8,
                            device=dev) for layer in layers[:1]]
     q0 = inputs[0][0][0]
-    a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    torch.cuda.synchronize()
-    a0.record(stream)
-    for _ in range(attn_reps):
+    def attend_all(_=None):
         for layer in layers:
             pkg.mikv_decode_attention(layer.cache, layer.n_lo, q0, layer.sm_scale, out, ws_attn[0])
-    a1.record(stream)
+
     torch.cuda.synchronize()
-    attn_ms = a0.elapsed_time(a1) / (attn_reps * L)
+    if scrub is None:
+        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        for _ in range(attn_reps):
+            attend_all()
+        a1.record(stream)
+        torch.cuda.synchronize()
+        attn_ms = a0.elapsed_time(a1) / (attn_reps * L)
+    else:
+        attn_ms = timed_with_flush(attend_all, max(attn_reps, K), scrub, stream) / (max(attn_reps, K) * L)
     attn_bytes = sum(layer.cache.nbytes_attended(layer.n_lo) for layer in layers) / L
 
     # ---- end to end through the C ABI with host buffers: H2D inputs, D2H outputs, every step
@@ -282,20 +307,25 @@ def run_mikv(args):
     torch.cuda.synchronize()
     if dist:
         dist.barrier()
-    t0 = time.perf_counter()
+    e2e_s = 0.0
     for s in range(e2e_steps):
+        if scrub is not None:  # flushed L2 before every step, outside the timed span
+            scrub.add_(1)
+            torch.cuda.current_stream().synchronize()
+        t0 = time.perf_counter()
         dev_flat.copy_(host_flat, non_blocking=True)
         for li, layer in enumerate(layers):
             layer.step(dev_in[li][0], dev_in[li][1], dev_in[li][2], dev_out[li])
         host_out.copy_(dev_out, non_blocking=True)
         torch.cuda.current_stream().synchronize()
-    e2e_ms = (time.perf_counter() - t0) * 1e3 / e2e_steps
+        e2e_s += time.perf_counter() - t0
+    e2e_ms = e2e_s * 1e3 / e2e_steps
     e2e_ms = max_over_ranks(dist, e2e_ms)
     for layer in layers:
         pkg.mikv_workspace_check(layer.ws)
 
     peak, peak_kind = _peaks()
-    ratio = profiled_traffic_ratio()
+    ratio = profiled_traffic_ratio(w.name)
     traffic = None if ratio is None else int(ratio * attn_bytes)
     value = world * bytes_per_step / (ms * 1e-3) / 1e9
     achieved = attn_bytes / (attn_ms * 1e-3) / 1e9
@@ -318,7 +348,9 @@ def run_mikv(args):
         "data": "synthetic",
         "config": {"workload": w.name, "batch": w.batch, "layers": L, "heads_q": w.heads_q, "heads_kv": w.heads_kv,
                    "context": w.context, "bits": w.bits, "group": w.group, "importance_ratio": w.ratio,
-                   "compressed_bytes_per_step": int(bytes_per_step), "l2": "cache larger than L2, no flush",
+                   "compressed_bytes_per_step": int(bytes_per_step), "l2": ("cache larger than L2, no flush" if scrub is None else
+                         f"cache smaller than L2: L2 flushed by a {L2_FLUSH_BYTES >> 20} MiB write before every "
+                         "timed step and launch (not timed); per-step CUDA events summed"),
                    "parallelism": f"replicas{world}"},
         "roofline": {"kernel": "decode attention (split-K + merge)", "bound": "hbm", "achieved": round(achieved, 1),
                      "peak": peak, "unit": "GB/s", "frac": round(achieved / peak, 3),
@@ -357,17 +389,23 @@ def _oracle_head(w, b, h, steps_cap):
     ks, vs = mi.bf16_bits(k[b:b + 1]), mi.bf16_bits(v[b:b + 1])
     sc = scores.numpy()
     del k, v, q_pre
-    dem, kept = oracle.select_demote(sc, w.context - w.budget)
+    k_b = oracle.budget(w.context, w.ratio)  # the oracle's own importance-ratio rule
+    lo_cap = _lo_cap(w.context - k_b + steps_cap, w.k_channel)
+    dem, kept = oracle.select_demote(sc, w.context - k_b)
     if w.k_channel:  # per-channel retained keys: no balancer, the last incomplete group staged in bf16
-        c = oracle.empty_cache(1, 1, w.head_dim, w.bits, w.group, w.hi_cap, w.lo_cap_for(steps_cap), k_channel=True)
+        c = oracle.empty_cache(1, 1, w.head_dim, w.bits, w.group, k_b + 1, lo_cap, k_channel=True)
         oracle.gather_hi(c, ks, vs, kept, src_scores=sc)
         oracle.append_retained(c, ks, vs, dem, 0)
     else:
-        c = oracle.empty_cache(1, 1, w.head_dim, w.bits, w.group, w.hi_cap, w.lo_cap_for(steps_cap),
-                               hi_bits=w.hi_bits)
+        c = oracle.empty_cache(1, 1, w.head_dim, w.bits, w.group, k_b + 1, lo_cap, hi_bits=w.hi_bits)
         oracle.gather_hi(c, ks, vs, kept, src_scores=sc, balancer_=bal)
         oracle.quantize_pack(c, ks, vs, dem, 0, balancer_=bal)
-    return c, bal, np.array([[w.budget]], np.int32)
+    return c, bal, np.array([[k_b]], np.int32)
+
+
+def _lo_cap(rows: int, k_channel: bool) -> int:
+    q = 64 if k_channel else 16
+    return max(q, (rows + q - 1) // q * q)
 
 
 def _oracle_step(w, c, bal, slots, n_lo, pos, q, kn, vn):
@@ -377,7 +415,7 @@ def _oracle_step(w, c, bal, slots, n_lo, pos, q, kn, vn):
     G = w.heads_q // w.heads_kv
     oracle.insert_token(c, kn, vn, pos, slots, balancer_=bal)
     _, hl, ml = oracle.decode_attention(c, q, n_lo, 1 / math.sqrt(w.head_dim), balancer_=bal)
-    hc = w.hi_cap
+    hc = oracle.budget(w.context, w.ratio) + 1
     acc = oracle.update_importance(c["acc"][:, :, :hc], hl[:, :, :hc].astype(np.float32), ml.astype(np.float32), G)
     c["acc"][:, :, :hc] = acc
     dem, _ = oracle.select_demote(acc, 1, c["hi_tok"][:, :, :hc], want_kept=False)
@@ -389,19 +427,22 @@ def _oracle_step(w, c, bal, slots, n_lo, pos, q, kn, vn):
 
 
 def _head_bytes(w, n_lo):
+    import oracle
+    hi_cap = oracle.budget(w.context, w.ratio) + 1
     lo = 2 * (w.head_dim * w.bits // 8 + 4 * (w.head_dim // w.group))
     if w.k_channel:  # keys: codes per token, (alpha, beta) per channel and 64 tokens; staged rows in bf16
         lo = 2 * w.head_dim * w.bits // 8 + 4 * (w.head_dim // w.group) + 4 * w.head_dim // 64
-        return w.hi_cap * 4 * w.head_dim + (n_lo // 64 * 64) * lo + (n_lo % 64) * 4 * w.head_dim
+        return hi_cap * 4 * w.head_dim + (n_lo // 64 * 64) * lo + (n_lo % 64) * 4 * w.head_dim
     hi = 4 * w.head_dim if w.hi_bits >= 16 else 2 * (w.head_dim * w.hi_bits // 8 + 4 * (w.head_dim // 64))
-    return w.hi_cap * hi + n_lo * lo
+    return hi_cap * hi + n_lo * lo
 
 
 def _oracle_steps(w, c, bal, slots, seconds: float, steps=None):
     """Whole decode steps of one KV head on the oracle until `seconds` of oracle time (or `steps` steps)
     have passed; returns (compressed bytes attended, oracle seconds, steps). Input generation is untimed."""
     G = w.heads_q // w.heads_kv
-    n_lo = w.n_lo0
+    import oracle
+    n_lo = w.context - oracle.budget(w.context, w.ratio)
     done_bytes, elapsed, n = 0, 0.0, 0
     while (steps is None and elapsed < seconds) or (steps is not None and n < steps):
         q, kn, vn = mi.decode_inputs(w, 0, n, "cpu", rows=[0], kv_heads=[0])
@@ -514,8 +555,8 @@ def run_sweep(args):
     points = []
     for w in mi.sweep_workloads():
         K, W = args.steps, args.warmup
-        shape = pkg.Shape(w.batch, w.heads_q, w.heads_kv, w.bits, w.group, w.hi_cap, w.lo_cap_for(K + W + 4),
-                          hi_bits=w.hi_bits)
+        shape = pkg.shape_for_context(w.batch, w.heads_q, w.heads_kv, w.bits, w.group, w.context, w.ratio, K + W + 4,
+                                      hi_bits=w.hi_bits)
         k, v = mi.prefill_kv(w, 0, dev)
         sc = mi.initial_scores(w, 0, dev)
         qp = mi.prefill_queries(w, 0, dev)
@@ -569,7 +610,7 @@ def run_reference(args):
     oracle.build()
     G = w.heads_q // w.heads_kv
     c, bal, slots = _oracle_head(w, 0, 0, W + K + 4)
-    n_lo = w.n_lo0
+    n_lo = w.context - oracle.budget(w.context, w.ratio)
     times, nbytes = [], []
     for s in range(W + K):
         q, kn, vn = mi.decode_inputs(w, 0, s, "cpu", rows=[0], kv_heads=[0])

@@ -273,20 +273,27 @@ mikv_status mikv_decode_step(const mikv_shape* shape, const mikv_cache* cache, i
  * workspace, and keeps its split partials in a scratch buffer that the library itself declares as a
  * fixed-size device array of MIKV_NOALLOC_SCRATCH_BYTES bytes. Every GPU that loads the library holds
  * that buffer until the process exits.
- *   - The first call on a device looks up the buffer's device address (cudaGetSymbolAddress) with that
- *     device current; make that first call before any stream capture.
+ *   - Every call looks up the buffer's device address in the current context (cudaGetSymbolAddress,
+ *     which allocates nothing). The first call on a device (in a context) also loads the library's device
+ *     code there: make that first call before any stream capture.
  *   - The call itself allocates nothing and frees nothing; it zeroes the buffer's status word on
  *     `stream` before launching.
- *   - All calls share the one buffer: calls that can overlap on the GPU (different streams without
- *     ordering between them) race on it and must not be issued.
+ *   - All calls share the one buffer, which keeps the last call's contents: calls that can overlap on
+ *     the GPU (different streams without ordering between them) race on it and must not be issued.
  *   - A problem whose scratch (mikv_workspace_bytes(shape, MIKV_WS_ATTENTION, n_lo)) exceeds the
  *     buffer returns MIKV_ERR_SCRATCH and launches nothing.
- *   - A kernel-side failure is recorded in the buffer's status word only; it is not reported here.
+ *   - A kernel-side failure (a wait that ran out of its time limit) is recorded in the buffer's status
+ *     word, not in the return code (the call returns before the kernels run): mikv_noalloc_check reads it.
  */
 #define MIKV_NOALLOC_SCRATCH_BYTES (8u << 20)
 mikv_status mikv_decode_attention_noalloc(const mikv_shape* shape, const mikv_cache* cache, int32_t n_lo,
                                           const void* q, float sm_scale, void* out, int32_t out_dtype,
                                           float* hi_logits, float* ml, void* stream);
+
+/* Status of the built-in buffer of mikv_decode_attention_noalloc: synchronises `stream`, reads the buffer's
+ * status word (left by the last mikv_decode_attention_noalloc call, which zeroed it first) and returns
+ * MIKV_ERR_DEVICE if a kernel reported a failure, else MIKV_OK. Allocates nothing. */
+mikv_status mikv_noalloc_check(void* stream);
 
 /*
  * KV-cache size as a fraction of an all-fp16 cache (the "Cache size" columns of Tables 2-3): a ratio
@@ -296,6 +303,16 @@ mikv_status mikv_decode_attention_noalloc(const mikv_shape* shape, const mikv_ca
  * Host-only, pure.
  */
 double mikv_cache_fraction(int32_t bits, int32_t group, double ratio, int32_t hi_bits);
+
+/*
+ * Important-set budget from the importance ratio (the "Importance ratio" column of Tables 1-3: the share
+ * of tokens kept in high precision): k = floor(ratio * T + 0.5), the ratio times the context length
+ * rounded half up, evaluated in IEEE double arithmetic. A cache built for context T keeps k important
+ * tokens and attends hi_cap = k + 1 important slots (one staging slot receives each decoded token before
+ * the step's demotion frees a slot again). Returns -1 for T < 0 or a ratio outside [0, 1] (NaN included).
+ * Host-only, pure.
+ */
+int32_t mikv_budget(int32_t T, double ratio);
 
 /* Bytes of one retained row (codes + parameters, K or V) and of one important row (K or V). */
 size_t mikv_retained_row_bytes(int32_t bits, int32_t group, int32_t head_dim);

@@ -34,33 +34,12 @@ class Workload:
     layers: int
     bits: int             # retained-set code width (0: no retained set, the H2O eviction baseline)
     group: int            # channels per quantization group
-    ratio: float          # fraction of tokens kept in bf16 (importance ratio)
+    ratio: float          # fraction of tokens kept in bf16 (importance ratio; each side turns it into a
+                          # token count with its own budget function)
     seed: int = 0
     head_dim: int = HEAD_DIM
     hi_bits: int = 16     # important-set precision: 16 = bf16, or 8 / 4 / 2-bit codes in groups of 64
     k_channel: bool = False  # retained keys per channel over groups of 64 tokens (App. C)
-
-    @property
-    def budget(self) -> int:
-        """k, the number of important tokens: ratio * T rounded half up."""
-        return int(self.ratio * self.context + 0.5)
-
-    @property
-    def hi_cap(self) -> int:
-        return self.budget + 1  # plus one staging slot for the incoming token
-
-    @property
-    def hi_stride(self) -> int:
-        return (self.hi_cap + 15) // 16 * 16
-
-    @property
-    def n_lo0(self) -> int:
-        """Retained rows after the cache build."""
-        return self.context - self.budget
-
-    def lo_cap_for(self, steps: int) -> int:
-        q = 64 if self.k_channel else 16
-        return max(q, (self.n_lo0 + steps + q - 1) // q * q)
 
 
 WORKLOADS = {
@@ -97,6 +76,11 @@ def sweep_workloads() -> List[Workload]:
                 out.append(Workload(f"sweep-b64-h32-t4096-int{bits}-g{group}-r{int(ratio * 100)}", 64, 32,
                                     32, 4096, 1, bits, group, ratio))
     return out
+
+
+# every sweep point under its own short name (e.g. "sweep-int3-g128-r0"), so one point can be run alone
+for _w in sweep_workloads():
+    WORKLOADS[f"sweep-int{_w.bits}-g{_w.group}-r{int(_w.ratio * 100)}"] = _w
 
 
 def scaled(w: Workload, **kw) -> Workload:

@@ -73,6 +73,7 @@ def _load():
                 "mikv_ref_insert_token": (I, [I, I, I, I, P, P, I, P, P, P, P, P]),
                 "mikv_ref_gather_hi": (I, [I, I, I, I, P, P, P, P, I, P, I, P, P, P, P]),
                 "mikv_ref_cache_fraction": (D, [I, I, D, I]),
+                "mikv_ref_budget": (I, [I, D]),
                 "mikv_ref_dequantize_row_f32": (I, [P, P, I, I, I, P]),
                 "mikv_ref_prefill_scores": (I, [I, I, I, I, I, P, P, D, P]),
                 "mikv_ref_quantize_channel_group": (I, [P, I, I, P, P]),
@@ -422,6 +423,15 @@ def prefill_scores(q_pre, k_pre, sm_scale: float):
 
 def cache_fraction(bits: int, g: int, ratio: float, hi_bits: int = 16) -> float:
     return float(_load().mikv_ref_cache_fraction(bits, g, ratio, hi_bits))
+
+
+def budget(T: int, ratio: float) -> int:
+    """Important tokens for importance ratio `ratio` over T tokens (Tables 1-3): nearest integer to
+    ratio * T, halves up (reading R10)."""
+    k = int(_load().mikv_ref_budget(int(T), float(ratio)))
+    if k < 0:
+        raise ValueError(f"budget: invalid T={T} or ratio={ratio}")
+    return k
 
 
 def empty_cache(B: int, Hkv: int, d: int, bits: int, g: int, hi_cap: int, lo_cap: int, hi_bits: int = 16,

@@ -839,3 +839,18 @@ double mikv_ref_cache_fraction(int bits, int g, double ratio, int hi_bits) {
   double lo = (bits + 32.0 / g) / 16.0;
   return ratio * hi + (1.0 - ratio) * lo;
 }
+
+/* ---------------------------------------------------------------- importance budget */
+
+/*
+ * Tables 1-3 state the important set as a ratio of the tokens; the count is the ratio times the context
+ * length rounded to the nearest integer, a half rounded up (reading R10). Written as: take the whole part
+ * of the product, then add one when the remaining fraction is at least one half.
+ */
+int mikv_ref_budget(int T, double ratio) {
+  if (T < 0 || ratio != ratio || ratio < 0.0 || ratio > 1.0) return -1;
+  double x = ratio * (double)T;
+  int whole = (int)x; /* x >= 0: truncation is the floor */
+  if (x - (double)whole >= 0.5) whole += 1;
+  return whole;
+}

@@ -22,7 +22,8 @@ __all__ = [
     "mikv_workspace_reset", "mikv_workspace_check", "mikv_compute_balancer", "mikv_quantize_pack",
     "mikv_decode_attention", "mikv_update_importance", "mikv_select_demote", "mikv_insert_token",
     "mikv_gather_hi", "mikv_decode_step", "mikv_cache_fraction", "mikv_retained_row_bytes",
-    "mikv_decode_attention_noalloc", "NOALLOC_SCRATCH_BYTES", "mikv_prefill_scores",
+    "mikv_decode_attention_noalloc", "mikv_noalloc_check", "NOALLOC_SCRATCH_BYTES", "mikv_prefill_scores",
+    "mikv_budget", "shape_for_context",
     "WS_ATTENTION", "WS_BALANCER", "WS_STEP", "WS_PREFILL", "OUT_BF16", "OUT_F32", "HEAD_DIM",
 ]
 
@@ -84,6 +85,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
                 "mikv_gather_hi": (I, [SP, CP, P, P, P, P, I, P, I, P]),
                 "mikv_decode_step": (I, [SP, CP, I, P, P, P, I, P, F, P, I, P, Z, P]),
                 "mikv_decode_attention_noalloc": (I, [SP, CP, I, P, F, P, I, P, P, P]),
+                "mikv_noalloc_check": (I, [P]),
+                "mikv_budget": (I, [I, ctypes.c_double]),
                 "mikv_prefill_scores": (I, [SP, P, P, I, F, P, P, Z, P]),
                 "mikv_cache_fraction": (ctypes.c_double, [I, I, ctypes.c_double, I]),
                 "mikv_retained_row_bytes": (Z, [I, I, I]),
@@ -142,6 +145,18 @@ class Shape:
     def c(self) -> _Shape:
         return _Shape(self.batch, self.heads_q, self.heads_kv, self.head_dim, self.bits, self.group,
                       self.hi_cap, self.hi_stride, self.lo_cap, self.hi_bits, self.hi_group, self.k_channel_group)
+
+
+def shape_for_context(batch: int, heads_q: int, heads_kv: int, bits: int, group: int, context: int, ratio: float,
+                      steps: int, hi_bits: int = 16, k_channel_group: int = 0) -> Shape:
+    """Shape of a cache built from `context` prefill tokens with importance ratio `ratio`: k = mikv_budget(
+    context, ratio) important tokens (hi_cap = k + 1 slots) and room for the other context - k tokens plus
+    `steps` decode steps in the retained set (a multiple of 16 rows; of 64 with per-channel keys)."""
+    k = mikv_budget(context, ratio)
+    q = 64 if k_channel_group else 16
+    lo_cap = max(q, (context - k + steps + q - 1) // q * q)
+    return Shape(batch, heads_q, heads_kv, bits, group, k + 1, lo_cap, hi_bits=hi_bits,
+                 k_channel_group=k_channel_group)
 
 
 class LayerCache:
@@ -243,6 +258,12 @@ def mikv_decode_attention_noalloc(cache: LayerCache, n_lo: int, q, sm_scale: flo
         out_dtype, _ptr(hi_logits), _ptr(ml), _stream(stream)))
 
 
+def mikv_noalloc_check(stream=None):
+    """Raise MikvError(MIKV_ERR_DEVICE) if the last mikv_decode_attention_noalloc call's kernels reported a
+    failure in the built-in buffer's status word (synchronises the stream)."""
+    _check("mikv_noalloc_check", load().mikv_noalloc_check(_stream(stream)))
+
+
 def mikv_update_importance(cache: LayerCache, hi_logits, ml, stream=None):
     _check("mikv_update_importance", load().mikv_update_importance(
         ctypes.byref(cache.shape.c()), ctypes.byref(cache.c()), _ptr(hi_logits), _ptr(ml), _stream(stream)))
@@ -286,6 +307,15 @@ def mikv_prefill_scores(shape: Shape, q_pre, k_pre, scores, workspace, sm_scale:
 
 def mikv_cache_fraction(bits: int, group: int, ratio: float, hi_bits: int = 16) -> float:
     return float(load(build_if_missing=False).mikv_cache_fraction(bits, group, ratio, hi_bits))
+
+
+def mikv_budget(T: int, ratio: float) -> int:
+    """Important tokens k for importance ratio `ratio` over T tokens (Tables 1-3): floor(ratio * T + 0.5).
+    A cache for context T then attends hi_cap = k + 1 important slots."""
+    k = int(load(build_if_missing=False).mikv_budget(int(T), float(ratio)))
+    if k < 0:
+        raise ValueError(f"mikv_budget: invalid T={T} or ratio={ratio}")
+    return k
 
 
 def mikv_retained_row_bytes(bits: int, group: int, head_dim: int = HEAD_DIM) -> int:

@@ -1,8 +1,9 @@
 // mikv_abi.cu — host side of the libmikv C ABI (include/mikv.h): argument validation, tensor-map
 // encoding for TMA, workspace layout and kernel dispatch. Nothing here allocates device memory or
-// synchronises, except mikv_workspace_check which reads the status word on request.
+// synchronises, except mikv_workspace_check and mikv_noalloc_check, which read a status word on request.
 #include <cuda.h>
 #include <cuda_runtime.h>
+#include <math.h>
 #include <stdio.h>
 #include <string.h>
 
@@ -512,6 +513,11 @@ double mikv_cache_fraction(int32_t bits, int32_t group, double ratio, int32_t hi
   return ratio * hi + (1.0 - ratio) * lo;
 }
 
+int32_t mikv_budget(int32_t T, double ratio) {
+  if (T < 0 || !(ratio >= 0.0 && ratio <= 1.0)) return -1;
+  return (int32_t)floor(ratio * (double)T + 0.5);
+}
+
 size_t mikv_retained_row_bytes(int32_t bits, int32_t group, int32_t head_dim) {
   if (bits <= 0 || group <= 0 || head_dim <= 0 || head_dim % group) return 0;
   return (size_t)head_dim * bits / 8 + (size_t)4 * (head_dim / group);
@@ -531,23 +537,14 @@ namespace {
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[MIKV_NOALLOC_SCRATCH_BYTES];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_noalloc_mu;
-void* g_noalloc_ptr[kMaxDevices] = {};
-
-// Device address of the buffer on the current device, looked up once per device. The name of a
-// __device__ array in host code is only a host-side stand-in, so the address must come from the runtime.
+// Device address of the buffer in the current context. The name of a __device__ array in host code is only
+// a host-side stand-in, so the address must come from the runtime. It is looked up on every call (the lookup
+// allocates nothing): an address kept from an earlier call would dangle after cudaDeviceReset or when the
+// caller makes another context current. The first lookup in a context loads the library's device code there.
 mikv_status noalloc_scratch(void** out) {
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return MIKV_ERR_CUDA;
-  if (dev < 0 || dev >= kMaxDevices) return MIKV_ERR_UNSUPPORTED;
-  std::lock_guard<std::mutex> lock(g_noalloc_mu);
-  if (!g_noalloc_ptr[dev]) {
-    void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return MIKV_ERR_CUDA;
-    g_noalloc_ptr[dev] = p;
-  }
-  *out = g_noalloc_ptr[dev];
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return MIKV_ERR_CUDA;
+  *out = p;
   return MIKV_OK;
 }
 
@@ -566,4 +563,11 @@ extern "C" mikv_status mikv_decode_attention_noalloc(const mikv_shape* shape, co
   if (cudaMemsetAsync(ws, 0, sizeof(int), s) != cudaSuccess) return MIKV_ERR_CUDA;  // status word starts at 0
   return attention_impl(shape, cache, n_lo, q, sm_scale, out, out_dtype, hi_logits, ml, ws,
                         MIKV_NOALLOC_SCRATCH_BYTES, s);
+}
+
+extern "C" mikv_status mikv_noalloc_check(void* stream) {
+  void* ws = nullptr;
+  mikv_status st = noalloc_scratch(&ws);
+  if (st != MIKV_OK) return st;
+  return mikv_workspace_check(ws, stream);
 }

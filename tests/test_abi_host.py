@@ -153,3 +153,29 @@ def test_argument_validation_before_launch(lib):
                                 None) == 3
     # gather beyond the important capacity
     assert lib.mikv_gather_hi(ctypes.byref(s), ctypes.byref(c), P, P, None, None, 40, P, 21, None) == 3
+
+
+def test_budget_on_the_boundary_matches_oracle(lib):
+    """mikv_budget (the library's importance-ratio rule) against the oracle's independent budget function over
+    every workload, the sweep and a grid of ratios and lengths; invalid arguments give -1."""
+    import mikv_inputs as mi
+    cases = [(w.context, w.ratio) for w in mi.WORKLOADS.values()]
+    cases += [(T, r / 100) for T in (0, 1, 2, 3, 10, 257, 512, 611, 999, 4096, 8192, 32768) for r in range(101)]
+    for T, r in cases:
+        assert pkg.mikv_budget(T, r) == oracle.budget(T, r), (T, r)
+    for T, r in ((-1, 0.5), (10, -0.01), (10, 1.01), (10, float("nan"))):
+        assert lib.mikv_budget(T, r) == -1
+
+
+def test_shape_for_context_capacities(lib):
+    """The cache shape derived from a context and a ratio: hi_cap = budget + 1, hi_stride a multiple of 16, and
+    retained capacity for the rest of the context plus the requested steps (multiple of 16; 64 with per-channel
+    keys)."""
+    for T, r in ((32768, 0.2), (4096, 0.0), (100, 1.0), (611, 0.15)):
+        for steps in (0, 1, 17, 100):
+            for kcg in (0, 64):
+                s = pkg.shape_for_context(2, 8, 2, 2, 32, T, r, steps, k_channel_group=kcg)
+                k = oracle.budget(T, r)
+                assert s.hi_cap == k + 1 and s.hi_stride % 16 == 0 and s.hi_stride >= s.hi_cap + (64 if kcg else 0)
+                q = 64 if kcg else 16
+                assert s.lo_cap % q == 0 and s.lo_cap >= T - k + steps and s.lo_cap >= q

@@ -14,7 +14,7 @@ import mikv_inputs as mi
 import oracle
 import paper_2402_18096_gb300 as pkg
 from paper_2402_18096_gb300.layer import oracle_eviction_attention
-from _cases import bits16, gpu_layer, raw_inputs, sm_scale, vmax_per_head
+from _cases import bits16, gpu_layer, raw_inputs, ref_sizes, sm_scale, vmax_per_head
 
 pytestmark = pytest.mark.gpu
 
@@ -23,8 +23,9 @@ def _oracle_h2o(w, raw, b, h):
     k, v, scores, _ = raw
     ks, vs = bits16(k[b:b + 1, h:h + 1]), bits16(v[b:b + 1, h:h + 1])
     sc = scores[b:b + 1, h:h + 1].numpy()
-    _, kept = oracle.select_demote(sc, w.context - w.budget)
-    c = oracle.empty_cache(1, 1, w.head_dim, 2, 32, w.hi_cap, 16)
+    R = ref_sizes(w)
+    _, kept = oracle.select_demote(sc, w.context - R.budget)
+    c = oracle.empty_cache(1, 1, w.head_dim, 2, 32, R.hi_cap, 16)
     oracle.gather_hi(c, ks, vs, kept, src_scores=sc)
     return c
 
@@ -39,7 +40,9 @@ def test_h2o_eviction_steps(w):
     G = w.heads_q // w.heads_kv
     dev = torch.device("cuda")
     refs = {(b, h): _oracle_h2o(w, raw, b, h) for b in range(w.batch) for h in range(w.heads_kv)}
-    slots_ref = {key: np.array([[w.budget]], np.int32) for key in refs}
+    R = ref_sizes(w)
+    assert layer.shape.hi_cap == R.hi_cap
+    slots_ref = {key: np.array([[R.budget]], np.int32) for key in refs}
     near_ties = 0
     for step in range(steps):
         q, k_new, v_new = mi.decode_inputs(w, 0, step)
@@ -54,7 +57,7 @@ def test_h2o_eviction_steps(w):
             oracle.insert_token(c, bits16(k_new[b:b + 1, h:h + 1]), bits16(v_new[b:b + 1, h:h + 1]), w.context + step,
                                 slot)
             # the important set holds exactly the oracle's tokens
-            assert sorted(layer.cache.hi_tok[b, h, :w.hi_cap].tolist()) == sorted(c["hi_tok"][0, 0].tolist())
+            assert sorted(layer.cache.hi_tok[b, h, :R.hi_cap].tolist()) == sorted(c["hi_tok"][0, 0].tolist())
             qb = bits16(q[b:b + 1, h * G:(h + 1) * G])
             ref_o, hl, ml = oracle.decode_attention(c, qb, 0, sm_scale())
             err = np.abs(out[b, h * G:(h + 1) * G].cpu().numpy() - ref_o[0])

@@ -10,8 +10,8 @@ import torch
 import mikv_inputs as mi
 import oracle
 import paper_2402_18096_gb300 as pkg
-from _cases import (attention_tolerance, bits16, gpu_layer, new_workspace, oracle_layer, raw_inputs, sm_scale,
-                    vmax_per_head)
+from _cases import (assert_attention_close, bits16, gpu_layer, logit_bounds, new_workspace, oracle_layer, raw_inputs,
+                    ref_sizes, sm_scale, softmax_stat_bounds, vmax_per_head)
 
 pytestmark = pytest.mark.gpu
 
@@ -30,7 +30,9 @@ def _u16(t: torch.Tensor) -> np.ndarray:
 
 
 def _check_hi_cache(layer, refs, w):
-    k_b = w.budget
+    R = ref_sizes(w)
+    assert layer.shape.hi_cap == R.hi_cap and layer.n_lo == R.n_lo0  # library budget = oracle budget
+    k_b = R.budget
     for r in refs:
         b, h, c = r["b"], r["h"], r["cache"]
         for name in ("k_hi", "v_hi"):
@@ -40,23 +42,11 @@ def _check_hi_cache(layer, refs, w):
             np.testing.assert_array_equal(_u16(getattr(layer.cache, gname)[b, h, :k_b]), c[oname][0, 0, :k_b],
                                           err_msg=gname)
         np.testing.assert_array_equal(layer.cache.hi_tok[b, h, :k_b].cpu().numpy(), c["hi_tok"][0, 0, :k_b])
-        n_lo = w.n_lo0
+        n_lo = R.n_lo0
         for name in ("k_codes", "v_codes", "lo_tok"):
             np.testing.assert_array_equal(getattr(layer.cache, name)[b, h, :n_lo].cpu().numpy(), c[name][0, 0, :n_lo])
         for name in ("k_params", "v_params"):
             np.testing.assert_array_equal(_u16(getattr(layer.cache, name)[b, h, :n_lo]), c[name][0, 0, :n_lo])
-
-
-def _logit_bound(c, q_bits, bal, w, n_lo):
-    """|GPU - oracle| bound for logits: fp16 rounding of q / b and of every dequantized key (2^-11 relative
-    each) plus fp32 accumulation: 2^-9 * scale * max_t sum_c |q_c k_tc|, over both coded sets."""
-    q = (q_bits.astype(np.uint32) << 16).view(np.float32).astype(np.float64)[0]
-    qh = q / (bal[0] if bal is not None else 1.0)
-    rows = [oracle.dequantize_row(c["k_hi"][0, 0, i], c["k_hp"][0, 0, i], w.hi_bits, 64) for i in range(w.hi_cap)]
-    rows += [oracle.dequantize_row(c["k_codes"][0, 0, t], c["k_params"][0, 0, t], w.bits, w.group)
-             for t in range(n_lo)]
-    worst = (np.abs(qh) @ np.abs(np.stack(rows)).T).max(axis=1) * 2.0 ** -9
-    return sm_scale() * worst + 1e-6
 
 
 @pytest.mark.parametrize("name", list(CASES))
@@ -68,6 +58,7 @@ def test_coded_important_set_attention(name, out_dtype):
     assert layer.shape.hi_coded
     refs = oracle_layer(w, raw, layer.shape.lo_cap)
     _check_hi_cache(layer, refs, w)
+    R = ref_sizes(w)
 
     q, k_new, v_new = mi.decode_inputs(w, 0, 0)
     dev = torch.device("cuda")
@@ -77,29 +68,34 @@ def test_coded_important_set_attention(name, out_dtype):
     out = torch.empty(w.batch, w.heads_q, w.head_dim, dtype=out_dtype, device=dev)
     hl = torch.full((w.batch, w.heads_q, s.hi_stride), float("nan"), device=dev)
     ml = torch.empty(w.batch, w.heads_q, 2, device=dev)
-    ws = new_workspace(s, pkg.WS_ATTENTION, w.n_lo0)
-    pkg.mikv_decode_attention(layer.cache, w.n_lo0, q.to(dev), sm_scale(), out, ws, hi_logits=hl, ml=ml)
+    ws = new_workspace(s, pkg.WS_ATTENTION, layer.n_lo)
+    pkg.mikv_decode_attention(layer.cache, layer.n_lo, q.to(dev), sm_scale(), out, ws, hi_logits=hl, ml=ml)
     pkg.mikv_workspace_check(ws)
-    out_c, hl_c, ml_c = out.float().cpu().numpy(), hl.cpu().numpy(), ml.cpu().numpy()
+    out_c, hl_c, ml_c = out.cpu(), hl.cpu().numpy(), ml.cpu().numpy()
+    out32 = None
+    if out_dtype == torch.bfloat16:  # the same call with fp32 output: the bf16 output must be its rounding
+        out32 = torch.empty(w.batch, w.heads_q, w.head_dim, dtype=torch.float32, device=dev)
+        pkg.mikv_decode_attention(layer.cache, layer.n_lo, q.to(dev), sm_scale(), out32, ws)
+        pkg.mikv_workspace_check(ws)
+        out32 = out32.cpu()
     vmax = vmax_per_head(raw[1], v_new)
     for r in refs:
         b, h, c = r["b"], r["h"], r["cache"]
         oracle.insert_token(c, bits16(k_new[b:b + 1, h:h + 1]), bits16(v_new[b:b + 1, h:h + 1]), w.context,
-                            np.array([[w.budget]], np.int32), balancer_=r["balancer"])
+                            np.array([[R.budget]], np.int32), balancer_=r["balancer"])
         # the inserted slot's codes are bit-exact too
-        np.testing.assert_array_equal(layer.cache.k_hi[b, h, w.budget].cpu().numpy(), c["k_hi"][0, 0, w.budget])
-        np.testing.assert_array_equal(_u16(layer.cache.v_hi_params[b, h, w.budget]), c["v_hp"][0, 0, w.budget])
+        np.testing.assert_array_equal(layer.cache.k_hi[b, h, R.budget].cpu().numpy(), c["k_hi"][0, 0, R.budget])
+        np.testing.assert_array_equal(_u16(layer.cache.v_hi_params[b, h, R.budget]), c["v_hp"][0, 0, R.budget])
         qb = bits16(q[b:b + 1, h * G:(h + 1) * G])
-        ref_o, ref_l, ref_ml = oracle.decode_attention(c, qb, w.n_lo0, sm_scale(), balancer_=r["balancer"])
-        got = out_c[b, h * G:(h + 1) * G]
-        tol = attention_tolerance(vmax[b, h], ref_o[0], out_dtype == torch.bfloat16)
-        err = np.abs(got - ref_o[0])
-        assert np.all(err <= tol), f"{name} b{b} h{h}: max err {err.max():.3e}, tol {tol.min():.3e}"
-        bound = _logit_bound(c, qb, r["balancer"], w, w.n_lo0)
-        np.testing.assert_allclose(hl_c[b, h * G:(h + 1) * G, :w.hi_cap], ref_l[0], atol=float(bound.max()), rtol=0)
-        dm = np.abs(ml_c[b, h * G:(h + 1) * G, 0] - ref_ml[0, :, 0])
-        assert np.all(dm <= bound), (dm, bound)
-        np.testing.assert_allclose(ml_c[b, h * G:(h + 1) * G, 1], ref_ml[0, :, 1], rtol=4 * float(bound.max()) + 1e-5)
+        ref_o, ref_l, ref_ml = oracle.decode_attention(c, qb, R.n_lo0, sm_scale(), balancer_=r["balancer"])
+        sl = slice(h * G, (h + 1) * G)
+        assert_attention_close(out_c[b, sl], ref_o[0], vmax[b, h], f32=None if out32 is None else out32[b, sl],
+                               msg=f"{name} b{b} h{h}")
+        hb, lb = logit_bounds(c, qb, r["balancer"], w.bits, w.group, R.n_lo0, sm_scale(), hi_bits=w.hi_bits)
+        E, l_rtol = softmax_stat_bounds(hb, lb, R.hi_cap + R.n_lo0)
+        assert np.all(np.abs(hl_c[b, sl, :R.hi_cap] - ref_l[0]) <= hb), "important-set logits"
+        assert np.all(np.abs(ml_c[b, sl, 0] - ref_ml[0, :, 0]) <= E), "softmax max"
+        assert np.all(np.abs(ml_c[b, sl, 1] / ref_ml[0, :, 1] - 1) <= l_rtol), "softmax sum"
 
 
 @pytest.mark.parametrize("hi_bits,bits,group", [(8, 2, 64), (4, 3, 32), (2, 4, 128)])
@@ -114,13 +110,15 @@ def test_coded_important_set_decode_steps(hi_bits, bits, group):
     refs = oracle_layer(w, raw, s.lo_cap)
     G = w.heads_q // w.heads_kv
     dev = torch.device("cuda")
-    slots_ref = {(r["b"], r["h"]): np.array([[w.budget]], np.int32) for r in refs}
+    R = ref_sizes(w)
+    slots_ref = {(r["b"], r["h"]): np.array([[R.budget]], np.int32) for r in refs}
     near_ties = 0
     acc_tol = {}
     for step in range(steps):
         q, k_new, v_new = mi.decode_inputs(w, 0, step)
         out = torch.empty(w.batch, w.heads_q, w.head_dim, dtype=torch.float32, device=dev)
-        n_lo = layer.n_lo
+        n_lo = R.n_lo0 + step  # the oracle's retained length; the library's must agree
+        assert layer.n_lo == n_lo
         layer.step(q.to(dev), k_new.to(dev), v_new.to(dev), out)
         pkg.mikv_workspace_check(layer.ws)
         gslots = layer.slots.cpu().numpy()
@@ -136,10 +134,15 @@ def test_coded_important_set_decode_steps(hi_bits, bits, group):
             assert np.all(err <= 2e-3 * vmax[b, h]), (step, b, h, err.max())
             acc_before = c["acc"][0, 0].astype(np.float64)
             c["acc"] = oracle.update_importance(c["acc"], hl.astype(np.float32), ml.astype(np.float32), G)
-            tol = acc_tol.setdefault((b, h), np.zeros(w.hi_cap))
+            # a softmax weight's relative error: its logit's plus m's and l's (logit_bounds), plus 2^-21 for its fp32
+            # roundings; the fp32 add into the score rounds once (2^-24, taken twice); errors add up over steps
+            hb, lb = logit_bounds(c, qb, r["balancer"], w.bits, w.group, n_lo, sm_scale(), hi_bits=w.hi_bits)
+            E, l_rtol = softmax_stat_bounds(hb, lb, R.hi_cap + n_lo)
+            inc_rtol = float((np.expm1(2 * E) + l_rtol).max()) + 2.0 ** -21
+            tol = acc_tol.setdefault((b, h), np.zeros(R.hi_cap))
             tol[slot[0, 0]] = 0.0
-            tol += 3e-3 * np.abs(c["acc"][0, 0] - acc_before) + 2e-7 * np.abs(acc_before) + 1e-9
-            acc_gpu = layer.cache.acc[b, h, :w.hi_cap].cpu().numpy()
+            tol += inc_rtol * np.abs(c["acc"][0, 0] - acc_before) + 2.0 ** -23 * np.abs(c["acc"][0, 0])
+            acc_gpu = layer.cache.acc[b, h, :R.hi_cap].cpu().numpy()
             assert np.all(np.abs(acc_gpu - c["acc"][0, 0]) <= tol), (step, b, h)
             dem, _ = oracle.select_demote(c["acc"], 1, c["hi_tok"], want_kept=False)
             victim = int(dem[0, 0, 0])

@@ -10,8 +10,8 @@ import torch
 import mikv_inputs as mi
 import oracle
 import paper_2402_18096_gb300 as pkg
-from _cases import (attention_tolerance, bits16, gpu_layer, new_workspace, oracle_layer, raw_inputs, sm_scale,
-                    vmax_per_head)
+from _cases import (assert_attention_close, bits16, gpu_layer, new_workspace, oracle_layer, raw_inputs, ref_sizes,
+                    sm_scale, vmax_per_head)
 
 pytestmark = pytest.mark.gpu
 
@@ -21,6 +21,8 @@ def _u16(t):
 
 
 def _check_kch_cache(layer, refs, w, n_lo):
+    R = ref_sizes(w)
+    assert layer.shape.hi_cap == R.hi_cap
     n_q, n_st = n_lo // 64 * 64, n_lo % 64
     for r in refs:
         b, h, c = r["b"], r["h"], r["cache"]
@@ -29,7 +31,7 @@ def _check_kch_cache(layer, refs, w, n_lo):
                                           err_msg=name)
         np.testing.assert_array_equal(_u16(layer.cache.k_params[b, h, :n_q // 64]), c["k_params"][0, 0, :n_q // 64])
         np.testing.assert_array_equal(_u16(layer.cache.v_params[b, h, :n_q]), c["v_params"][0, 0, :n_q])
-        rows = slice(w.hi_cap, w.hi_cap + n_st)  # the staged retained tokens
+        rows = slice(R.hi_cap, R.hi_cap + n_st)  # the staged retained tokens
         np.testing.assert_array_equal(bits16(layer.cache.k_hi[b, h, rows]), c["k_hi"][0, 0, rows])
         np.testing.assert_array_equal(bits16(layer.cache.v_hi[b, h, rows]), c["v_hi"][0, 0, rows])
         np.testing.assert_array_equal(layer.cache.hi_tok[b, h, rows].cpu().numpy(), c["hi_tok"][0, 0, rows])
@@ -42,7 +44,7 @@ def _kch_logit_bound(c, q_bits, w, n_lo):
     and fp32 sums. 2^-9 (4x margin) of max_t sum_c |q_c alpha_c code_tc| plus 2^-20 of the exact parts."""
     q = np.abs((q_bits.astype(np.uint32) << 16).view(np.float32).astype(np.float64)[0])  # [G, d]
     n_q, n_st = n_lo // 64 * 64, n_lo % 64
-    kh = (c["k_hi"][0, 0, :w.hi_cap + n_st].astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    kh = (c["k_hi"][0, 0, :ref_sizes(w).hi_cap + n_st].astype(np.uint32) << 16).view(np.float32).astype(np.float64)
     worst = (q @ np.abs(kh).T).max(axis=1) * 2.0 ** -20
     for j in range(n_q // 64):
         par = c["k_params"][0, 0, j].view(np.float16).astype(np.float64)  # [d, 2]: alpha, beta
@@ -67,7 +69,8 @@ def test_kch_attention(name, out_dtype):
     raw = raw_inputs(w)
     layer = gpu_layer(w, raw)
     refs = oracle_layer(w, raw, layer.shape.lo_cap)
-    _check_kch_cache(layer, refs, w, w.n_lo0)
+    R = ref_sizes(w)
+    _check_kch_cache(layer, refs, w, R.n_lo0)
     q, k_new, v_new = mi.decode_inputs(w, 0, 0)
     dev = torch.device("cuda")
     s = layer.shape
@@ -76,22 +79,28 @@ def test_kch_attention(name, out_dtype):
     out = torch.empty(w.batch, w.heads_q, w.head_dim, dtype=out_dtype, device=dev)
     hl = torch.full((w.batch, w.heads_q, s.hi_stride), float("nan"), device=dev)
     ml = torch.empty(w.batch, w.heads_q, 2, device=dev)
-    ws = new_workspace(s, pkg.WS_ATTENTION, w.n_lo0)
-    pkg.mikv_decode_attention(layer.cache, w.n_lo0, q.to(dev), sm_scale(), out, ws, hi_logits=hl, ml=ml)
+    ws = new_workspace(s, pkg.WS_ATTENTION, layer.n_lo)
+    pkg.mikv_decode_attention(layer.cache, layer.n_lo, q.to(dev), sm_scale(), out, ws, hi_logits=hl, ml=ml)
     pkg.mikv_workspace_check(ws)
-    out_c, hl_c, ml_c = out.float().cpu().numpy(), hl.cpu().numpy(), ml.cpu().numpy()
+    out_c, hl_c, ml_c = out.cpu(), hl.cpu().numpy(), ml.cpu().numpy()
+    out32 = None
+    if out_dtype == torch.bfloat16:  # the same call with fp32 output: the bf16 output must be its rounding
+        out32 = torch.empty(w.batch, w.heads_q, w.head_dim, dtype=torch.float32, device=dev)
+        pkg.mikv_decode_attention(layer.cache, layer.n_lo, q.to(dev), sm_scale(), out32, ws)
+        pkg.mikv_workspace_check(ws)
+        out32 = out32.cpu()
     vmax = vmax_per_head(raw[1], v_new)
     for r in refs:
         b, h, c = r["b"], r["h"], r["cache"]
         oracle.insert_token(c, bits16(k_new[b:b + 1, h:h + 1]), bits16(v_new[b:b + 1, h:h + 1]), w.context,
-                            np.array([[w.budget]], np.int32))
+                            np.array([[R.budget]], np.int32))
         qb = bits16(q[b:b + 1, h * G:(h + 1) * G])
-        ref_o, ref_l, ref_ml = oracle.decode_attention(c, qb, w.n_lo0, sm_scale())
-        tol = attention_tolerance(vmax[b, h], ref_o[0], out_dtype == torch.bfloat16)
-        err = np.abs(out_c[b, h * G:(h + 1) * G] - ref_o[0])
-        assert np.all(err <= tol), f"{name} b{b} h{h}: max err {err.max():.3e}, tol {tol.min():.3e}"
-        bound = _kch_logit_bound(c, qb, w, w.n_lo0)
-        np.testing.assert_allclose(hl_c[b, h * G:(h + 1) * G, :w.hi_cap], ref_l[0, :, :w.hi_cap],
+        ref_o, ref_l, ref_ml = oracle.decode_attention(c, qb, R.n_lo0, sm_scale())
+        sl = slice(h * G, (h + 1) * G)
+        assert_attention_close(out_c[b, sl], ref_o[0], vmax[b, h], f32=None if out32 is None else out32[b, sl],
+                               msg=f"{name} b{b} h{h}")
+        bound = _kch_logit_bound(c, qb, w, R.n_lo0)
+        np.testing.assert_allclose(hl_c[b, h * G:(h + 1) * G, :R.hi_cap], ref_l[0, :, :R.hi_cap],
                                    atol=float(bound.max()), rtol=0)
         dm = np.abs(ml_c[b, h * G:(h + 1) * G, 0] - ref_ml[0, :, 0])
         assert np.all(dm <= bound), (dm, bound)
@@ -103,19 +112,21 @@ def test_kch_decode_steps_across_a_group(bits, group):
     """61 staged tokens after the build: the third step completes the group, which is quantized per channel
     from the staged rows bit for bit; outputs, scores and victims follow the oracle's steps."""
     w = mi.Workload("kct", 2, 8, 2, 396, 1, bits, group, 0.2, seed=85 + bits, k_channel=True)
-    assert w.n_lo0 % 64 == 61
+    R = ref_sizes(w)
+    assert R.n_lo0 % 64 == 61
     steps = 6
     raw = raw_inputs(w)
     layer = gpu_layer(w, raw, steps=steps)
     refs = oracle_layer(w, raw, layer.shape.lo_cap)
     G = w.heads_q // w.heads_kv
     dev = torch.device("cuda")
-    slots_ref = {(r["b"], r["h"]): np.array([[w.budget]], np.int32) for r in refs}
+    slots_ref = {(r["b"], r["h"]): np.array([[R.budget]], np.int32) for r in refs}
     near_ties = 0
     for step in range(steps):
         q, k_new, v_new = mi.decode_inputs(w, 0, step)
         out = torch.empty(w.batch, w.heads_q, w.head_dim, dtype=torch.float32, device=dev)
-        n_lo = layer.n_lo
+        n_lo = R.n_lo0 + step  # the oracle's retained length; the library's must agree
+        assert layer.n_lo == n_lo
         layer.step(q.to(dev), k_new.to(dev), v_new.to(dev), out)
         pkg.mikv_workspace_check(layer.ws)
         gslots = layer.slots.cpu().numpy()
@@ -128,10 +139,10 @@ def test_kch_decode_steps_across_a_group(bits, group):
             ref_o, hl, ml = oracle.decode_attention(c, qb, n_lo, sm_scale())
             err = np.abs(out[b, h * G:(h + 1) * G].cpu().numpy() - ref_o[0])
             assert np.all(err <= 2e-3 * vmax[b, h]), (step, b, h, err.max())
-            acc = c["acc"][:, :, :w.hi_cap]
-            acc = oracle.update_importance(acc, hl[:, :, :w.hi_cap].astype(np.float32), ml.astype(np.float32), G)
-            c["acc"][:, :, :w.hi_cap] = acc
-            dem, _ = oracle.select_demote(acc, 1, c["hi_tok"][:, :, :w.hi_cap], want_kept=False)
+            acc = c["acc"][:, :, :R.hi_cap]
+            acc = oracle.update_importance(acc, hl[:, :, :R.hi_cap].astype(np.float32), ml.astype(np.float32), G)
+            c["acc"][:, :, :R.hi_cap] = acc
+            dem, _ = oracle.select_demote(acc, 1, c["hi_tok"][:, :, :R.hi_cap], want_kept=False)
             victim = int(dem[0, 0, 0])
             if gslots[b, h] != victim:
                 a_sorted = np.sort(acc[0, 0])

@@ -41,7 +41,7 @@ def test_fused_step_equals_separate_calls(w, out_dtype):
         pkg.mikv_decode_attention(sep.cache, n_lo, q, sm_scale(), out_s, ws, hi_logits=hl, ml=ml)
         pkg.mikv_update_importance(sep.cache, hl, ml)
         victim = torch.empty(w.batch, w.heads_kv, 1, dtype=torch.int32, device=dev)
-        pkg.mikv_select_demote(sep.cache.acc, w.hi_cap, 1, victim, ids=sep.cache.hi_tok)
+        pkg.mikv_select_demote(sep.cache.acc, s.hi_cap, 1, victim, ids=sep.cache.hi_tok)
         pkg.mikv_quantize_pack(sep.cache, sep.cache.k_hi, sep.cache.v_hi, victim, n_lo, src_tok=sep.cache.hi_tok)
         pkg.mikv_workspace_check(ws)
         sep.slots.copy_(victim[..., 0])
@@ -49,7 +49,7 @@ def test_fused_step_equals_separate_calls(w, out_dtype):
         sep.pos += 1
 
         assert torch.equal(out_f, out_s), step
-        assert torch.equal(fused.cache.acc[..., :w.hi_cap], sep.cache.acc[..., :w.hi_cap]), step
+        assert torch.equal(fused.cache.acc[..., :s.hi_cap], sep.cache.acc[..., :s.hi_cap]), step
         assert torch.equal(fused.slots, sep.slots), step
         for name in ("k_codes", "v_codes", "k_params", "v_params", "lo_tok"):
             assert torch.equal(getattr(fused.cache, name)[:, :, n_lo], getattr(sep.cache, name)[:, :, n_lo]), (name, step)

@@ -74,17 +74,8 @@ def test_normal_draws_and_lognormal_scores():
     assert bool((mi.initial_scores(W, 0) > 0).all())
 
 
-def test_budget_rounds_half_up_and_capacities():
-    assert mi.WORKLOADS["llama2-7b"].budget == 819           # 0.2 * 4096 = 819.2
-    assert mi.WORKLOADS["llama2-13b"].budget == 819          # 0.1 * 8192 = 819.2
-    assert mi.WORKLOADS["mistral-7b"].budget == 6554         # 0.2 * 32768 = 6553.6
-    assert mi.scaled(W, context=10, ratio=0.25).budget == 3  # 2.5 rounds up
-    w = mi.WORKLOADS["mistral-7b"]
-    assert w.hi_cap == w.budget + 1 and w.hi_stride % 16 == 0 and w.hi_stride >= w.hi_cap
-    assert w.n_lo0 == w.context - w.budget
-    for steps in (0, 1, 17, 100):
-        cap = w.lo_cap_for(steps)
-        assert cap % 16 == 0 and cap >= w.n_lo0 + steps
-        kc = mi.scaled(w, k_channel=True).lo_cap_for(steps)
-        assert kc % 64 == 0 and kc >= w.n_lo0 + steps
+def test_workload_table():
     assert len(mi.sweep_workloads()) == 30
+    for w in mi.sweep_workloads():  # every sweep point is also reachable by its short name
+        assert mi.WORKLOADS[f"sweep-int{w.bits}-g{w.group}-r{int(w.ratio * 100)}"] == w
+    assert not hasattr(mi.Workload, "budget")  # the ratio -> token count rule lives on each side, not here

@@ -157,3 +157,36 @@ def test_cache_fraction_limits():
     assert oracle.cache_fraction(2, 64, 1.0) == 1.0                    # everything fp16
     assert oracle.cache_fraction(4, 128, 0.0) == (4 + 0.25) / 16       # uniform RTN baseline
     assert oracle.cache_fraction(8, 64, 1.0, 8) == (8 + 0.5) / 16
+
+
+def test_budget_hand_values():
+    """Tables 1-3 give the important set as a ratio of the tokens; the oracle's count (reading R10) is the
+    nearest integer to ratio * T, halves rounded up. Hand-computed values of the benchmark shapes and ties."""
+    assert oracle.budget(4096, 0.2) == 819       # 819.2
+    assert oracle.budget(8192, 0.1) == 819       # 819.2
+    assert oracle.budget(32768, 0.2) == 6554     # 6553.6
+    assert oracle.budget(512, 0.2) == 102        # 102.4
+    assert oracle.budget(4096, 0.05) == 205      # 204.8
+    assert oracle.budget(10, 0.25) == 3          # 2.5: a half rounds up
+    assert oracle.budget(1, 0.5) == 1            # 0.5
+    assert oracle.budget(3, 0.5) == 2            # 1.5
+    assert oracle.budget(6, 0.25) == 2           # 1.5
+    assert oracle.budget(1, 0.2) == 0            # 0.2
+    assert oracle.budget(0, 0.7) == 0
+    assert oracle.budget(4096, 0.0) == 0 and oracle.budget(4096, 1.0) == 4096
+    for bad in ((-1, 0.5), (10, -0.1), (10, 1.5), (10, float("nan"))):
+        with pytest.raises(ValueError):
+            oracle.budget(*bad)
+
+
+def test_budget_brute_force_exact_ratios():
+    """For ratios k/64 (exact in binary) the budget is the integer n minimising |n - ratio * T| in exact
+    rational arithmetic, the larger n on a tie."""
+    from fractions import Fraction
+    for num in range(65):
+        r = Fraction(num, 64)
+        for T in (0, 1, 2, 3, 5, 7, 31, 64, 100, 127, 4095, 4096):
+            x = r * T
+            lo = x.numerator // x.denominator
+            want = lo + 1 if x - lo >= Fraction(1, 2) else lo
+            assert oracle.budget(T, num / 64) == want, (num, T)
