@@ -29,7 +29,7 @@
  * c = 16 m + u (u = c mod 16, m = c div 16) and a plane is a sequence of little-endian 16-bit units.
  * In a plane of f-bit fields (f in {2, 4, 8}) with P = 16 / f codes per unit, channel c sits in unit
  * 8 * (2 * (m div P) + (u div 8)) + (u mod 8) at bits [f * (m mod P), f * (m mod P) + f). In a plane of
- * 1-bit fields, channel c sits in unit (u mod 8) at bit 8 * (u div 8) + m. N = 2, 4 and 8 use one
+ * 1-bit fields, channel c sits in unit (u mod 8) at bit 2 * m + (u div 8). N = 2, 4 and 8 use one
  * plane of N-bit fields; N = 3 uses a plane of 2-bit fields (code bits 0..1) followed by a plane of
  * 1-bit fields (code bit 2). The quantization parameters of a row are d / group pairs of fp16
  * (alpha, beta), alpha first; the dequantized value is alpha * code + beta.

@@ -126,7 +126,7 @@ int mikv_ref_quantize_group(const float* x, int g, int bits, int32_t* codes, uin
  * u = c mod 16 and m = c div 16. A plane is a sequence of little-endian 16-bit units.
  *  - plane of f-bit fields, f in {2, 4, 8}: P = 16 / f codes per unit; the code of channel c sits in
  *    unit 8 * (2 * (m div P) + (u div 8)) + (u mod 8), at bits [f * (m mod P), f * (m mod P) + f).
- *  - plane of 1-bit fields: the bit of channel c sits in unit (u mod 8), at bit 8 * (u div 8) + m.
+ *  - plane of 1-bit fields: the bit of channel c sits in unit (u mod 8), at bit 2 * m + (u div 8).
  * N = 2, 4, 8: one plane of N-bit fields. N = 3: a plane of 2-bit fields holding bits 0..1 of each
  * code, then a plane of 1-bit fields holding bit 2. A row takes 16 * N bytes.
  */
@@ -134,7 +134,7 @@ static void field_position(int c, int f, int* unit, int* bit) {
   int u = c % 16, m = c / 16;
   if (f == 1) {
     *unit = u % 8;
-    *bit = 8 * (u / 8) + m;
+    *bit = 2 * m + u / 8;
     return;
   }
   int P = 16 / f;

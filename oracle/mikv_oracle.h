@@ -19,7 +19,7 @@
  * little-endian 16-bit units. In a plane of f-bit fields (f in {2, 4, 8}) with P = 16 / f codes per
  * unit, channel c sits in unit 8 * (2 * (m div P) + (u div 8)) + (u mod 8) at bits
  * [f * (m mod P), f * (m mod P) + f). In a plane of 1-bit fields, channel c sits in unit u mod 8 at
- * bit 8 * (u div 8) + m. N in {2, 4, 8}: one plane of N-bit fields. N = 3: a plane of 2-bit fields
+ * bit 2 * m + (u div 8). N in {2, 4, 8}: one plane of N-bit fields. N = 3: a plane of 2-bit fields
  * holding bits 0..1 of each code, then a plane of 1-bit fields holding bit 2. A row takes 16 * N
  * bytes. Quantization parameters of a row are d/g pairs of fp16 (alpha, beta), alpha first.
  */
@@ -163,6 +163,11 @@ int mikv_ref_prefill_scores(int B, int Hq, int Hkv, int T, int d, const uint16_t
  * (16 = fp16, else hi_bits-bit codes with fp16 alpha/beta per group g) plus (1 - r) at bits-bit codes
  * with fp16 alpha/beta per group g. */
 double mikv_ref_cache_fraction(int bits, int g, double ratio, int hi_bits);
+
+/* Number of important tokens for importance ratio `ratio` over T tokens (Tables 1-3 "Importance ratio"):
+ * the integer nearest ratio * T (double product), halves rounded up. -1 if T < 0 or ratio is outside
+ * [0, 1]. */
+int mikv_ref_budget(int T, double ratio);
 
 #ifdef __cplusplus
 }

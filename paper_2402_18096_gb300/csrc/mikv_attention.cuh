@@ -250,11 +250,25 @@ __device__ __forceinline__ uint32_t code8(uint32_t r, int hi) {
   return exact_codes(prmt(r, 0x64646464u, hi ? 0x4341u : 0x4240u), 0x64006400u);
 }
 
-// 3-bit code: bits 0..1 at position j of r, bit 2 at bit hb of each unit of h.
-__device__ __forceinline__ uint32_t code3(uint32_t r, uint32_t h, int j, int hb) {
-  const uint32_t lo = and_or(r >> (2 * j), 0x00030003u, 0x64006400u);
-  return exact_codes(lo | (((h >> hb) << 2) & 0x00040004u), 0x64006400u);
+// 3-bit code with its low bits at [p, p + 2) of r and its high bit at p + 2 of hs (each unit), OR-ed under
+// `magic`, the fp16 exponent that makes bit p weigh 1: the pair holds magic + code exactly. In the 1-bit plane
+// the bits of the two channels u and u + 8 of a unit alternate (bit 2 m + (u div 8) for channel 16 m + u), so
+// one shift of the plane word lines up the high bit of every code of a channel with its low bits.
+__device__ __forceinline__ uint32_t or_code3(uint32_t r, uint32_t hs, int p, uint32_t magic) {
+  return and_or(hs, 0x00040004u << p, and_or(r, 0x00030003u << p, magic));
 }
+
+// Key codes (exact) of k-step ks, N = 3: kr = a fragment register of the 2-bit plane (its codes for ks at bits
+// 2 ks), kr8 = kr >> 8; he / he8 the 1-bit plane word shifted so that the high bits of ks <= 3 / ks >= 4 land
+// at 2 ks + 2 / 2 (ks - 4) + 2.
+__device__ __forceinline__ uint32_t kcode3(uint32_t kr, uint32_t kr8, uint32_t he, uint32_t he8, int ks) {
+  const int j = ks & 3;
+  return exact_codes(or_code3(ks < 4 ? kr : kr8, ks < 4 ? he : he8, 2 * j, mag2(j)), mag2(j));
+}
+
+// Value codes, N = 3, take a code offset M in {64, 16} like vcode2: code mt is read at bit 4 + 2 (mt & 1) of the
+// words shifted by 4 - 4 (mt div 2) (the low bits) and by two more (the high bit).
+__host__ __device__ constexpr float voff3(int mt) { return (mt & 1) ? 16.f : 64.f; }
 
 // Value codes (N = 2, 4) skip the subtraction: the code is placed at a mantissa position where it
 // weighs 1 under a magic M in {4, 16, 64}, so the fp16 pair holds M + code exactly. The PV sums then
@@ -280,7 +294,7 @@ __host__ __device__ constexpr float voff4(int p) { return p < 2 ? 64.f : 16.f; }
 
 template <int BITS>
 __host__ __device__ constexpr float voff(int mt) {
-  return BITS == 2 ? voff2(mt) : BITS == 4 ? voff4(mt & 3) : 0.f;
+  return BITS == 2 ? voff2(mt) : BITS == 4 ? voff4(mt & 3) : BITS == 3 ? voff3(mt) : 0.f;
 }
 
 // ---------------------------------------------------------------------- one important block
@@ -415,8 +429,13 @@ __device__ __forceinline__ void lo_logits(uint32_t unit, int b, int valid, const
       if (BITS == 3) ldsm_x2(ka + (lane & 15) * U.pitch + U.plane_b, kb0, kb1);
     }
 #pragma unroll
-    for (int i = 0; i < NR; ++i) kh[i] = kr[i] >> (BITS == 4 ? 8 : 10);
+    for (int i = 0; i < NR; ++i) kh[i] = kr[i] >> (BITS == 2 ? 10 : 8);
   }
+  // N = 3: the 1-bit plane words of tokens g (kb0) and g + 8 (kb1) shifted so that the high bit of code ks sits
+  // two bits above its low bits: channels 2t, 2t+1 use the even bits (<< 2 for ks <= 3, >> 6 for ks >= 4),
+  // channels 2t+8, 2t+9 the odd bits (<< 1, >> 7)
+  const uint32_t he0 = kb0 << 2, he1 = kb1 << 2, ho0 = kb0 << 1, ho1 = kb1 << 1;
+  const uint32_t he0s = kb0 >> 6, he1s = kb1 >> 6, ho0s = kb0 >> 7, ho1s = kb1 >> 7;
 #pragma unroll
   for (int ks = 0; ks < 8; ++ks) {
     const int gi = (16 * ks) / GROUP;
@@ -430,10 +449,10 @@ __device__ __forceinline__ void lo_logits(uint32_t unit, int b, int valid, const
 #pragma unroll
       for (int i = 0; i < 4; ++i) c[i] = code2(kr[i], kh[i], ks);
     } else {
-      c[0] = code3(kr[0], kb0, ks, ks);
-      c[1] = code3(kr[1], kb1, ks, ks);
-      c[2] = code3(kr[2], kb0, ks, 8 + ks);
-      c[3] = code3(kr[3], kb1, ks, 8 + ks);
+      c[0] = kcode3(kr[0], kh[0], he0, he0s, ks);
+      c[1] = kcode3(kr[1], kh[1], he1, he1s, ks);
+      c[2] = kcode3(kr[2], kh[2], ho0, ho0s, ks);
+      c[3] = kcode3(kr[3], kh[3], ho1, ho1s, ks);
     }
     if constexpr (KCH) {
       mma_f16(accs[ks % QACC], c, qh[ks][0], qh[ks][1]);
@@ -487,6 +506,7 @@ __device__ __forceinline__ void kch_prepare(uint32_t kp, const uint32_t (&qh)[8]
 template <int BITS, int GROUP, int NB, bool EXACT, bool KCH = false>
 __device__ __forceinline__ void lo_values(uint32_t unit, int b, int valid, const float (&p)[4], float (&o)[8][4],
                                           float (&ob)[NB][4], int lane) {
+  static_assert(!(EXACT && BITS == 3), "coded important sets use 8-, 4- or 2-bit codes");
   constexpr LoUnit U = KCH ? lo_unit_layout_kch(BITS, GROUP) : lo_unit_layout(BITS, GROUP);
   constexpr int NG = kHeadDim / GROUP;
   constexpr int PR = U.param_row;
@@ -566,7 +586,7 @@ __device__ __forceinline__ void lo_values(uint32_t unit, int b, int valid, const
     pa0[gi] = h2_as_u32(__hmul2(u32_as_h2(pb0), u32_as_h2(prmt(pv0[gi], pv1[gi], 0x5410u))));
     pa1[gi] = h2_as_u32(__hmul2(u32_as_h2(pb1), u32_as_h2(prmt(pv8[gi], pv9[gi], 0x5410u))));
   }
-  if (!EXACT && BITS != 3) {
+  if (!EXACT) {
     // sum of p * alpha per group, from the same fp16 operands as the code MMAs: ones in rows 0..7
     // (even groups) or 8..15 (odd groups), so ob[1 + gi / 2] holds two groups per fragment
     constexpr uint32_t kOne = 0x3C003C00u;
@@ -617,10 +637,15 @@ __device__ __forceinline__ void lo_values(uint32_t unit, int b, int valid, const
           a[i] = vcode2(vr[i] << 4, vr[i], vr[i] >> 6, mt);  // the shifted copies are shared by all mt
       }
     } else {
-      a[0] = code3(vr[0], vb0, mt, mt);
-      a[1] = code3(vr[1], vb0, mt, 8 + mt);
-      a[2] = code3(vr[2], vb1, mt, mt);
-      a[3] = code3(vr[3], vb1, mt, 8 + mt);
+      // vr[0], vr[2]: channel g (tokens 2t, 2t+1 and 2t+8, 2t+9), whose high bits are the even bits of vb0, vb1;
+      // vr[1], vr[3]: channel g + 8, the odd bits
+      const int k = mt >> 1, s = 4 - 4 * k;  // codes 2k, 2k+1 read at bits 4, 6 of the words shifted by s
+      auto sh = [](uint32_t x, int n) { return n >= 0 ? x << n : x >> -n; };
+      const uint32_t r4[4] = {sh(vr[0], s), sh(vr[1], s), sh(vr[2], s), sh(vr[3], s)};
+      const uint32_t h4[4] = {sh(vb0, s + 2), sh(vb0, s + 1), sh(vb1, s + 2), sh(vb1, s + 1)};
+      const int p = 4 + 2 * (mt & 1);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) a[i] = or_code3(r4[i], h4[i], p, mag2(p >> 1));
     }
     mma_f16(o[mt], a, pa0[gi], pa1[gi]);  // sums p * alpha * (code + offset)
   }
@@ -683,7 +708,7 @@ __device__ __forceinline__ void write_partial(const AttnArgs& a, int slot, Softm
       for (int mt = 0; mt < 8; ++mt) {
         const int gi = (16 * mt) / GROUP;
         float z = hd ? bz1[mt >> 1] : bz0[mt >> 1];
-        if (BITS != 3) z = fmaf(-voff<BITS>(mt), ob[1 + gi / 2][2 * (gi & 1) + hd], z);
+        z = fmaf(-voff<BITS>(mt), ob[1 + gi / 2][2 * (gi & 1) + hd], z);
         po[16 * mt + g] = (o[mt][hd] + z) * inv[hd];
         po[16 * mt + 8 + g] = (o[mt][2 + hd] + z) * inv[hd];
       }
@@ -854,7 +879,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
 
   const int g = lane >> 2, t = lane & 3;
   uint32_t qb[8][2], qh[8][2];
-  constexpr int NB = 1 + (BITS == 3 ? 0 : (kHeadDim / GROUP + 1) / 2);  // beta rows + alpha-sum pairs
+  constexpr int NB = 1 + (kHeadDim / GROUP + 1) / 2;  // beta rows + alpha-sum pairs
   Softmax st;
   float o[8][4], ob[NB][4];
   __shared__ int s_ins[kWarps];  // each warp's insertion slot of its current head (fused insertion; kept out of

@@ -147,11 +147,11 @@ __global__ void __launch_bounds__(256) quantize_pack_kernel(const QPArgs a) {
     const uint32_t wd = reduce_scatter<8, 4>(L, l8);
     if (valid) row[l8] = wd;
     if constexpr (BITS == 3) {
-      // high bits: channel 16 l8 + u sits in unit u & 7 at bit 8 (u >> 3) + l8 (words 8..11 of the row);
+      // high bits: channel 16 l8 + u sits in unit u & 7 at bit 2 l8 + (u >> 3) (words 8..11 of the row);
       // after two rounds a lane pair holds one word, and the pair's even lane stores it
       uint32_t H[4] = {0u, 0u, 0u, 0u};
 #pragma unroll
-      for (int u = 0; u < 16; ++u) H[(u & 7) >> 1] |= (code[u] >> 2) << (16 * (u & 1) + 8 * (u >> 3) + l8);
+      for (int u = 0; u < 16; ++u) H[(u & 7) >> 1] |= (code[u] >> 2) << (16 * (u & 1) + 2 * l8 + (u >> 3));
       uint32_t K[2];
 #pragma unroll
       for (int k = 0; k < 2; ++k) {

@@ -12,9 +12,9 @@ namespace mikv {
 // Bit position of channel c (= 16 m + u) in a plane of f-bit fields: 16-bit unit and bit offset.
 __device__ __forceinline__ void field_pos(int c, int f, int& unit, int& bit) {
   const int u = c & 15, m = c >> 4;
-  if (f == 1) {
+  if (f == 1) {  // the two channels u and u + 8 of a unit alternate: their bits for m sit at 2 m and 2 m + 1
     unit = u & 7;
-    bit = 8 * (u >> 3) + m;
+    bit = 2 * m + (u >> 3);
   } else {
     const int P = 16 / f;
     unit = 8 * (2 * (m / P) + (u >> 3)) + (u & 7);

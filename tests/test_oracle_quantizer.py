@@ -168,10 +168,13 @@ def test_pack_layout_hand_examples():
     assert p[50] == 0xA0 and int(p.sum()) == 0xA0
     p = one(4, 16 * 2 + 3, 0x7)          # m 2, u 3 -> unit 3, bits 8..11 -> byte 7 = 0x07
     assert p[7] == 0x07 and int(p.sum()) == 7
-    # N = 3: 2-bit plane (32 bytes) then 1-bit plane: bit of c in unit u%8 at bit 8*(u//8) + m.
+    # N = 3: 2-bit plane (32 bytes) then 1-bit plane: bit of c in unit u%8 at bit 2*m + u//8.
     p = one(3, 16 * 6 + 12, 0b101)      # low bits 01 -> unit 12 bits 12-13 -> byte 25 = 0x10;
-    assert p[25] == 0x10                 # bit 2 -> plane 2 unit 4, bit 8 + 6 = 14 -> byte 32+9 = 0x40
-    assert p[41] == 0x40 and int(p.sum()) == 0x50
+    assert p[25] == 0x10                 # bit 2 -> plane 2 unit 4, bit 2*6 + 1 = 13 -> byte 32+9 bit 5 = 0x20
+    assert p[41] == 0x20 and int(p.sum()) == 0x30
+    p = one(3, 16 * 3 + 5, 0b110)       # low bits 10 -> unit 5 bits 6-7 -> byte 10 = 0x80;
+    assert p[10] == 0x80                 # bit 2 -> plane 2 unit 5, bit 2*3 + 0 = 6 -> byte 32+10 = 0x40
+    assert p[42] == 0x40 and int(p.sum()) == 0xC0
     # N = 8: P = 2; unit 8*(2*(m//2) + u//8) + u%8, bits 8*(m%2).
     p = one(8, 16 * 3 + 8, 0xC3)         # m 3, u 8 -> unit 8*(2+1)+0 = 24, high byte -> byte 49
     assert p[49] == 0xC3 and int(p.sum()) == 0xC3
