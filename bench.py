@@ -37,7 +37,7 @@ METRIC = "decode-attn compressed-KV GB/s and % of GB300 HBM peak; us per decode 
 UNIT = "GB/s"
 DEFAULT_WORKLOAD = "mistral-7b"
 L2_BYTES = 129 * 10 ** 6          # GB300 L2
-L2_FLUSH_BYTES = 512 << 20        # a write this large evicts every cache line of L2
+L2_FLUSH_BYTES = 1024 << 20       # flush buffer: a 512 MiB write, then a 512 MiB read (each far larger than L2)
 
 
 ATTN_SOURCES = ["mikv_attention.cuh", "mikv_attention.cu", "mikv_attn_h16.cu", "mikv_device.cuh", "mikv_internal.h",
@@ -70,12 +70,20 @@ def profiled_traffic_ratio(workload: str):
         return None
 
 
+def flush_l2(scrub: torch.Tensor):
+    """Evict L2: write the first half of `scrub` (larger than L2), then read its second half, so that the dirty
+    lines of the write are written back before whatever follows (only clean lines of `scrub` remain)."""
+    half = scrub.numel() // 2
+    scrub[:half].add_(1)
+    scrub[half:].max()
+
+
 def timed_with_flush(fn, n: int, scrub: torch.Tensor, stream) -> float:
-    """Milliseconds of n calls fn(i), each timed alone with CUDA events on `stream` after a write of
-    `scrub` (larger than L2) has evicted whatever the previous call left in L2."""
+    """Milliseconds of n calls fn(i), each timed alone with CUDA events on `stream` after an L2 flush
+    (flush_l2) has evicted whatever the previous call left in L2."""
     evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
     for i in range(n):
-        scrub.add_(1)
+        flush_l2(scrub)
         evs[i][0].record(stream)
         fn(i)
         evs[i][1].record(stream)
@@ -215,7 +223,6 @@ def run_mikv(args):
         w = mi.scaled(w, layers=args.layers)
     K, W = args.steps, args.warmup
     e2e_steps = max(2, K // 2)
-    attn_reps = 2
     steps_cap = W + K + W + e2e_steps + 4
     shape, layers, build = build_model(w, steps_cap, dev, rank)
     L = len(layers)
@@ -279,6 +286,8 @@ def run_mikv(args):
         for layer in layers:
             pkg.mikv_decode_attention(layer.cache, layer.n_lo, q0, layer.sm_scale, out, ws_attn[0])
 
+    attn_reps = max(2, -(-16 // L))  # at least 16 launches
+    attend_all()  # untimed: the first launches of this entry point's kernels (module loading, attributes)
     torch.cuda.synchronize()
     if scrub is None:
         a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -310,7 +319,7 @@ def run_mikv(args):
     e2e_s = 0.0
     for s in range(e2e_steps):
         if scrub is not None:  # flushed L2 before every step, outside the timed span
-            scrub.add_(1)
+            flush_l2(scrub)
             torch.cuda.current_stream().synchronize()
         t0 = time.perf_counter()
         dev_flat.copy_(host_flat, non_blocking=True)
@@ -349,8 +358,9 @@ def run_mikv(args):
         "config": {"workload": w.name, "batch": w.batch, "layers": L, "heads_q": w.heads_q, "heads_kv": w.heads_kv,
                    "context": w.context, "bits": w.bits, "group": w.group, "importance_ratio": w.ratio,
                    "compressed_bytes_per_step": int(bytes_per_step), "l2": ("cache larger than L2, no flush" if scrub is None else
-                         f"cache smaller than L2: L2 flushed by a {L2_FLUSH_BYTES >> 20} MiB write before every "
-                         "timed step and launch (not timed); per-step CUDA events summed"),
+                         f"cache smaller than L2: L2 flushed before every timed step and launch (not timed) by a "
+                         f"{L2_FLUSH_BYTES >> 21} MiB write and a {L2_FLUSH_BYTES >> 21} MiB read; per-step CUDA "
+                         "events summed"),
                    "parallelism": f"replicas{world}"},
         "roofline": {"kernel": "decode attention (split-K + merge)", "bound": "hbm", "achieved": round(achieved, 1),
                      "peak": peak, "unit": "GB/s", "frac": round(achieved / peak, 3),
@@ -579,6 +589,7 @@ def run_sweep(args):
                                                                      - layer.cache.nbytes_attended(0)) / 2
         ws = torch.zeros(pkg.mikv_workspace_bytes(shape, pkg.WS_ATTENTION, layer.n_lo) + 256, dtype=torch.uint8,
                          device=dev)
+        pkg.mikv_decode_attention(layer.cache, layer.n_lo, ins[0][0], layer.sm_scale, out, ws)  # untimed first call
         a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a0.record()
         for _ in range(K):

@@ -296,6 +296,20 @@ mikv_status mikv_decode_attention_noalloc(const mikv_shape* shape, const mikv_ca
 mikv_status mikv_noalloc_check(void* stream);
 
 /*
+ * Debug builds. Every kernel that takes an index from device memory (an insertion slot in `slots`, a source row in
+ * `rows`, the victim of a step) skips the access when the index is out of range, without error. A library built
+ * with -DMIKV_DEBUG also records each such skip, and the internal invariants of the attention work split, as a
+ * failure: in the workspace status word for the entry points with a workspace (read by mikv_workspace_check), and
+ * in a status word of its own for mikv_insert_token, mikv_gather_hi and mikv_quantize_pack. No kernel traps.
+ *   mikv_debug_enabled  1 if this library was built with -DMIKV_DEBUG, else 0. Host-only.
+ *   mikv_debug_check    synchronises `stream`, reads and clears the library's own status word and returns
+ *                       MIKV_ERR_DEVICE if an index check failed since the last call, else MIKV_OK (always
+ *                       MIKV_OK in release builds).
+ */
+int32_t mikv_debug_enabled(void);
+mikv_status mikv_debug_check(void* stream);
+
+/*
  * KV-cache size as a fraction of an all-fp16 cache (the "Cache size" columns of Tables 2-3): a ratio
  * `ratio` of tokens kept at hi_bits (16 = fp16; otherwise hi_bits-bit codes plus fp16 alpha/beta per
  * group) and the rest at `bits`-bit codes plus fp16 alpha/beta per `group` channels:

@@ -23,7 +23,7 @@ __all__ = [
     "mikv_decode_attention", "mikv_update_importance", "mikv_select_demote", "mikv_insert_token",
     "mikv_gather_hi", "mikv_decode_step", "mikv_cache_fraction", "mikv_retained_row_bytes",
     "mikv_decode_attention_noalloc", "mikv_noalloc_check", "NOALLOC_SCRATCH_BYTES", "mikv_prefill_scores",
-    "mikv_budget", "shape_for_context",
+    "mikv_budget", "shape_for_context", "mikv_debug_check", "debug_build",
     "WS_ATTENTION", "WS_BALANCER", "WS_STEP", "WS_PREFILL", "OUT_BF16", "OUT_F32", "HEAD_DIM",
 ]
 
@@ -59,15 +59,18 @@ _lock = threading.Lock()
 
 
 def load(build_if_missing: bool = True) -> ctypes.CDLL:
-    """Load libmikv.so (building it with nvcc first when it is missing or stale)."""
+    """Load libmikv.so (building it with nvcc first when it is missing or stale). With MIKV_DEBUG=1 in the
+    environment the checked build (libmikv_debug.so, -DMIKV_DEBUG) is loaded instead."""
     global _lib
     with _lock:
         if _lib is None:
-            if build_if_missing and not _build.up_to_date():
-                _build.build()
-            if not os.path.exists(_build.LIB):
-                raise RuntimeError(f"libmikv is not built ({_build.LIB}); run paper_2402_18096_gb300.build")
-            lib = ctypes.CDLL(_build.LIB)
+            debug = os.environ.get("MIKV_DEBUG", "") == "1"
+            path = _build.LIB_DEBUG if debug else _build.LIB
+            if build_if_missing and not _build.up_to_date(debug):
+                _build.build(debug=debug)
+            if not os.path.exists(path):
+                raise RuntimeError(f"libmikv is not built ({path}); run paper_2402_18096_gb300.build")
+            lib = ctypes.CDLL(path)
             P, I, Z, F = ctypes.c_void_p, ctypes.c_int32, ctypes.c_size_t, ctypes.c_float
             SP = ctypes.POINTER(_Shape)
             CP = ctypes.POINTER(_Cache)
@@ -87,6 +90,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
                 "mikv_decode_attention_noalloc": (I, [SP, CP, I, P, F, P, I, P, P, P]),
                 "mikv_noalloc_check": (I, [P]),
                 "mikv_budget": (I, [I, ctypes.c_double]),
+                "mikv_debug_enabled": (I, []),
+                "mikv_debug_check": (I, [P]),
                 "mikv_prefill_scores": (I, [SP, P, P, I, F, P, P, Z, P]),
                 "mikv_cache_fraction": (ctypes.c_double, [I, I, ctypes.c_double, I]),
                 "mikv_retained_row_bytes": (Z, [I, I, I]),
@@ -262,6 +267,17 @@ def mikv_noalloc_check(stream=None):
     """Raise MikvError(MIKV_ERR_DEVICE) if the last mikv_decode_attention_noalloc call's kernels reported a
     failure in the built-in buffer's status word (synchronises the stream)."""
     _check("mikv_noalloc_check", load().mikv_noalloc_check(_stream(stream)))
+
+
+def debug_build() -> bool:
+    """Whether the loaded library is the checked build (-DMIKV_DEBUG)."""
+    return bool(load().mikv_debug_enabled())
+
+
+def mikv_debug_check(stream=None):
+    """Raise MikvError(MIKV_ERR_DEVICE) if a kernel of a checked build found an out-of-range index since the last
+    call (entry points without a workspace); clears the word. A release build always passes."""
+    _check("mikv_debug_check", load().mikv_debug_check(_stream(stream)))
 
 
 def mikv_update_importance(cache: LayerCache, hi_logits, ml, stream=None):

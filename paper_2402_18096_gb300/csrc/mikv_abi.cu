@@ -15,6 +15,18 @@
 
 using namespace mikv;
 
+// The library's own status word for the index checks of debug builds (-DMIKV_DEBUG) in the entry points that take
+// no workspace (insertion, gather, quantize/pack). Looked up in the current context on every use.
+#ifdef MIKV_DEBUG
+static __device__ int g_debug_status;
+int* mikv::debug_status_word() {
+  void* p = nullptr;
+  return cudaGetSymbolAddress(&p, g_debug_status) == cudaSuccess ? static_cast<int*>(p) : nullptr;
+}
+#else
+int* mikv::debug_status_word() { return nullptr; }
+#endif
+
 namespace {
 
 mikv_status cuda_status(cudaError_t e) { return e == cudaSuccess ? MIKV_OK : MIKV_ERR_CUDA; }
@@ -468,6 +480,7 @@ mikv_status mikv_decode_step(const mikv_shape* shape, const mikv_cache* cache, i
                            v_new, tok)) != MIKV_OK)
     return st;
   StepPostArgs p;
+  p.status = a.status;
   p.part_o = a.part_o;
   p.part_ml = a.part_ml;
   p.out = out;
@@ -570,4 +583,28 @@ extern "C" mikv_status mikv_noalloc_check(void* stream) {
   mikv_status st = noalloc_scratch(&ws);
   if (st != MIKV_OK) return st;
   return mikv_workspace_check(ws, stream);
+}
+
+extern "C" int32_t mikv_debug_enabled(void) {
+#ifdef MIKV_DEBUG
+  return 1;
+#else
+  return 0;
+#endif
+}
+
+extern "C" mikv_status mikv_debug_check(void* stream) {
+#ifdef MIKV_DEBUG
+  int* w = debug_status_word();
+  if (!w) return MIKV_ERR_CUDA;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int v = 0;
+  if (cudaMemcpyAsync(&v, w, sizeof v, cudaMemcpyDeviceToHost, st) != cudaSuccess) return MIKV_ERR_CUDA;
+  if (cudaMemsetAsync(w, 0, sizeof(int), st) != cudaSuccess) return MIKV_ERR_CUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return MIKV_ERR_CUDA;
+  return v == 0 ? MIKV_OK : MIKV_ERR_DEVICE;
+#else
+  (void)stream;
+  return MIKV_OK;
+#endif
 }

@@ -61,6 +61,9 @@ namespace {
 #ifndef MIKV_PAIR_ACC
 #define MIKV_PAIR_ACC 1
 #endif
+#ifndef MIKV_L2_AHEAD
+#define MIKV_L2_AHEAD 2
+#endif
 constexpr int kWarps = MIKV_ATTN_WARPS;     // independent warps per CTA
 constexpr int kThreads = kWarps * 32;
 constexpr int kNS = MIKV_ATTN_STAGES;       // ring stages per warp
@@ -71,6 +74,7 @@ constexpr int kHiBlockBytes = 8192;         // K and V of 16 tokens: 4 boxes of 
 constexpr int kCtasPerSm = MIKV_ATTN_CTAS;
 constexpr int kQkAcc = MIKV_QK_ACC;         // independent accumulators of the QK^T MMA chain
 constexpr int kUnitsPerWarp = 24;    // target share per warp (sizes the grid for small caches)
+constexpr int kL2Ahead = MIKV_L2_AHEAD;  // units a warp prefetches into L2 beyond its shared-memory ring
 constexpr float kLog2e = 1.4426950408889634f;
 
 __host__ __device__ constexpr int smem_bytes() { return 1024 + kWarps * kNS * kStageBytes + kWarps * kNS * 8; }
@@ -139,41 +143,48 @@ __device__ __forceinline__ void sum_acc(const float (&accs)[Q][4], float (&acc)[
 // more than kLazy; otherwise the block reuses the old reference, so probabilities stay below e^kLazy.
 constexpr float kLazy = 4.f;
 
-template <int NB, int NK>
+// ODD: whether head 2t + 1 can exist (G > 1). With one query head per KV head only column 0 of the MMA tiles
+// (lanes with t = 0, head 0) is real, so the odd column's statistics and probabilities are skipped (its
+// probabilities are 0, which keeps the column's output sums at 0).
+template <int NB, int NK, bool ODD = true>
 __device__ __forceinline__ void softmax_blocks(const float (&s)[NK][4], Softmax& st, float (&o)[8][4],
                                                float (&ob)[NB][4], float (&p)[NK][4]) {
-  float bm0 = fmaxf(s[0][0], s[0][2]), bm1 = fmaxf(s[0][1], s[0][3]);
+  float bm0 = fmaxf(s[0][0], s[0][2]), bm1 = ODD ? fmaxf(s[0][1], s[0][3]) : -INFINITY;
 #pragma unroll
   for (int k = 1; k < NK; ++k) {
     bm0 = fmaxf(bm0, fmaxf(s[k][0], s[k][2]));
-    bm1 = fmaxf(bm1, fmaxf(s[k][1], s[k][3]));
+    if (ODD) bm1 = fmaxf(bm1, fmaxf(s[k][1], s[k][3]));
   }
   st.mx[0] = fmaxf(st.mx[0], bm0);
-  st.mx[1] = fmaxf(st.mx[1], bm1);
-  if (__any_sync(0xffffffffu, bm0 > st.m[0] + kLazy || bm1 > st.m[1] + kLazy)) {
+  if (ODD) st.mx[1] = fmaxf(st.mx[1], bm1);
+  if (__any_sync(0xffffffffu, bm0 > st.m[0] + kLazy || (ODD && bm1 > st.m[1] + kLazy))) {
 #pragma unroll
     for (int off = 4; off < 32; off <<= 1) {
       bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, off));
-      bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, off));
+      if (ODD) bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, off));
     }
-    const float mn0 = fmaxf(st.m[0], bm0), mn1 = fmaxf(st.m[1], bm1);
+    const float mn0 = fmaxf(st.m[0], bm0), mn1 = ODD ? fmaxf(st.m[1], bm1) : st.m[1];
     const float c0 = mn0 == st.m[0] ? 1.f : fast_exp2((st.m[0] - mn0) * kLog2e);
-    const float c1 = mn1 == st.m[1] ? 1.f : fast_exp2((st.m[1] - mn1) * kLog2e);
+    const float c1 = !ODD || mn1 == st.m[1] ? 1.f : fast_exp2((st.m[1] - mn1) * kLog2e);
     st.l[0] *= c0;
-    st.l[1] *= c1;
+    if (ODD) st.l[1] *= c1;
 #pragma unroll
     for (int mt = 0; mt < 8; ++mt) {
       o[mt][0] *= c0;
-      o[mt][1] *= c1;
       o[mt][2] *= c0;
-      o[mt][3] *= c1;
+      if (ODD) {
+        o[mt][1] *= c1;
+        o[mt][3] *= c1;
+      }
     }
 #pragma unroll
     for (int i = 0; i < NB; ++i) {
       ob[i][0] *= c0;
-      ob[i][1] *= c1;
       ob[i][2] *= c0;
-      ob[i][3] *= c1;
+      if (ODD) {
+        ob[i][1] *= c1;
+        ob[i][3] *= c1;
+      }
     }
     st.m[0] = mn0;
     st.m[1] = mn1;
@@ -182,11 +193,15 @@ __device__ __forceinline__ void softmax_blocks(const float (&s)[NK][4], Softmax&
 #pragma unroll
   for (int k = 0; k < NK; ++k) {
     p[k][0] = fast_exp2(fmaf(s[k][0], kLog2e, -ml0));
-    p[k][1] = fast_exp2(fmaf(s[k][1], kLog2e, -ml1));
     p[k][2] = fast_exp2(fmaf(s[k][2], kLog2e, -ml0));
-    p[k][3] = fast_exp2(fmaf(s[k][3], kLog2e, -ml1));
     st.l[0] += p[k][0] + p[k][2];
-    st.l[1] += p[k][1] + p[k][3];
+    if (ODD) {
+      p[k][1] = fast_exp2(fmaf(s[k][1], kLog2e, -ml1));
+      p[k][3] = fast_exp2(fmaf(s[k][3], kLog2e, -ml1));
+      st.l[1] += p[k][1] + p[k][3];
+    } else {
+      p[k][1] = p[k][3] = 0.f;
+    }
   }
 }
 
@@ -319,7 +334,7 @@ __device__ __forceinline__ void process_hi(uint32_t blk, int valid, int slot0, c
   sum_acc(accs, acc);
   float s[1][4], p[1][4];
   finish_logits<G>(acc, scale, valid, g, t, logit_base, hi_stride, slot0, s[0]);
-  softmax_blocks(s, st, o, ob, p);
+  softmax_blocks<NB, 1, (G > 1)>(s, st, o, ob, p);
   const uint32_t pb0 = movmatrix_t(pack_bf16(p[0][0], p[0][1]));
   const uint32_t pb1 = movmatrix_t(pack_bf16(p[0][2], p[0][3]));
   {
@@ -666,7 +681,7 @@ __device__ __forceinline__ void process_coded(uint32_t unit, int b, int n_left, 
     lo_logits<BITS, GROUP, G, NK == 1 ? kQkAcc : kPairAcc, KCH>(unit, b + k, min(16, n_left - 16 * k), qh, scale,
                                                                 s[k], lane, HI ? logit_base : nullptr, hi_stride,
                                                                 slot0 + 16 * k, kbias);
-  softmax_blocks(s, st, o, ob, p);
+  softmax_blocks<NB, NK, (G > 1)>(s, st, o, ob, p);
 #pragma unroll
   for (int k = 0; k < NK; ++k)
     lo_values<BITS, GROUP, NB, HI, KCH>(unit, b + k, min(16, n_left - 16 * k), p[k], o, ob, lane);
@@ -737,6 +752,8 @@ __device__ __forceinline__ void issue_unit(const AttnArgs& a, const Cursor& c, u
       return;
     }
   }
+  MIKV_DEBUG_ASSERT(c.bh < a.batch * a.heads_kv && c.i < a.n_u, a.status);
+  MIKV_DEBUG_ASSERT(k.hi ? 16 * k.index < a.hi_stride : 16 * U.blocks * k.index < a.lo_cap, a.status);
   if (k.hi) {
     const int row = c.bh * a.hi_stride + 16 * k.index;
     mbar_arrive_expect_tx(bar, kHiBlockBytes);
@@ -862,11 +879,18 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
       prefetch_tensormap(&a.map_v_par);
     }
   }
-  if (lane == 0)  // warm L2 with this warp's first units while the previous kernel drains (reads only)
-    for (int k = 0; k < kNS && u0 + k < u1; ++k) {
-      Cursor cp = cursor_at(u0 + k, hu, n_u);
+  // L2 look-ahead: besides the kNS units in its ring, each warp keeps kL2Ahead further units on their way into
+  // L2 (a prefetch needs no shared memory), so a warp that waits on memory has twice the data in flight. The
+  // first ones are requested while the previous kernel drains (reads only; L2 stays coherent with its writes).
+  __shared__ Cursor s_pf[kWarps];  // next unit to prefetch into L2 (lane 0)
+  if (lane == 0) {
+    Cursor cp = cursor_at(u0, hu, n_u);
+    for (int k = 0; k < kNS + kL2Ahead && u0 + k < u1; ++k) {
       prefetch_unit<BITS, GROUP, HB, KCH>(a, cp);
+      cursor_next(cp, hu, n_u);
     }
+    s_pf[warp] = cp;  // unit u0 + kNS + kL2Ahead
+  }
   grid_dependency_wait();  // the cache and the query come from the kernels before this one
   allow_dependent_launch();
   if (lane == 0) {
@@ -924,7 +948,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
         __syncwarp();
         if (lane == 0) {
           const int sl = a.ins_slots[cur];
-          s_ins[warp] = sl < a.hi_cap ? sl : -1;
+          const bool ok = sl >= 0 && sl < a.hi_cap;  // an out-of-range slot inserts nothing
+          if (!ok) MIKV_BOUNDS_FAIL(a.status);
+          s_ins[warp] = ok ? sl : -1;
         }
         __syncwarp();
       }
@@ -992,6 +1018,12 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
       fence_proxy_async();  // our generic reads of this stage precede the next asynchronous write
       issue_unit<BITS, GROUP, HB, KCH>(a, ci, stage, bars + 8 * s, pol);
       cursor_next(ci, hu, n_u);
+      if (kL2Ahead > 0 && u + kNS + kL2Ahead < u1) {
+        Cursor cp = s_pf[warp];
+        prefetch_unit<BITS, GROUP, HB, KCH>(a, cp);
+        cursor_next(cp, hu, n_u);
+        s_pf[warp] = cp;
+      }
     }
   }
   if (failed) {

@@ -14,7 +14,7 @@ constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s: a correct pipeline nev
 
 // Workspace header: status word set by kernels on an internal failure (0 = none).
 constexpr size_t kWsHeader = 256;
-enum DeviceError : int { kErrFullTimeout = 1, kErrEmptyTimeout = 2, kErrDrainTimeout = 3 };
+enum DeviceError : int { kErrFullTimeout = 1, kErrEmptyTimeout = 2, kErrDrainTimeout = 3, kErrBounds = 4 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -235,6 +235,22 @@ __device__ __forceinline__ uint32_t pack_f16(float lo, float hi) {
 __device__ __forceinline__ void record_error(int* status, int code) {
   if (status) atomicCAS(status, 0, code);
 }
+
+// Index checks. Every kernel that takes an index from device memory (an insertion slot, a source row, a victim)
+// skips the access when the index is out of range. A debug build (-DMIKV_DEBUG) also records each such skip, and
+// the by-construction invariants of the work split, as kErrBounds in a status word (the workspace's, or the
+// library's own debug word for the entry points without a workspace); a release build skips silently. Neither
+// traps.
+#ifdef MIKV_DEBUG
+#define MIKV_BOUNDS_FAIL(status) ::mikv::record_error((status), ::mikv::kErrBounds)
+#define MIKV_DEBUG_ASSERT(cond, status) \
+  do {                                  \
+    if (!(cond)) MIKV_BOUNDS_FAIL(status); \
+  } while (0)
+#else
+#define MIKV_BOUNDS_FAIL(status) ((void)0)
+#define MIKV_DEBUG_ASSERT(cond, status) ((void)0)
+#endif
 
 // Packed pairs of fp32 (one 64-bit register, low word first) for the two-wide fp32 instructions of sm_100-class
 // GPUs: half the instructions of the scalar forms.

@@ -11,6 +11,10 @@
 
 namespace mikv {
 
+// The library's status word for index checks of the entry points without a workspace (debug builds, -DMIKV_DEBUG;
+// nullptr in release builds). Defined in mikv_abi.cu; read by mikv_debug_check.
+int* debug_status_word();
+
 // Shared-memory layout of one retained unit: up to `blocks` consecutive 16-token blocks loaded with
 // one TMA box per array (codes of K, codes of V, parameters of K, parameters of V; N = 3 adds the
 // 1-bit planes). Offsets are in bytes from the unit's stage; each section starts on the alignment its
@@ -156,6 +160,7 @@ struct StepPostArgs {
   int hi_bits;              // 16 = bf16 important rows; 8, 4, 2 = coded (groups of kHiGroup)
   int evict;                // no retained set: the victim's slot is freed, nothing is demoted
   int kch;                  // per-channel retained keys: the victim is staged at important row hi_cap + n_lo % 64
+  int* status;              // the workspace status word (index checks of debug builds)
   int batch, heads_q, heads_kv, hi_cap, hi_stride, lo_cap, n_lo;
   int n_u, n_units, n_warps;
 };

@@ -151,12 +151,15 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const float* scores
 __global__ void __launch_bounds__(64) insert_kernel(__nv_bfloat16* k_hi, __nv_bfloat16* v_hi, int32_t* hi_tok,
                                                     float* acc, const __nv_bfloat16* k_new,
                                                     const __nv_bfloat16* v_new, int tok, const int32_t* slots,
-                                                    int hi_cap, int hi_stride) {
+                                                    int hi_cap, int hi_stride, int* dbg) {
   const int bh = blockIdx.x, tid = threadIdx.x;
   grid_dependency_wait();  // the slot comes from the previous step's tail
   allow_dependent_launch();
   const int s = slots[bh];
-  if (s < 0 || s >= hi_cap) return;
+  if (s < 0 || s >= hi_cap) {  // an out-of-range slot is skipped (recorded in debug builds)
+    if (tid == 0) MIKV_BOUNDS_FAIL(dbg);
+    return;
+  }
   const size_t row = (size_t)bh * hi_stride + s;
   if (tid < 32) {
     reinterpret_cast<uint2*>(k_hi + row * kHeadDim)[tid] =
@@ -175,12 +178,15 @@ __global__ void __launch_bounds__(256) gather_kernel(__nv_bfloat16* k_hi, __nv_b
                                                      float* acc, const __nv_bfloat16* k_src,
                                                      const __nv_bfloat16* v_src, const int32_t* src_tok,
                                                      const float* src_scores, int n_src, const int32_t* rows,
-                                                     int n_rows, int hi_stride) {
+                                                     int n_rows, int hi_stride, int* dbg) {
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int i = blockIdx.x * 8 + w, bh = blockIdx.y;
   if (i >= n_rows) return;
   const int r = rows[(size_t)bh * n_rows + i];
-  if (r < 0 || r >= n_src) return;
+  if (r < 0 || r >= n_src) {  // an out-of-range source row is skipped (recorded in debug builds)
+    if (lane == 0) MIKV_BOUNDS_FAIL(dbg);
+    return;
+  }
   const size_t src = ((size_t)bh * n_src + r) * kHeadDim, dst = ((size_t)bh * hi_stride + i) * kHeadDim;
   reinterpret_cast<uint2*>(k_hi + dst)[lane] = reinterpret_cast<const uint2*>(k_src + src)[lane];
   reinterpret_cast<uint2*>(v_hi + dst)[lane] = reinterpret_cast<const uint2*>(v_src + src)[lane];
@@ -213,7 +219,7 @@ cudaError_t launch_insert(const mikv_shape& s, const mikv_cache& c, const void* 
   return launch_chained(insert_kernel, dim3(s.batch * s.heads_kv), dim3(64), 0, st,
                         static_cast<__nv_bfloat16*>(c.k_hi), static_cast<__nv_bfloat16*>(c.v_hi), c.hi_tok, c.acc,
                         static_cast<const __nv_bfloat16*>(k_new), static_cast<const __nv_bfloat16*>(v_new), tok, slots,
-                        s.hi_cap, s.hi_stride);
+                        s.hi_cap, s.hi_stride, debug_status_word());
 }
 
 cudaError_t launch_gather(const mikv_shape& s, const mikv_cache& c, const void* k_src, const void* v_src,
@@ -226,7 +232,7 @@ cudaError_t launch_gather(const mikv_shape& s, const mikv_cache& c, const void* 
   gather_kernel<<<grid, 256, 0, st>>>(static_cast<__nv_bfloat16*>(c.k_hi), static_cast<__nv_bfloat16*>(c.v_hi),
                                       c.hi_tok, c.acc, static_cast<const __nv_bfloat16*>(k_src),
                                       static_cast<const __nv_bfloat16*>(v_src), src_tok, src_scores, n_src, rows,
-                                      n_rows, s.hi_stride);
+                                      n_rows, s.hi_stride, debug_status_word());
   return cudaGetLastError();
 }
 

@@ -25,6 +25,7 @@ struct QPArgs {
   __half2* k_params;
   __half2* v_params;
   int32_t* lo_tok;
+  int* dbg;  // debug builds: the library's status word for index checks (nullptr otherwise)
   int heads_kv, n_src, n_rows, lo_start, lo_cap;
 };
 
@@ -65,6 +66,7 @@ __global__ void __launch_bounds__(256) quantize_pack_kernel(const QPArgs a) {
   const int i = (blockIdx.x * 4 + (w >> 1)) * kQpRowsPerWarp + (lane >> 3);
   const int r = i < a.n_rows ? a.rows[(size_t)bh * a.n_rows + i] : -1;
   const bool valid = r >= 0 && r < a.n_src;  // out-of-range rows are skipped (documented in the ABI)
+  if (i < a.n_rows && !valid && l8 == 0 && !is_v) MIKV_BOUNDS_FAIL(a.dbg);
   // invalid rows run the arithmetic on zeros (every lane takes part in the shuffles) and store nothing
   uint4 raw[2] = {make_uint4(0u, 0u, 0u, 0u), make_uint4(0u, 0u, 0u, 0u)};
   if (valid) {
@@ -200,6 +202,7 @@ struct HiQArgs {
   __half2* v_hp;
   int32_t* hi_tok;
   float* acc;
+  int* dbg;  // debug builds: the library's status word for index checks (nullptr otherwise)
   int heads_kv, hi_cap, hi_stride, n_src, n_rows, tok;
 };
 
@@ -216,13 +219,19 @@ __global__ void __launch_bounds__(256) hi_quant_kernel(const HiQArgs a) {
   if (a.rows) {
     if (i >= a.n_rows) return;
     r = a.rows[(size_t)bh * a.n_rows + i];
-    if (r < 0 || r >= a.n_src) return;  // out-of-range rows are skipped, as in quantize_pack
+    if (r < 0 || r >= a.n_src) {  // out-of-range rows are skipped, as in quantize_pack
+      if (lane == 0 && !is_v) MIKV_BOUNDS_FAIL(a.dbg);
+      return;
+    }
     slot = i;
     src = (is_v ? a.v_src : a.k_src) + ((size_t)bh * a.n_src + r) * kHeadDim;
   } else {
     if (i > 0) return;
     slot = a.slots[bh];
-    if (slot < 0 || slot >= a.hi_cap) return;
+    if (slot < 0 || slot >= a.hi_cap) {
+      if (lane == 0 && !is_v) MIKV_BOUNDS_FAIL(a.dbg);
+      return;
+    }
     src = (is_v ? a.v_src : a.k_src) + (size_t)bh * kHeadDim;
   }
   const size_t row = (size_t)bh * a.hi_stride + slot;
@@ -253,6 +262,7 @@ struct KchArgs {
   __half2* k_params;  // [B][Hkv][lo_cap / 64][128]
   __half2* v_params;
   int32_t* lo_tok;
+  int* dbg;  // debug builds: the library's status word for index checks (nullptr otherwise)
   int heads_kv, hi_cap, hi_stride, lo_cap, n_src, n_rows, p0, p_end, g0;
 };
 
@@ -268,7 +278,10 @@ __device__ __forceinline__ const __nv_bfloat16* kch_row(const KchArgs& a, int bh
   }
   const int r = a.rows[(size_t)bh * a.n_rows + (p - a.p0)];
   if (tok) *tok = (r >= 0 && r < a.n_src) ? (a.src_tok ? a.src_tok[(size_t)bh * a.n_src + r] : r) : -1;
-  if (r < 0 || r >= a.n_src) return nullptr;
+  if (r < 0 || r >= a.n_src) {
+    if (key) MIKV_BOUNDS_FAIL(a.dbg);
+    return nullptr;
+  }
   return (key ? a.k_src : a.v_src) + ((size_t)bh * a.n_src + r) * kHeadDim;
 }
 
@@ -397,7 +410,8 @@ cudaError_t launch_quantize_pack(const mikv_shape& s, const mikv_cache& c, const
                                  const void* v_src, const int32_t* src_tok, int n_src,
                                  const int32_t* rows, int n_rows, int lo_start, cudaStream_t st) {
   if (n_rows == 0) return cudaSuccess;
-  QPArgs a;
+  QPArgs a = {};
+  a.dbg = debug_status_word();
   a.k_src = static_cast<const __nv_bfloat16*>(k_src);
   a.v_src = static_cast<const __nv_bfloat16*>(v_src);
   a.src_tok = src_tok;
@@ -425,7 +439,8 @@ cudaError_t launch_quantize_pack(const mikv_shape& s, const mikv_cache& c, const
 cudaError_t launch_hi_quant(const mikv_shape& s, const mikv_cache& c, const void* k_src, const void* v_src,
                             const int32_t* src_tok, const float* src_scores, int n_src, const int32_t* rows,
                             int n_rows, const int32_t* slots, int tok, cudaStream_t st) {
-  HiQArgs a;
+  HiQArgs a = {};
+  a.dbg = debug_status_word();
   a.k_src = static_cast<const __nv_bfloat16*>(k_src);
   a.v_src = static_cast<const __nv_bfloat16*>(v_src);
   a.src_tok = src_tok;
@@ -458,7 +473,8 @@ cudaError_t launch_hi_quant(const mikv_shape& s, const mikv_cache& c, const void
 cudaError_t launch_kch_append(const mikv_shape& s, const mikv_cache& c, const void* k_src, const void* v_src,
                               const int32_t* src_tok, int n_src, const int32_t* rows, int n_rows, int p0,
                               cudaStream_t st) {
-  KchArgs a;
+  KchArgs a = {};
+  a.dbg = debug_status_word();
   a.k_src = static_cast<const __nv_bfloat16*>(k_src);
   a.v_src = static_cast<const __nv_bfloat16*>(v_src);
   a.src_tok = src_tok;

@@ -161,7 +161,12 @@ __global__ void __launch_bounds__(kPostThreads, 2) step_post_kernel(const StepPo
     }
   }
   const int victim = s_victim;
-  if (victim < 0) return;  // unreachable for valid scores (hi_cap >= 1, no NaN)
+  if (victim < 0 || victim >= a.hi_cap) {  // unreachable for valid scores (hi_cap >= 1, no NaN)
+    if (tid == 0) MIKV_BOUNDS_FAIL(a.status);
+    return;
+  }
+  MIKV_DEBUG_ASSERT(a.evict || a.n_lo < a.lo_cap, a.status);
+  MIKV_DEBUG_ASSERT(!a.kch || a.hi_cap + a.n_lo % kKchGroup < a.hi_stride, a.status);
 
   // 4. demote the victim: quantize its key (balanced, Eq. 3) and value rows into retained row n_lo; a
   // coded important row is re-quantized from its fp32 dequantized values (already balanced, Sec. 3.3)
