@@ -61,9 +61,6 @@ namespace {
 #ifndef MIKV_PAIR_ACC
 #define MIKV_PAIR_ACC 1
 #endif
-#ifndef MIKV_L2_AHEAD
-#define MIKV_L2_AHEAD 2
-#endif
 constexpr int kWarps = MIKV_ATTN_WARPS;     // independent warps per CTA
 constexpr int kThreads = kWarps * 32;
 constexpr int kNS = MIKV_ATTN_STAGES;       // ring stages per warp
@@ -74,7 +71,6 @@ constexpr int kHiBlockBytes = 8192;         // K and V of 16 tokens: 4 boxes of 
 constexpr int kCtasPerSm = MIKV_ATTN_CTAS;
 constexpr int kQkAcc = MIKV_QK_ACC;         // independent accumulators of the QK^T MMA chain
 constexpr int kUnitsPerWarp = 24;    // target share per warp (sizes the grid for small caches)
-constexpr int kL2Ahead = MIKV_L2_AHEAD;  // units a warp prefetches into L2 beyond its shared-memory ring
 constexpr float kLog2e = 1.4426950408889634f;
 
 __host__ __device__ constexpr int smem_bytes() { return 1024 + kWarps * kNS * kStageBytes + kWarps * kNS * 8; }
@@ -879,17 +875,14 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
       prefetch_tensormap(&a.map_v_par);
     }
   }
-  // L2 look-ahead: besides the kNS units in its ring, each warp keeps kL2Ahead further units on their way into
-  // L2 (a prefetch needs no shared memory), so a warp that waits on memory has twice the data in flight. The
-  // first ones are requested while the previous kernel drains (reads only; L2 stays coherent with its writes).
-  __shared__ Cursor s_pf[kWarps];  // next unit to prefetch into L2 (lane 0)
+  // warm L2 with this warp's first units while the previous kernel drains (reads only; L2 stays coherent with
+  // its writes). Prefetching further ahead than the ring during the stream measured slower on every shape.
   if (lane == 0) {
     Cursor cp = cursor_at(u0, hu, n_u);
-    for (int k = 0; k < kNS + kL2Ahead && u0 + k < u1; ++k) {
+    for (int k = 0; k < kNS && u0 + k < u1; ++k) {
       prefetch_unit<BITS, GROUP, HB, KCH>(a, cp);
       cursor_next(cp, hu, n_u);
     }
-    s_pf[warp] = cp;  // unit u0 + kNS + kL2Ahead
   }
   grid_dependency_wait();  // the cache and the query come from the kernels before this one
   allow_dependent_launch();
@@ -1018,12 +1011,6 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
       fence_proxy_async();  // our generic reads of this stage precede the next asynchronous write
       issue_unit<BITS, GROUP, HB, KCH>(a, ci, stage, bars + 8 * s, pol);
       cursor_next(ci, hu, n_u);
-      if (kL2Ahead > 0 && u + kNS + kL2Ahead < u1) {
-        Cursor cp = s_pf[warp];
-        prefetch_unit<BITS, GROUP, HB, KCH>(a, cp);
-        cursor_next(cp, hu, n_u);
-        s_pf[warp] = cp;
-      }
     }
   }
   if (failed) {
