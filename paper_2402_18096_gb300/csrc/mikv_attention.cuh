@@ -61,6 +61,9 @@ namespace {
 #ifndef MIKV_PAIR_ACC
 #define MIKV_PAIR_ACC 1
 #endif
+#ifndef MIKV_MHA_PATH
+#define MIKV_MHA_PATH 1
+#endif
 constexpr int kWarps = MIKV_ATTN_WARPS;     // independent warps per CTA
 constexpr int kThreads = kWarps * 32;
 constexpr int kNS = MIKV_ATTN_STAGES;       // ring stages per warp
@@ -308,6 +311,131 @@ __host__ __device__ constexpr float voff(int mt) {
   return BITS == 2 ? voff2(mt) : BITS == 4 ? voff4(mt & 3) : BITS == 3 ? voff3(mt) : 0.f;
 }
 
+// The code fragments of one 16-token block (N = 2, 3, 4). KeyFrag: the QK^T A operand (tokens g, g + 8 on M,
+// channels on K) with exact codes; ValFrag: the PV A operand (channels on M, tokens 2t, 2t+1, 2t+8, 2t+9 on K) with
+// the codes offset by voff (or exact). `rows` is the block's first code row in the stage (pitch U.pitch bytes).
+template <int BITS, int PITCH>
+struct KeyFrag {
+  static constexpr int NR = BITS == 4 ? 8 : 4;
+  uint32_t kr[NR], kh[NR];
+  uint32_t he0, he1, ho0, ho1, he0s, he1s, ho0s, ho1s;  // N = 3 only
+
+  __device__ __forceinline__ void load(uint32_t rows, int lane) {
+    const int r8 = lane & 7, j = lane >> 3;
+    const int tok = r8 + 8 * (j & 1);
+    uint32_t kb0 = 0, kb1 = 0;
+    if (BITS == 4) {
+      const int o0 = tok * 64 + 16 * (j >> 1), sw = ((tok >> 1) & 3) << 4;
+      uint32_t r0[4], r1[4];
+      ldsm_x4(rows + (o0 ^ sw), r0);
+      ldsm_x4(rows + ((o0 + 32) ^ sw), r1);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        kr[i] = r0[i];
+        kr[(NR == 8 ? 4 : 0) + i] = r1[i];
+      }
+    } else {
+      // N = 2: 32-byte tokens under the 64B swizzle (bits 4..5 ^= bits 7..8); N = 3: 48-byte tokens, unswizzled
+      const int o0 = tok * PITCH + 16 * (j >> 1), sw = BITS == 2 ? ((tok >> 2) & 3) << 4 : 0;
+      uint32_t r0[4];
+      ldsm_x4(rows + (o0 ^ sw), r0);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) kr[i] = r0[i];
+      if (BITS == 3) ldsm_x2(rows + (lane & 15) * PITCH + 32, kb0, kb1);
+    }
+#pragma unroll
+    for (int i = 0; i < NR; ++i) kh[i] = kr[i] >> (BITS == 2 ? 10 : 8);
+    // N = 3: the 1-bit plane words of tokens g (kb0) and g + 8 (kb1) shifted so that the high bit of code ks sits
+    // two bits above its low bits: channels 2t, 2t+1 use the even bits (<< 2 for ks <= 3, >> 6 for ks >= 4),
+    // channels 2t+8, 2t+9 the odd bits (<< 1, >> 7)
+    he0 = kb0 << 2, he1 = kb1 << 2, ho0 = kb0 << 1, ho1 = kb1 << 1;
+    he0s = kb0 >> 6, he1s = kb1 >> 6, ho0s = kb0 >> 7, ho1s = kb1 >> 7;
+  }
+
+  // exact codes of k-step ks (channels 16 ks .. 16 ks + 15) as fp16 pairs
+  __device__ __forceinline__ void code(int ks, uint32_t (&c)[4]) const {
+    if (BITS == 4) {
+      const int ri = (ks >> 2) * 4, p = ks & 3;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) c[i] = code4(kr[ri + i], kh[ri + i], p);
+    } else if (BITS == 2) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) c[i] = code2(kr[i], kh[i], ks);
+    } else {
+      c[0] = kcode3(kr[0], kh[0], he0, he0s, ks);
+      c[1] = kcode3(kr[1], kh[1], he1, he1s, ks);
+      c[2] = kcode3(kr[2], kh[2], ho0, ho0s, ks);
+      c[3] = kcode3(kr[3], kh[3], ho1, ho1s, ks);
+    }
+  }
+};
+
+template <int BITS, int PITCH, bool EXACT>
+struct ValFrag {
+  static constexpr int NR = BITS == 4 ? 8 : 4;
+  uint32_t vr[NR];
+  uint32_t vb0, vb1;  // N = 3: the 1-bit plane words of tokens (2t, 2t+1) and (2t+8, 2t+9)
+
+  __device__ __forceinline__ void load(uint32_t rows, int lane) {
+    const int r8 = lane & 7, j = lane >> 3;
+    const int tok = r8 + 8 * (j >> 1);
+    vb0 = vb1 = 0;
+    if (BITS == 4) {
+      const int o0 = tok * 64 + 16 * (j & 1), sw = ((tok >> 1) & 3) << 4;
+      uint32_t r0[4], r1[4];
+      ldsm_x4_t(rows + (o0 ^ sw), r0);
+      ldsm_x4_t(rows + ((o0 + 32) ^ sw), r1);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        vr[i] = r0[i];
+        vr[(NR == 8 ? 4 : 0) + i] = r1[i];
+      }
+    } else {
+      const int o0 = tok * PITCH + 16 * (j & 1), sw = BITS == 2 ? ((tok >> 2) & 3) << 4 : 0;
+      uint32_t r0[4];
+      ldsm_x4_t(rows + (o0 ^ sw), r0);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) vr[i] = r0[i];
+      if (BITS == 3) ldsm_x2_t(rows + (lane & 15) * PITCH + 32, vb0, vb1);
+    }
+  }
+
+  // codes of channels 16 mt .. 16 mt + 15 (EXACT: exact codes; else the codes plus voff<BITS>(mt))
+  __device__ __forceinline__ void code(int mt, uint32_t (&a)[4]) const {
+    if (BITS == 4) {
+      const int ri = (mt >> 2) * 4, pp = mt & 3;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const uint32_t w = vr[ri + i];
+        if (EXACT) {
+          a[i] = code4(w, w >> 8, pp);
+        } else {
+          const uint32_t c4[4] = {w << 4, w, w >> 2, w >> 6};  // shared by the four mt of this word
+          a[i] = vcode4(c4, pp);
+        }
+      }
+    } else if (BITS == 2) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        if (EXACT)
+          a[i] = code2(vr[i], vr[i] >> 10, mt);
+        else
+          a[i] = vcode2(vr[i] << 4, vr[i], vr[i] >> 6, mt);  // the shifted copies are shared by all mt
+      }
+    } else {
+      // vr[0], vr[2]: channel g (tokens 2t, 2t+1 and 2t+8, 2t+9), whose high bits are the even bits of vb0, vb1;
+      // vr[1], vr[3]: channel g + 8, the odd bits
+      const int k = mt >> 1, s = 4 - 4 * k;  // codes 2k, 2k+1 read at bits 4, 6 of the words shifted by s
+      auto sh = [](uint32_t x, int n) { return n >= 0 ? x << n : x >> -n; };
+      const uint32_t r4[4] = {sh(vr[0], s), sh(vr[1], s), sh(vr[2], s), sh(vr[3], s)};
+      const uint32_t h4[4] = {sh(vb0, s + 2), sh(vb0, s + 1), sh(vb1, s + 2), sh(vb1, s + 1)};
+      const int p = 4 + 2 * (mt & 1);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) a[i] = or_code3(r4[i], h4[i], p, mag2(p >> 1));
+    }
+  }
+};
+
 // ---------------------------------------------------------------------- one important block
 
 template <int G, int NB>
@@ -377,7 +505,6 @@ __device__ __forceinline__ void lo_logits(uint32_t unit, int b, int valid, const
   // this block's rows inside the unit's sections
   const uint32_t ka = unit + U.k_a + b * 16 * U.pitch;
   const uint32_t kp = unit + U.k_p + b * 16 * PR;
-  constexpr int NR = BITS == 4 ? 8 : 4;
   const int g = lane >> 2, t = lane & 3, r8 = lane & 7, j = lane >> 3;
 
   uint32_t pk0[NG], pk1[NG];
@@ -416,55 +543,14 @@ __device__ __forceinline__ void lo_logits(uint32_t unit, int b, int valid, const
   }
 
   // ---- keys of tokens g and g+8
-  uint32_t kr[NR], kh[NR];
-  uint32_t kb0 = 0, kb1 = 0;
-  {
-    const int tok = r8 + 8 * (j & 1);
-    if (BITS == 4) {
-      const int o0 = tok * 64 + 16 * (j >> 1), sw = ((tok >> 1) & 3) << 4;
-      uint32_t r0[4], r1[4];
-      ldsm_x4(ka + (o0 ^ sw), r0);
-      ldsm_x4(ka + ((o0 + 32) ^ sw), r1);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        kr[i] = r0[i];
-        kr[(NR == 8 ? 4 : 0) + i] = r1[i];
-      }
-    } else {
-      // N = 2: 32-byte tokens under the 64B swizzle (bits 4..5 ^= bits 7..8); N = 3: 48-byte tokens, unswizzled
-      const int o0 = tok * U.pitch + 16 * (j >> 1), sw = BITS == 2 ? ((tok >> 2) & 3) << 4 : 0;
-      uint32_t r0[4];
-      ldsm_x4(ka + (o0 ^ sw), r0);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) kr[i] = r0[i];
-      if (BITS == 3) ldsm_x2(ka + (lane & 15) * U.pitch + U.plane_b, kb0, kb1);
-    }
-#pragma unroll
-    for (int i = 0; i < NR; ++i) kh[i] = kr[i] >> (BITS == 2 ? 10 : 8);
-  }
-  // N = 3: the 1-bit plane words of tokens g (kb0) and g + 8 (kb1) shifted so that the high bit of code ks sits
-  // two bits above its low bits: channels 2t, 2t+1 use the even bits (<< 2 for ks <= 3, >> 6 for ks >= 4),
-  // channels 2t+8, 2t+9 the odd bits (<< 1, >> 7)
-  const uint32_t he0 = kb0 << 2, he1 = kb1 << 2, ho0 = kb0 << 1, ho1 = kb1 << 1;
-  const uint32_t he0s = kb0 >> 6, he1s = kb1 >> 6, ho0s = kb0 >> 7, ho1s = kb1 >> 7;
+  KeyFrag<BITS, U.pitch> kf;
+  kf.load(ka, lane);
 #pragma unroll
   for (int ks = 0; ks < 8; ++ks) {
     const int gi = (16 * ks) / GROUP;
     // (alpha, alpha) and (beta, beta) of tokens g and g + 8: half-broadcasts the HFMA2 operand selectors absorb
     uint32_t c[4];
-    if (BITS == 4) {
-      const int ri = (ks >> 2) * 4, p = ks & 3;
-#pragma unroll
-      for (int i = 0; i < 4; ++i) c[i] = code4(kr[ri + i], kh[ri + i], p);
-    } else if (BITS == 2) {
-#pragma unroll
-      for (int i = 0; i < 4; ++i) c[i] = code2(kr[i], kh[i], ks);
-    } else {
-      c[0] = kcode3(kr[0], kh[0], he0, he0s, ks);
-      c[1] = kcode3(kr[1], kh[1], he1, he1s, ks);
-      c[2] = kcode3(kr[2], kh[2], ho0, ho0s, ks);
-      c[3] = kcode3(kr[3], kh[3], ho1, ho1s, ks);
-    }
+    kf.code(ks, c);
     if constexpr (KCH) {
       mma_f16(accs[ks % QACC], c, qh[ks][0], qh[ks][1]);
     } else {
@@ -523,36 +609,14 @@ __device__ __forceinline__ void lo_values(uint32_t unit, int b, int valid, const
   constexpr int PR = U.param_row;
   const uint32_t va = unit + U.v_a + b * 16 * U.pitch;
   const uint32_t vp = unit + U.v_p + b * 16 * PR;
-  constexpr int NR = BITS == 4 ? 8 : 4;
   const int g = lane >> 2, t = lane & 3, r8 = lane & 7, j = lane >> 3;
   const uint32_t pb0 = movmatrix_t(pack_f16(p[0], p[1]));  // (P[2t][head g], P[2t+1][head g])
   const uint32_t pb1 = movmatrix_t(pack_f16(p[2], p[3]));  // tokens 2t+8, 2t+9
 
   // ---- values of tokens (2t, 2t+1) and (2t+8, 2t+9), channels 16 mt + g and 16 mt + 8 + g
-  uint32_t vr[NR];
-  uint32_t vb0 = 0, vb1 = 0;
   const int vtok = r8 + 8 * (j >> 1);
-  if constexpr (BITS != 8) {
-    const int tok = vtok;
-    if (BITS == 4) {
-      const int o0 = tok * 64 + 16 * (j & 1), sw = ((tok >> 1) & 3) << 4;
-      uint32_t r0[4], r1[4];
-      ldsm_x4_t(va + (o0 ^ sw), r0);
-      ldsm_x4_t(va + ((o0 + 32) ^ sw), r1);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        vr[i] = r0[i];
-        vr[(NR == 8 ? 4 : 0) + i] = r1[i];
-      }
-    } else {
-      const int o0 = tok * U.pitch + 16 * (j & 1), sw = BITS == 2 ? ((tok >> 2) & 3) << 4 : 0;
-      uint32_t r0[4];
-      ldsm_x4_t(va + (o0 ^ sw), r0);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) vr[i] = r0[i];
-      if (BITS == 3) ldsm_x2_t(va + (lane & 15) * U.pitch + U.plane_b, vb0, vb1);
-    }
-  }
+  ValFrag<BITS == 8 ? 2 : BITS, U.pitch, EXACT> vf;
+  if constexpr (BITS != 8) vf.load(va, lane);
   // (alpha, beta) of the four tokens for every group; zero past the end (exact zeros in the sums)
   const int t0 = 2 * t, t1 = 2 * t + 1, t8 = 2 * t + 8, t9 = 2 * t + 9;
   uint32_t pv0[NG], pv1[NG], pv8[NG], pv9[NG];
@@ -627,37 +691,7 @@ __device__ __forceinline__ void lo_values(uint32_t unit, int b, int valid, const
   for (int mt = 0; mt < 8; ++mt) {
     const int gi = (16 * mt) / GROUP;
     uint32_t a[4];
-    if (BITS == 4) {
-      const int ri = (mt >> 2) * 4, pp = mt & 3;
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const uint32_t w = vr[ri + i];
-        if (EXACT) {
-          a[i] = code4(w, w >> 8, pp);
-        } else {
-          const uint32_t c4[4] = {w << 4, w, w >> 2, w >> 6};  // shared by the four mt of this word
-          a[i] = vcode4(c4, pp);
-        }
-      }
-    } else if (BITS == 2) {
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        if (EXACT)
-          a[i] = code2(vr[i], vr[i] >> 10, mt);
-        else
-          a[i] = vcode2(vr[i] << 4, vr[i], vr[i] >> 6, mt);  // the shifted copies are shared by all mt
-      }
-    } else {
-      // vr[0], vr[2]: channel g (tokens 2t, 2t+1 and 2t+8, 2t+9), whose high bits are the even bits of vb0, vb1;
-      // vr[1], vr[3]: channel g + 8, the odd bits
-      const int k = mt >> 1, s = 4 - 4 * k;  // codes 2k, 2k+1 read at bits 4, 6 of the words shifted by s
-      auto sh = [](uint32_t x, int n) { return n >= 0 ? x << n : x >> -n; };
-      const uint32_t r4[4] = {sh(vr[0], s), sh(vr[1], s), sh(vr[2], s), sh(vr[3], s)};
-      const uint32_t h4[4] = {sh(vb0, s + 2), sh(vb0, s + 1), sh(vb1, s + 2), sh(vb1, s + 1)};
-      const int p = 4 + 2 * (mt & 1);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) a[i] = or_code3(r4[i], h4[i], p, mag2(p >> 1));
-    }
+    vf.code(mt, a);
     mma_f16(o[mt], a, pa0[gi], pa1[gi]);  // sums p * alpha * (code + offset)
   }
 }
@@ -728,6 +762,302 @@ __device__ __forceinline__ void write_partial(const AttnArgs& a, int slot, Softm
         a.part_ml[((size_t)slot * G + head) * 2 + 1] = st.l[hd] * c[hd];
       }
     }
+  }
+}
+
+// ---------------------------------------------------------------------- one query head per KV head (G = 1)
+//
+// With G = 1 only one of the eight columns of the QK^T and PV tiles would hold a query head. This path (bf16
+// important set, per-token retained keys) gives the other columns work, indexed by the quantization group
+// (NG = 128 / group groups per row):
+//  - keys: column n of the query operand holds the balanced query on the channels of group n mod NG and zeros
+//    elsewhere, so the MMA over exact key codes gives every token one partial dot product per group. The token's
+//    (alpha, beta) then enter in fp32, s = scale * sum_g (alpha_g (q . code)_g + beta_g (sum of q over g)): no key
+//    element is dequantized (Eq. 1 and Eq. 3-4 regrouped per group).
+//  - values: column n < NG of the probability operand holds p * alpha of group n, column NG holds p, and one
+//    more MMA, whose row n < NG holds beta of group n and row NG ones, gives the beta sums, the alpha sums that
+//    remove the code offsets, and the normaliser (the sum of the probabilities as the MMAs used them).
+// Every lane then holds the logits of its tokens g and g + 8 (the important blocks replicate the query over all
+// columns; the group sums of a retained block are complete in every lane, after one shuffle when NG = 4), which
+// is what movmatrix needs to place the probabilities of every column.
+
+constexpr uint32_t kOnesF16 = 0x3C003C00u, kOnesBf16 = 0x3F803F80u;
+
+// Per-head query operands. Lane (g, t) holds channels 16 ks + 2t (+1) (r = 0) and 16 ks + 2t + 8 (+9) (r = 1) of
+// every k-step: qb, the bf16 query, in every column (important blocks); qh, the fp16 balanced query q / b (Eq. 4),
+// in the columns of its group (retained blocks); qs0 / qs1, the fp32 sums of qh over the groups of this lane's
+// columns 2t and 2t + 1.
+template <int GROUP>
+__device__ __forceinline__ void mha_query(const AttnArgs& a, int b, int h, int lane, uint32_t (&qb)[8][2],
+                                          uint32_t (&qh)[8][2], float& qs0, float& qs1) {
+  constexpr int NG = kHeadDim / GROUP;
+  const int g = lane >> 2, t = lane & 3;
+  const __nv_bfloat16* qp = static_cast<const __nv_bfloat16*>(a.q) + (size_t)(b * a.heads_q + h) * kHeadDim;
+  float cs[8];  // this lane's four channels of each k-step
+#pragma unroll
+  for (int ks = 0; ks < 8; ++ks) {
+    const bool mine = g % NG == (16 * ks) / GROUP;
+    cs[ks] = 0.f;
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      const int c = 16 * ks + 2 * t + 8 * r;
+      const uint32_t w = *reinterpret_cast<const uint32_t*>(qp + c);
+      qb[ks][r] = w;
+      const float q0 = __uint_as_float(w << 16), q1 = __uint_as_float(w & 0xffff0000u);
+      const float b0 = a.balancer ? a.balancer[h * kHeadDim + c] : 1.f;
+      const float b1 = a.balancer ? a.balancer[h * kHeadDim + c + 1] : 1.f;
+      const uint32_t f = pack_f16(__fdiv_rn(q0, b0), __fdiv_rn(q1, b1));
+      qh[ks][r] = mine ? f : 0u;
+      cs[ks] += __low2float(u32_as_h2(f)) + __high2float(u32_as_h2(f));
+    }
+  }
+  float gs[NG];
+#pragma unroll
+  for (int i = 0; i < NG; ++i) gs[i] = 0.f;
+#pragma unroll
+  for (int ks = 0; ks < 8; ++ks) {  // k-step sums over the four lanes t (the same bits in each), then per group
+    float v = cs[ks];
+    v += __shfl_xor_sync(0xffffffffu, v, 1);
+    v += __shfl_xor_sync(0xffffffffu, v, 2);
+    gs[(16 * ks) / GROUP] += v;
+  }
+  qs0 = gs[(2 * t) % NG];
+  qs1 = gs[(2 * t + 1) % NG];
+}
+
+// Online-softmax update for NK blocks of the G = 1 path: s[k] = logits of tokens g and g + 8 of block k (the same
+// in the four lanes of a row); p = unnormalised probabilities. All four columns of o and ob belong to the one
+// head and are rescaled together when the reference max moves (lazily, as in softmax_blocks).
+template <int NK>
+__device__ __forceinline__ void mha_softmax(const float (&s)[NK][2], Softmax& st, float (&o)[8][4], float (&ob)[4],
+                                            float (&p)[NK][2]) {
+  float bm = fmaxf(s[0][0], s[0][1]);
+#pragma unroll
+  for (int k = 1; k < NK; ++k) bm = fmaxf(bm, fmaxf(s[k][0], s[k][1]));
+  st.mx[0] = fmaxf(st.mx[0], bm);
+  if (__any_sync(0xffffffffu, bm > st.m[0] + kLazy)) {
+#pragma unroll
+    for (int off = 4; off < 32; off <<= 1) bm = fmaxf(bm, __shfl_xor_sync(0xffffffffu, bm, off));
+    const float mn = fmaxf(st.m[0], bm);
+    const float c = mn == st.m[0] ? 1.f : fast_exp2((st.m[0] - mn) * kLog2e);
+    st.l[0] *= c;
+#pragma unroll
+    for (int mt = 0; mt < 8; ++mt)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) o[mt][e] *= c;
+#pragma unroll
+    for (int e = 0; e < 4; ++e) ob[e] *= c;
+    st.m[0] = mn;
+  }
+  const float ml = st.m[0] * kLog2e;
+#pragma unroll
+  for (int k = 0; k < NK; ++k) {
+    p[k][0] = fast_exp2(fmaf(s[k][0], kLog2e, -ml));
+    p[k][1] = fast_exp2(fmaf(s[k][1], kLog2e, -ml));
+    st.l[0] += p[k][0] + p[k][1];
+  }
+}
+
+// One bf16 important block on the G = 1 path: logits (stored for the importance update), softmax, PV, and the
+// block's probabilities (as the bf16 MMA uses them) into the normaliser, entry (NG, NG) of the correction tile.
+template <int NG>
+__device__ __forceinline__ void mha_hi(uint32_t blk, int valid, int slot0, const uint32_t (&qb)[8][2], float scale,
+                                       float* logit_base, Softmax& st, float (&o)[8][4], float (&ob)[4], int lane) {
+  const int g = lane >> 2, t = lane & 3, r8 = lane & 7, j = lane >> 3;
+  float accs[kQkAcc][4];
+#pragma unroll
+  for (int q = 0; q < kQkAcc; ++q) accs[q][0] = accs[q][1] = accs[q][2] = accs[q][3] = 0.f;
+  const int krow = r8 + 8 * (j & 1);
+#pragma unroll
+  for (int ks = 0; ks < 8; ++ks) {
+    const int chunk = 2 * (ks & 3) + (j >> 1);
+    uint32_t a[4];
+    ldsm_x4(blk + (ks >> 2) * 2048 + krow * 128 + ((chunk ^ (krow & 7)) << 4), a);
+    mma_bf16(accs[ks % kQkAcc], a, qb[ks][0], qb[ks][1]);
+  }
+  float acc[4];
+  sum_acc(accs, acc);
+  float s[1][2], p[1][2];
+  s[0][0] = g < valid ? acc[0] * scale : -INFINITY;
+  s[0][1] = g + 8 < valid ? acc[2] * scale : -INFINITY;
+  if (logit_base && t == 0) {
+    if (g < valid) logit_base[slot0 + g] = s[0][0];
+    if (g + 8 < valid) logit_base[slot0 + g + 8] = s[0][1];
+  }
+  mha_softmax<1>(s, st, o, ob, p);
+  const uint32_t pb0 = movmatrix_t(pack_bf16(p[0][0], p[0][0]));  // tokens 2t, 2t+1, every column
+  const uint32_t pb1 = movmatrix_t(pack_bf16(p[0][1], p[0][1]));  // tokens 2t+8, 2t+9
+  {
+    const uint32_t one = g == NG ? kOnesBf16 : 0u;
+    const uint32_t a[4] = {one, 0u, one, 0u};
+    mma_bf16(ob, a, g == NG ? pb0 : 0u, g == NG ? pb1 : 0u);
+  }
+  uint32_t m01 = 0xffffffffu, m89 = 0xffffffffu;
+  if (valid < 16) {
+    m01 = (2 * t < valid ? 0x0000ffffu : 0u) | (2 * t + 1 < valid ? 0xffff0000u : 0u);
+    m89 = (2 * t + 8 < valid ? 0x0000ffffu : 0u) | (2 * t + 9 < valid ? 0xffff0000u : 0u);
+  }
+  const int vtok = r8 + 8 * (j >> 1);
+#pragma unroll
+  for (int mt = 0; mt < 8; ++mt) {
+    const int chunk = 2 * (mt & 3) + (j & 1);
+    uint32_t a[4];
+    ldsm_x4_t(blk + 4096 + (mt >> 2) * 2048 + vtok * 128 + ((chunk ^ (vtok & 7)) << 4), a);
+    if (valid < 16) {  // rows past the end may hold any bits: zero them (P is 0 there, NaN * 0 is not)
+      a[0] &= m01;
+      a[1] &= m01;
+      a[2] &= m89;
+      a[3] &= m89;
+    }
+    mma_bf16(o[mt], a, pb0, pb1);
+  }
+}
+
+// Logits of retained block b (tokens g, g + 8; -inf past valid) on the G = 1 path.
+template <int BITS, int GROUP, int QACC>
+__device__ __forceinline__ void mha_lo_logits(uint32_t unit, int b, int valid, const uint32_t (&qh)[8][2], float qs0,
+                                              float qs1, float scale, float (&s)[2], int lane) {
+  constexpr LoUnit U = lo_unit_layout(BITS, GROUP);
+  constexpr int NG = kHeadDim / GROUP;
+  constexpr int PR = U.param_row;
+  const uint32_t ka = unit + U.k_a + b * 16 * U.pitch;
+  const uint32_t kp = unit + U.k_p + b * 16 * PR;
+  const int g = lane >> 2, t = lane & 3;
+  // (alpha, beta) of tokens g and g + 8 for the groups of columns 2t, 2t + 1
+  uint32_t pg[2], p8[2];
+  if constexpr (NG == 1) {
+    pg[0] = pg[1] = lds32(kp + g * PR);
+    p8[0] = p8[1] = lds32(kp + (g + 8) * PR);
+  } else {
+    const int off = NG == 4 ? 8 * (t & 1) : 0;
+    lds_vec<2>(kp + g * PR + off, pg);
+    lds_vec<2>(kp + (g + 8) * PR + off, p8);
+  }
+  float accs[QACC][4];
+#pragma unroll
+  for (int q = 0; q < QACC; ++q) accs[q][0] = accs[q][1] = accs[q][2] = accs[q][3] = 0.f;
+  KeyFrag<BITS, U.pitch> kf;
+  kf.load(ka, lane);
+#pragma unroll
+  for (int ks = 0; ks < 8; ++ks) {
+    uint32_t c[4];
+    kf.code(ks, c);
+    mma_f16(accs[ks % QACC], c, qh[ks][0], qh[ks][1]);
+  }
+  float acc[4];
+  sum_acc(accs, acc);
+  const __half2 g0 = u32_as_h2(pg[0]), e0 = u32_as_h2(p8[0]);
+  float sg = fmaf(__low2float(g0), acc[0], __high2float(g0) * qs0);
+  float s8 = fmaf(__low2float(e0), acc[2], __high2float(e0) * qs0);
+  if constexpr (NG >= 2) {
+    const __half2 g1 = u32_as_h2(pg[1]), e1 = u32_as_h2(p8[1]);
+    sg += fmaf(__low2float(g1), acc[1], __high2float(g1) * qs1);
+    s8 += fmaf(__low2float(e1), acc[3], __high2float(e1) * qs1);
+  }
+  if constexpr (NG == 4) {  // lanes t and t ^ 1 hold the group pairs (0, 1) and (2, 3)
+    sg += __shfl_xor_sync(0xffffffffu, sg, 1);
+    s8 += __shfl_xor_sync(0xffffffffu, s8, 1);
+  }
+  s[0] = g < valid ? sg * scale : -INFINITY;
+  s[1] = g + 8 < valid ? s8 * scale : -INFINITY;
+}
+
+// Values of retained block b on the G = 1 path: o += the block's codes (plus voff) times the group-column
+// probability operand; the correction tile ob += beta sums, alpha sums and the normaliser.
+template <int BITS, int GROUP>
+__device__ __forceinline__ void mha_lo_values(uint32_t unit, int b, int valid, const float (&p)[2], float (&o)[8][4],
+                                              float (&ob)[4], int lane) {
+  constexpr LoUnit U = lo_unit_layout(BITS, GROUP);
+  constexpr int NG = kHeadDim / GROUP;
+  constexpr int PR = U.param_row;
+  const uint32_t va = unit + U.v_a + b * 16 * U.pitch;
+  const uint32_t vp = unit + U.v_p + b * 16 * PR;
+  const int g = lane >> 2, t = lane & 3;
+  const uint32_t pb0 = movmatrix_t(pack_f16(p[0], p[0]));  // tokens 2t, 2t+1, every column
+  const uint32_t pb1 = movmatrix_t(pack_f16(p[1], p[1]));  // tokens 2t+8, 2t+9
+  ValFrag<BITS, U.pitch, false> vf;
+  vf.load(va, lane);
+  // (alpha, beta) of group g (lanes g < NG; the others read group 0 and do not use it) for the four tokens
+  const uint32_t gp = vp + 4 * (g < NG ? g : 0);
+  uint32_t w0 = lds32(gp + (2 * t) * PR), w1 = lds32(gp + (2 * t + 1) * PR);
+  uint32_t w8 = lds32(gp + (2 * t + 8) * PR), w9 = lds32(gp + (2 * t + 9) * PR);
+  if (valid < 16) {  // exact zeros past the end
+    if (2 * t >= valid) w0 = 0u;
+    if (2 * t + 1 >= valid) w1 = 0u;
+    if (2 * t + 8 >= valid) w8 = 0u;
+    if (2 * t + 9 >= valid) w9 = 0u;
+  }
+  uint32_t B0, B1, A0, A2;
+  if (g < NG) {
+    B0 = h2_as_u32(__hmul2(u32_as_h2(pb0), u32_as_h2(prmt(w0, w1, 0x5410u))));
+    B1 = h2_as_u32(__hmul2(u32_as_h2(pb1), u32_as_h2(prmt(w8, w9, 0x5410u))));
+    A0 = prmt(w0, w1, 0x7632u);
+    A2 = prmt(w8, w9, 0x7632u);
+  } else {
+    B0 = g == NG ? pb0 : 0u;
+    B1 = g == NG ? pb1 : 0u;
+    A0 = A2 = g == NG ? kOnesF16 : 0u;
+  }
+  {
+    const uint32_t a[4] = {A0, 0u, A2, 0u};
+    mma_f16(ob, a, B0, B1);
+  }
+#pragma unroll
+  for (int mt = 0; mt < 8; ++mt) {
+    uint32_t a[4];
+    vf.code(mt, a);
+    mma_f16(o[mt], a, B0, B1);  // column g < NG: sums p * alpha_g * (code + offset)
+  }
+}
+
+template <int BITS, int GROUP, int NK>
+__device__ __forceinline__ void mha_coded(uint32_t unit, int b, int n_left, const uint32_t (&qh)[8][2], float qs0,
+                                          float qs1, float scale, Softmax& st, float (&o)[8][4], float (&ob)[4],
+                                          int lane) {
+  float s[NK][2], p[NK][2];
+#pragma unroll
+  for (int k = 0; k < NK; ++k)
+    mha_lo_logits<BITS, GROUP, NK == 1 ? kQkAcc : kPairAcc>(unit, b + k, min(16, n_left - 16 * k), qh, qs0, qs1,
+                                                             scale, s[k], lane);
+  mha_softmax<NK>(s, st, o, ob, p);
+#pragma unroll
+  for (int k = 0; k < NK; ++k) mha_lo_values<BITS, GROUP>(unit, b + k, min(16, n_left - 16 * k), p[k], o, ob, lane);
+}
+
+// The partial of the G = 1 path (same content as write_partial): channel c of tile mt (group gi) is read from column
+// gi, out = (o - voff * alpha sum + beta sum) / normaliser, with the sums taken from the correction tile.
+template <int BITS, int GROUP>
+__device__ __forceinline__ void mha_write_partial(const AttnArgs& a, int slot, Softmax& st, const float (&o)[8][4],
+                                                  const float (&ob)[4], int lane) {
+  constexpr int NG = kHeadDim / GROUP;
+  const int g = lane >> 2, t = lane & 3;
+#pragma unroll
+  for (int off = 4; off < 32; off <<= 1) {  // over the rows g (the four lanes of a row hold the same tokens)
+    st.l[0] += __shfl_xor_sync(0xffffffffu, st.l[0], off);
+    st.mx[0] = fmaxf(st.mx[0], __shfl_xor_sync(0xffffffffu, st.mx[0], off));
+  }
+  const float c = st.mx[0] == st.m[0] ? 1.f : fast_exp2((st.m[0] - st.mx[0]) * kLog2e);
+  // correction tile entry (r, n) sits in lane 4 r + n / 2, element n & 1 (rows r < 8)
+  const float inv = 1.f / __shfl_sync(0xffffffffu, ob[NG & 1], 4 * NG + NG / 2);
+  float za[NG], zb[NG];
+#pragma unroll
+  for (int gi = 0; gi < NG; ++gi) {
+    za[gi] = __shfl_sync(0xffffffffu, ob[gi & 1], 4 * NG + gi / 2);  // sum of p * alpha of group gi
+    zb[gi] = __shfl_sync(0xffffffffu, ob[NG & 1], 4 * gi + NG / 2);  // sum of p * beta of group gi
+  }
+  float* po = a.part_o + (size_t)slot * kHeadDim;
+#pragma unroll
+  for (int mt = 0; mt < 8; ++mt) {
+    const int gi = (16 * mt) / GROUP;
+    if (t == gi / 2) {
+      const float z = fmaf(-voff<BITS>(mt), za[gi], zb[gi]);
+      po[16 * mt + g] = (o[mt][gi & 1] + z) * inv;
+      po[16 * mt + 8 + g] = (o[mt][2 + (gi & 1)] + z) * inv;
+    }
+  }
+  if (lane == 0) {
+    a.part_ml[(size_t)slot * 2] = st.mx[0];
+    a.part_ml[(size_t)slot * 2 + 1] = st.l[0] * c;
   }
 }
 
@@ -846,6 +1176,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
   constexpr LoUnit H = lo_unit_layout(HB == 16 ? 2 : HB, kHiGroup);
   static_assert(U.total <= kStageBytes && H.total <= kStageBytes, "unit too large for a stage");
   static_assert(!KCH || HB == 16, "per-channel retained keys need a bf16 important set");
+  // one query head per KV head with a bf16 important set and per-token retained keys: the group-column path
+  constexpr bool MHA = MIKV_MHA_PATH && G == 1 && HB == 16 && !KCH;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -903,17 +1235,25 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
                                  // the register file)
   if (lane == 0) s_ins[warp] = -1;
   float* logit_base = nullptr;
+  float qs0 = 0.f, qs1 = 0.f;  // G = 1 path: sums of the balanced query over the groups of columns 2t, 2t + 1
   Cursor cc = cursor_at(u0, hu, n_u);  // unit being consumed
   int cur = -1;
   bool failed = false;
   int u = u0;
   for (; u < u1; ++u) {
     if (cc.bh != cur) {
-      if (cur >= 0) write_partial<BITS, GROUP, G, NB>(a, wg + cur, st, o, ob, lane);
+      if (cur >= 0) {
+        if constexpr (MHA)
+          mha_write_partial<BITS, GROUP>(a, wg + cur, st, o, ob[0], lane);
+        else
+          write_partial<BITS, GROUP, G, NB>(a, wg + cur, st, o, ob, lane);
+      }
       cur = cc.bh;
       const int b = cur / a.heads_kv, h = cur - b * a.heads_kv;
       // query fragments (B operand: head g; channels 16 ks + 2t (+1) and 16 ks + 2t + 8 (+9))
-      if (g < G) {
+      if constexpr (MHA) {
+        mha_query<GROUP>(a, b, h, lane, qb, qh, qs0, qs1);
+      } else if (g < G) {
         const __nv_bfloat16* qp =
             static_cast<const __nv_bfloat16*>(a.q) + (size_t)(b * a.heads_q + h * G + g) * kHeadDim;
 #pragma unroll
@@ -970,8 +1310,12 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
           const int sl = s_ins[warp];
           if (sl >= 0 && (sl >> 4) == k.index) insert_row(a, cur, sl, stage, lane);
         }
-        process_hi<G, NB>(stage, min(16, a.hi_cap - 16 * k.index), 16 * k.index, qb, a.sm_scale, logit_base,
-                          a.hi_stride, st, o, ob, lane);
+        if constexpr (MHA)
+          mha_hi<kHeadDim / GROUP>(stage, min(16, a.hi_cap - 16 * k.index), 16 * k.index, qb, a.sm_scale, logit_base,
+                                   st, o, ob[0], lane);
+        else
+          process_hi<G, NB>(stage, min(16, a.hi_cap - 16 * k.index), 16 * k.index, qb, a.sm_scale, logit_base,
+                            a.hi_stride, st, o, ob, lane);
       } else {
         const int first = k.index * H.blocks;
         const int nb = min(H.blocks, a.hi_blocks - first);
@@ -995,6 +1339,13 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
         for (; b + 1 < nb; b += 2)
           process_coded<BITS, GROUP, G, NB, 2, false, true>(stage, b, a.n_lo - 16 * (first + b), qk, a.sm_scale, st,
                                                             o, ob, lane, nullptr, 0, 0, kbias);
+      } else if constexpr (MHA) {
+        if (kLoPair)
+          for (; b + 1 < nb; b += 2)
+            mha_coded<BITS, GROUP, 2>(stage, b, a.n_lo - 16 * (first + b), qh, qs0, qs1, a.sm_scale, st, o, ob[0],
+                                      lane);
+        for (; b < nb; ++b)
+          mha_coded<BITS, GROUP, 1>(stage, b, a.n_lo - 16 * (first + b), qh, qs0, qs1, a.sm_scale, st, o, ob[0], lane);
       } else {
         if (kLoPair)
           for (; b + 1 < nb; b += 2)
@@ -1022,7 +1373,12 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
       }
     return;
   }
-  if (cur >= 0) write_partial<BITS, GROUP, G, NB>(a, wg + cur, st, o, ob, lane);
+  if (cur >= 0) {
+    if constexpr (MHA)
+      mha_write_partial<BITS, GROUP>(a, wg + cur, st, o, ob[0], lane);
+    else
+      write_partial<BITS, GROUP, G, NB>(a, wg + cur, st, o, ob, lane);
+  }
 }
 
 template <int BITS, int GROUP, int HB, int G, bool KCH = false>

@@ -144,9 +144,14 @@ def logit_bounds(c, q_bits, bal, bits: int, group: int, n_lo: int, scale: float,
     """Per-token bound on |GPU logit - oracle logit| for one (b, KV head) of a cache with a bf16 important set and
     per-token retained keys, from the kernel's documented arithmetic (the oracle evaluates in fp64):
       important rows: bf16 q times bf16 k, exact products, fp32 accumulation, times the fp32 scale;
-      retained rows (and important rows of a coded important set, hi_bits < 16, groups of 64): q_hat =
-                      fp16(fp32 q / fp32 b) and k_hat = fp16(alpha * code + beta) (HFMA2, one rounding) as MMA
-                      operands, exact products, fp32 accumulation.
+      retained rows (and important rows of a coded important set, hi_bits < 16, groups of 64), G > 1 or a coded
+                      important set: q_hat = fp16(fp32 q / fp32 b) and k_hat = fp16(alpha * code + beta) (HFMA2, one
+                      rounding) as MMA operands, exact products, fp32 accumulation;
+      retained rows, G = 1 with a bf16 important set (the group-column path): the MMA sums q_hat * code (exact
+                      integer codes) per group in fp32, and alpha, beta enter in fp32 afterwards,
+                      s = scale * sum_g (alpha_g * (q_hat . code)_g + beta_g * sum_g q_hat): bounded by the q_hat
+                      rounding (evaluated exactly) plus (ACC_GAMMA + 2^-22) * sum_c |q_hat_c| (alpha code_c + |beta|)
+                      for the fp32 accumulations and the few fp32 roundings that combine the groups.
     The operand roundings are evaluated exactly (numpy's IEEE fp32 division and correctly rounded fp16 casts);
     only the accumulation is bounded (ACC_GAMMA * sum |products|, plus 2^-24 of the scaling multiply).
     q_bits uint16 [1, G, d]; returns (hi [G, hi_cap], lo [G, n_lo])."""
@@ -171,8 +176,17 @@ def logit_bounds(c, q_bits, bal, bits: int, group: int, n_lo: int, scale: float,
         hi = s32 * (ACC_GAMMA + 2.0 ** -24) * (np.abs(qd) @ np.abs(kh).T) + abs(s32 - scale) * np.abs(qd @ kh.T)
     if n_lo == 0:
         return hi, np.zeros((q.shape[0], 0))
-    return hi, coded(np.stack([oracle.dequantize_row(c["k_codes"][0, 0, t], c["k_params"][0, 0, t], bits, group)
-                               for t in range(n_lo)]))
+    rows = np.stack([oracle.dequantize_row(c["k_codes"][0, 0, t], c["k_params"][0, 0, t], bits, group)
+                     for t in range(n_lo)])
+    if q.shape[0] > 1 or hi_bits < 16:
+        return hi, coded(rows)
+    # G = 1 group-column path: exact keys alpha * code + beta; |alpha code| = |k - beta|
+    beta = np.stack([np.repeat(c["k_params"][0, 0, t][:, 1].view(np.float16).astype(np.float64), group)
+                     for t in range(n_lo)])
+    mag = np.abs(rows - beta) + np.abs(beta)
+    lo = (np.abs(s32 * (q16 @ rows.T) - scale * (qhat @ rows.T))
+          + s32 * (ACC_GAMMA + 2.0 ** -22) * (np.abs(q16) @ mag.T))
+    return hi, lo
 
 
 def softmax_stat_bounds(hi, lo, n_tokens: int):

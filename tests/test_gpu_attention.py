@@ -31,10 +31,13 @@ CASES = {
     "one-token": mi.Workload("t1", 1, 4, 4, 1, 1, 3, 32, 0.2, seed=6),
     "exact-16": mi.Workload("x16", 1, 4, 1, 160, 1, 4, 32, 0.09375, seed=7),  # hi_cap = 16
 }
-# every retained layout (bits x group): ragged lengths, several units per head
+# every retained layout (bits x group): ragged lengths, several units per head; with two query heads per KV head
+# and with one (the group-column path of G = 1)
 for _b in (2, 3, 4):
     for _g in (32, 64, 128):
         CASES[f"layout-int{_b}-g{_g}"] = mi.Workload(f"l{_b}{_g}", 1, 4, 2, 611, 1, _b, _g, 0.15, seed=10 * _b + _g)
+        CASES[f"layout-mha-int{_b}-g{_g}"] = mi.Workload(f"m{_b}{_g}", 1, 3, 3, 611, 1, _b, _g, 0.15,
+                                                         seed=100 + 10 * _b + _g)
 
 
 def _check_cache(layer, refs, w):
@@ -103,10 +106,12 @@ def test_attention_matches_oracle(name, out_dtype):
         assert np.all(np.abs(ml_c[b, sl, 1] / ref_ml[0, :, 1] - 1) <= l_rtol), "softmax sum"
 
 
-def test_decode_steps_trajectory():
+@pytest.mark.parametrize("w", [mi.Workload("traj", 2, 8, 2, 500, 1, 2, 32, 0.2, seed=21),
+                               mi.Workload("traj-mha", 2, 4, 4, 500, 1, 3, 64, 0.1, seed=22)], ids=lambda w: w.name)
+def test_decode_steps_trajectory(w):
     """Several whole decode steps (insert, attend, update, select, demote) through mikv_decode_step
-    against the oracle's step sequence: chosen victims, appended retained rows and outputs."""
-    w = mi.Workload("traj", 2, 8, 2, 500, 1, 2, 32, 0.2, seed=21)
+    against the oracle's step sequence: chosen victims, appended retained rows and outputs (G = 4, and G = 1 on
+    the group-column path)."""
     steps = 6
     raw = raw_inputs(w)
     layer = gpu_layer(w, raw, steps=steps)
