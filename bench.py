@@ -680,20 +680,28 @@ def run_prefill(args):
     # algorithmic work: two passes (row statistics, column sums) over the causal triangle of Q K^T
     flops = 2.0 * w.batch * w.heads_q * (T * (T + 1) / 2) * 2 * w.head_dim
     tflops = flops / ms / 1e9
+    # a timed loop of a second or more runs under the power cap: it is judged against the sustained bf16 peak,
+    # shorter ones against the burst peak
+    sustained = ms * args.steps >= 1000.0
     peak, kind = None, "fallback"
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
         with open(p) as f:
-            peak, kind = float(json.load(f)["bf16_tflops"]), "measured"
+            mp = json.load(f)
+        if sustained and "bf16_tflops_sustained" in mp:
+            peak, kind = float(mp["bf16_tflops_sustained"]), "measured"
+        else:
+            peak, kind, sustained = float(mp["bf16_tflops"]), "measured", False
     if peak is None:
-        peak = 1900.0
+        peak = 1700.0 if sustained else 1900.0
     print(json.dumps({
         "metric": "prefill importance (accumulated causal attention) TFLOP/s", "value": round(tflops, 1),
         "unit": "TFLOP/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_layer": round(ms, 3),
         "higher_is_better": True, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": w.name, "batch": w.batch, "heads_q": w.heads_q, "heads_kv": w.heads_kv, "context": T},
         "roofline": {"kernel": "prefill_rows_kernel + prefill_cols_kernel", "bound": "tensor", "achieved": round(tflops, 1),
-                     "peak": peak, "peak_kind": kind + " bf16 burst", "unit": "TFLOP/s", "frac": round(tflops / peak, 3)},
+                     "peak": peak, "peak_kind": kind + (" bf16 sustained" if sustained else " bf16 burst"), "unit": "TFLOP/s",
+                     "frac": round(tflops / peak, 3)},
         "clocks": clocks}))
 
 
