@@ -45,12 +45,37 @@ ATTN_SOURCES = ["mikv_attention.cuh", "mikv_attention.cu", "mikv_attn_h16.cu", "
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "attention_traffic.json")
 
 
+def _code_only(text: str) -> str:
+    """C++ source without its comments and with whitespace collapsed: what the compiler sees of it (a change
+    of a comment alone leaves the kernel, and so its profile, as it was)."""
+    import re
+    out, i, n = [], 0, len(text)
+    while i < n:
+        if text.startswith("//", i):
+            j = text.find("\n", i)
+            i = n if j < 0 else j
+        elif text.startswith("/*", i):
+            j = text.find("*/", i + 2)
+            i = n if j < 0 else j + 2
+        elif text[i] in "\"'":  # string and character literals are kept whole
+            q, j = text[i], i + 1
+            while j < n and text[j] != q:
+                j += 2 if text[j] == "\\" else 1
+            out.append(text[i:j + 1])
+            i = j + 1
+        else:
+            out.append(text[i])
+            i += 1
+    return re.sub(r"\s+", " ", "".join(out)).strip()
+
+
 def attention_source_sha256() -> str:
+    """Hash of the attention kernel's sources, comments left out."""
     import hashlib
     h = hashlib.sha256()
     for f in ATTN_SOURCES:
-        with open(os.path.join(ROOT, "paper_2402_18096_gb300", "csrc", f), "rb") as fh:
-            h.update(fh.read())
+        with open(os.path.join(ROOT, "paper_2402_18096_gb300", "csrc", f), encoding="utf-8") as fh:
+            h.update(_code_only(fh.read()).encode())
     return h.hexdigest()
 
 

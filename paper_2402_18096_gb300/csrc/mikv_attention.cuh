@@ -31,6 +31,11 @@
 // value scale is folded into the probabilities (p * alpha per token and group) and the zero into one
 // extra MMA row (sum of p * beta per group), so values need no HFMA2. Online softmax in fp32;
 // movmatrix turns probabilities into the PV operand without shared memory.
+//
+// With one query head per KV head (G = 1, bf16 important set, per-token retained keys) the N columns that no
+// head would use carry the quantization groups instead (the mha_* functions): the keys' alpha and beta are
+// applied per group after the MMA in fp32, and the values' beta sums, alpha sums and normaliser come from one
+// correction MMA.
 #pragma once
 
 #include <math.h>

@@ -18,3 +18,11 @@ def test_cpu_baseline_one_and_all_cores():
 def test_cpu_baseline_single_core_only():
     r = bench.cpu_baseline(mi.WORKLOADS["tiny"], seconds=0.2, all_cores=False)
     assert r["cores"] == 1 and r["value"] == r["single_core_value"]
+
+
+def test_source_hash_ignores_comments_only():
+    """The attention-source hash that gates the profiled traffic figure follows the code, not its comments."""
+    a = 'int x = 1; // one\n/* block\n comment */ const char* s = "// kept"; char c = \'/\';'
+    b = 'int x = 1;\nconst char* s = "// kept";   char c = \'/\';  // other'
+    assert bench._code_only(a) == bench._code_only(b) == 'int x = 1; const char* s = "// kept"; char c = \'/\';'
+    assert bench._code_only("a = b;") != bench._code_only("a = c;")
