@@ -798,6 +798,16 @@ __device__ __forceinline__ void mha_query(const AttnArgs& a, int b, int h, int l
   constexpr int NG = kHeadDim / GROUP;
   const int g = lane >> 2, t = lane & 3;
   const __nv_bfloat16* qp = static_cast<const __nv_bfloat16*>(a.q) + (size_t)(b * a.heads_q + h) * kHeadDim;
+  // every load first (the divisions below branch, which would otherwise keep later loads behind earlier ones)
+  float2 bal[8][2];
+#pragma unroll
+  for (int ks = 0; ks < 8; ++ks)
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      const int c = 16 * ks + 2 * t + 8 * r;
+      qb[ks][r] = *reinterpret_cast<const uint32_t*>(qp + c);
+      bal[ks][r] = a.balancer ? *reinterpret_cast<const float2*>(a.balancer + h * kHeadDim + c) : make_float2(1.f, 1.f);
+    }
   float cs[8];  // this lane's four channels of each k-step
 #pragma unroll
   for (int ks = 0; ks < 8; ++ks) {
@@ -805,13 +815,9 @@ __device__ __forceinline__ void mha_query(const AttnArgs& a, int b, int h, int l
     cs[ks] = 0.f;
 #pragma unroll
     for (int r = 0; r < 2; ++r) {
-      const int c = 16 * ks + 2 * t + 8 * r;
-      const uint32_t w = *reinterpret_cast<const uint32_t*>(qp + c);
-      qb[ks][r] = w;
+      const uint32_t w = qb[ks][r];
       const float q0 = __uint_as_float(w << 16), q1 = __uint_as_float(w & 0xffff0000u);
-      const float b0 = a.balancer ? a.balancer[h * kHeadDim + c] : 1.f;
-      const float b1 = a.balancer ? a.balancer[h * kHeadDim + c + 1] : 1.f;
-      const uint32_t f = pack_f16(__fdiv_rn(q0, b0), __fdiv_rn(q1, b1));
+      const uint32_t f = pack_f16(__fdiv_rn(q0, bal[ks][r].x), __fdiv_rn(q1, bal[ks][r].y));
       qh[ks][r] = mine ? f : 0u;
       cs[ks] += __low2float(u32_as_h2(f)) + __high2float(u32_as_h2(f));
     }
@@ -1261,20 +1267,27 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
       } else if (g < G) {
         const __nv_bfloat16* qp =
             static_cast<const __nv_bfloat16*>(a.q) + (size_t)(b * a.heads_q + h * G + g) * kHeadDim;
+        // every load first (the divisions below branch, which would otherwise keep later loads behind earlier ones)
+        float2 bal[8][2];
 #pragma unroll
         for (int ks = 0; ks < 8; ++ks)
 #pragma unroll
           for (int r = 0; r < 2; ++r) {
             const int c = 16 * ks + 2 * t + 8 * r;
-            const uint32_t w = *reinterpret_cast<const uint32_t*>(qp + c);
-            qb[ks][r] = w;
+            qb[ks][r] = *reinterpret_cast<const uint32_t*>(qp + c);
+            bal[ks][r] = !KCH && a.balancer ? *reinterpret_cast<const float2*>(a.balancer + h * kHeadDim + c)
+                                            : make_float2(1.f, 1.f);
+          }
+#pragma unroll
+        for (int ks = 0; ks < 8; ++ks)
+#pragma unroll
+          for (int r = 0; r < 2; ++r) {
+            const uint32_t w = qb[ks][r];
             const float q0 = __uint_as_float(w << 16), q1 = __uint_as_float(w & 0xffff0000u);
             if constexpr (KCH) {  // per-channel retained keys are not balanced
               qh[ks][r] = pack_f16(q0, q1);
             } else {
-              const float b0 = a.balancer ? a.balancer[h * kHeadDim + c] : 1.f;
-              const float b1 = a.balancer ? a.balancer[h * kHeadDim + c + 1] : 1.f;
-              qh[ks][r] = pack_f16(__fdiv_rn(q0, b0), __fdiv_rn(q1, b1));  // Eq. 4
+              qh[ks][r] = pack_f16(__fdiv_rn(q0, bal[ks][r].x), __fdiv_rn(q1, bal[ks][r].y));  // Eq. 4
             }
           }
       } else {
