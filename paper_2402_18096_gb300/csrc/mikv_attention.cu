@@ -20,8 +20,7 @@ __global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a, int G) {
   const int w0 = owner_warp((long long)bh * a.n_u, a.n_units, a.n_warps);
   const int w1 = owner_warp((long long)(bh + 1) * a.n_u - 1, a.n_units, a.n_warps);
   float r[4], M, L;
-  merge_stats_warp(a.part_ml, G, bh, jh, w0, w1, lane, M, L);
-  merge_output_warp(a.part_o, a.part_ml, G, bh, jh, w0, w1, lane, M, L, r);
+  merge_head_warp<12>(a.part_o, a.part_ml, G, bh, jh, w0, w1, lane, M, L, r);
   if (OUT_F32) {
     reinterpret_cast<float4*>(static_cast<float*>(a.out) + (size_t)bq * kHeadDim)[lane] = make_float4(r[0], r[1], r[2], r[3]);
   } else {

@@ -86,6 +86,52 @@ __device__ __forceinline__ void merge_output_warp(const float* part_o, const flo
   for (int i = 0; i < 4; ++i) out[i] = O[i] / L;
 }
 
+// Both steps at once when the head has at most NB partials: every load (each partial's statistics and output)
+// is issued before any is used, so the merge costs one round of loads; the arithmetic, and its order, is that of
+// merge_stats_warp followed by merge_output_warp, so the bits are the same. More partials take those two.
+template <int NB>
+__device__ __forceinline__ void merge_head_warp(const float* part_o, const float* part_ml, int G, int bh, int jh,
+                                                int w0, int w1, int lane, float& M, float& L, float (&out)[4]) {
+  constexpr float kLog2e = 1.4426950408889634f;
+  const int n = w1 - w0 + 1;
+  if (n > NB || n > 32) {
+    merge_stats_warp(part_ml, G, bh, jh, w0, w1, lane, M, L);
+    merge_output_warp(part_o, part_ml, G, bh, jh, w0, w1, lane, M, L, out);
+    return;
+  }
+  float4 po[NB];
+#pragma unroll
+  for (int k = 0; k < NB; ++k)
+    if (k < n) po[k] = __ldcg(reinterpret_cast<const float4*>(part_o + ((size_t)(w0 + k + bh) * G + jh) * kHeadDim) + lane);
+  float ms = -INFINITY, ls = 0.f;
+  if (lane < n) {
+    const float2 v = __ldcg(reinterpret_cast<const float2*>(part_ml + ((size_t)(w0 + lane + bh) * G + jh) * 2));
+    ms = v.x;
+    ls = v.y;
+  }
+  M = ms;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+  const float wt = lane < n && ms != -INFINITY ? fast_exp2((ms - M) * kLog2e) * ls : 0.f;
+  float Lp = wt;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) Lp += __shfl_xor_sync(0xffffffffu, Lp, off);
+  L = Lp;
+  float O[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int k = 0; k < NB; ++k) {
+    if (k < n) {
+      const float ws = __shfl_sync(0xffffffffu, wt, k);
+      O[0] += ws * po[k].x;
+      O[1] += ws * po[k].y;
+      O[2] += ws * po[k].z;
+      O[3] += ws * po[k].w;
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) out[i] = O[i] / L;
+}
+
 // Importance weight of one slot for one query head: exp(s - M) / L, as exp2((s - M) log2 e) times the
 // reciprocal of L (the same arithmetic in the fused step tail and in mikv_update_importance).
 __device__ __forceinline__ float importance_weight(float s, float M, float inv_L) {
