@@ -798,16 +798,21 @@ __device__ __forceinline__ void mha_query(const AttnArgs& a, int b, int h, int l
   constexpr int NG = kHeadDim / GROUP;
   const int g = lane >> 2, t = lane & 3;
   const __nv_bfloat16* qp = static_cast<const __nv_bfloat16*>(a.q) + (size_t)(b * a.heads_q + h) * kHeadDim;
-  // every load first (the divisions below branch, which would otherwise keep later loads behind earlier ones)
-  float2 bal[8][2];
+  // Every row of lanes needs the same fragments: lane (g, t) loads and divides (Eq. 4) those of k-step ks = g only,
+  // every load before any division (the divisions branch), and the fragments reach the other rows by shuffles.
+  uint32_t qw[2], fw[2];
+  float2 bal[2];
 #pragma unroll
-  for (int ks = 0; ks < 8; ++ks)
+  for (int r = 0; r < 2; ++r) {
+    const int c = 16 * g + 2 * t + 8 * r;
+    qw[r] = *reinterpret_cast<const uint32_t*>(qp + c);
+    bal[r] = a.balancer ? *reinterpret_cast<const float2*>(a.balancer + h * kHeadDim + c) : make_float2(1.f, 1.f);
+  }
 #pragma unroll
-    for (int r = 0; r < 2; ++r) {
-      const int c = 16 * ks + 2 * t + 8 * r;
-      qb[ks][r] = *reinterpret_cast<const uint32_t*>(qp + c);
-      bal[ks][r] = a.balancer ? *reinterpret_cast<const float2*>(a.balancer + h * kHeadDim + c) : make_float2(1.f, 1.f);
-    }
+  for (int r = 0; r < 2; ++r) {
+    const float q0 = __uint_as_float(qw[r] << 16), q1 = __uint_as_float(qw[r] & 0xffff0000u);
+    fw[r] = pack_f16(__fdiv_rn(q0, bal[r].x), __fdiv_rn(q1, bal[r].y));
+  }
   float cs[8];  // this lane's four channels of each k-step
 #pragma unroll
   for (int ks = 0; ks < 8; ++ks) {
@@ -815,9 +820,8 @@ __device__ __forceinline__ void mha_query(const AttnArgs& a, int b, int h, int l
     cs[ks] = 0.f;
 #pragma unroll
     for (int r = 0; r < 2; ++r) {
-      const uint32_t w = qb[ks][r];
-      const float q0 = __uint_as_float(w << 16), q1 = __uint_as_float(w & 0xffff0000u);
-      const uint32_t f = pack_f16(__fdiv_rn(q0, bal[ks][r].x), __fdiv_rn(q1, bal[ks][r].y));
+      qb[ks][r] = __shfl_sync(0xffffffffu, qw[r], 4 * ks + t);
+      const uint32_t f = __shfl_sync(0xffffffffu, fw[r], 4 * ks + t);
       qh[ks][r] = mine ? f : 0u;
       cs[ks] += __low2float(u32_as_h2(f)) + __high2float(u32_as_h2(f));
     }
@@ -1264,35 +1268,45 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
       // query fragments (B operand: head g; channels 16 ks + 2t (+1) and 16 ks + 2t + 8 (+9))
       if constexpr (MHA) {
         mha_query<GROUP>(a, b, h, lane, qb, qh, qs0, qs1);
-      } else if (g < G) {
-        const __nv_bfloat16* qp =
-            static_cast<const __nv_bfloat16*>(a.q) + (size_t)(b * a.heads_q + h * G + g) * kHeadDim;
-        // every load first (the divisions below branch, which would otherwise keep later loads behind earlier ones)
-        float2 bal[8][2];
-#pragma unroll
-        for (int ks = 0; ks < 8; ++ks)
-#pragma unroll
-          for (int r = 0; r < 2; ++r) {
-            const int c = 16 * ks + 2 * t + 8 * r;
-            qb[ks][r] = *reinterpret_cast<const uint32_t*>(qp + c);
-            bal[ks][r] = !KCH && a.balancer ? *reinterpret_cast<const float2*>(a.balancer + h * kHeadDim + c)
-                                            : make_float2(1.f, 1.f);
-          }
-#pragma unroll
-        for (int ks = 0; ks < 8; ++ks)
-#pragma unroll
-          for (int r = 0; r < 2; ++r) {
-            const uint32_t w = qb[ks][r];
-            const float q0 = __uint_as_float(w << 16), q1 = __uint_as_float(w & 0xffff0000u);
-            if constexpr (KCH) {  // per-channel retained keys are not balanced
-              qh[ks][r] = pack_f16(q0, q1);
-            } else {
-              qh[ks][r] = pack_f16(__fdiv_rn(q0, bal[ks][r].x), __fdiv_rn(q1, bal[ks][r].y));  // Eq. 4
-            }
-          }
       } else {
+        // Column g < G holds query head g. The RQ = 8 / G rows of lanes g' = g + G j (j < RQ) share head g's
+        // fragments: row g' loads and divides (Eq. 4) the k-steps ks = j (mod RQ), every load before any division
+        // (the divisions branch), and the fragments reach row g by shuffles; rows g >= G then hold zeros.
+        constexpr int RQ = 8 / G;
+        const int hq = g % G, j = g / G;
+        const __nv_bfloat16* qp =
+            static_cast<const __nv_bfloat16*>(a.q) + (size_t)(b * a.heads_q + h * G + hq) * kHeadDim;
+        uint32_t qw[8 / RQ][2], fw[8 / RQ][2];
+        float2 bal[8 / RQ][2];
 #pragma unroll
-        for (int ks = 0; ks < 8; ++ks) qb[ks][0] = qb[ks][1] = qh[ks][0] = qh[ks][1] = 0u;
+        for (int m = 0; m < 8 / RQ; ++m)
+#pragma unroll
+          for (int r = 0; r < 2; ++r) {
+            const int c = 16 * (j + RQ * m) + 2 * t + 8 * r;
+            qw[m][r] = *reinterpret_cast<const uint32_t*>(qp + c);
+            bal[m][r] = !KCH && a.balancer ? *reinterpret_cast<const float2*>(a.balancer + h * kHeadDim + c)
+                                           : make_float2(1.f, 1.f);
+          }
+#pragma unroll
+        for (int m = 0; m < 8 / RQ; ++m)
+#pragma unroll
+          for (int r = 0; r < 2; ++r) {
+            const float q0 = __uint_as_float(qw[m][r] << 16), q1 = __uint_as_float(qw[m][r] & 0xffff0000u);
+            if constexpr (KCH)  // per-channel retained keys are not balanced
+              fw[m][r] = pack_f16(q0, q1);
+            else
+              fw[m][r] = pack_f16(__fdiv_rn(q0, bal[m][r].x), __fdiv_rn(q1, bal[m][r].y));
+          }
+#pragma unroll
+        for (int ks = 0; ks < 8; ++ks)
+#pragma unroll
+          for (int r = 0; r < 2; ++r) {  // k-step ks of head g: row g + G (ks mod RQ), its entry ks div RQ
+            const int src = 4 * ((g < G ? g : 0) + G * (ks % RQ)) + t;
+            const uint32_t wq = __shfl_sync(0xffffffffu, qw[ks / RQ][r], src);
+            const uint32_t wf = __shfl_sync(0xffffffffu, fw[ks / RQ][r], src);
+            qb[ks][r] = g < G ? wq : 0u;
+            qh[ks][r] = g < G ? wf : 0u;
+          }
       }
       logit_base = a.hi_logits ? a.hi_logits + (size_t)(b * a.heads_q + h * G) * a.hi_stride : nullptr;
       if (HB == 16 && a.ins_slots) {
