@@ -69,6 +69,10 @@ namespace {
 #ifndef MIKV_MHA_PATH
 #define MIKV_MHA_PATH 1
 #endif
+// L2 prefetch of the first head's query and balancer rows before the grid-dependency wait (0 turns it off).
+#ifndef MIKV_Q_PREFETCH
+#define MIKV_Q_PREFETCH 1
+#endif
 constexpr int kWarps = MIKV_ATTN_WARPS;     // independent warps per CTA
 constexpr int kThreads = kWarps * 32;
 constexpr int kNS = MIKV_ATTN_STAGES;       // ring stages per warp
@@ -1229,6 +1233,19 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) attention_kernel(const _
     for (int k = 0; k < kNS && u0 + k < u1; ++k) {
       prefetch_unit<BITS, GROUP, HB, KCH>(a, cp);
       cursor_next(cp, hu, n_u);
+    }
+  }
+  // the first head's query rows (G x 256 bytes) and balancer row (512 bytes) into L2, every line of both
+  if (MIKV_Q_PREFETCH && u0 < u1) {
+    const int b0 = ci.bh / a.heads_kv, h0 = ci.bh - b0 * a.heads_kv;
+    const char* qrow =
+        reinterpret_cast<const char*>(static_cast<const __nv_bfloat16*>(a.q) + (size_t)(b0 * a.heads_q + h0 * G) * kHeadDim);
+    constexpr int nq = 2 * G + 1;  // the rows need not start on a line
+    static_assert(nq + 5 <= 32, "one line per lane");
+    if (lane < nq) prefetch_l2(qrow + (lane < 2 * G ? 128 * lane : 256 * G - 1));
+    if (!KCH && a.balancer && lane >= nq && lane < nq + 5) {
+      const char* brow = reinterpret_cast<const char*>(a.balancer + h0 * kHeadDim);
+      prefetch_l2(brow + (lane - nq < 4 ? 128 * (lane - nq) : 4 * kHeadDim - 1));
     }
   }
   grid_dependency_wait();  // the cache and the query come from the kernels before this one

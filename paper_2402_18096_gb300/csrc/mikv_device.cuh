@@ -96,6 +96,11 @@ __device__ __forceinline__ void tma_prefetch_2d(const CUtensorMap* map, int x, i
                : "memory");
 }
 
+// Prefetch of the 128-byte line holding p into L2 only.
+__device__ __forceinline__ void prefetch_l2(const void* p) {
+  asm volatile("prefetch.global.L2 [%0];" ::"l"(reinterpret_cast<uint64_t>(p)) : "memory");
+}
+
 // L2 policy for data a kernel streams through once: its lines are evicted before others, so what the
 // kernel writes for the next one (logits, split partials) stays in L2 across the stream.
 __device__ __forceinline__ uint64_t l2_evict_first() {
