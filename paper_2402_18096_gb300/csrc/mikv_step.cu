@@ -29,12 +29,23 @@ struct SlotQuad {
 };
 
 template <int G>
-__device__ __forceinline__ void load_quad(const float* logit, const float* acc, const int32_t* tok, int hi_stride,
-                                          int v, SlotQuad<G>& q) {
+__device__ __forceinline__ void load_logits(const float* logit, int hi_stride, int v, SlotQuad<G>& q) {
 #pragma unroll
   for (int j = 0; j < G; ++j) q.lg[j] = reinterpret_cast<const float4*>(logit + (size_t)j * hi_stride)[v];
-  q.ac = reinterpret_cast<const float4*>(acc)[v];
-  q.tk = reinterpret_cast<const int4*>(tok)[v];
+}
+
+// Scores and ids through L2 only: also read before the grid-dependency wait (see step_post_kernel).
+template <int G>
+__device__ __forceinline__ void load_scores(const float* acc, const int32_t* tok, int v, SlotQuad<G>& q) {
+  q.ac = __ldcg(reinterpret_cast<const float4*>(acc) + v);
+  q.tk = __ldcg(reinterpret_cast<const int4*>(tok) + v);
+}
+
+template <int G>
+__device__ __forceinline__ void load_quad(const float* logit, const float* acc, const int32_t* tok, int hi_stride,
+                                          int v, SlotQuad<G>& q) {
+  load_logits<G>(logit, hi_stride, v, q);
+  load_scores<G>(acc, tok, v, q);
 }
 
 // Importance update of the slots of q below hi_cap (the arithmetic of update_importance_kernel: the
@@ -72,19 +83,37 @@ __global__ void __launch_bounds__(kPostThreads, 2) step_post_kernel(const StepPo
   __shared__ int s_victim;
   const int bh = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int b = bh / a.heads_kv, h = bh - b * a.heads_kv;
-  grid_dependency_wait();  // logits and partials come from the attention kernel
-  allow_dependent_launch();
   float* acc = a.acc + (size_t)bh * a.hi_stride;
   const int32_t* tok = a.hi_tok + (size_t)bh * a.hi_stride;
   const float* logit = a.hi_logits + (size_t)(b * a.heads_q + h * G) * a.hi_stride;
   const int nv = (a.hi_cap + 3) / 4;  // groups of four slots
 
-  // 0. this thread's first groups of slots are loaded before the statistics, which they do not depend on
-  // (two groups each where registers allow: those loads overlap the statistics' loads below)
+  // 0. Scores and ids are read before the grid-dependency wait. This kernel starts only once every block of
+  // the attention kernel has passed its own wait, so every kernel before the attention kernel has completed;
+  // the attention kernel itself writes one of them: the slot it inserts the new token into (slots[bh], set by
+  // the previous step's tail), whose group is read again after the wait. The first groups of this thread go
+  // to registers, every line of the rest into L2.
   constexpr int kPre = G <= 4 ? 2 : 1;
   SlotQuad<G> q0, qp;
-  if (tid < nv) load_quad<G>(logit, acc, tok, a.hi_stride, tid, q0);
-  if (kPre == 2 && tid + kPostThreads < nv) load_quad<G>(logit, acc, tok, a.hi_stride, tid + kPostThreads, qp);
+  const int ins = a.slots[bh];
+  if (tid < nv) load_scores<G>(acc, tok, tid, q0);
+  if (kPre == 2 && tid + kPostThreads < nv) load_scores<G>(acc, tok, tid + kPostThreads, qp);
+  for (int l = kPre * kPostThreads / 8 + tid; l < (nv + 7) / 8; l += kPostThreads) {  // 8 groups per line
+    prefetch_l2(acc + 32 * l);
+    prefetch_l2(tok + 32 * l);
+  }
+  grid_dependency_wait();  // logits, partials and the inserted slot come from the attention kernel
+  allow_dependent_launch();
+  // the first groups' logits are loaded before the statistics, which they do not depend on (two groups each
+  // where registers allow: those loads overlap the statistics' loads below)
+  if (tid < nv) {
+    load_logits<G>(logit, a.hi_stride, tid, q0);
+    if (ins >> 2 == tid) load_scores<G>(acc, tok, tid, q0);
+  }
+  if (kPre == 2 && tid + kPostThreads < nv) {
+    load_logits<G>(logit, a.hi_stride, tid + kPostThreads, qp);
+    if (ins >> 2 == tid + kPostThreads) load_scores<G>(acc, tok, tid + kPostThreads, qp);
+  }
 
   // 1. softmax statistics (M, L) of query heads h*G .. h*G+G-1 from the split partials (one warp per head)
   const int w0 = owner_warp((long long)bh * a.n_u, a.n_units, a.n_warps);
