@@ -24,6 +24,10 @@
  *   - Layouts are dense row-major in the index order written next to each argument.
  *   - The head dimension d is 128; the query-head group size G = heads_q / heads_kv is 1, 2, 4 or 8
  *     (grouped-query attention: query head j reads KV head j / G).
+ *   - Each compute entry point (balancer, quantize/pack, prefill scores, attention, importance update,
+ *     select/demote, insert, gather, decode step) marks its host time with one NVTX range named after
+ *     the call (NVTX v3, header-only: inert unless a tool such as Nsight is attached; a build with
+ *     -DMIKV_NVTX=0 leaves the ranges out).
  *
  * Packed-code layout of one retained row (d = 128, N bits, 16 * N bytes): channel c is written
  * c = 16 m + u (u = c mod 16, m = c div 16) and a plane is a sequence of little-endian 16-bit units.

@@ -9,11 +9,35 @@
 
 #include <mutex>
 
+#ifndef MIKV_NVTX
+#define MIKV_NVTX 1
+#endif
+#if MIKV_NVTX
+#include <nvtx3/nvToolsExt.h>
+#endif
+
 #include "mikv_device.cuh"
 #include "mikv_internal.h"
 #include "mikv_prefill.h"
 
 using namespace mikv;
+
+namespace {
+// One NVTX range per compute entry point, named after the call, around its validation and launches (host time:
+// the kernels run later on the stream). Without a tool attached, push and pop return at once; -DMIKV_NVTX=0
+// leaves them out.
+struct CallRange {
+#if MIKV_NVTX
+  explicit CallRange(const char* name) { nvtxRangePushA(name); }
+  ~CallRange() { nvtxRangePop(); }
+#else
+  explicit CallRange(const char*) {}
+#endif
+  CallRange(const CallRange&) = delete;
+  CallRange& operator=(const CallRange&) = delete;
+};
+}  // namespace
+#define MIKV_CALL_RANGE() const CallRange mikv_call_range_(__func__)
 
 // The library's own status word for the index checks of debug builds (-DMIKV_DEBUG) in the entry points that take
 // no workspace (insertion, gather, quantize/pack). Looked up in the current context on every use.
@@ -336,6 +360,7 @@ mikv_status mikv_workspace_check(const void* workspace, void* stream) {
 
 mikv_status mikv_compute_balancer(const mikv_shape* shape, const void* q_pre, const void* k_pre, int32_t T,
                                   float* balancer_out, void* workspace, size_t ws_bytes, void* stream) {
+  MIKV_CALL_RANGE();
   mikv_status st = shape_supported(shape);
   if (st != MIKV_OK) return st;
   if (!q_pre || !k_pre || !balancer_out || T <= 0) return MIKV_ERR_ARG;
@@ -349,6 +374,7 @@ mikv_status mikv_compute_balancer(const mikv_shape* shape, const void* q_pre, co
 mikv_status mikv_quantize_pack(const mikv_shape* shape, const mikv_cache* cache, const void* k_src,
                                const void* v_src, const int32_t* src_tok, int32_t n_src, const int32_t* rows,
                                int32_t n_rows, int32_t lo_start, void* stream) {
+  MIKV_CALL_RANGE();
   mikv_status st = shape_supported(shape);
   if (st != MIKV_OK) return st;
   if (evicting(*shape)) return MIKV_ERR_UNSUPPORTED;  // no retained set to write
@@ -370,6 +396,7 @@ mikv_status mikv_quantize_pack(const mikv_shape* shape, const mikv_cache* cache,
 
 mikv_status mikv_prefill_scores(const mikv_shape* shape, const void* q_pre, const void* k_pre, int32_t T,
                                 float sm_scale, float* scores, void* workspace, size_t ws_bytes, void* stream) {
+  MIKV_CALL_RANGE();
   mikv_status st = shape_supported(shape);
   if (st != MIKV_OK) return st;
   if (!q_pre || !k_pre || !scores || T <= 0) return MIKV_ERR_ARG;
@@ -407,6 +434,7 @@ mikv_status mikv_prefill_scores(const mikv_shape* shape, const void* q_pre, cons
 mikv_status mikv_decode_attention(const mikv_shape* shape, const mikv_cache* cache, int32_t n_lo, const void* q,
                                   float sm_scale, void* out, int32_t out_dtype, float* hi_logits, float* ml,
                                   void* workspace, size_t ws_bytes, void* stream) {
+  MIKV_CALL_RANGE();
   mikv_status st = attention_args_ok(shape, cache, n_lo, q, out, out_dtype);
   if (st != MIKV_OK) return st;
   if (!workspace || !aligned(workspace, 256)) return MIKV_ERR_WORKSPACE;
@@ -416,6 +444,7 @@ mikv_status mikv_decode_attention(const mikv_shape* shape, const mikv_cache* cac
 
 mikv_status mikv_update_importance(const mikv_shape* shape, const mikv_cache* cache, const float* hi_logits,
                                    const float* ml, void* stream) {
+  MIKV_CALL_RANGE();
   mikv_status st = shape_supported(shape);
   if (st != MIKV_OK) return st;
   if (!cache_ok(cache, shape) || !hi_logits || !ml) return MIKV_ERR_ARG;
@@ -425,6 +454,7 @@ mikv_status mikv_update_importance(const mikv_shape* shape, const mikv_cache* ca
 
 mikv_status mikv_select_demote(int32_t batch, int32_t heads, const float* scores, const int32_t* ids, int32_t n,
                                int32_t stride, int32_t n_demote, int32_t* demoted, int32_t* kept, void* stream) {
+  MIKV_CALL_RANGE();
   if (batch <= 0 || heads <= 0 || !scores || n < 0 || stride < n || n_demote < 0 || n_demote > n) return MIKV_ERR_ARG;
   if (n_demote > 0 && !demoted) return MIKV_ERR_ARG;
   if ((int64_t)batch * heads > 2147483647) return MIKV_ERR_UNSUPPORTED;
@@ -435,6 +465,7 @@ mikv_status mikv_select_demote(int32_t batch, int32_t heads, const float* scores
 
 mikv_status mikv_insert_token(const mikv_shape* shape, const mikv_cache* cache, const void* k_new,
                               const void* v_new, int32_t tok, const int32_t* slots, void* stream) {
+  MIKV_CALL_RANGE();
   mikv_status st = shape_supported(shape);
   if (st != MIKV_OK) return st;
   if (!cache_ok(cache, shape) || !k_new || !v_new || !slots) return MIKV_ERR_ARG;
@@ -445,6 +476,7 @@ mikv_status mikv_insert_token(const mikv_shape* shape, const mikv_cache* cache, 
 mikv_status mikv_gather_hi(const mikv_shape* shape, const mikv_cache* cache, const void* k_src, const void* v_src,
                            const int32_t* src_tok, const float* src_scores, int32_t n_src, const int32_t* rows,
                            int32_t n_rows, void* stream) {
+  MIKV_CALL_RANGE();
   mikv_status st = shape_supported(shape);
   if (st != MIKV_OK) return st;
   if (!cache_ok(cache, shape) || !k_src || !v_src || n_src <= 0 || n_rows < 0 || (n_rows > 0 && !rows))
@@ -457,6 +489,7 @@ mikv_status mikv_gather_hi(const mikv_shape* shape, const mikv_cache* cache, con
 mikv_status mikv_decode_step(const mikv_shape* shape, const mikv_cache* cache, int32_t n_lo, const void* q,
                              const void* k_new, const void* v_new, int32_t tok, int32_t* slots, float sm_scale,
                              void* out, int32_t out_dtype, void* workspace, size_t ws_bytes, void* stream) {
+  MIKV_CALL_RANGE();
   mikv_status st = shape_supported(shape);
   if (st != MIKV_OK) return st;
   if (!cache_ok(cache, shape) || !q || !k_new || !v_new || !slots || !out || n_lo < 0) return MIKV_ERR_ARG;
@@ -566,6 +599,7 @@ mikv_status noalloc_scratch(void** out) {
 extern "C" mikv_status mikv_decode_attention_noalloc(const mikv_shape* shape, const mikv_cache* cache, int32_t n_lo,
                                                      const void* q, float sm_scale, void* out, int32_t out_dtype,
                                                      float* hi_logits, float* ml, void* stream) {
+  MIKV_CALL_RANGE();
   mikv_status st = attention_args_ok(shape, cache, n_lo, q, out, out_dtype);
   if (st != MIKV_OK) return st;
   const size_t need = attention_workspace_bytes(*shape, n_lo, num_sms());
