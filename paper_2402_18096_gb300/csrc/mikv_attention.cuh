@@ -82,7 +82,8 @@ constexpr int kStageBytes = kUnitBytes;
 constexpr int kHiBlockBytes = 8192;         // K and V of 16 tokens: 4 boxes of 16 rows x 64 bf16
 constexpr int kCtasPerSm = MIKV_ATTN_CTAS;
 constexpr int kQkAcc = MIKV_QK_ACC;         // independent accumulators of the QK^T MMA chain
-constexpr int kUnitsPerWarp = 24;    // target share per warp (sizes the grid for small caches)
+constexpr int kUnitsPerWarp = 24;    // share the grid sizing starts from; the plan then fills every warp slot
+                                     // it can (min(units, slots) warps)
 constexpr float kLog2e = 1.4426950408889634f;
 
 __host__ __device__ constexpr int smem_bytes() { return 1024 + kWarps * kNS * kStageBytes + kWarps * kNS * 8; }
