@@ -705,7 +705,7 @@ def run_prefill(args):
     # algorithmic work: two passes (row statistics, column sums) over the causal triangle of Q K^T
     flops = 2.0 * w.batch * w.heads_q * (T * (T + 1) / 2) * 2 * w.head_dim
     tflops = flops / ms / 1e9
-    # a timed loop of a second or more runs under the power cap: it is judged against the sustained bf16 peak,
+    # a timed loop of a second or more runs under the power cap: it is compared with the sustained bf16 peak,
     # shorter ones against the burst peak
     sustained = ms * args.steps >= 1000.0
     peak, kind = None, "fallback"
